@@ -1,0 +1,157 @@
+"""Group-wise asymmetric min-max quantizer and Hadamard pre-rotation (oracle).
+
+TEST INFRASTRUCTURE ONLY -- see ``oracle/__init__.py``.
+
+Paper passages followed
+-----------------------
+* Sec. 2 / Sec. 4.1 "Base quantizers": KIVI quantizes keys per channel and
+  values per token; QuaRot rotates with a Hadamard matrix and then quantizes
+  per token.
+* App. W "KIVI kernel": K_hat[:, j] = Q_b(K[:, j], scale_j) (per channel),
+  V_hat[t, :] = Q_b(V[t, :], scale_t) (per token).
+* App. W "QuaRot kernel": X_hat = Q_b(X R) R^T with R orthogonal.
+
+The paper gives no formula for the asymmetric min-max quantizer Q_b. The
+reading used here (every step in the stated precision, in this order) is:
+
+  for one group x[0..31] (fp16/bf16 values, exact in fp32) and b in 1..8:
+    v   = fp32(x) + 0.0f              (turns -0 into +0; min/max then unique)
+    mn  = min v,  mx = max v          (exact)
+    L   = 2^b - 1
+    s32 = fp32_rn(fp32_rn(mx - mn) / L)
+    scale = fp16_rn(s32),  zero = fp16_rn(mn)        (both stored)
+    sf = fp32(scale), zf = fp32(zero)
+    if sf == 0: every code is 0
+    else:  inv = fp32_rn(1 / sf)
+           c_j = clamp(rint_half_even(fp32_rn(fp32_rn(v_j - zf) * inv)), 0, L)
+    dequantized value  x_hat_j = fp32_rn(fp32_rn(fp32(c_j) * sf) + zf)
+
+  A group holding a non-finite value, or whose fp16 scale or zero overflows,
+  is a numeric failure: codes 0, scale 0, zero 0, and the failure is reported.
+
+Rotation (QuaRot reading of "Hadamard" / "random orthogonal R"):
+  y = FWHT(x * sigma) * fp32_rn(1/sqrt(128)), in fp32, butterfly stages with
+  stride 1, 2, 4, ..., 64 in that order; each stage maps the pair (i, i+h),
+  i with bit h clear, to (a + b, a - b). sigma is a caller-supplied +-1 vector
+  (all +1 when absent). R = diag(sigma) H / sqrt(128) is orthogonal.
+"""
+from __future__ import annotations
+
+import numpy as np
+
+GROUP = 32
+HEAD_DIM = 128
+PER_TOKEN = 0
+PER_CHANNEL = 1
+
+# fp32 round-to-nearest of 1/sqrt(128) = 2^-3.5
+INV_SQRT_128_F32 = np.float32(0.08838834764831845)
+
+
+def canonical(v: np.ndarray) -> np.ndarray:
+    """fp32 values with -0 replaced by +0 (IEEE: -0 + +0 = +0)."""
+    return (np.asarray(v, dtype=np.float32) + np.float32(0.0)).astype(np.float32)
+
+
+def hadamard_rotate(x: np.ndarray, signs: np.ndarray | None) -> np.ndarray:
+    """Rotate the last axis (length 128) by R = diag(signs) H / sqrt(128), fp32."""
+    y = np.array(x, dtype=np.float32, copy=True)
+    assert y.shape[-1] == HEAD_DIM
+    if signs is not None:
+        y = y * np.asarray(signs, dtype=np.float32)
+    lead = y.shape[:-1]
+    h = 1
+    while h < HEAD_DIM:
+        y = y.reshape(lead + (HEAD_DIM // (2 * h), 2, h))
+        a = y[..., 0, :]
+        b = y[..., 1, :]
+        y = np.stack([a + b, a - b], axis=-2).reshape(lead + (HEAD_DIM,))
+        h *= 2
+    return (y * INV_SQRT_128_F32).astype(np.float32)
+
+
+def quantize_groups(v: np.ndarray, b: int):
+    """Quantize groups along the last axis (length 32) at b bits.
+
+    Returns (codes uint8, scale float16, zero float16, bad bool), the last
+    three with the group shape (last axis removed).
+    """
+    assert 1 <= b <= 8
+    v = canonical(v)
+    assert v.shape[-1] == GROUP
+    with np.errstate(all="ignore"):
+        finite = np.isfinite(v).all(axis=-1)
+        vv = np.where(finite[..., None], v, np.float32(0.0))
+        mn = vv.min(axis=-1)
+        mx = vv.max(axis=-1)
+        L = np.float32(2 ** b - 1)
+        s32 = ((mx - mn).astype(np.float32) / L).astype(np.float32)
+        scale = s32.astype(np.float16)
+        zero = mn.astype(np.float16)
+        bad = (~finite) | (~np.isfinite(scale)) | (~np.isfinite(zero))
+        sf = scale.astype(np.float32)
+        zf = zero.astype(np.float32)
+        ok = (~bad) & (sf != np.float32(0.0))
+        inv = (np.float32(1.0) / np.where(ok, sf, np.float32(1.0))).astype(np.float32)
+        d = (vv - zf[..., None]).astype(np.float32)
+        t = (d * inv[..., None]).astype(np.float32)
+        c = np.clip(np.rint(t), np.float32(0.0), L)
+        codes = np.where(ok[..., None], c, np.float32(0.0)).astype(np.uint8)
+    scale = np.where(bad, np.float16(0.0), scale).astype(np.float16)
+    zero = np.where(bad, np.float16(0.0), zero).astype(np.float16)
+    return codes, scale, zero, bad
+
+
+def dequantize_groups(codes: np.ndarray, scale: np.ndarray, zero: np.ndarray) -> np.ndarray:
+    """x_hat = fp32(c) * sf + zf as two rounded fp32 operations (no FMA)."""
+    sf = np.asarray(scale, dtype=np.float16).astype(np.float32)[..., None]
+    zf = np.asarray(zero, dtype=np.float16).astype(np.float32)[..., None]
+    prod = (codes.astype(np.float32) * sf).astype(np.float32)
+    return (prod + zf).astype(np.float32)
+
+
+def to_groups(x: np.ndarray, grouping: int) -> np.ndarray:
+    """View one stream x[S, 128] as groups of 32.
+
+    PER_TOKEN:   groups[t, G, :]   = x[t, 32G : 32G+32]
+    PER_CHANNEL: groups[blk, c, :] = x[32 blk : 32 blk + 32, c]   (S % 32 == 0)
+    """
+    S, d = x.shape
+    assert d == HEAD_DIM
+    if grouping == PER_TOKEN:
+        return x.reshape(S, HEAD_DIM // GROUP, GROUP)
+    assert S % GROUP == 0, "per-channel groups need S % 32 == 0"
+    return x.reshape(S // GROUP, GROUP, HEAD_DIM).transpose(0, 2, 1)
+
+
+def from_groups(g: np.ndarray, grouping: int) -> np.ndarray:
+    """Inverse of ``to_groups``: back to [S, 128]."""
+    if grouping == PER_TOKEN:
+        S = g.shape[0]
+        return g.reshape(S, HEAD_DIM)
+    nblk = g.shape[0]
+    return g.transpose(0, 2, 1).reshape(nblk * GROUP, HEAD_DIM)
+
+
+def quantize_stream(x: np.ndarray, grouping: int, b: int, signs: np.ndarray | None = None,
+                    hadamard: bool = False):
+    """Quantize one (batch, head, K/V) stream x[S, 128].
+
+    Returns dict with the quantizer-domain values ``y`` [S,128] (rotated when
+    ``hadamard``), ``codes`` [S,128] uint8 (element order), group-shaped
+    ``scale``/``zero``/``bad``, and ``xhat`` [S,128] fp32 in the quantizer domain.
+    """
+    x = np.asarray(x, dtype=np.float32)
+    y = hadamard_rotate(x, signs) if hadamard else x.astype(np.float32)
+    y = canonical(y)
+    g = to_groups(y, grouping)
+    codes, scale, zero, bad = quantize_groups(g, b)
+    xhat = dequantize_groups(codes, scale, zero)
+    return {
+        "y": y,
+        "codes": from_groups(codes, grouping),
+        "scale": scale,
+        "zero": zero,
+        "bad": bad,
+        "xhat": from_groups(xhat, grouping),
+    }

@@ -1,0 +1,179 @@
+"""Pins for the oracle quantizer and rotation (CPU only).
+
+Each test checks the oracle against something other than itself: exact
+reconstruction cases, the uniform-quantization noise law s^2/12, the error
+bound |x - x_hat| <= s/2, monotonicity in b, and the textbook Sylvester /
+scipy Hadamard matrix.
+"""
+import numpy as np
+import pytest
+import scipy.linalg
+
+from oracle import quant
+from oracle.attention import rotation_matrix, sylvester_hadamard
+
+
+@pytest.mark.parametrize("b", range(1, 9))
+def test_constant_group_is_exact(b):
+    # A constant group has zero range: scale 0, every code 0, x_hat = x
+    # exactly when the value is representable in fp16 (App. W KIVI kernel,
+    # 8-bit case included).
+    for val in (0.0, 1.5, -3.25, 1000.0, 2.0 ** -14):
+        x = np.full((3, 32), val, dtype=np.float32)
+        codes, scale, zero, bad = quant.quantize_groups(x, b)
+        assert not bad.any()
+        assert (codes == 0).all()
+        assert (scale == 0).all()
+        xhat = quant.dequantize_groups(codes, scale, zero)
+        assert np.array_equal(xhat, x)
+
+
+def test_integer_group_at_8_bits_is_exact():
+    # Values 0..255 in one group of 32 (min 0, max 255): scale = 255/255 = 1,
+    # zero = 0, codes equal the values, reconstruction is exact.
+    rng = np.random.default_rng(1)
+    x = rng.integers(0, 256, size=(64, 32)).astype(np.float32)
+    x[:, 0] = 0.0
+    x[:, 1] = 255.0
+    codes, scale, zero, bad = quant.quantize_groups(x, 8)
+    assert (scale == 1.0).all() and (zero == 0.0).all() and not bad.any()
+    assert np.array_equal(codes.astype(np.float32), x)
+    assert np.array_equal(quant.dequantize_groups(codes, scale, zero), x)
+
+
+@pytest.mark.parametrize("b", range(1, 9))
+def test_error_bound_half_step(b):
+    # Asymmetric min-max rounding: |x - x_hat| <= s/2 plus the fp16 rounding
+    # of the zero-point and of the scale times the code range.
+    rng = np.random.default_rng(b)
+    x = rng.standard_normal((2048, 32)).astype(np.float32) * 3.0
+    codes, scale, zero, bad = quant.quantize_groups(x, b)
+    xhat = quant.dequantize_groups(codes, scale, zero)
+    sf = scale.astype(np.float64)[:, None]
+    mn = x.min(axis=1, keepdims=True).astype(np.float64)
+    zslack = np.abs(zero.astype(np.float64)[:, None] - mn)
+    L = 2 ** b - 1
+    s_exact = (x.max(axis=1, keepdims=True) - mn) / L
+    sslack = L * np.abs(sf - s_exact)
+    err = np.abs(x.astype(np.float64) - xhat)
+    assert (err <= sf / 2 + zslack + sslack + 1e-6).all()
+    assert codes.max() <= L
+
+
+def test_mse_decreases_with_bits():
+    # D(b) strictly decreasing in b on Gaussian groups (Assumption 1, beta > 1).
+    rng = np.random.default_rng(7)
+    x = rng.standard_normal((65536 // 32 * 32, 32)).astype(np.float32)
+    mse = []
+    for b in range(1, 9):
+        codes, scale, zero, _ = quant.quantize_groups(x, b)
+        xhat = quant.dequantize_groups(codes, scale, zero)
+        mse.append(np.mean((x.astype(np.float64) - xhat) ** 2))
+    assert all(mse[i + 1] < mse[i] for i in range(7)), mse
+
+
+@pytest.mark.parametrize("b", [2, 4, 6])
+def test_uniform_noise_law(b):
+    # Uniform data filling [0, 1] with both ends present: the error of a
+    # uniform quantizer with step s is uniform on [-s/2, s/2], MSE = s^2/12
+    # (textbook high-resolution result). 3-sigma of the estimate ~ 2e-3.
+    rng = np.random.default_rng(100 + b)
+    n = 65536
+    x = rng.random((n, 32)).astype(np.float32)
+    x[:, 0] = 0.0
+    x[:, 1] = 1.0
+    codes, scale, zero, _ = quant.quantize_groups(x, b)
+    xhat = quant.dequantize_groups(codes, scale, zero)
+    # the two forced endpoints sit on grid points; measure the other 30 columns
+    mse = np.mean((x[:, 2:].astype(np.float64) - xhat[:, 2:]) ** 2)
+    s = float(scale[0])
+    assert (scale == scale[0]).all()
+    assert abs(mse / (s * s / 12.0) - 1.0) < 0.01
+
+
+def test_rounding_is_half_even_and_codes_use_stored_scale():
+    # One group, b = 2: values chosen so (x - zero)/scale lands exactly on .5.
+    # min 0, max 3 -> scale 1, zero 0; 0.5 -> 0, 1.5 -> 2, 2.5 -> 2 (ties to even).
+    x = np.zeros((1, 32), dtype=np.float32)
+    x[0, 1] = 3.0
+    x[0, 2] = 0.5
+    x[0, 3] = 1.5
+    x[0, 4] = 2.5
+    codes, scale, zero, _ = quant.quantize_groups(x, 2)
+    assert scale[0] == 1.0 and zero[0] == 0.0
+    assert list(codes[0, :5]) == [0, 3, 0, 2, 2]
+
+
+def test_negative_zero_is_canonical():
+    # -0 and +0 quantize the same way; the stored zero-point is +0.
+    x = np.zeros((2, 32), dtype=np.float32)
+    x[0, :] = -0.0
+    codes, scale, zero, bad = quant.quantize_groups(x, 3)
+    assert np.array_equal(zero.view(np.uint16), np.zeros(2, np.uint16))
+
+
+def test_numeric_failures_are_flagged():
+    x = np.zeros((4, 32), dtype=np.float32)
+    x[0, 3] = np.nan
+    x[1, 5] = np.inf
+    x[2, 0] = 1e6           # zero-point or range overflows fp16
+    x[2, 1] = -1e6
+    x[3, :] = np.arange(32)
+    codes, scale, zero, bad = quant.quantize_groups(x, 4)
+    assert list(bad) == [True, True, True, False]
+    assert (codes[:3] == 0).all() and (scale[:3] == 0).all() and (zero[:3] == 0).all()
+
+
+def test_grouping_views_round_trip():
+    rng = np.random.default_rng(3)
+    x = rng.standard_normal((96, 128)).astype(np.float32)
+    for gp in (quant.PER_TOKEN, quant.PER_CHANNEL):
+        g = quant.to_groups(x, gp)
+        assert np.array_equal(quant.from_groups(g, gp), x)
+    g = quant.to_groups(x, quant.PER_CHANNEL)
+    assert np.array_equal(g[1, 5], x[32:64, 5])          # 32 tokens of channel 5
+    g = quant.to_groups(x, quant.PER_TOKEN)
+    assert np.array_equal(g[7, 2], x[7, 64:96])          # channels 64..95 of token 7
+
+
+def test_sylvester_matches_scipy():
+    assert np.array_equal(sylvester_hadamard(128), scipy.linalg.hadamard(128))
+
+
+def test_rotation_orthogonal():
+    rng = np.random.default_rng(5)
+    signs = rng.choice([-1, 1], size=128).astype(np.int8)
+    R = rotation_matrix(signs)
+    assert np.allclose(R @ R.T, np.eye(128), atol=1e-12)
+
+
+def test_fwht_of_unit_vectors_is_hadamard_column():
+    # FWHT(e_k)/sqrt(128) is row k of H/sqrt(128) (H symmetric).
+    H = scipy.linalg.hadamard(128).astype(np.float64) / np.sqrt(128)
+    E = np.eye(128, dtype=np.float32)
+    Y = quant.hadamard_rotate(E, None).astype(np.float64)
+    assert np.allclose(Y, H, rtol=1e-7, atol=0)
+
+
+def test_fwht_matches_matrix_product():
+    rng = np.random.default_rng(9)
+    signs = rng.choice([-1, 1], size=128).astype(np.int8)
+    x = rng.standard_normal((200, 128)).astype(np.float32)
+    y = quant.hadamard_rotate(x, signs).astype(np.float64)
+    ref = x.astype(np.float64) @ (np.diag(signs.astype(np.float64))
+                                  @ scipy.linalg.hadamard(128) / np.sqrt(128))
+    assert np.allclose(y, ref, rtol=0, atol=1e-5 * np.abs(ref).max())
+
+
+def test_rotation_preserves_mse():
+    # R orthogonal: the error measured in the rotated domain equals the error
+    # after rotating back, up to fp32/fp64 rounding.
+    rng = np.random.default_rng(11)
+    signs = rng.choice([-1, 1], size=128).astype(np.int8)
+    x = rng.standard_normal((256, 128)).astype(np.float32)
+    r = quant.quantize_stream(x, quant.PER_TOKEN, 4, signs, hadamard=True)
+    e_rot = np.mean((r["y"].astype(np.float64) - r["xhat"]) ** 2)
+    R = rotation_matrix(signs)
+    back = r["xhat"].astype(np.float64) @ R.T
+    e_orig = np.mean((x.astype(np.float64) - back) ** 2)
+    assert abs(e_rot / e_orig - 1.0) < 1e-5
