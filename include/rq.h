@@ -1,0 +1,195 @@
+/*
+ * rq.h -- C ABI of librq, the GB300 (sm_103a) hot path of RateQuant
+ * (arXiv 2605.06675): per-head mixed-bit KV-cache quantization chosen by
+ * reverse waterfilling, bit-packing, and decode attention that reads the
+ * packed cache directly.
+ *
+ * Conventions for every entry point
+ * ---------------------------------
+ * - Plain C types only. Device pointers are ordinary pointers into device
+ *   memory the caller owns; `stream` is a cudaStream_t passed as void*
+ *   (NULL = legacy default stream). librq never allocates memory and keeps no
+ *   state between calls apart from a cached per-device SM count.
+ * - Arguments are validated on the host before anything is launched; a bad
+ *   argument returns an error code and launches nothing. A failed launch
+ *   returns RQ_ERR_CUDA. Device entry points are asynchronous on `stream`.
+ * - Conditions the device detects (non-finite input, a bit-width outside
+ *   1..8 in the device table) are OR-ed into `*status_dev` (a device uint32;
+ *   may be NULL) as RQ_STATUS_* bits; the kernels still write defined values
+ *   and never trap or spin.
+ * - Host-only functions are pure and thread-safe.
+ *
+ * Indexing
+ * --------
+ * - Component index of (layer l, kv head h, kind): i = (l * H_kv + h) * 2 + kind,
+ *   kind 0 = K, 1 = V (Sec. 3.4 "K/V separation": 2N components share one budget).
+ * - Bit table: uint8 bits[L][H_kv][2], the paper's static per-head lookup
+ *   table (Sec. 3.4 "Pipeline summary"; App. M "No runtime overhead").
+ * - GQA: query head j reads kv head j / (H_q / H_kv) (Sec. 4.1 "Models").
+ * - Caches: one layer's K and V are [B][H_kv][S][d] contiguous, fp16 or bf16.
+ */
+#ifndef RQ_H
+#define RQ_H
+
+#include <stddef.h>
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+#define RQ_ABI_VERSION 1
+#define RQ_HEAD_DIM 128
+#define RQ_GROUP 32
+#define RQ_MAX_GQA 8
+
+typedef enum {
+  RQ_OK = 0,
+  RQ_ERR_INVALID_ARG = 1, /* NULL pointer, bad enum, n <= 0, ... */
+  RQ_ERR_INFEASIBLE = 2,  /* budget not reachable with the allowed bit set */
+  RQ_ERR_SHAPE = 3,       /* unsupported shape (d != 128, S % 32 != 0, ...) */
+  RQ_ERR_ALIGNMENT = 4,   /* a device pointer is not 16-byte aligned */
+  RQ_ERR_WORKSPACE = 5,   /* workspace smaller than the *_workspace_bytes query */
+  RQ_ERR_CUDA = 6         /* a CUDA runtime call or launch failed */
+} rq_status;
+
+/* bits OR-ed into *status_dev by the kernels */
+#define RQ_STATUS_NUMERIC 1u  /* a group held NaN/inf or its fp16 scale/zero overflowed */
+#define RQ_STATUS_BAD_BITS 2u /* a device bit-table entry was outside 1..8; stream skipped */
+
+typedef enum { RQ_F16 = 0, RQ_BF16 = 1 } rq_dtype;
+
+/* RQ_PER_TOKEN: a group is 32 consecutive channels of one token (KIVI values,
+ * QuaRot); RQ_PER_CHANNEL: 32 consecutive tokens of one channel (KIVI keys).
+ * Sec. 2 "KV cache quantization", App. W "KIVI kernel". */
+typedef enum { RQ_PER_TOKEN = 0, RQ_PER_CHANNEL = 1 } rq_grouping;
+
+/* allocation flags */
+#define RQ_CAP_5X 1u /* w_i <- min(w_i, 5 * mean w) first (App. W "Mitigation") */
+
+typedef struct {
+  int32_t L;          /* layers */
+  int32_t B;          /* batch */
+  int32_t H_kv;       /* kv heads */
+  int32_t H_q;        /* query heads; H_q % H_kv == 0, H_q / H_kv <= 8 */
+  int32_t S;          /* cached tokens; S % 32 == 0 */
+  int32_t d;          /* head dim; must be 128 */
+  int32_t group;      /* group size; must be 32 */
+  int32_t dtype;      /* rq_dtype of K, V and q */
+  int32_t k_grouping; /* rq_grouping of keys */
+  int32_t v_grouping; /* rq_grouping of values */
+  int32_t hadamard;   /* 1: rotate K and V per token by R = diag(signs) H / sqrt(128)
+                         before quantizing (QuaRot, App. W "QuaRot kernel") */
+} rq_cache_desc;
+
+const char* rq_status_string(rq_status s);
+int32_t rq_abi_version(void);
+
+/* ---------------------------------------------------------------- host ---- */
+
+/* Fit D(b) = alpha * beta^-b per component by unweighted least squares of
+ * ln D on b over b in [b_lo, b_hi] with D(b) > 0 (Assumption 1; Alg. 1 stage 2;
+ * Sec. 3.4 "Distortion calibration"). mse: host [n][8], column k = D(k+1).
+ * R^2 on ln D is returned in r2. If r2_min > 0, a component with
+ * R^2 < r2_min gets beta = min(beta, mean fitted beta of its class)
+ * (App. W "Outlier heads"); classes: host [n] (NULL = one class).
+ * Fewer than two positive points: alpha = 0, beta = +inf, r2 = 1.
+ * Outputs: host arrays of n doubles. Errors: RQ_ERR_INVALID_ARG. */
+rq_status rq_fit_distortion(int32_t n, const double* mse, int32_t b_lo, int32_t b_hi,
+                            double r2_min, const int32_t* classes, double* alpha,
+                            double* beta, double* r2);
+
+/* Integer allocation of Eq. 1: minimise sum_i w_i alpha_i beta_i^-b_i with
+ * sum_i b_i = B = floor(avg_bits * n + 0.5) and every b_i in the allowed set
+ * (bit k of allowed_mask set <=> k bits allowed, k in 1..8).
+ * A contiguous set uses the greedy max-heap of Alg. 2 (marginal gain
+ * w alpha beta^-b (1 - 1/beta), ties to the lower index; optimal by Prop. 3).
+ * A non-contiguous set (e.g. {2,3,4,8}) uses an exact dynamic programme
+ * (ties: the larger bit-width for the lower index).
+ * flags: RQ_CAP_5X. Inputs/outputs are host arrays; bits_out: n uint8;
+ * objective_out (nullable): the minimised objective.
+ * Errors: RQ_ERR_INVALID_ARG, RQ_ERR_INFEASIBLE (B not reachable). */
+rq_status rq_alloc(int32_t n, const double* w, const double* alpha, const double* beta,
+                   double avg_bits, uint32_t allowed_mask, uint32_t flags, uint8_t* bits_out,
+                   double* objective_out);
+
+/* Continuous reverse waterfilling (Thm. 1, Eq. 2; App. B.1): free components
+ * satisfy w_i alpha_i ln(beta_i) beta_i^-b_i = lambda with sum b_i = avg_bits * n;
+ * components leaving [b_min, b_max] are clipped, fixed, and the rest
+ * re-solved until none leaves (App. B.1 "Iterative waterfilling").
+ * Requires beta_i > 1, w_i, alpha_i > 0. b_out: host n doubles.
+ * Errors: RQ_ERR_INVALID_ARG, RQ_ERR_INFEASIBLE. */
+rq_status rq_alloc_continuous(int32_t n, const double* w, const double* alpha,
+                              const double* beta, double avg_bits, double b_min, double b_max,
+                              double* b_out);
+
+/* Byte offsets of every packed stream and the buffer size.
+ * bits: host [L][H_kv][2]. offsets: host [L][B][H_kv][2] (uint64), filled in
+ * (layer, batch, head, kind) order. A stream of S tokens at b bits is S/32
+ * blocks of 512*(b+1) bytes: 512*b bytes of codes (32 lanes x 4b words in
+ * MMA-fragment order) then 512 bytes of fp16 scale/zero metadata.
+ * Errors: RQ_ERR_INVALID_ARG, RQ_ERR_SHAPE. */
+rq_status rq_packed_layout(const rq_cache_desc* desc, const uint8_t* bits, uint64_t* offsets,
+                           uint64_t* total_bytes);
+
+/* -------------------------------------------------------------- device ---- */
+
+/* Size of the workspace rq_calibrate_distortion needs for n components of T
+ * tokens: n * (T/32) * 8 doubles. */
+size_t rq_calibrate_workspace_bytes(int32_t n, int32_t T);
+
+/* Distortion sweep (Alg. 1 stage 2; Sec. 3.4 "Distortion calibration"):
+ * for every component i and b = 1..8, quantize-dequantize every group with
+ * the asymmetric min-max quantizer (after the per-token Hadamard rotation
+ * when `hadamard`) and store mse_dev[i][b-1] = mean over the component's
+ * T*128 elements of (y - y_hat)^2 in the quantizer's domain, fp64.
+ * x: device [n][T][128] of `dtype`; component i is a key (grouping
+ * k_grouping) when i is even, a value (v_grouping) when odd.
+ * signs_dev: device int8 [128] of +-1 (NULL = all +1; used when hadamard).
+ * ws: device workspace of rq_calibrate_workspace_bytes(n, T) bytes.
+ * Deterministic (fixed reduction order).
+ * Errors: RQ_ERR_INVALID_ARG, RQ_ERR_SHAPE (T % 32), RQ_ERR_ALIGNMENT,
+ * RQ_ERR_WORKSPACE, RQ_ERR_CUDA. */
+rq_status rq_calibrate_distortion(const void* x, int32_t dtype, int32_t n, int32_t T,
+                                  int32_t k_grouping, int32_t v_grouping, int32_t hadamard,
+                                  const int8_t* signs_dev, double* mse_dev, void* ws,
+                                  size_t ws_bytes, uint32_t* status_dev, void* stream);
+
+/* Quantize and pack one layer (the quantizer kernel indexing the per-head
+ * table, App. M / App. U): for every (batch, kv head, kind) stream, every
+ * group gets scale = fp16(fp32(max - min) / (2^b - 1)), zero = fp16(min),
+ * codes c = clamp(rint((x - zero) * (1/scale)), 0, 2^b - 1) (fp32), written
+ * to packed + offsets[layer][batch][head][kind] in the block format of
+ * rq_packed_layout. k, v: device [B][H_kv][S][128] of desc->dtype (16-byte
+ * aligned). bits_dev: device [L][H_kv][2]; offsets_dev: device copy of the
+ * rq_packed_layout offsets; packed: device buffer of total_bytes (16-byte
+ * aligned). signs_dev as in rq_calibrate_distortion.
+ * Errors: RQ_ERR_INVALID_ARG, RQ_ERR_SHAPE, RQ_ERR_ALIGNMENT, RQ_ERR_CUDA. */
+rq_status rq_quantize_pack(const rq_cache_desc* desc, int32_t layer, const void* k,
+                           const void* v, const int8_t* signs_dev, const uint8_t* bits_dev,
+                           const uint64_t* offsets_dev, void* packed, uint32_t* status_dev,
+                           void* stream);
+
+/* Workspace rq_decode_attention needs on the current device (split-K partials). */
+rq_status rq_decode_workspace_bytes(const rq_cache_desc* desc, size_t* bytes);
+
+/* Decode attention of one query per (batch, query head) over all S cached
+ * tokens of one layer, reading the packed mixed-bit cache directly
+ * (App. W "Kernel fusion"): out[b][j] = sum_t softmax_t(q_j . k_hat_t / sqrt(128)) v_hat_t
+ * with k_hat, v_hat the dequantized cache of kv head j / (H_q / H_kv); with
+ * desc->hadamard the rotated cache is used as Q(XR)R^T (App. W "QuaRot kernel").
+ * Split-K over the sequence with a log-sum-exp merge.
+ * q: device [B][H_q][128] of desc->dtype; out: device fp32 [B][H_q][128];
+ * ws: device workspace of at least rq_decode_workspace_bytes.
+ * Errors: RQ_ERR_INVALID_ARG, RQ_ERR_SHAPE (S == 0, S % 32, GQA > 8),
+ * RQ_ERR_ALIGNMENT, RQ_ERR_WORKSPACE, RQ_ERR_CUDA. */
+rq_status rq_decode_attention(const rq_cache_desc* desc, int32_t layer, const void* q,
+                              const void* packed, const uint8_t* bits_dev,
+                              const uint64_t* offsets_dev, const int8_t* signs_dev, float* out,
+                              void* ws, size_t ws_bytes, uint32_t* status_dev, void* stream);
+
+#ifdef __cplusplus
+}
+#endif
+
+#endif /* RQ_H */

@@ -93,40 +93,52 @@ def lane_word_to_block_word(lane: np.ndarray, w: np.ndarray) -> np.ndarray:
     return 128 * (w // 4) + 4 * lane + (w % 4)
 
 
-def pack_codes_block(tile: np.ndarray, kind: int, b: int) -> np.ndarray:
-    """Pack a 32x128 code tile into 128*b uint32 words (bit by bit)."""
-    tile = np.asarray(tile, dtype=np.int64)
-    assert tile.shape == (BLOCK_TOKENS, HEAD_DIM)
-    assert tile.min() >= 0 and tile.max() < (1 << b)
+def pack_codes_blocks(tiles: np.ndarray, kind: int, b: int) -> np.ndarray:
+    """Pack code tiles [nb, 32, 128] into [nb, 128*b] uint32 words, bit by bit."""
+    tiles = np.asarray(tiles).astype(np.int64)
+    nb = tiles.shape[0]
+    assert tiles.shape[1:] == (BLOCK_TOKENS, HEAD_DIM)
+    assert nb == 0 or (tiles.min() >= 0 and tiles.max() < (1 << b))
     lane, bitpos = code_positions(kind, b)
-    bits = np.zeros((32, 128 * b), dtype=np.int64)        # lane bit streams
+    bits = np.zeros((nb, 32, 128 * b), dtype=np.uint8)      # lane bit streams
     for k in range(b):
-        bits[lane, bitpos + k] = (tile >> k) & 1
-    lane_words = np.zeros((32, 4 * b), dtype=np.int64)
+        bits[:, lane, bitpos + k] = ((tiles >> k) & 1).astype(np.uint8)
+    lane_words = np.zeros((nb, 32, 4 * b), dtype=np.uint64)
     for j in range(32):
-        lane_words |= bits[:, j::32] << j
-    out = np.zeros(128 * b, dtype=np.uint32)
+        lane_words |= bits[:, :, j::32].astype(np.uint64) << np.uint64(j)
+    out = np.zeros((nb, 128 * b), dtype=np.uint32)
     L = np.arange(32)[:, None] * np.ones((1, 4 * b), dtype=np.int64)
     W = np.ones((32, 1), dtype=np.int64) * np.arange(4 * b)[None, :]
-    out[lane_word_to_block_word(L, W)] = lane_words.astype(np.uint32)
+    out[:, lane_word_to_block_word(L, W)] = lane_words.astype(np.uint32)
     return out
+
+
+def unpack_codes_blocks(words: np.ndarray, kind: int, b: int) -> np.ndarray:
+    """Inverse of ``pack_codes_blocks``: [nb, 128*b] words -> [nb, 32, 128] codes."""
+    words = np.asarray(words, dtype=np.uint32)
+    nb = words.shape[0]
+    assert words.shape[1:] == (128 * b,)
+    L = np.arange(32)[:, None] * np.ones((1, 4 * b), dtype=np.int64)
+    W = np.ones((32, 1), dtype=np.int64) * np.arange(4 * b)[None, :]
+    lane_words = words[:, lane_word_to_block_word(L, W)].astype(np.uint64)
+    bits = np.zeros((nb, 32, 128 * b), dtype=np.uint8)
+    for j in range(32):
+        bits[:, :, j::32] = ((lane_words >> np.uint64(j)) & np.uint64(1)).astype(np.uint8)
+    lane, bitpos = code_positions(kind, b)
+    tile = np.zeros((nb, BLOCK_TOKENS, HEAD_DIM), dtype=np.int64)
+    for k in range(b):
+        tile |= bits[:, lane, bitpos + k].astype(np.int64) << k
+    return tile.astype(np.uint8)
+
+
+def pack_codes_block(tile: np.ndarray, kind: int, b: int) -> np.ndarray:
+    """Pack a 32x128 code tile into 128*b uint32 words (bit by bit)."""
+    return pack_codes_blocks(np.asarray(tile)[None], kind, b)[0]
 
 
 def unpack_codes_block(words: np.ndarray, kind: int, b: int) -> np.ndarray:
     """Inverse of ``pack_codes_block``."""
-    words = np.asarray(words, dtype=np.uint32).astype(np.int64)
-    assert words.shape == (128 * b,)
-    L = np.arange(32)[:, None] * np.ones((1, 4 * b), dtype=np.int64)
-    W = np.ones((32, 1), dtype=np.int64) * np.arange(4 * b)[None, :]
-    lane_words = words[lane_word_to_block_word(L, W)]
-    bits = np.zeros((32, 128 * b), dtype=np.int64)
-    for j in range(32):
-        bits[:, j::32] = (lane_words >> j) & 1
-    lane, bitpos = code_positions(kind, b)
-    tile = np.zeros((BLOCK_TOKENS, HEAD_DIM), dtype=np.int64)
-    for k in range(b):
-        tile |= bits[lane, bitpos + k] << k
-    return tile.astype(np.uint8)
+    return unpack_codes_blocks(np.asarray(words)[None], kind, b)[0]
 
 
 def meta_layout(kind: int, grouping: int) -> str:
@@ -170,56 +182,64 @@ def meta_positions(kind: int, grouping: int):
     return 16 * (c % 8) + 2 * (c // 16) + (c // 8) % 2, None
 
 
-def pack_meta_block(scale: np.ndarray, zero: np.ndarray, kind: int, grouping: int) -> np.ndarray:
-    """Pack one block's 128 group (scale, zero) fp16 values into 128 words."""
-    s = np.asarray(scale, dtype=np.float16).reshape(-1).view(np.uint16).astype(np.uint32)
-    z = np.asarray(zero, dtype=np.float16).reshape(-1).view(np.uint16).astype(np.uint32)
-    assert s.shape == (128,) and z.shape == (128,)
+def pack_meta_blocks(scale: np.ndarray, zero: np.ndarray, kind: int, grouping: int) -> np.ndarray:
+    """Pack per-block group (scale, zero) fp16 values [nb, 128] into [nb, 128] words."""
+    s = np.asarray(scale, dtype=np.float16).reshape(-1, 128).view(np.uint16).astype(np.uint32)
+    z = np.asarray(zero, dtype=np.float16).reshape(-1, 128).view(np.uint16).astype(np.uint32)
+    nb = s.shape[0]
     word, half = meta_positions(kind, grouping)
-    out = np.zeros(META_WORDS, dtype=np.uint32)
+    out = np.zeros((nb, META_WORDS), dtype=np.uint32)
     if half is None:
-        out[word] = s | (z << 16)
+        out[:, word] = s | (z << np.uint32(16))
     else:
         # two groups share a word: one pass per half so no index repeats
         for h in (0, 1):
             m = half == h
-            out[word[m]] |= s[m] << np.uint32(16 * h)
-            out[64 + word[m]] |= z[m] << np.uint32(16 * h)
+            out[:, word[m]] |= s[:, m] << np.uint32(16 * h)
+            out[:, 64 + word[m]] |= z[:, m] << np.uint32(16 * h)
     return out
 
 
-def unpack_meta_block(words: np.ndarray, kind: int, grouping: int):
+def pack_meta_block(scale: np.ndarray, zero: np.ndarray, kind: int, grouping: int) -> np.ndarray:
+    """Pack one block's 128 group (scale, zero) fp16 values into 128 words."""
+    return pack_meta_blocks(np.asarray(scale)[None], np.asarray(zero)[None], kind, grouping)[0]
+
+
+def unpack_meta_blocks(words: np.ndarray, kind: int, grouping: int):
     words = np.asarray(words, dtype=np.uint32)
     word, half = meta_positions(kind, grouping)
     if half is None:
-        s = (words[word] & 0xFFFF).astype(np.uint16)
-        z = (words[word] >> 16).astype(np.uint16)
+        s = (words[:, word] & 0xFFFF).astype(np.uint16)
+        z = (words[:, word] >> 16).astype(np.uint16)
     else:
         sh = (16 * half).astype(np.uint32)
-        s = ((words[word] >> sh) & 0xFFFF).astype(np.uint16)
-        z = ((words[64 + word] >> sh) & 0xFFFF).astype(np.uint16)
+        s = ((words[:, word] >> sh) & 0xFFFF).astype(np.uint16)
+        z = ((words[:, 64 + word] >> sh) & 0xFFFF).astype(np.uint16)
     return s.view(np.float16), z.view(np.float16)
 
 
+def unpack_meta_block(words: np.ndarray, kind: int, grouping: int):
+    s, z = unpack_meta_blocks(np.asarray(words)[None], kind, grouping)
+    return s[0], z[0]
+
+
 def pack_stream(codes: np.ndarray, scale: np.ndarray, zero: np.ndarray, kind: int,
-                grouping: int, b: int) -> np.ndarray:
+                grouping: int, b: int, chunk: int = 256) -> np.ndarray:
     """Pack one stream: codes [S,128] (element order) and group-shaped
-    scale/zero (as returned by ``quant.quantize_stream``) into uint32 words."""
+    scale/zero (as returned by ``quant.quantize_stream``) into uint32 words:
+    block j = codes image of tokens [32j, 32j+32) then its meta image."""
     S = codes.shape[0]
     assert S % BLOCK_TOKENS == 0
     nblk = S // BLOCK_TOKENS
-    if grouping == PER_TOKEN:
-        sc = np.asarray(scale).reshape(nblk, BLOCK_TOKENS * 4)
-        ze = np.asarray(zero).reshape(nblk, BLOCK_TOKENS * 4)
-    else:
-        sc = np.asarray(scale).reshape(nblk, HEAD_DIM)
-        ze = np.asarray(zero).reshape(nblk, HEAD_DIM)
-    out = []
-    for j in range(nblk):
-        tile = codes[j * BLOCK_TOKENS:(j + 1) * BLOCK_TOKENS]
-        out.append(pack_codes_block(tile, kind, b))
-        out.append(pack_meta_block(sc[j], ze[j], kind, grouping))
-    return np.concatenate(out) if out else np.zeros(0, dtype=np.uint32)
+    tiles = np.asarray(codes).reshape(nblk, BLOCK_TOKENS, HEAD_DIM)
+    sc = np.asarray(scale).reshape(nblk, 128)
+    ze = np.asarray(zero).reshape(nblk, 128)
+    out = np.zeros((nblk, 128 * (b + 1)), dtype=np.uint32)
+    for j0 in range(0, nblk, chunk):
+        j1 = min(nblk, j0 + chunk)
+        out[j0:j1, :128 * b] = pack_codes_blocks(tiles[j0:j1], kind, b)
+        out[j0:j1, 128 * b:] = pack_meta_blocks(sc[j0:j1], ze[j0:j1], kind, grouping)
+    return out.reshape(-1)
 
 
 def unpack_stream(words: np.ndarray, S: int, kind: int, grouping: int, b: int):
@@ -228,21 +248,12 @@ def unpack_stream(words: np.ndarray, S: int, kind: int, grouping: int, b: int):
     per = 128 * (b + 1)
     words = np.asarray(words, dtype=np.uint32)
     assert words.shape == (nblk * per,)
-    codes, scs, zes = [], [], []
-    for j in range(nblk):
-        blk = words[j * per:(j + 1) * per]
-        codes.append(unpack_codes_block(blk[:128 * b], kind, b))
-        s, z = unpack_meta_block(blk[128 * b:], kind, grouping)
-        scs.append(s)
-        zes.append(z)
-    codes = np.concatenate(codes) if codes else np.zeros((0, HEAD_DIM), np.uint8)
+    w = words.reshape(nblk, per)
+    codes = unpack_codes_blocks(w[:, :128 * b], kind, b).reshape(S, HEAD_DIM)
+    s, z = unpack_meta_blocks(w[:, 128 * b:], kind, grouping)
     if grouping == PER_TOKEN:
-        scale = np.concatenate(scs).reshape(S, 4) if scs else np.zeros((0, 4), np.float16)
-        zero = np.concatenate(zes).reshape(S, 4) if zes else np.zeros((0, 4), np.float16)
-    else:
-        scale = np.stack(scs) if scs else np.zeros((0, HEAD_DIM), np.float16)
-        zero = np.stack(zes) if zes else np.zeros((0, HEAD_DIM), np.float16)
-    return codes, scale, zero
+        return codes, s.reshape(S, 4), z.reshape(S, 4)
+    return codes, s.reshape(nblk, HEAD_DIM), z.reshape(nblk, HEAD_DIM)
 
 
 def stream_offsets(L: int, B: int, H: int, S: int, bits: np.ndarray) -> tuple[np.ndarray, int]:

@@ -1,0 +1,331 @@
+// Host half of librq: distortion-model fit, integer and continuous bit
+// allocation, packed layout. Pure C++17, no CUDA.
+//
+// RateQuant (arXiv 2605.06675):
+//   Assumption 1        D(b) = alpha * beta^-b
+//   Alg. 1 stage 2      least squares of ln D on b at b = 2..6
+//   App. W              poor fits (R^2 < 0.96) fall back to min(beta, beta_bar)
+//   Eq. 1               min sum w_i D_i(b_i), sum b_i = B, bounds
+//   Alg. 2, Prop. 3     greedy max-heap on marginal gain, optimal for convex D
+//   Thm. 1, App. B.1    continuous reverse waterfilling with iterative clipping
+#include <cmath>
+#include <cstdint>
+#include <cstring>
+#include <limits>
+#include <queue>
+#include <vector>
+
+#include "rq.h"
+
+namespace {
+
+bool is_contiguous_mask(uint32_t mask, int* lo, int* hi) {
+  int first = -1, last = -1;
+  for (int k = 1; k <= 8; ++k)
+    if ((mask >> k) & 1u) {
+      if (first < 0) first = k;
+      last = k;
+    }
+  if (first < 0) return false;
+  *lo = first;
+  *hi = last;
+  for (int k = first; k <= last; ++k)
+    if (!((mask >> k) & 1u)) return false;
+  return true;
+}
+
+// w alpha beta^-b, evaluated as ((w * alpha) * beta^-b)
+inline double component_cost(double w, double a, double beta, int b) {
+  return (w * a) * std::pow(beta, -static_cast<double>(b));
+}
+
+// gain of the (b+1)-th bit: w alpha beta^-b (1 - 1/beta)
+inline double marginal_gain(double w, double a, double beta, int b) {
+  return ((w * a) * std::pow(beta, -static_cast<double>(b))) * (1.0 - 1.0 / beta);
+}
+
+struct HeapItem {
+  double gain;
+  int32_t index;
+};
+// std::priority_queue pops the "largest"; larger gain first, then lower index
+struct HeapOrder {
+  bool operator()(const HeapItem& a, const HeapItem& b) const {
+    if (a.gain != b.gain) return a.gain < b.gain;
+    return a.index > b.index;
+  }
+};
+
+rq_status greedy_alloc(int32_t n, const std::vector<double>& w, const double* alpha,
+                       const double* beta, int64_t B, int lo, int hi, uint8_t* bits) {
+  if (B < static_cast<int64_t>(n) * lo || B > static_cast<int64_t>(n) * hi)
+    return RQ_ERR_INFEASIBLE;
+  for (int32_t i = 0; i < n; ++i) bits[i] = static_cast<uint8_t>(lo);
+  int64_t remaining = B - static_cast<int64_t>(n) * lo;
+  std::priority_queue<HeapItem, std::vector<HeapItem>, HeapOrder> heap;
+  if (lo < hi)
+    for (int32_t i = 0; i < n; ++i) heap.push({marginal_gain(w[i], alpha[i], beta[i], lo), i});
+  while (remaining > 0) {
+    HeapItem top = heap.top();
+    heap.pop();
+    const int32_t i = top.index;
+    bits[i] = static_cast<uint8_t>(bits[i] + 1);
+    --remaining;
+    if (bits[i] < hi) heap.push({marginal_gain(w[i], alpha[i], beta[i], bits[i]), i});
+  }
+  return RQ_OK;
+}
+
+// Exact optimum for any allowed set: suffix table g[i][r] = least cost of
+// components i..n-1 spending r bits above the smallest allowed width.
+rq_status dp_alloc(int32_t n, const std::vector<double>& w, const double* alpha,
+                   const double* beta, int64_t B, uint32_t mask, uint8_t* bits) {
+  std::vector<int> widths;
+  for (int k = 1; k <= 8; ++k)
+    if ((mask >> k) & 1u) widths.push_back(k);
+  const int lo = widths.front();
+  const int64_t R = B - static_cast<int64_t>(n) * lo;
+  if (R < 0) return RQ_ERR_INFEASIBLE;
+  if (static_cast<double>(n + 1) * static_cast<double>(R + 1) > 4.0e8) return RQ_ERR_INVALID_ARG;
+  const double inf = std::numeric_limits<double>::infinity();
+  const size_t W = static_cast<size_t>(R + 1);
+  std::vector<double> g(static_cast<size_t>(n + 1) * W, inf);
+  g[static_cast<size_t>(n) * W + 0] = 0.0;
+  const size_t nw = widths.size();
+  std::vector<double> cost(static_cast<size_t>(n) * nw);
+  for (int32_t i = 0; i < n; ++i)
+    for (size_t k = 0; k < nw; ++k) cost[i * nw + k] = component_cost(w[i], alpha[i], beta[i], widths[k]);
+  for (int32_t i = n - 1; i >= 0; --i) {
+    double* gi = &g[static_cast<size_t>(i) * W];
+    const double* gn = &g[static_cast<size_t>(i + 1) * W];
+    for (int64_t r = 0; r <= R; ++r) {
+      double best = inf;
+      for (size_t k = 0; k < nw; ++k) {
+        const int64_t dlt = widths[k] - lo;
+        if (dlt > r || gn[r - dlt] == inf) continue;
+        const double v = cost[i * nw + k] + gn[r - dlt];
+        if (v < best) best = v;
+      }
+      gi[r] = best;
+    }
+  }
+  if (g[R] == inf) return RQ_ERR_INFEASIBLE;
+  int64_t r = R;
+  for (int32_t i = 0; i < n; ++i) {
+    const double* gi = &g[static_cast<size_t>(i) * W];
+    const double* gn = &g[static_cast<size_t>(i + 1) * W];
+    bool placed = false;
+    for (int k = static_cast<int>(nw) - 1; k >= 0; --k) {
+      const int64_t dlt = widths[k] - lo;
+      if (dlt > r || gn[r - dlt] == inf) continue;
+      if (cost[i * nw + k] + gn[r - dlt] == gi[r]) {
+        bits[i] = static_cast<uint8_t>(widths[k]);
+        r -= dlt;
+        placed = true;
+        break;
+      }
+    }
+    if (!placed) return RQ_ERR_INFEASIBLE;  // unreachable when g[R] is finite
+  }
+  return RQ_OK;
+}
+
+}  // namespace
+
+extern "C" {
+
+const char* rq_status_string(rq_status s) {
+  switch (s) {
+    case RQ_OK: return "ok";
+    case RQ_ERR_INVALID_ARG: return "invalid argument";
+    case RQ_ERR_INFEASIBLE: return "budget not reachable with the allowed bit-widths";
+    case RQ_ERR_SHAPE: return "unsupported shape";
+    case RQ_ERR_ALIGNMENT: return "device pointer not 16-byte aligned";
+    case RQ_ERR_WORKSPACE: return "workspace too small";
+    case RQ_ERR_CUDA: return "CUDA error";
+  }
+  return "unknown status";
+}
+
+int32_t rq_abi_version(void) { return RQ_ABI_VERSION; }
+
+rq_status rq_fit_distortion(int32_t n, const double* mse, int32_t b_lo, int32_t b_hi,
+                            double r2_min, const int32_t* classes, double* alpha, double* beta,
+                            double* r2) {
+  if (n <= 0 || !mse || !alpha || !beta || !r2) return RQ_ERR_INVALID_ARG;
+  if (b_lo < 1 || b_hi > 8 || b_lo >= b_hi) return RQ_ERR_INVALID_ARG;
+  const double inf = std::numeric_limits<double>::infinity();
+  for (int32_t i = 0; i < n; ++i) {
+    double xs[8], ys[8];
+    int m = 0;
+    for (int b = b_lo; b <= b_hi; ++b) {
+      const double D = mse[static_cast<size_t>(i) * 8 + (b - 1)];
+      if (D > 0.0) {
+        xs[m] = static_cast<double>(b);
+        ys[m] = std::log(D);
+        ++m;
+      }
+    }
+    if (m < 2) {
+      alpha[i] = 0.0;
+      beta[i] = inf;
+      r2[i] = 1.0;
+      continue;
+    }
+    double sx = 0.0, sy = 0.0;
+    for (int k = 0; k < m; ++k) {
+      sx += xs[k];
+      sy += ys[k];
+    }
+    const double mx = sx / m, my = sy / m;
+    double sxy = 0.0, sxx = 0.0;
+    for (int k = 0; k < m; ++k) {
+      sxy += (xs[k] - mx) * (ys[k] - my);
+      sxx += (xs[k] - mx) * (xs[k] - mx);
+    }
+    const double slope = sxy / sxx;
+    const double icept = my - slope * mx;
+    double ss_res = 0.0, ss_tot = 0.0;
+    for (int k = 0; k < m; ++k) {
+      const double res = ys[k] - (icept + slope * xs[k]);
+      ss_res += res * res;
+      ss_tot += (ys[k] - my) * (ys[k] - my);
+    }
+    alpha[i] = std::exp(icept);
+    beta[i] = std::exp(-slope);
+    r2[i] = (ss_tot == 0.0) ? (ss_res == 0.0 ? 1.0 : 0.0) : 1.0 - ss_res / ss_tot;
+  }
+  if (r2_min > 0.0) {
+    // class means of the fitted (finite) beta, before any fallback
+    std::vector<int32_t> cls(n, 0);
+    if (classes)
+      for (int32_t i = 0; i < n; ++i) cls[i] = classes[i];
+    std::vector<int32_t> keys;
+    for (int32_t i = 0; i < n; ++i) {
+      bool seen = false;
+      for (int32_t k : keys) seen = seen || (k == cls[i]);
+      if (!seen) keys.push_back(cls[i]);
+    }
+    std::vector<double> fitted(beta, beta + n);
+    for (int32_t key : keys) {
+      double s = 0.0;
+      int cnt = 0;
+      for (int32_t i = 0; i < n; ++i)
+        if (cls[i] == key && std::isfinite(fitted[i])) {
+          s += fitted[i];
+          ++cnt;
+        }
+      const double mean = cnt > 0 ? s / cnt : inf;
+      for (int32_t i = 0; i < n; ++i)
+        if (cls[i] == key && r2[i] < r2_min) beta[i] = std::fmin(fitted[i], mean);
+    }
+  }
+  return RQ_OK;
+}
+
+rq_status rq_alloc(int32_t n, const double* w, const double* alpha, const double* beta,
+                   double avg_bits, uint32_t allowed_mask, uint32_t flags, uint8_t* bits_out,
+                   double* objective_out) {
+  if (n <= 0 || !w || !alpha || !beta || !bits_out) return RQ_ERR_INVALID_ARG;
+  if ((allowed_mask & 0x1FEu) == 0 || (allowed_mask & ~0x1FEu) != 0) return RQ_ERR_INVALID_ARG;
+  if (!std::isfinite(avg_bits)) return RQ_ERR_INVALID_ARG;
+  std::vector<double> wv(w, w + n);
+  if (flags & RQ_CAP_5X) {
+    double mean = 0.0;
+    for (int32_t i = 0; i < n; ++i) mean += wv[i];
+    mean /= n;
+    for (int32_t i = 0; i < n; ++i) wv[i] = std::fmin(wv[i], 5.0 * mean);
+  }
+  const int64_t B = static_cast<int64_t>(std::floor(avg_bits * n + 0.5));
+  int lo = 0, hi = 0;
+  rq_status st = is_contiguous_mask(allowed_mask, &lo, &hi)
+                     ? greedy_alloc(n, wv, alpha, beta, B, lo, hi, bits_out)
+                     : dp_alloc(n, wv, alpha, beta, B, allowed_mask, bits_out);
+  if (st != RQ_OK) return st;
+  if (objective_out) {
+    double J = 0.0;
+    for (int32_t i = 0; i < n; ++i) J += component_cost(wv[i], alpha[i], beta[i], bits_out[i]);
+    *objective_out = J;
+  }
+  return RQ_OK;
+}
+
+rq_status rq_alloc_continuous(int32_t n, const double* w, const double* alpha,
+                              const double* beta, double avg_bits, double b_min, double b_max,
+                              double* b_out) {
+  if (n <= 0 || !w || !alpha || !beta || !b_out) return RQ_ERR_INVALID_ARG;
+  if (!(b_min <= b_max)) return RQ_ERR_INVALID_ARG;
+  for (int32_t i = 0; i < n; ++i)
+    if (!(w[i] > 0.0) || !(alpha[i] > 0.0) || !(beta[i] > 1.0)) return RQ_ERR_INVALID_ARG;
+  const double B = avg_bits * n;
+  if (B < n * b_min - 1e-9 || B > n * b_max + 1e-9) return RQ_ERR_INFEASIBLE;
+  // ln of w alpha ln(beta), and ln(beta)
+  std::vector<double> A(n), lb(n);
+  for (int32_t i = 0; i < n; ++i) {
+    A[i] = std::log(w[i] * alpha[i] * std::log(beta[i]));
+    lb[i] = std::log(beta[i]);
+  }
+  std::vector<char> fixed(n, 0);
+  std::vector<double> fixed_val(n, 0.0);
+  for (int32_t round = 0; round <= n; ++round) {
+    double Bf = B;
+    bool any_free = false;
+    for (int32_t i = 0; i < n; ++i) {
+      if (fixed[i]) Bf -= fixed_val[i];
+      else any_free = true;
+    }
+    if (!any_free) break;
+    // sum_F (A_i - ln lambda) / ln beta_i = B_F  ->  ln lambda in closed form
+    double num = 0.0, den = 0.0;
+    for (int32_t i = 0; i < n; ++i)
+      if (!fixed[i]) {
+        num += A[i] / lb[i];
+        den += 1.0 / lb[i];
+      }
+    const double ln_lambda = (num - Bf) / den;
+    bool changed = false;
+    for (int32_t i = 0; i < n; ++i) {
+      if (fixed[i]) continue;
+      const double b = (A[i] - ln_lambda) / lb[i];
+      if (b < b_min) {
+        fixed[i] = 1;
+        fixed_val[i] = b_min;
+        changed = true;
+      } else if (b > b_max) {
+        fixed[i] = 1;
+        fixed_val[i] = b_max;
+        changed = true;
+      } else {
+        b_out[i] = b;
+      }
+    }
+    if (!changed) break;
+  }
+  for (int32_t i = 0; i < n; ++i)
+    if (fixed[i]) b_out[i] = fixed_val[i];
+  return RQ_OK;
+}
+
+rq_status rq_packed_layout(const rq_cache_desc* desc, const uint8_t* bits, uint64_t* offsets,
+                           uint64_t* total_bytes) {
+  if (!desc || !bits || !total_bytes) return RQ_ERR_INVALID_ARG;
+  if (desc->L <= 0 || desc->B < 0 || desc->H_kv <= 0 || desc->S < 0) return RQ_ERR_INVALID_ARG;
+  if (desc->d != RQ_HEAD_DIM || desc->group != RQ_GROUP || desc->S % RQ_GROUP != 0)
+    return RQ_ERR_SHAPE;
+  const uint64_t nblk = static_cast<uint64_t>(desc->S / RQ_GROUP);
+  uint64_t pos = 0;
+  for (int32_t l = 0; l < desc->L; ++l)
+    for (int32_t b = 0; b < desc->B; ++b)
+      for (int32_t h = 0; h < desc->H_kv; ++h)
+        for (int32_t kind = 0; kind < 2; ++kind) {
+          const int bw = bits[(static_cast<size_t>(l) * desc->H_kv + h) * 2 + kind];
+          if (bw < 1 || bw > 8) return RQ_ERR_INVALID_ARG;
+          if (offsets)
+            offsets[((static_cast<size_t>(l) * desc->B + b) * desc->H_kv + h) * 2 + kind] = pos;
+          pos += nblk * 512ull * static_cast<uint64_t>(bw + 1);
+        }
+  *total_bytes = pos;
+  return RQ_OK;
+}
+
+}  // extern "C"

@@ -1,0 +1,132 @@
+"""librq host half on the CPU: the library builds, loads and exports every
+symbol include/rq.h declares; its host functions (fit, allocation, layout)
+agree with the oracle on identical inputs. No CUDA compute is launched."""
+import math
+import os
+import re
+
+import numpy as np
+import pytest
+
+from oracle import alloc as oalloc
+from oracle import calib as ocalib
+from oracle import pack as opack
+
+ROOT = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
+
+
+@pytest.fixture(scope="session")
+def rq():
+    from paper_2605_06675_gb300 import build, rq as binding
+    srcs = [os.path.join(build.CSRC, f) for f in os.listdir(build.CSRC)]
+    srcs.append(os.path.join(build.INCLUDE, "rq.h"))
+    if not os.path.exists(build.LIB) or os.path.getmtime(build.LIB) < max(map(os.path.getmtime, srcs)):
+        build.build()
+    binding.lib()
+    return binding
+
+
+def test_exports_every_header_symbol(rq):
+    header = open(os.path.join(ROOT, "include", "rq.h")).read()
+    declared = sorted(set(re.findall(r"\b(rq_[a-z_]+)\s*\(", header)))
+    assert declared, "no declarations found"
+    lib = rq.lib()
+    for name in declared:
+        assert hasattr(lib, name), name
+    assert sorted(rq.EXPORTS) == declared
+    assert rq.rq_abi_version() == 1
+    assert rq.rq_status_string(3) == "unsupported shape"
+
+
+def _mse_rows(rng, n):
+    a = rng.uniform(0.5, 20, n)
+    beta = rng.uniform(3.5, 6.0, n)
+    b = np.arange(1, 9)
+    mse = a[:, None] * beta[:, None] ** (-b[None, :])
+    return mse * np.exp(rng.normal(0, 0.05, mse.shape))
+
+
+def test_fit_matches_oracle(rq):
+    rng = np.random.default_rng(0)
+    n = 64
+    mse = _mse_rows(rng, n)
+    mse[3] = [1.0, 0.9, 1e-3, 1e-2, 1e-6, 1e-5, 1e-9, 1e-9]     # poor fit -> fallback
+    mse[5] = 0.0                                                 # degenerate
+    classes = np.arange(n) % 2
+    for lo, hi, r2min in ((2, 6, 0.96), (1, 8, 0.96), (2, 6, 0.0)):
+        a, b, r2 = rq.rq_fit_distortion(mse, lo, hi, r2min, classes)
+        oa, ob, or2 = ocalib.fit_distortion(mse, lo, hi, r2min, classes)
+        assert np.array_equal(a, oa) and np.array_equal(b, ob) and np.array_equal(r2, or2)
+    assert rq.rq_fit_distortion(mse, 2, 6, 0.96, None)[1].shape == (n,)
+
+
+def test_table8_through_the_library(rq):
+    # the paper's Table 8 fit (alpha ~ 1.36, beta ~ 3.48) through the C ABI
+    row = np.zeros((1, 8))
+    row[0, :6] = [3.634e-01, 1.175e-01, 3.455e-02, 9.501e-03, 2.512e-03, 7.647e-04]
+    a, b, r2 = rq.rq_fit_distortion(row, 1, 6, 0.0)
+    assert abs(a[0] - 1.36) < 0.005 and abs(b[0] - 3.48) < 0.005 and r2[0] > 0.99
+
+
+@pytest.mark.parametrize("allowed,avg", [((2, 3, 4), 2.5), ((2, 3, 4), 3.0),
+                                         ((2, 3, 4, 5, 6, 7, 8), 4.0), ((2, 3, 4, 8), 3.0),
+                                         ((1, 2, 3, 4, 5, 6, 7, 8), 3.3), ((2, 8), 4.0)])
+def test_alloc_matches_oracle(rq, allowed, avg):
+    rng = np.random.default_rng(int(avg * 10) + len(allowed))
+    n = 96
+    w = np.exp(rng.normal(0, 0.76, n))
+    a = rng.uniform(0.5, 20, n)
+    beta = rng.uniform(3.5, 6.0, n)
+    mask = sum(1 << k for k in allowed)
+    for cap in (False, True):
+        bits, J = rq.rq_alloc(w, a, beta, avg, mask, rq.RQ_CAP_5X if cap else 0)
+        obits, oJ = oalloc.allocate(w, a, beta, avg, mask, cap)
+        assert obits is not None
+        assert list(bits) == obits
+        assert J == oJ
+        assert int(bits.sum()) == oalloc.budget(avg, n)
+
+
+def test_alloc_ties_and_errors(rq):
+    n = 10
+    bits, _ = rq.rq_alloc([1.0] * n, [1.0] * n, [4.0] * n, 3.4, 0b1111100)
+    assert list(bits) == [4, 4, 4, 4, 3, 3, 3, 3, 3, 3]
+    with pytest.raises(rq.RQError) as e:
+        rq.rq_alloc([1.0] * 3, [1.0] * 3, [4.0] * 3, 7.0 / 3.0, (1 << 2) | (1 << 8))
+    assert e.value.status == 2            # 7 bits over {2, 8} is unreachable
+    with pytest.raises(rq.RQError) as e:
+        rq.rq_alloc([1.0] * 3, [1.0] * 3, [4.0] * 3, 3.0, 1)       # bit 0 is not a width
+    assert e.value.status == 1
+
+
+def test_continuous_matches_oracle(rq):
+    rng = np.random.default_rng(3)
+    n = 80
+    w = np.exp(rng.normal(0, 1.2, n))
+    a = rng.uniform(1, 10, n)
+    beta = rng.uniform(3.5, 5.5, n)
+    for lo, hi, avg in ((2.0, 4.0, 3.0), (0.0, 16.0, 4.0), (3.0, 6.0, 4.5)):
+        got = rq.rq_alloc_continuous(w, a, beta, avg, lo, hi)
+        ref = oalloc.continuous(list(w), list(a), list(beta), avg, lo, hi)
+        assert np.array_equal(got, np.array(ref))
+        assert abs(got.sum() - avg * n) < 1e-8
+    with pytest.raises(rq.RQError):
+        rq.rq_alloc_continuous(w, a, beta, 5.0, 2.0, 4.0)
+
+
+def test_packed_layout_matches_oracle(rq):
+    rng = np.random.default_rng(4)
+    L, B, H, S = 3, 2, 4, 96
+    bits = rng.integers(1, 9, size=(L, H, 2)).astype(np.uint8)
+    desc = rq.make_desc(L, B, H, 4 * H, S, rq.RQ_BF16, rq.RQ_PER_CHANNEL, rq.RQ_PER_TOKEN)
+    off, total = rq.rq_packed_layout(desc, bits)
+    ooff, ototal = opack.stream_offsets(L, B, H, S, bits)
+    assert total == ototal and np.array_equal(off, ooff)
+    assert all(int(o) % 512 == 0 for o in off.reshape(-1))
+    bad = rq.make_desc(L, B, H, 4 * H, 100, rq.RQ_BF16, 1, 0)
+    with pytest.raises(rq.RQError) as e:
+        rq.rq_packed_layout(bad, bits)
+    assert e.value.status == 3
+    bits[0, 0, 0] = 9
+    with pytest.raises(rq.RQError):
+        rq.rq_packed_layout(desc, bits)
