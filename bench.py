@@ -50,6 +50,8 @@ def _parse():
     ap.add_argument("--warmup", type=int, default=3)
     ap.add_argument("--impl", choices=["ours", "reference"], default="ours")
     ap.add_argument("--workload", default=None)
+    ap.add_argument("--layers", type=int, default=None,
+                    help="run only the first N layers (small cases for profiling)")
     ap.add_argument("--no-e2e", action="store_true")
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--cpu-leg", action="store_true", help=argparse.SUPPRESS)
@@ -405,11 +407,14 @@ def run_e2e(args, wl, path, K, V, Q, OUT, X, w, cap, dev, stream, step_bytes, wo
 # the CPU oracle (cpu_baseline leg and --impl reference)
 # --------------------------------------------------------------------------
 
-def oracle_sample_run(wl, tokens: int, n_calib: int):
-    """One bounded sample of the workload on the CPU oracle; returns
-    (algorithmic bytes, seconds, description)."""
+def oracle_sample_run(wl, tokens: int, n_calib: int, heads: int = 1, budget_s: float = 0.0):
+    """Bounded sample of the workload on the CPU oracle: the calibration sweep
+    of ``n_calib`` components, fit + allocation of every component, then
+    quantize + pack + decode attention of (batch 0, kv head h) K+V stream pairs
+    of ``tokens`` tokens for h = 0, 1, ... until ``heads`` pairs are done or
+    ``budget_s`` seconds have passed. Returns (algorithmic bytes, seconds,
+    description)."""
     import numpy as np
-    import torch
 
     from oracle import alloc as oalloc
     from oracle import calib as ocalib
@@ -417,14 +422,15 @@ def oracle_sample_run(wl, tokens: int, n_calib: int):
     from paper_2605_06675_gb300 import synth
 
     S = min(tokens, wl.S)
-    k, v = synth.kv_layer(1, 1, S, wl.dtype, wl.seed, 0, wl.value_dist, "cpu")
-    q = synth.queries(1, wl.g, wl.dtype, wl.seed, 0, "cpu")
+    H = max(1, min(wl.H_kv, heads))
+    k, v = synth.kv_layer(1, H, S, wl.dtype, wl.seed, 0, wl.value_dist, "cpu")
+    q = synth.queries(1, wl.H_q, wl.dtype, wl.seed, 0, "cpu")
     X = synth.calibration_sample(wl.scaled(L=1, H_kv=max(1, n_calib // 2)), device="cpu")
     signs = synth.hadamard_signs(wl.seed).numpy() if wl.hadamard else None
     ks, vs, qs, xs = (t.float().numpy() for t in (k, v, q, X))
     n = wl.n_components
     w = synth.importances(n, wl.sigma_lnw, wl.seed)
-    bits_layer = np.array([[wl.allowed[0], wl.allowed[-1]]], dtype=np.uint8)
+    allowed = list(wl.allowed)
 
     t0 = time.perf_counter()
     groupings = [wl.k_grouping if i % 2 == 0 else wl.v_grouping for i in range(xs.shape[0])]
@@ -432,24 +438,32 @@ def oracle_sample_run(wl, tokens: int, n_calib: int):
     mse_all = np.resize(mse, (n, 8))
     a, b, _ = ocalib.fit_distortion(mse_all, 2, 6, 0.96, np.arange(n) % 2)
     oalloc.allocate(w, a, b, wl.avg_bits, wl.allowed_mask)
-    ol = opipe.quantize_layer(ks, vs, bits_layer, wl.k_grouping, wl.v_grouping, wl.hadamard, signs)
-    opipe.attend_layer(qs, ol)
-    el = time.perf_counter() - t0
-
+    nbytes = calib_bytes(wl, xs.shape[0], xs.shape[1])
     nblk = S // 32
-    qbytes = 2 * S * 128 * 2 + sum(nblk * 512 * (int(x) + 1) for x in bits_layer.reshape(-1))
-    dbytes = sum(nblk * 512 * (int(x) + 1) for x in bits_layer.reshape(-1)) + wl.g * 128 * 6
-    cbytes = calib_bytes(wl, xs.shape[0], xs.shape[1])
-    desc = (f"oracle on 1 (batch, kv head) K+V stream pair of {S} tokens "
-            f"(bits {bits_layer.reshape(-1).tolist()}), calibration sweep of {xs.shape[0]} "
-            f"components x {xs.shape[1]} tokens, fit + allocation of all {n} components")
-    return qbytes + dbytes + cbytes, el, desc
+    done = []
+    for h in range(H):
+        bl = np.array([[allowed[(2 * h) % len(allowed)], allowed[(2 * h + 1) % len(allowed)]]],
+                      dtype=np.uint8)
+        ol = opipe.quantize_layer(ks[:, h:h + 1], vs[:, h:h + 1], bl, wl.k_grouping,
+                                  wl.v_grouping, wl.hadamard, signs)
+        opipe.attend_layer(qs[:, h * wl.g:(h + 1) * wl.g], ol)
+        packed = sum(nblk * 512 * (int(x) + 1) for x in bl.reshape(-1))
+        nbytes += 2 * S * 128 * 2 + packed                      # quantize: read + write
+        nbytes += packed + wl.g * 128 * (2 + 4)                  # decode: packed + q + out
+        done.append(bl.reshape(-1).tolist())
+        if budget_s and time.perf_counter() - t0 > budget_s:
+            break
+    el = time.perf_counter() - t0
+    desc = (f"oracle: calibration sweep of {xs.shape[0]} components x {xs.shape[1]} tokens, "
+            f"fit + allocation of all {n} components, then quantize + pack + decode attention "
+            f"of {len(done)} (batch 0, kv head) K+V stream pairs of {S} tokens (bits {done})")
+    return nbytes, el, desc
 
 
 def cpu_leg_main(args, wl):
     os.environ.setdefault("OMP_NUM_THREADS", "1")
-    tokens = args.cpu_tokens or 8192
-    nbytes, el, desc = oracle_sample_run(wl, tokens, 8)
+    tokens = args.cpu_tokens or wl.S
+    nbytes, el, desc = oracle_sample_run(wl, tokens, 8, heads=wl.H_kv, budget_s=10.0)
     print(json.dumps({"value": nbytes / el / 1e9, "unit": "GB/s", "cores": 1, "kind": "oracle",
                       "sample": desc, "seconds": el}))
 
@@ -478,11 +492,11 @@ def run_cpu_leg_subprocess(wl, tokens=None):
 def run_reference(args, wl, world):
     """--impl reference: the CPU oracle as it stands, bounded sample per step."""
     times = []
-    tokens = min(wl.S, 4096)
+    tokens = min(wl.S, 8192)
     nbytes = 0
     desc = ""
     for i in range(args.warmup + args.steps):
-        nbytes, el, desc = oracle_sample_run(wl, tokens, 4)
+        nbytes, el, desc = oracle_sample_run(wl, tokens, 4, heads=1)
         if i >= args.warmup:
             times.append(el)
     ms = statistics.mean(times) * 1e3
@@ -504,6 +518,8 @@ def main():
     args = _parse()
     table, default = _workloads()
     wl = table[args.workload] if args.workload else default
+    if args.layers:
+        wl = wl.scaled(L=min(args.layers, wl.L))
     if args.cpu_leg:
         cpu_leg_main(args, wl)
         return
