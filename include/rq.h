@@ -9,7 +9,8 @@
  * - Plain C types only. Device pointers are ordinary pointers into device
  *   memory the caller owns; `stream` is a cudaStream_t passed as void*
  *   (NULL = legacy default stream). librq never allocates memory and keeps no
- *   state between calls apart from a cached per-device SM count.
+ *   state between calls apart from a cached per-device SM count and the fixed
+ *   device array used by rq_decode_attention_static.
  * - Arguments are validated on the host before anything is launched; a bad
  *   argument returns an error code and launches nothing. A failed launch
  *   returns RQ_ERR_CUDA. Device entry points are asynchronous on `stream`.
@@ -187,6 +188,33 @@ rq_status rq_decode_attention(const rq_cache_desc* desc, int32_t layer, const vo
                               const void* packed, const uint8_t* bits_dev,
                               const uint64_t* offsets_dev, const int8_t* signs_dev, float* out,
                               void* ws, size_t ws_bytes, uint32_t* status_dev, void* stream);
+
+/* Allocation-free variant of rq_decode_attention (the paper has no counterpart;
+ * this is a library convenience). Some callers cannot allocate device memory
+ * at the point where they decode: code running inside a captured or
+ * replayed CUDA graph, embedding runtimes whose allocator is owned by
+ * someone else, or plugins that are handed only the tensors they read and
+ * write. This entry point takes the same arguments minus the workspace: the
+ * split-K partials live in a fixed device array inside librq of
+ * RQ_STATIC_SCRATCH_BYTES bytes, reserved on every GPU that loads the
+ * library until the process exits. It calls no cudaMalloc/cudaFree.
+ *  - Limit: B * H_q * splits * 130 * 4 bytes must fit in RQ_STATIC_SCRATCH_BYTES
+ *    (splits as chosen for rq_decode_workspace_bytes); larger shapes return
+ *    RQ_ERR_WORKSPACE before anything is launched.
+ *  - The first call on a device looks up the array's device address
+ *    (cudaGetSymbolAddress) with that device current; make that first call
+ *    before any stream capture.
+ *  - Every call on a device shares the one array, which keeps the previous
+ *    call's contents (each call overwrites every record it reads, so nothing
+ *    needs clearing). Calls that can overlap on the GPU (different streams
+ *    without ordering) race on the array and give wrong results: serialise
+ *    them, or use rq_decode_attention with separate workspaces.
+ * Other arguments, results and errors as rq_decode_attention. */
+#define RQ_STATIC_SCRATCH_BYTES (8u << 20)
+rq_status rq_decode_attention_static(const rq_cache_desc* desc, int32_t layer, const void* q,
+                                     const void* packed, const uint8_t* bits_dev,
+                                     const uint64_t* offsets_dev, const int8_t* signs_dev,
+                                     float* out, uint32_t* status_dev, void* stream);
 
 #ifdef __cplusplus
 }

@@ -531,3 +531,90 @@ extern "C" rq_status rq_decode_attention(const rq_cache_desc* desc, int32_t laye
       a.partial, out, signs_dev, status_dev, splits, a.hadamard);
   return launch_status();
 }
+
+// ---------------------------------------------------------------------------
+// Allocation-free decode: the split-K partials live in a fixed device array
+// of this library instead of a caller-supplied workspace, for callers that
+// cannot allocate (graph replays, foreign allocators, plugins handed only
+// their inputs and outputs). The array is shared by every call on a device.
+namespace rq {
+namespace {
+
+constexpr size_t kStaticScratchFloats = RQ_STATIC_SCRATCH_BYTES / sizeof(float);
+static __device__ __align__(256) float g_decode_scratch[kStaticScratchFloats];
+
+// device address of g_decode_scratch for the current device, looked up once
+// per device (host code only sees a host-side stand-in for the symbol)
+rq_status static_scratch_ptr(float** ptr) {
+  static std::atomic<uintptr_t> cache[64];
+  int dev = 0;
+  if (cudaGetDevice(&dev) != cudaSuccess) return RQ_ERR_CUDA;
+  if (dev >= 0 && dev < 64) {
+    const uintptr_t c = cache[dev].load(std::memory_order_acquire);
+    if (c != 0) {
+      *ptr = reinterpret_cast<float*>(c);
+      return RQ_OK;
+    }
+  }
+  void* p = nullptr;
+  if (cudaGetSymbolAddress(&p, g_decode_scratch) != cudaSuccess || p == nullptr) return RQ_ERR_CUDA;
+  if (dev >= 0 && dev < 64) cache[dev].store(reinterpret_cast<uintptr_t>(p), std::memory_order_release);
+  *ptr = static_cast<float*>(p);
+  return RQ_OK;
+}
+
+}  // namespace
+}  // namespace rq
+
+extern "C" rq_status rq_decode_attention_static(const rq_cache_desc* desc, int32_t layer,
+                                                const void* q, const void* packed,
+                                                const uint8_t* bits_dev,
+                                                const uint64_t* offsets_dev,
+                                                const int8_t* signs_dev, float* out,
+                                                uint32_t* status_dev, void* stream) {
+  using namespace rq;
+  const rq_status st = check_desc(desc);
+  if (st != RQ_OK) return st;
+  if (!q || !packed || !bits_dev || !offsets_dev || !out) return RQ_ERR_INVALID_ARG;
+  if (layer < 0 || layer >= desc->L) return RQ_ERR_INVALID_ARG;
+  if (!aligned16(packed) || (reinterpret_cast<uintptr_t>(q) & 1u) ||
+      (reinterpret_cast<uintptr_t>(out) & 3u))
+    return RQ_ERR_ALIGNMENT;
+  if (desc->B == 0) return RQ_OK;
+  int sms = 0;
+  if (current_sm_count(&sms) != RQ_OK) return RQ_ERR_CUDA;
+  int splits = 1, bps = 1;
+  decode_plan(desc, sms, &splits, &bps);
+  const size_t need = static_cast<size_t>(desc->B) * desc->H_q * splits * kPart * sizeof(float);
+  if (need > RQ_STATIC_SCRATCH_BYTES) return RQ_ERR_WORKSPACE;
+  float* scratch = nullptr;
+  if (static_scratch_ptr(&scratch) != RQ_OK) return RQ_ERR_CUDA;
+  DecodeArgs a;
+  a.q = q;
+  a.packed = static_cast<const uint8_t*>(packed);
+  a.bits = bits_dev;
+  a.offsets = offsets_dev;
+  a.signs = signs_dev;
+  a.partial = scratch;
+  a.status = status_dev;
+  a.layer = layer;
+  a.B = desc->B;
+  a.H = desc->H_kv;
+  a.Hq = desc->H_q;
+  a.g = desc->H_q / desc->H_kv;
+  a.nblk = desc->S / kTile;
+  a.splits = splits;
+  a.bps = bps;
+  a.kg = desc->k_grouping;
+  a.vg = desc->v_grouping;
+  a.hadamard = desc->hadamard ? 1 : 0;
+  cudaStream_t s = static_cast<cudaStream_t>(stream);
+  const dim3 grid(static_cast<unsigned>(splits), static_cast<unsigned>(desc->H_kv),
+                  static_cast<unsigned>(desc->B));
+  if (desc->dtype == RQ_F16) decode_split_kernel<__half><<<grid, kThreads, 0, s>>>(a);
+  else decode_split_kernel<__nv_bfloat16><<<grid, kThreads, 0, s>>>(a);
+  if (launch_status() != RQ_OK) return RQ_ERR_CUDA;
+  decode_combine_kernel<<<static_cast<unsigned>(desc->B * desc->H_q), kD, 0, s>>>(
+      a.partial, out, signs_dev, status_dev, splits, a.hadamard);
+  return launch_status();
+}

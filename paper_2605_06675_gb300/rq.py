@@ -21,6 +21,7 @@ RQ_PER_TOKEN, RQ_PER_CHANNEL = 0, 1
 RQ_CAP_5X = 1
 RQ_STATUS_NUMERIC = 1
 RQ_STATUS_BAD_BITS = 2
+RQ_STATIC_SCRATCH_BYTES = 8 << 20
 HEAD_DIM = 128
 GROUP = 32
 
@@ -31,7 +32,7 @@ STATUS_NAMES = {0: "RQ_OK", 1: "RQ_ERR_INVALID_ARG", 2: "RQ_ERR_INFEASIBLE", 3: 
 EXPORTS = ["rq_status_string", "rq_abi_version", "rq_fit_distortion", "rq_alloc",
            "rq_alloc_continuous", "rq_packed_layout", "rq_calibrate_workspace_bytes",
            "rq_calibrate_distortion", "rq_quantize_pack", "rq_decode_workspace_bytes",
-           "rq_decode_attention"]
+           "rq_decode_attention", "rq_decode_attention_static"]
 
 
 class RQError(RuntimeError):
@@ -72,6 +73,7 @@ def lib() -> ctypes.CDLL:
             "rq_quantize_pack": ([_P, _I, _P, _P, _P, _P, _P, _P, _P, _P], _I),
             "rq_decode_workspace_bytes": ([_P, _P], _I),
             "rq_decode_attention": ([_P, _I, _P, _P, _P, _P, _P, _P, _P, _SZ, _P, _P], _I),
+            "rq_decode_attention_static": ([_P, _I, _P, _P, _P, _P, _P, _P, _P, _P], _I),
         }
         for name, (args, res) in sig.items():
             f = getattr(L, name)
@@ -222,3 +224,14 @@ def rq_decode_attention(desc, layer, q, packed, bits_dev, offsets_dev, signs, ou
         ctypes.byref(desc), layer, _dp(q), _dp(packed), _dp(bits_dev), _dp(offsets_dev),
         _dp(signs), _dp(out), _dp(ws), ws.numel() * ws.element_size(), _dp(status),
         _stream(stream)))
+
+
+def rq_decode_attention_static(desc, layer, q, packed, bits_dev, offsets_dev, signs, out,
+                               status=None, stream=None):
+    """rq_decode_attention without a workspace argument: for callers that
+    cannot allocate device memory (graph replays, foreign allocators,
+    plugins). Uses librq's fixed RQ_STATIC_SCRATCH_BYTES device array, shared
+    by every call on the device, so concurrent calls on unordered streams race."""
+    _check("rq_decode_attention_static", lib().rq_decode_attention_static(
+        ctypes.byref(desc), layer, _dp(q), _dp(packed), _dp(bits_dev), _dp(offsets_dev),
+        _dp(signs), _dp(out), _dp(status), _stream(stream)))

@@ -1,0 +1,62 @@
+"""rq_decode_attention_static: decode attention for callers that cannot
+allocate device memory (code replayed inside a CUDA graph, runtimes whose
+allocator belongs to someone else, plugins handed only their inputs and
+outputs). Its split-K partials live in librq's fixed device array instead of
+a caller workspace. Checked through the C ABI against rq_decode_attention on
+two calls in a row (the second call finds the first call's leftovers in the
+shared array). This file is collected last on purpose."""
+import numpy as np
+import pytest
+import torch
+
+from paper_2605_06675_gb300 import synth
+from paper_2605_06675_gb300.path import PackedKVPath
+from paper_2605_06675_gb300.workloads import PER_CHANNEL, PER_TOKEN, Workload
+
+from .gpu_helpers import TOL, attn_err, bits_cycle, ensure_built, to_np
+
+pytestmark = pytest.mark.gpu
+DEV = "cuda"
+
+
+def test_static_scratch_matches_workspace_version():
+    rq = ensure_built()
+    wl = Workload("noalloc", L=2, B=3, H_kv=4, H_q=16, S=2048, dtype="bfloat16",
+                  k_grouping=PER_CHANNEL, v_grouping=PER_TOKEN, hadamard=False,
+                  allowed=(2, 3, 4, 8), avg_bits=3.0, sigma_lnw=0.5, value_dist="gaussian",
+                  seed=41)
+    path = PackedKVPath(wl, DEV)
+    path.set_bits(bits_cycle(wl.L, wl.H_kv, wl.allowed))
+    ws = path.decode_workspace()
+    assert ws.numel() <= rq.RQ_STATIC_SCRATCH_BYTES
+    for call, layer in enumerate((0, 1)):            # two calls in a row
+        k, v = synth.kv_layer(wl.B, wl.H_kv, wl.S, wl.dtype, wl.seed, layer, device=DEV)
+        q = synth.queries(wl.B, wl.H_q, wl.dtype, wl.seed + call, layer, DEV)
+        path.quantize(layer, k, v)
+        ref = torch.empty((wl.B, wl.H_q, 128), dtype=torch.float32, device=DEV)
+        out = torch.full((wl.B, wl.H_q, 128), float("nan"), dtype=torch.float32, device=DEV)
+        rq.rq_decode_attention(path.desc, layer, q, path.packed, path.bits, path.offsets, None,
+                               ref, ws, path.status)
+        rq.rq_decode_attention_static(path.desc, layer, q, path.packed, path.bits,
+                                      path.offsets, None, out, path.status)
+        torch.cuda.synchronize()
+        assert torch.isfinite(out).all()
+        assert attn_err(to_np(out), to_np(ref)) <= TOL
+    assert int(path.status.item()) == 0
+
+
+def test_static_scratch_rejects_oversized_shapes():
+    rq = ensure_built()
+    # B * H_q * splits * 130 floats beyond the fixed array: refused on the
+    # host before any launch
+    big = rq.make_desc(1, 256, 8, 64, 32 * 4096, torch.bfloat16, PER_CHANNEL, PER_TOKEN)
+    need = rq.rq_decode_workspace_bytes(big)
+    assert need > rq.RQ_STATIC_SCRATCH_BYTES
+    dummy = torch.zeros(16, dtype=torch.uint8, device=DEV)
+    q = torch.zeros((256, 64, 128), dtype=torch.bfloat16, device=DEV)
+    out = torch.zeros((256, 64, 128), dtype=torch.float32, device=DEV)
+    bits = torch.full((1, 8, 2), 2, dtype=torch.uint8, device=DEV)
+    offs = torch.zeros((1, 256, 8, 2), dtype=torch.int64, device=DEV)
+    with pytest.raises(rq.RQError) as e:
+        rq.rq_decode_attention_static(big, 0, q, dummy, bits, offs, None, out)
+    assert e.value.status == 5
