@@ -19,7 +19,10 @@ BUILD = os.path.join(PKG, "_build")
 LIB = os.path.join(PKG, "librq.so")
 
 ARCH = ["-gencode", "arch=compute_103a,code=sm_103a"]
+# host code does exactly the written IEEE operations on every platform (no
+# FMA contraction on aarch64), so fits and allocations are bit-reproducible
 NVCC_FLAGS = ["-O3", "-lineinfo", "-std=c++17", "-Xcompiler", "-fPIC", "-Xcompiler", "-O2",
+              "-Xcompiler", "-ffp-contract=off",
               "-prec-div=true", "-prec-sqrt=true", f"-I{INCLUDE}", f"-I{CSRC}"]
 SOURCES = ["host.cpp", "quantize.cu", "decode.cu"]
 
