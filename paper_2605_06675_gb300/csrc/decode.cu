@@ -13,9 +13,15 @@
 //   online softmax in fp32 (log2 domain), P^T via movmatrix.trans
 //   o^T[128 x 8 heads]       += V_hat^T[128 x 32] . P^T    (16 x mma m16n8k16)
 // The GQA group (g <= 8 query heads) is the MMA n dimension, so it is never
-// padded to 16. Codes are read in the MMA-fragment order the quantizer wrote,
-// turned into exact fp16 integers with the 1024-exponent trick and dequantized
-// with one fp16x2 FMA (scale, zero) in registers.
+// padded to 16. Each warp streams its K and V block images through its own
+// ring of shared-memory slots with cp.async, several entries ahead of use.
+// Codes are read in the MMA-fragment order the quantizer wrote and turned into
+// exact fp16 integers with the fp16-1024 exponent trick (a code placed in the
+// mantissa of 1024, scaled by a power of two, removed with one fp16x2 FMA).
+// For the KIVI layouts (per-channel keys, per-token values) the group scale
+// is folded into the small MMA operand (q or P) and the zero-points are added
+// by extra MMAs, so the codes enter the tensor cores undequantized; the other
+// layouts dequantize in registers with one fp16x2 FMA (scale, zero).
 #include <algorithm>
 #include <atomic>
 
@@ -46,8 +52,13 @@ namespace {
 
 constexpr int kWarps = 4;
 constexpr int kThreads = 32 * kWarps;
-constexpr int kPart = kD + 2;   // partial record: o[128], m (log2 domain), l
-constexpr int kMaxHeads = 8;    // MMA n
+constexpr int kPart = kD + 2;        // partial record: o[128], m (log2 domain), l
+constexpr int kMaxHeads = 8;         // MMA n
+constexpr int kRingBytes = 12800;    // per-warp ring of shared-memory slots
+constexpr int kMaxSlots = 8;
+constexpr int kQBytes = kMaxHeads * kD * 4;
+constexpr int kSmemBytes = kQBytes + kWarps * kRingBytes;   // 55296: 4 CTAs per SM
+static_assert(kWarps * kMaxHeads * kD * 4 <= kWarps * kRingBytes, "merge buffer aliases rings");
 
 struct DecodeArgs {
   const void* q;
@@ -80,12 +91,48 @@ __device__ __forceinline__ uint32_t movmatrix_trans(uint32_t x) {
   return y;
 }
 
-// lane's 4*BW code words of one block: 16-byte piece i of lane L at 16*(32 i + L)
+__device__ __forceinline__ uint32_t smem_u32(const void* p) {
+  return static_cast<uint32_t>(__cvta_generic_to_shared(p));
+}
+
+__device__ __forceinline__ void cp_async16(uint32_t dst, const void* src) {
+  asm volatile("cp.async.cg.shared.global [%0], [%1], 16;\n" ::"r"(dst), "l"(src));
+}
+__device__ __forceinline__ void cp_async_commit() { asm volatile("cp.async.commit_group;\n" ::); }
+template <int N>
+__device__ __forceinline__ void cp_async_wait() { asm volatile("cp.async.wait_group %0;\n" ::"n"(N)); }
+__device__ __forceinline__ void cp_async_wait_dyn(int n) {
+  switch (n) {
+    case 0: cp_async_wait<0>(); break;
+    case 1: cp_async_wait<1>(); break;
+    case 2: cp_async_wait<2>(); break;
+    case 3: cp_async_wait<3>(); break;
+    case 4: cp_async_wait<4>(); break;
+    case 5: cp_async_wait<5>(); break;
+    case 6: cp_async_wait<6>(); break;
+    default: cp_async_wait<7>(); break;
+  }
+}
+
+// 2^x with the MUFU approximation (x <= 0 or small; -inf gives 0)
+__device__ __forceinline__ float fast_exp2(float x) {
+  float y;
+  asm("ex2.approx.ftz.f32 %0, %1;" : "=f"(y) : "f"(x));
+  return y;
+}
+
+__device__ __forceinline__ uint4 lds128(const uint8_t* p) {
+  return *reinterpret_cast<const uint4*>(p);
+}
+
+// ------------------------------------------------------- code extraction ----
+// The lane's 4*BW code words of one block image (16-byte piece i of lane L at
+// byte 16*(32 i + L)).
 template <int BW>
-__device__ __forceinline__ void load_lane_codes(const uint8_t* blk, int lane, uint32_t (&w)[4 * BW]) {
+__device__ __forceinline__ void lane_words(const uint8_t* img, int lane, uint32_t (&w)[4 * BW]) {
 #pragma unroll
   for (int i = 0; i < BW; ++i) {
-    const uint4 u = ldg_stream(blk + 16 * (32 * i + lane));
+    const uint4 u = lds128(img + 16 * (32 * i + lane));
     w[4 * i + 0] = u.x;
     w[4 * i + 1] = u.y;
     w[4 * i + 2] = u.z;
@@ -93,7 +140,6 @@ __device__ __forceinline__ void load_lane_codes(const uint8_t* blk, int lane, ui
   }
 }
 
-// BW-bit code at lane-stream bit p (p is a compile-time constant after unrolling)
 template <int BW>
 __device__ __forceinline__ uint32_t lane_code(const uint32_t (&w)[4 * BW], int p) {
   const int wi = p >> 5, sh = p & 31;
@@ -102,155 +148,261 @@ __device__ __forceinline__ uint32_t lane_code(const uint32_t (&w)[4 * BW], int p
   return v & ((1u << BW) - 1u);
 }
 
-// Register k of the A fragment of fragment phi: codes (a_2k, a_2k+1) at slot
-// positions k and 4+k, as exact fp16 integers: the code is OR-ed into the
-// mantissa of fp16 1024.0 and 1024.0 is subtracted.
-template <int BW>
-__device__ __forceinline__ __half2 code_pair(const uint32_t (&w)[4 * BW], int phi, int k) {
-  const int base = 8 * BW * phi;
-  const uint32_t lo = lane_code<BW>(w, base + BW * k);
-  const uint32_t hi = lane_code<BW>(w, base + BW * (4 + k));
-  constexpr uint32_t kMagic = 0x64006400u;
-  return __hsub2(u2h(lo | (hi << 16) | kMagic), u2h(kMagic));
+constexpr uint32_t kMagic = 0x64006400u;      // fp16 1024.0 in both halves
+constexpr uint32_t kMagicBytes = 0x64646464u;
+
+__device__ __forceinline__ uint32_t hfma2u(uint32_t x, uint32_t m, uint32_t a) {
+  return h2u(__hfma2(u2h(x), u2h(m), u2h(a)));
+}
+__device__ __forceinline__ uint32_t hsub2u(uint32_t x, uint32_t y) {
+  return h2u(__hsub2(u2h(x), u2h(y)));
 }
 
-// 16 meta words of this lane starting at uint4 index q4
-__device__ __forceinline__ void load_meta16(const uint4* meta, int q4, uint32_t (&m)[16]) {
+// Fragment f of the lane stream: register k holds the code pair
+// (a_2k, a_2k+1) = (slot k, slot 4+k) as exact fp16 integers.
+template <int BW>
+__device__ __forceinline__ void frag_codes(const uint32_t (&w)[4 * BW], int f, uint32_t (&c)[4]) {
+  if constexpr (BW == 1) {
+    // byte = (a0 a2 a4 a6 | a1 a3 a5 a7) bits; both halves get the byte under 0x64
+    const int bi = f & 3;
+    const uint32_t W = __byte_perm(w[f >> 2], kMagicBytes, 0x4040u | (bi << 8) | bi);
+    // half0 keeps bit k (2^k a), half1 bit 4+k (2^(4+k) a'); scales are exact
+    const uint32_t mul[4] = {0x2C003C00u, 0x28003800u, 0x24003400u, 0x20003000u};
+    const uint32_t add[4] = {0xD400E400u, 0xD000E000u, 0xCC00DC00u, 0xC800D800u};
 #pragma unroll
-  for (int i = 0; i < 4; ++i) {
-    const uint4 u = ldg_stream(meta + q4 + i);
-    m[4 * i + 0] = u.x;
-    m[4 * i + 1] = u.y;
-    m[4 * i + 2] = u.z;
-    m[4 * i + 3] = u.w;
+    for (int k = 0; k < 4; ++k)
+      c[k] = hfma2u(W & (kMagic | (1u << k) | (1u << (20 + k))), mul[k], add[k]);
+  } else if constexpr (BW == 2) {
+    // 16-bit fragment: low byte (a0 a2 a4 a6) -> half0, high byte -> half1
+    const int lb = 2 * (f & 1);
+    const uint32_t W = __byte_perm(w[f >> 1], kMagicBytes, 0x4040u | ((lb + 1) << 8) | lb);
+    const uint32_t mul[4] = {0x3C003C00u, 0x34003400u, 0x2C002C00u, 0x24002400u};   // 4^-k
+    const uint32_t add[4] = {0xE400E400u, 0xDC00DC00u, 0xD400D400u, 0xCC00CC00u};   // -1024 4^-k
+#pragma unroll
+    for (int k = 0; k < 4; ++k) c[k] = hfma2u(W & (kMagic | (0x00030003u << (2 * k))), mul[k], add[k]);
+  } else if constexpr (BW == 3) {
+    // 24-bit fragment: low 12 bits -> half0, next 12 bits -> half1
+    const int base = 3 * (f >> 2), s = f & 3;
+    uint32_t X;
+    if (s == 0) X = w[base];
+    else if (s == 1) X = __funnelshift_r(w[base], w[base + 1], 24);
+    else if (s == 2) X = __funnelshift_r(w[base + 1], w[base + 2], 16);
+    else X = w[base + 2] >> 8;
+    const uint32_t W = (X & 0xFFFFu) | ((X << 4) & 0xFFFF0000u);
+    const uint32_t mul[3] = {0x3C003C00u, 0x30003000u, 0x24002400u};   // 8^-k
+    const uint32_t add[3] = {0xE400E400u, 0xD800D800u, 0xCC00CC00u};   // -1024 8^-k
+#pragma unroll
+    for (int k = 0; k < 3; ++k) c[k] = hfma2u((W & (0x00070007u << (3 * k))) | kMagic, mul[k], add[k]);
+    c[3] = hfma2u(((W >> 3) & 0x01C001C0u) | kMagic, 0x24002400u, 0xCC00CC00u);
+  } else if constexpr (BW == 4) {
+    // one word: low half nibbles a0 a2 a4 a6, high half a1 a3 a5 a7
+    const uint32_t X = w[f], Y = X >> 8;
+    c[0] = hsub2u((X & 0x000F000Fu) | kMagic, kMagic);
+    c[1] = hfma2u((X & 0x00F000F0u) | kMagic, 0x2C002C00u, 0xD400D400u);   // /16 - 64
+    c[2] = hsub2u((Y & 0x000F000Fu) | kMagic, kMagic);
+    c[3] = hfma2u((Y & 0x00F000F0u) | kMagic, 0x2C002C00u, 0xD400D400u);
+  } else if constexpr (BW == 8) {
+    // two words: bytes a0 a2 a4 a6 | a1 a3 a5 a7
+    const uint32_t X0 = w[2 * f], X1 = w[2 * f + 1];
+    const uint32_t Y0 = __byte_perm(X0, X1, 0x5140u);   // a0 a1 a2 a3
+    const uint32_t Y1 = __byte_perm(X0, X1, 0x7362u);   // a4 a5 a6 a7
+    c[0] = hsub2u(__byte_perm(Y0, kMagicBytes, 0x4140u), kMagic);
+    c[1] = hsub2u(__byte_perm(Y0, kMagicBytes, 0x4342u), kMagic);
+    c[2] = hsub2u(__byte_perm(Y1, kMagicBytes, 0x4140u), kMagic);
+    c[3] = hsub2u(__byte_perm(Y1, kMagicBytes, 0x4342u), kMagic);
+  } else {
+    const int base = 8 * BW * f;
+#pragma unroll
+    for (int k = 0; k < 4; ++k) {
+      const uint32_t lo = lane_code<BW>(w, base + BW * k);
+      const uint32_t hi = lane_code<BW>(w, base + BW * (4 + k));
+      c[k] = hsub2u(lo | (hi << 16) | kMagic, kMagic);
+    }
   }
 }
 
-// scores^T[mt] (tokens 16 mt + gid (+8), heads 2 tig (+1)) for one K block
+// ------------------------------------------------------------ block math ----
+
+// scores^T[mt] (tokens 16 mt + gid (+8), heads 2 tig (+1)) of one K block image.
+// Per-channel keys: k_hat[t][c] = code s_c + z_c, so
+//   scores[t][j] = sum_c code[t][c] (q_jc s_c) + sum_c z_c q_jc:
+// the scale is folded into q (one fp16x2 multiply per q pair) and the
+// zero-point term, the same for every token, comes from MMAs whose A operand
+// repeats z in every row and initialises the accumulators. The codes enter
+// the MMA as exact fp16 integers.
 template <int BW, int KG>
-__device__ __forceinline__ void qk_block(const uint8_t* blk, int lane, const uint32_t (&qb)[8][2],
+__device__ __forceinline__ void qk_block(const uint8_t* img, int lane, const uint32_t (&qb)[8][2],
                                          float (&s)[2][4]) {
   const int gid = lane >> 2, tig = lane & 3;
   uint32_t w[4 * BW];
-  load_lane_codes<BW>(blk, lane, w);
-  const uint4* meta = reinterpret_cast<const uint4*>(blk + 512 * BW);
-  uint32_t ms[16], mz[16];
-  if (KG == RQ_PER_CHANNEL) {   // scale pairs at words 16 tig.., zero pairs at 64 + 16 tig..
-    load_meta16(meta, 4 * tig, ms);
-    load_meta16(meta, 16 + 4 * tig, mz);
-  } else {                      // (scale, zero) words at 16 gid..
-    load_meta16(meta, 4 * gid, ms);
-  }
+  lane_words<BW>(img, lane, w);
+  const uint8_t* meta = img + 512 * BW;
+  if constexpr (KG == RQ_PER_CHANNEL) {
+    uint32_t qs2[8][2];
+    float zb[4] = {0.0f, 0.0f, 0.0f, 0.0f};
 #pragma unroll
-  for (int mt = 0; mt < 2; ++mt)
-#pragma unroll
-    for (int r = 0; r < 4; ++r) s[mt][r] = 0.0f;
-#pragma unroll
-  for (int ks = 0; ks < 8; ++ks) {
-#pragma unroll
-    for (int mt = 0; mt < 2; ++mt) {
-      const int phi = 2 * ks + mt;
-      uint32_t a[4];
-#pragma unroll
-      for (int k = 0; k < 4; ++k) {
-        const __half2 c = code_pair<BW>(w, phi, k);
-        __half2 sc, zr;
-        if (KG == RQ_PER_CHANNEL) {        // channels 16 ks + 8 (k>>1) + 2 tig, +1
-          const int wd = 2 * ks + (k >> 1);
-          sc = u2h(ms[wd]);
-          zr = u2h(mz[wd]);
-        } else {                           // token 16 mt + gid + 8 (k&1), group ks/2
-          const __half2 sz = u2h(ms[4 * (2 * mt + (k & 1)) + (ks >> 1)]);
-          sc = __low2half2(sz);
-          zr = __high2half2(sz);
-        }
-        a[k] = h2u(__hfma2(c, sc, zr));
-      }
-      mma16816(s[mt], a, qb[ks][0], qb[ks][1]);
+    for (int ks = 0; ks < 8; ++ks) {   // channel pairs 16 ks + 8 h + 2 tig: words 16 tig + 2 ks + h
+      const uint2 s2 = *reinterpret_cast<const uint2*>(meta + 4 * (16 * tig + 2 * ks));
+      const uint2 z2 = *reinterpret_cast<const uint2*>(meta + 256 + 4 * (16 * tig + 2 * ks));
+      qs2[ks][0] = h2u(__hmul2(u2h(qb[ks][0]), u2h(s2.x)));
+      qs2[ks][1] = h2u(__hmul2(u2h(qb[ks][1]), u2h(s2.y)));
+      const uint32_t az[4] = {z2.x, z2.x, z2.y, z2.y};
+      mma16816(zb, az, qb[ks][0], qb[ks][1]);
     }
+#pragma unroll
+    for (int mt = 0; mt < 2; ++mt)
+#pragma unroll
+      for (int r = 0; r < 4; ++r) s[mt][r] = zb[r];
+#pragma unroll
+    for (int ks = 0; ks < 8; ++ks)
+#pragma unroll
+      for (int mt = 0; mt < 2; ++mt) {
+        uint32_t c[4];
+        frag_codes<BW>(w, 2 * ks + mt, c);
+        mma16816(s[mt], c, qs2[ks][0], qs2[ks][1]);
+      }
+  } else {                    // per-token keys: dequantize in registers
+    uint32_t sz[16];          // (scale, zero) of groups (gid + 8m, G): words 16 gid ..
+#pragma unroll
+    for (int i = 0; i < 4; ++i) {
+      const uint4 u = lds128(meta + 64 * gid + 16 * i);
+      sz[4 * i] = u.x;
+      sz[4 * i + 1] = u.y;
+      sz[4 * i + 2] = u.z;
+      sz[4 * i + 3] = u.w;
+    }
+#pragma unroll
+    for (int mt = 0; mt < 2; ++mt)
+#pragma unroll
+      for (int r = 0; r < 4; ++r) s[mt][r] = 0.0f;
+#pragma unroll
+    for (int ks = 0; ks < 8; ++ks)
+#pragma unroll
+      for (int mt = 0; mt < 2; ++mt) {
+        uint32_t c[4], a[4];
+        frag_codes<BW>(w, 2 * ks + mt, c);
+#pragma unroll
+        for (int k = 0; k < 4; ++k) {     // token 16 mt + gid + 8 (k&1), group ks/2
+          const __half2 szh = u2h(sz[4 * (2 * mt + (k & 1)) + (ks >> 1)]);
+          a[k] = hfma2u(c[k], h2u(__low2half2(szh)), h2u(__high2half2(szh)));
+        }
+        mma16816(s[mt], a, qb[ks][0], qb[ks][1]);
+      }
   }
 }
 
-// o^T[mt] (channels 16 mt + gid (+8), heads 2 tig (+1)) += V_hat^T . P^T for one V block
+// o^T[mt] (channels 16 mt + gid (+8), heads 2 tig (+1)) += V_hat^T . P^T of one V block image.
+// Per-token values: v_hat[t][c] = code s_tG + z_tG (G = c / 32), so
+//   o[c][j] += sum_t code[t][c] (p_tj s_tG) + sum_t z_tG p_tj:
+// the scale is folded into P^T per channel group (one fp16x2 multiply per
+// pair) and the zero-point term comes from MMAs whose A operand repeats z_tG
+// down every channel row of the group.
 template <int BW, int VG>
-__device__ __forceinline__ void pv_block(const uint8_t* blk, int lane, const uint32_t (&pb)[2][2],
+__device__ __forceinline__ void pv_block(const uint8_t* img, int lane, const uint32_t (&pb)[2][2],
                                          float (&o)[8][4]) {
   const int gid = lane >> 2, tig = lane & 3;
   uint32_t w[4 * BW];
-  load_lane_codes<BW>(blk, lane, w);
-  const uint4* meta = reinterpret_cast<const uint4*>(blk + 512 * BW);
-  uint32_t ms[16], mz[16];
-  if (VG == RQ_PER_TOKEN) {
-    load_meta16(meta, 4 * tig, ms);
-    load_meta16(meta, 16 + 4 * tig, mz);
-  } else {
-    load_meta16(meta, 4 * gid, ms);
-  }
+  lane_words<BW>(img, lane, w);
+  const uint8_t* meta = img + 512 * BW;
+  if constexpr (VG == RQ_PER_TOKEN) {
+    uint32_t ms[16], mz[16];  // token pairs (tig + 4j) x group G: words 16 tig + 4 j + G
 #pragma unroll
-  for (int ks = 0; ks < 2; ++ks) {
-#pragma unroll
-    for (int mt = 0; mt < 8; ++mt) {
-      const int phi = 8 * ks + mt;
-      uint32_t a[4];
-#pragma unroll
-      for (int k = 0; k < 4; ++k) {
-        const __half2 c = code_pair<BW>(w, phi, k);
-        __half2 sc, zr;
-        if (VG == RQ_PER_TOKEN) {          // tokens 16 ks + 8 (k>>1) + 2 tig, +1; group mt/2
-          const int wd = 4 * (2 * ks + (k >> 1)) + (mt >> 1);
-          sc = u2h(ms[wd]);
-          zr = u2h(mz[wd]);
-        } else {                           // channel 16 mt + gid + 8 (k&1)
-          const __half2 sz = u2h(ms[2 * mt + (k & 1)]);
-          sc = __low2half2(sz);
-          zr = __high2half2(sz);
-        }
-        a[k] = h2u(__hfma2(c, sc, zr));
-      }
-      mma16816(o[mt], a, pb[ks][0], pb[ks][1]);
+    for (int i = 0; i < 4; ++i) {
+      const uint4 u = lds128(meta + 64 * tig + 16 * i);
+      const uint4 z = lds128(meta + 256 + 64 * tig + 16 * i);
+      ms[4 * i] = u.x;
+      ms[4 * i + 1] = u.y;
+      ms[4 * i + 2] = u.z;
+      ms[4 * i + 3] = u.w;
+      mz[4 * i] = z.x;
+      mz[4 * i + 1] = z.y;
+      mz[4 * i + 2] = z.z;
+      mz[4 * i + 3] = z.w;
     }
+#pragma unroll
+    for (int ks = 0; ks < 2; ++ks) {
+#pragma unroll
+      for (int G = 0; G < 4; ++G) {
+        // B fragment rows: tokens 16 ks + 2 tig (+1) and + 8  ->  pair words j = 2 ks, 2 ks + 1
+        const uint32_t b0 = h2u(__hmul2(u2h(pb[ks][0]), u2h(ms[4 * (2 * ks) + G])));
+        const uint32_t b1 = h2u(__hmul2(u2h(pb[ks][1]), u2h(ms[4 * (2 * ks + 1) + G])));
+        const uint32_t az[4] = {mz[4 * (2 * ks) + G], mz[4 * (2 * ks) + G],
+                                mz[4 * (2 * ks + 1) + G], mz[4 * (2 * ks + 1) + G]};
+#pragma unroll
+        for (int h = 0; h < 2; ++h) {
+          const int mt = 2 * G + h;
+          uint32_t c[4];
+          frag_codes<BW>(w, 8 * ks + mt, c);
+          mma16816(o[mt], c, b0, b1);
+          mma16816(o[mt], az, pb[ks][0], pb[ks][1]);
+        }
+      }
+    }
+  } else {                    // per-channel values: dequantize in registers
+    uint32_t ms[16];          // (scale, zero) of channels 16 mt + gid + 8 h: words 16 gid ..
+#pragma unroll
+    for (int i = 0; i < 4; ++i) {
+      const uint4 u = lds128(meta + 64 * gid + 16 * i);
+      ms[4 * i] = u.x;
+      ms[4 * i + 1] = u.y;
+      ms[4 * i + 2] = u.z;
+      ms[4 * i + 3] = u.w;
+    }
+#pragma unroll
+    for (int ks = 0; ks < 2; ++ks)
+#pragma unroll
+      for (int mt = 0; mt < 8; ++mt) {
+        uint32_t c[4], a[4];
+        frag_codes<BW>(w, 8 * ks + mt, c);
+#pragma unroll
+        for (int k = 0; k < 4; ++k) {     // channel 16 mt + gid + 8 (k&1)
+          const __half2 szh = u2h(ms[2 * mt + (k & 1)]);
+          a[k] = hfma2u(c[k], h2u(__low2half2(szh)), h2u(__high2half2(szh)));
+        }
+        mma16816(o[mt], a, pb[ks][0], pb[ks][1]);
+      }
   }
 }
 
 template <int BW>
-__device__ __forceinline__ void qk_dispatch_g(int kg, const uint8_t* blk, int lane,
+__device__ __forceinline__ void qk_dispatch_g(int kg, const uint8_t* img, int lane,
                                               const uint32_t (&qb)[8][2], float (&s)[2][4]) {
-  if (kg == RQ_PER_CHANNEL) qk_block<BW, RQ_PER_CHANNEL>(blk, lane, qb, s);
-  else qk_block<BW, RQ_PER_TOKEN>(blk, lane, qb, s);
+  if (kg == RQ_PER_CHANNEL) qk_block<BW, RQ_PER_CHANNEL>(img, lane, qb, s);
+  else qk_block<BW, RQ_PER_TOKEN>(img, lane, qb, s);
 }
 
 template <int BW>
-__device__ __forceinline__ void pv_dispatch_g(int vg, const uint8_t* blk, int lane,
+__device__ __forceinline__ void pv_dispatch_g(int vg, const uint8_t* img, int lane,
                                               const uint32_t (&pb)[2][2], float (&o)[8][4]) {
-  if (vg == RQ_PER_TOKEN) pv_block<BW, RQ_PER_TOKEN>(blk, lane, pb, o);
-  else pv_block<BW, RQ_PER_CHANNEL>(blk, lane, pb, o);
+  if (vg == RQ_PER_TOKEN) pv_block<BW, RQ_PER_TOKEN>(img, lane, pb, o);
+  else pv_block<BW, RQ_PER_CHANNEL>(img, lane, pb, o);
 }
 
-__device__ __forceinline__ void qk_dispatch(int bw, int kg, const uint8_t* blk, int lane,
+__device__ __forceinline__ void qk_dispatch(int bw, int kg, const uint8_t* img, int lane,
                                             const uint32_t (&qb)[8][2], float (&s)[2][4]) {
   switch (bw) {
-    case 1: qk_dispatch_g<1>(kg, blk, lane, qb, s); break;
-    case 2: qk_dispatch_g<2>(kg, blk, lane, qb, s); break;
-    case 3: qk_dispatch_g<3>(kg, blk, lane, qb, s); break;
-    case 4: qk_dispatch_g<4>(kg, blk, lane, qb, s); break;
-    case 5: qk_dispatch_g<5>(kg, blk, lane, qb, s); break;
-    case 6: qk_dispatch_g<6>(kg, blk, lane, qb, s); break;
-    case 7: qk_dispatch_g<7>(kg, blk, lane, qb, s); break;
-    default: qk_dispatch_g<8>(kg, blk, lane, qb, s); break;
+    case 1: qk_dispatch_g<1>(kg, img, lane, qb, s); break;
+    case 2: qk_dispatch_g<2>(kg, img, lane, qb, s); break;
+    case 3: qk_dispatch_g<3>(kg, img, lane, qb, s); break;
+    case 4: qk_dispatch_g<4>(kg, img, lane, qb, s); break;
+    case 5: qk_dispatch_g<5>(kg, img, lane, qb, s); break;
+    case 6: qk_dispatch_g<6>(kg, img, lane, qb, s); break;
+    case 7: qk_dispatch_g<7>(kg, img, lane, qb, s); break;
+    default: qk_dispatch_g<8>(kg, img, lane, qb, s); break;
   }
 }
 
-__device__ __forceinline__ void pv_dispatch(int bw, int vg, const uint8_t* blk, int lane,
+__device__ __forceinline__ void pv_dispatch(int bw, int vg, const uint8_t* img, int lane,
                                             const uint32_t (&pb)[2][2], float (&o)[8][4]) {
   switch (bw) {
-    case 1: pv_dispatch_g<1>(vg, blk, lane, pb, o); break;
-    case 2: pv_dispatch_g<2>(vg, blk, lane, pb, o); break;
-    case 3: pv_dispatch_g<3>(vg, blk, lane, pb, o); break;
-    case 4: pv_dispatch_g<4>(vg, blk, lane, pb, o); break;
-    case 5: pv_dispatch_g<5>(vg, blk, lane, pb, o); break;
-    case 6: pv_dispatch_g<6>(vg, blk, lane, pb, o); break;
-    case 7: pv_dispatch_g<7>(vg, blk, lane, pb, o); break;
-    default: pv_dispatch_g<8>(vg, blk, lane, pb, o); break;
+    case 1: pv_dispatch_g<1>(vg, img, lane, pb, o); break;
+    case 2: pv_dispatch_g<2>(vg, img, lane, pb, o); break;
+    case 3: pv_dispatch_g<3>(vg, img, lane, pb, o); break;
+    case 4: pv_dispatch_g<4>(vg, img, lane, pb, o); break;
+    case 5: pv_dispatch_g<5>(vg, img, lane, pb, o); break;
+    case 6: pv_dispatch_g<6>(vg, img, lane, pb, o); break;
+    case 7: pv_dispatch_g<7>(vg, img, lane, pb, o); break;
+    default: pv_dispatch_g<8>(vg, img, lane, pb, o); break;
   }
 }
 
@@ -270,15 +422,245 @@ __device__ void fwht_smem(float* x, int rows) {
   }
 }
 
+// Issue the cp.async copies of one ring entry (the K or V image of one
+// block, `bytes` long, at `src`) into the slot at shared address `dst`; one
+// commit group per entry (empty when there is nothing left, so the group
+// count stays uniform).
+__device__ __forceinline__ void issue_entry(bool live, int lane, uint32_t dst, const uint8_t* src,
+                                            int bytes) {
+  if (live) {
+    const int chunks = bytes >> 4;
+    for (int ch = lane; ch < chunks; ch += 32) cp_async16(dst + 16 * ch, src + 16 * ch);
+  }
+  cp_async_commit();
+}
+
+// Per-warp streaming state: the warp's blocks are blk_first, blk_first + 4,
+// ... of one (batch, kv head) K and V stream; ring entry e is the K image
+// (e even) or V image (e odd) of the warp's block e / 2.
+struct WarpStream {
+  const uint8_t* kwarp;   // K image of the warp's first block
+  const uint8_t* vwarp;
+  uint8_t* ring_ptr;      // this warp's ring of slots
+  uint32_t ring;          // its shared-memory address
+  int lane, nb;
+};
+
+// online-softmax state of one warp: o^T accumulators and per-column max/sum
+struct SoftmaxAcc {
+  float o[8][4];
+  float m0, m1, l0, l1;
+};
+
+// softmax of one block's scores (log2 units) into the accumulator; returns
+// the B fragments of P^T. The running max only moves when a block max
+// exceeds it by more than 8, so p <= 2^8 and rescaling is rare.
+__device__ __forceinline__ void softmax_block(float (&s)[2][4], SoftmaxAcc& acc,
+                                              uint32_t (&pb)[2][2]) {
+  float bm0 = fmaxf(fmaxf(s[0][0], s[0][2]), fmaxf(s[1][0], s[1][2]));
+  float bm1 = fmaxf(fmaxf(s[0][1], s[0][3]), fmaxf(s[1][1], s[1][3]));
+#pragma unroll
+  for (int off = 4; off <= 16; off <<= 1) {
+    bm0 = fmaxf(bm0, __shfl_xor_sync(0xffffffffu, bm0, off));
+    bm1 = fmaxf(bm1, __shfl_xor_sync(0xffffffffu, bm1, off));
+  }
+  if (__any_sync(0xffffffffu, bm0 > acc.m0 + 8.0f || bm1 > acc.m1 + 8.0f)) {
+    const float nm0 = fmaxf(acc.m0, bm0), nm1 = fmaxf(acc.m1, bm1);
+    const float al0 = fast_exp2(acc.m0 - nm0), al1 = fast_exp2(acc.m1 - nm1);
+    acc.m0 = nm0;
+    acc.m1 = nm1;
+    acc.l0 *= al0;
+    acc.l1 *= al1;
+#pragma unroll
+    for (int mt = 0; mt < 8; ++mt) {
+      acc.o[mt][0] *= al0;
+      acc.o[mt][1] *= al1;
+      acc.o[mt][2] *= al0;
+      acc.o[mt][3] *= al1;
+    }
+  }
+  float p[2][4];
+#pragma unroll
+  for (int mt = 0; mt < 2; ++mt) {
+    p[mt][0] = fast_exp2(s[mt][0] - acc.m0);
+    p[mt][1] = fast_exp2(s[mt][1] - acc.m1);
+    p[mt][2] = fast_exp2(s[mt][2] - acc.m0);
+    p[mt][3] = fast_exp2(s[mt][3] - acc.m1);
+  }
+  acc.l0 += (p[0][0] + p[0][2]) + (p[1][0] + p[1][2]);
+  acc.l1 += (p[0][1] + p[0][3]) + (p[1][1] + p[1][3]);
+#pragma unroll
+  for (int ks = 0; ks < 2; ++ks) {
+    pb[ks][0] = movmatrix_trans(pack_f16x2(p[ks][0], p[ks][1]));
+    pb[ks][1] = movmatrix_trans(pack_f16x2(p[ks][2], p[ks][3]));
+  }
+}
+
+// ---- streaming with widths and groupings fixed at compile time: slot sizes,
+// slot counts, copy counts and the wait depth are constants, and the fp16
+// constants of the code extraction stay in registers across the loop.
+template <int BK, int BV>
+struct Ring {
+  static constexpr int kSK = 512 * (BK + 1), kSV = 512 * (BV + 1);
+  static constexpr int kSlot = kSK > kSV ? kSK : kSV;
+  static constexpr int kRaw = kRingBytes / kSlot;
+  static constexpr int kSlots = kRaw > kMaxSlots ? kMaxSlots : kRaw;
+};
+
+template <int BK, int BV>
+__device__ __forceinline__ void issue_static(const WarpStream& ws, int e, int slot) {
+  using R = Ring<BK, BV>;
+  if (e < 2 * ws.nb) {
+    const int i = e >> 1;
+    const uint32_t dst = ws.ring + slot * R::kSlot;
+    if ((e & 1) == 0) {
+      const uint8_t* src = ws.kwarp + i * (kWarps * R::kSK);
+#pragma unroll
+      for (int c = 0; c < R::kSK / 512; ++c) cp_async16(dst + 16 * (ws.lane + 32 * c), src + 16 * (ws.lane + 32 * c));
+    } else {
+      const uint8_t* src = ws.vwarp + i * (kWarps * R::kSV);
+#pragma unroll
+      for (int c = 0; c < R::kSV / 512; ++c) cp_async16(dst + 16 * (ws.lane + 32 * c), src + 16 * (ws.lane + 32 * c));
+    }
+  }
+  cp_async_commit();
+}
+
+template <int BK, int BV>
+__device__ __forceinline__ void prologue_static(const WarpStream& ws) {
+#pragma unroll
+  for (int e = 0; e < Ring<BK, BV>::kSlots - 1; ++e) issue_static<BK, BV>(ws, e, e);
+}
+
+template <int BK, int KG, int BV, int VG>
+__device__ __forceinline__ void blocks_static(const WarpStream& ws, const uint32_t (&qb)[8][2],
+                                              SoftmaxAcc& acc) {
+  using R = Ring<BK, BV>;
+  constexpr int NS = R::kSlots;
+  int use = 0, iss = NS - 1;          // slot of the next entry to use / to issue
+  for (int i = 0; i < ws.nb; ++i) {
+    issue_static<BK, BV>(ws, 2 * i + NS - 1, iss);
+    iss = iss + 1 == NS ? 0 : iss + 1;
+    cp_async_wait<NS - 1>();
+    __syncwarp();
+    float s[2][4];
+    qk_block<BK, KG>(ws.ring_ptr + use * R::kSlot, ws.lane, qb, s);
+    __syncwarp();
+    use = use + 1 == NS ? 0 : use + 1;
+    uint32_t pb[2][2];
+    softmax_block(s, acc, pb);
+    issue_static<BK, BV>(ws, 2 * i + NS, iss);
+    iss = iss + 1 == NS ? 0 : iss + 1;
+    cp_async_wait<NS - 1>();
+    __syncwarp();
+    pv_block<BV, VG>(ws.ring_ptr + use * R::kSlot, ws.lane, pb, acc.o);
+    __syncwarp();
+    use = use + 1 == NS ? 0 : use + 1;
+  }
+  cp_async_wait<0>();
+}
+
+// ---- streaming with runtime widths/groupings (every other combination)
+struct DynRing {
+  int bK, bV, kg, vg, sK, sV, slot, ns;
+};
+
+__device__ __forceinline__ void issue_dyn(const WarpStream& ws, const DynRing& r, int e, int slot) {
+  const int i = e >> 1;
+  const bool isK = (e & 1) == 0;
+  issue_entry(e < 2 * ws.nb, ws.lane, ws.ring + slot * r.slot,
+              isK ? ws.kwarp + i * (kWarps * r.sK) : ws.vwarp + i * (kWarps * r.sV), isK ? r.sK : r.sV);
+}
+
+__device__ __forceinline__ void prologue_dyn(const WarpStream& ws, const DynRing& r) {
+  for (int e = 0; e < r.ns - 1; ++e) issue_dyn(ws, r, e, e);
+}
+
+__device__ __forceinline__ void blocks_dyn(const WarpStream& ws, const DynRing& r,
+                                           const uint32_t (&qb)[8][2], SoftmaxAcc& acc) {
+  int use = 0, iss = r.ns - 1;
+  for (int i = 0; i < ws.nb; ++i) {
+    issue_dyn(ws, r, 2 * i + r.ns - 1, iss);
+    iss = iss + 1 == r.ns ? 0 : iss + 1;
+    cp_async_wait_dyn(r.ns - 1);
+    __syncwarp();
+    float s[2][4];
+    qk_dispatch(r.bK, r.kg, ws.ring_ptr + use * r.slot, ws.lane, qb, s);
+    __syncwarp();
+    use = use + 1 == r.ns ? 0 : use + 1;
+    uint32_t pb[2][2];
+    softmax_block(s, acc, pb);
+    issue_dyn(ws, r, 2 * i + r.ns, iss);
+    iss = iss + 1 == r.ns ? 0 : iss + 1;
+    cp_async_wait_dyn(r.ns - 1);
+    __syncwarp();
+    pv_dispatch(r.bV, r.vg, ws.ring_ptr + use * r.slot, ws.lane, pb, acc.o);
+    __syncwarp();
+    use = use + 1 == r.ns ? 0 : use + 1;
+  }
+  cp_async_wait<0>();
+}
+
+// KIVI layout (per-channel K, per-token V) at widths {2, 3, 4, 8}: key for
+// the compile-time path, or -1
+__device__ __forceinline__ int fast_key(int bK, int bV, int kg, int vg) {
+  auto idx = [](int b) { return b == 2 ? 0 : b == 3 ? 1 : b == 4 ? 2 : b == 8 ? 3 : -1; };
+  if (kg != RQ_PER_CHANNEL || vg != RQ_PER_TOKEN) return -1;
+  const int ik = idx(bK), iv = idx(bV);
+  return (ik < 0 || iv < 0) ? -1 : 4 * ik + iv;
+}
+
+#define RQ_FAST_CASES(X) \
+  X(0, 2, 2) X(1, 2, 3) X(2, 2, 4) X(3, 2, 8) X(4, 3, 2) X(5, 3, 3) X(6, 3, 4) X(7, 3, 8) \
+  X(8, 4, 2) X(9, 4, 3) X(10, 4, 4) X(11, 4, 8) X(12, 8, 2) X(13, 8, 3) X(14, 8, 4) X(15, 8, 8)
+
 template <typename T>
 __global__ void __launch_bounds__(kThreads) decode_split_kernel(DecodeArgs a) {
-  __shared__ float qs[kMaxHeads][kD];
-  __shared__ float red_o[kWarps][kMaxHeads][kD];
+  extern __shared__ __align__(16) unsigned char smem_raw[];
+  float* qs = reinterpret_cast<float*>(smem_raw);                  // [8][128]
+  uint8_t* rings = smem_raw + kQBytes;
   __shared__ float red_m[kWarps][kMaxHeads];
   __shared__ float red_l[kWarps][kMaxHeads];
   const int split = blockIdx.x, h = blockIdx.y, batch = blockIdx.z;
   const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
   const int gid = lane >> 2, tig = lane & 3;
+
+  const int bK = a.bits[(a.layer * a.H + h) * 2 + 0];
+  const int bV = a.bits[(a.layer * a.H + h) * 2 + 1];
+  const bool valid = bK >= 1 && bK <= 8 && bV >= 1 && bV <= 8;
+  if (!valid && threadIdx.x == 0) set_status(a.status, RQ_STATUS_BAD_BITS);
+  const uint64_t* offp =
+      a.offsets + ((static_cast<long long>(a.layer) * a.B + batch) * a.H + h) * 2;
+  const uint8_t* kbase = a.packed + (valid ? offp[0] : 0);
+  const uint8_t* vbase = a.packed + (valid ? offp[1] : 0);
+  DynRing dr;
+  dr.bK = bK;
+  dr.bV = bV;
+  dr.kg = a.kg;
+  dr.vg = a.vg;
+  dr.sK = 512 * (bK + 1);
+  dr.sV = 512 * (bV + 1);
+  dr.slot = max(dr.sK, dr.sV);
+  dr.ns = valid ? min(kMaxSlots, kRingBytes / dr.slot) : 2;
+  const int blk0 = split * a.bps;
+  const int blk1 = min(a.nblk, blk0 + a.bps);
+  const int blk_first = blk0 + warp;
+  WarpStream ws;
+  ws.lane = lane;
+  ws.nb = valid && blk_first < blk1 ? (blk1 - blk_first + kWarps - 1) / kWarps : 0;
+  ws.ring_ptr = rings + warp * kRingBytes;
+  ws.ring = smem_u32(ws.ring_ptr);
+  ws.kwarp = kbase + static_cast<size_t>(blk_first) * dr.sK;
+  ws.vwarp = vbase + static_cast<size_t>(blk_first) * dr.sV;
+  const int key = valid ? fast_key(bK, bV, a.kg, a.vg) : -1;
+
+  // start streaming the first entries before the q prologue
+  switch (key) {
+#define RQ_PRO(k, BK, BV) case k: prologue_static<BK, BV>(ws); break;
+    RQ_FAST_CASES(RQ_PRO)
+#undef RQ_PRO
+    default: prologue_dyn(ws, dr); break;
+  }
 
   // q of the g query heads of this kv head (rows >= g are zero), rotated
   // into the cache's domain when the cache is Hadamard-rotated
@@ -291,92 +673,52 @@ __global__ void __launch_bounds__(kThreads) decode_split_kernel(DecodeArgs a) {
       x = to_f32<T>(qp[n * kD + d]);
       if (a.hadamard && a.signs && a.signs[d] < 0) x = -x;
     }
-    qs[n][d] = x;
+    qs[idx] = x;
   }
   __syncthreads();
-  if (a.hadamard) fwht_smem(&qs[0][0], kMaxHeads);
+  if (a.hadamard) fwht_smem(qs, kMaxHeads);
   // softmax scale 1/sqrt(128) and log2(e) folded into q (scores in log2 units)
   const float qscale = kLog2e * kInvSqrt128 * (a.hadamard ? kInvSqrt128 : 1.0f);
   uint32_t qb[8][2];
 #pragma unroll
   for (int ks = 0; ks < 8; ++ks) {
-    const int c0 = 16 * ks + 2 * tig;
-    qb[ks][0] = pack_f16x2(qs[gid][c0] * qscale, qs[gid][c0 + 1] * qscale);
-    qb[ks][1] = pack_f16x2(qs[gid][c0 + 8] * qscale, qs[gid][c0 + 9] * qscale);
+    const float* qr = qs + gid * kD + 16 * ks + 2 * tig;
+    qb[ks][0] = pack_f16x2(qr[0] * qscale, qr[1] * qscale);
+    qb[ks][1] = pack_f16x2(qr[8] * qscale, qr[9] * qscale);
   }
 
-  const int bK = a.bits[(a.layer * a.H + h) * 2 + 0];
-  const int bV = a.bits[(a.layer * a.H + h) * 2 + 1];
-  const bool valid = bK >= 1 && bK <= 8 && bV >= 1 && bV <= 8;
-  if (!valid && threadIdx.x == 0) set_status(a.status, RQ_STATUS_BAD_BITS);
-  const uint64_t* offp =
-      a.offsets + ((static_cast<long long>(a.layer) * a.B + batch) * a.H + h) * 2;
-  const uint8_t* kbase = a.packed + offp[0];
-  const uint8_t* vbase = a.packed + offp[1];
-  const int blk0 = split * a.bps;
-  const int blk1 = min(a.nblk, blk0 + a.bps);
-
-  float o[8][4];
+  SoftmaxAcc acc;
 #pragma unroll
   for (int mt = 0; mt < 8; ++mt)
 #pragma unroll
-    for (int r = 0; r < 4; ++r) o[mt][r] = 0.0f;
-  float m0 = -INFINITY, m1 = -INFINITY, l0 = 0.0f, l1 = 0.0f;
+    for (int r = 0; r < 4; ++r) acc.o[mt][r] = 0.0f;
+  acc.m0 = acc.m1 = -INFINITY;
+  acc.l0 = acc.l1 = 0.0f;
 
-  if (valid) {
-    for (int blk = blk0 + warp; blk < blk1; blk += kWarps) {
-      float s[2][4];
-      qk_dispatch(bK, a.kg, kbase + static_cast<size_t>(blk) * 512u * (bK + 1), lane, qb, s);
-      // online softmax over this block's 32 tokens, per head column
-      float bm0 = fmaxf(fmaxf(s[0][0], s[0][2]), fmaxf(s[1][0], s[1][2]));
-      float bm1 = fmaxf(fmaxf(s[0][1], s[0][3]), fmaxf(s[1][1], s[1][3]));
-#pragma unroll
-      for (int off = 4; off <= 16; off <<= 1) {
-        bm0 = fmaxf(bm0, __shfl_xor_sync(0xffffffffu, bm0, off));
-        bm1 = fmaxf(bm1, __shfl_xor_sync(0xffffffffu, bm1, off));
-      }
-      const float nm0 = fmaxf(m0, bm0), nm1 = fmaxf(m1, bm1);
-      const float al0 = exp2f(m0 - nm0), al1 = exp2f(m1 - nm1);
-      m0 = nm0;
-      m1 = nm1;
-      float p[2][4];
-#pragma unroll
-      for (int mt = 0; mt < 2; ++mt) {
-        p[mt][0] = exp2f(s[mt][0] - m0);
-        p[mt][1] = exp2f(s[mt][1] - m1);
-        p[mt][2] = exp2f(s[mt][2] - m0);
-        p[mt][3] = exp2f(s[mt][3] - m1);
-      }
-      l0 = l0 * al0 + ((p[0][0] + p[0][2]) + (p[1][0] + p[1][2]));
-      l1 = l1 * al1 + ((p[0][1] + p[0][3]) + (p[1][1] + p[1][3]));
-#pragma unroll
-      for (int mt = 0; mt < 8; ++mt) {
-        o[mt][0] *= al0;
-        o[mt][1] *= al1;
-        o[mt][2] *= al0;
-        o[mt][3] *= al1;
-      }
-      uint32_t pb[2][2];
-#pragma unroll
-      for (int ks = 0; ks < 2; ++ks) {
-        pb[ks][0] = movmatrix_trans(pack_f16x2(p[ks][0], p[ks][1]));
-        pb[ks][1] = movmatrix_trans(pack_f16x2(p[ks][2], p[ks][3]));
-      }
-      pv_dispatch(bV, a.vg, vbase + static_cast<size_t>(blk) * 512u * (bV + 1), lane, pb, o);
-    }
+  switch (key) {
+#define RQ_BLK(k, BK, BV) case k: blocks_static<BK, RQ_PER_CHANNEL, BV, RQ_PER_TOKEN>(ws, qb, acc); break;
+    RQ_FAST_CASES(RQ_BLK)
+#undef RQ_BLK
+    default: blocks_dyn(ws, dr, qb, acc); break;
   }
+  float m0 = acc.m0, m1 = acc.m1, l0 = acc.l0, l1 = acc.l1;
 #pragma unroll
   for (int off = 4; off <= 16; off <<= 1) {
     l0 += __shfl_xor_sync(0xffffffffu, l0, off);
     l1 += __shfl_xor_sync(0xffffffffu, l1, off);
   }
-  // merge the four warps (log-sum-exp), one partial record per query head
+  // merge the four warps (log-sum-exp), one partial record per query head;
+  // the merge buffer reuses the rings
+  __syncthreads();
+  float* red_o = reinterpret_cast<float*>(rings);   // [warp][head][channel]
 #pragma unroll
   for (int mt = 0; mt < 8; ++mt) {
-    red_o[warp][2 * tig][16 * mt + gid] = o[mt][0];
-    red_o[warp][2 * tig + 1][16 * mt + gid] = o[mt][1];
-    red_o[warp][2 * tig][16 * mt + gid + 8] = o[mt][2];
-    red_o[warp][2 * tig + 1][16 * mt + gid + 8] = o[mt][3];
+    float* r0 = red_o + (warp * kMaxHeads + 2 * tig) * kD;
+    float* r1 = r0 + kD;
+    r0[16 * mt + gid] = acc.o[mt][0];
+    r1[16 * mt + gid] = acc.o[mt][1];
+    r0[16 * mt + gid + 8] = acc.o[mt][2];
+    r1[16 * mt + gid + 8] = acc.o[mt][3];
   }
   if (gid == 0) {
     red_m[warp][2 * tig] = m0;
@@ -395,7 +737,7 @@ __global__ void __launch_bounds__(kThreads) decode_split_kernel(DecodeArgs a) {
     for (int w = 0; w < kWarps; ++w) {
       const float mw = red_m[w][n];
       const float sc = (mw == -INFINITY) ? 0.0f : exp2f(mw - M);
-      osum += sc * red_o[w][n][d];
+      osum += sc * red_o[(w * kMaxHeads + n) * kD + d];
       lsum += sc * red_l[w][n];
     }
     float* dst = a.partial + ((static_cast<long long>(batch) * a.Hq + h * a.g + n) * a.splits + split) * kPart;
@@ -445,7 +787,7 @@ __global__ void __launch_bounds__(kD) decode_combine_kernel(const float* partial
 void decode_plan(const rq_cache_desc* desc, int sms, int* splits, int* bps) {
   const int nblk = desc->S / kTile;
   const long long units = static_cast<long long>(desc->B) * desc->H_kv;
-  const long long target = static_cast<long long>(sms) * 8;
+  const long long target = static_cast<long long>(sms) * 16;
   long long sp = units > 0 ? (target + units - 1) / units : 1;
   sp = std::max<long long>(1, std::min<long long>(sp, nblk));
   const int b = static_cast<int>((nblk + sp - 1) / sp);
@@ -464,6 +806,51 @@ rq_status check_desc(const rq_cache_desc* desc) {
     return RQ_ERR_SHAPE;
   if (desc->H_q % desc->H_kv != 0 || desc->H_q / desc->H_kv > kMaxHeads) return RQ_ERR_SHAPE;
   return RQ_OK;
+}
+
+void fill_args(DecodeArgs& a, const rq_cache_desc* desc, int32_t layer, const void* q,
+               const void* packed, const uint8_t* bits_dev, const uint64_t* offsets_dev,
+               const int8_t* signs_dev, float* partial, uint32_t* status_dev, int splits, int bps) {
+  a.q = q;
+  a.packed = static_cast<const uint8_t*>(packed);
+  a.bits = bits_dev;
+  a.offsets = offsets_dev;
+  a.signs = signs_dev;
+  a.partial = partial;
+  a.status = status_dev;
+  a.layer = layer;
+  a.B = desc->B;
+  a.H = desc->H_kv;
+  a.Hq = desc->H_q;
+  a.g = desc->H_q / desc->H_kv;
+  a.nblk = desc->S / kTile;
+  a.splits = splits;
+  a.bps = bps;
+  a.kg = desc->k_grouping;
+  a.vg = desc->v_grouping;
+  a.hadamard = desc->hadamard ? 1 : 0;
+}
+
+// split kernel + combine kernel on `stream`
+rq_status launch_decode(const DecodeArgs& a, const rq_cache_desc* desc, float* out,
+                        cudaStream_t s) {
+  const dim3 grid(static_cast<unsigned>(a.splits), static_cast<unsigned>(desc->H_kv),
+                  static_cast<unsigned>(desc->B));
+  if (desc->dtype == RQ_F16) {
+    if (cudaFuncSetAttribute(decode_split_kernel<__half>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                             kSmemBytes) != cudaSuccess)
+      return RQ_ERR_CUDA;
+    decode_split_kernel<__half><<<grid, kThreads, kSmemBytes, s>>>(a);
+  } else {
+    if (cudaFuncSetAttribute(decode_split_kernel<__nv_bfloat16>,
+                             cudaFuncAttributeMaxDynamicSharedMemorySize, kSmemBytes) != cudaSuccess)
+      return RQ_ERR_CUDA;
+    decode_split_kernel<__nv_bfloat16><<<grid, kThreads, kSmemBytes, s>>>(a);
+  }
+  if (launch_status() != RQ_OK) return RQ_ERR_CUDA;
+  decode_combine_kernel<<<static_cast<unsigned>(desc->B * desc->H_q), kD, 0, s>>>(
+      a.partial, out, a.signs, a.status, a.splits, a.hadamard);
+  return launch_status();
 }
 
 }  // namespace
@@ -503,33 +890,9 @@ extern "C" rq_status rq_decode_attention(const rq_cache_desc* desc, int32_t laye
   const size_t need = static_cast<size_t>(desc->B) * desc->H_q * splits * kPart * sizeof(float);
   if (ws_bytes < need) return RQ_ERR_WORKSPACE;
   DecodeArgs a;
-  a.q = q;
-  a.packed = static_cast<const uint8_t*>(packed);
-  a.bits = bits_dev;
-  a.offsets = offsets_dev;
-  a.signs = signs_dev;
-  a.partial = static_cast<float*>(ws);
-  a.status = status_dev;
-  a.layer = layer;
-  a.B = desc->B;
-  a.H = desc->H_kv;
-  a.Hq = desc->H_q;
-  a.g = desc->H_q / desc->H_kv;
-  a.nblk = desc->S / kTile;
-  a.splits = splits;
-  a.bps = bps;
-  a.kg = desc->k_grouping;
-  a.vg = desc->v_grouping;
-  a.hadamard = desc->hadamard ? 1 : 0;
-  cudaStream_t s = static_cast<cudaStream_t>(stream);
-  const dim3 grid(static_cast<unsigned>(splits), static_cast<unsigned>(desc->H_kv),
-                  static_cast<unsigned>(desc->B));
-  if (desc->dtype == RQ_F16) decode_split_kernel<__half><<<grid, kThreads, 0, s>>>(a);
-  else decode_split_kernel<__nv_bfloat16><<<grid, kThreads, 0, s>>>(a);
-  if (launch_status() != RQ_OK) return RQ_ERR_CUDA;
-  decode_combine_kernel<<<static_cast<unsigned>(desc->B * desc->H_q), kD, 0, s>>>(
-      a.partial, out, signs_dev, status_dev, splits, a.hadamard);
-  return launch_status();
+  fill_args(a, desc, layer, q, packed, bits_dev, offsets_dev, signs_dev, static_cast<float*>(ws),
+            status_dev, splits, bps);
+  return launch_decode(a, desc, out, static_cast<cudaStream_t>(stream));
 }
 
 // ---------------------------------------------------------------------------
@@ -590,31 +953,7 @@ extern "C" rq_status rq_decode_attention_static(const rq_cache_desc* desc, int32
   float* scratch = nullptr;
   if (static_scratch_ptr(&scratch) != RQ_OK) return RQ_ERR_CUDA;
   DecodeArgs a;
-  a.q = q;
-  a.packed = static_cast<const uint8_t*>(packed);
-  a.bits = bits_dev;
-  a.offsets = offsets_dev;
-  a.signs = signs_dev;
-  a.partial = scratch;
-  a.status = status_dev;
-  a.layer = layer;
-  a.B = desc->B;
-  a.H = desc->H_kv;
-  a.Hq = desc->H_q;
-  a.g = desc->H_q / desc->H_kv;
-  a.nblk = desc->S / kTile;
-  a.splits = splits;
-  a.bps = bps;
-  a.kg = desc->k_grouping;
-  a.vg = desc->v_grouping;
-  a.hadamard = desc->hadamard ? 1 : 0;
-  cudaStream_t s = static_cast<cudaStream_t>(stream);
-  const dim3 grid(static_cast<unsigned>(splits), static_cast<unsigned>(desc->H_kv),
-                  static_cast<unsigned>(desc->B));
-  if (desc->dtype == RQ_F16) decode_split_kernel<__half><<<grid, kThreads, 0, s>>>(a);
-  else decode_split_kernel<__nv_bfloat16><<<grid, kThreads, 0, s>>>(a);
-  if (launch_status() != RQ_OK) return RQ_ERR_CUDA;
-  decode_combine_kernel<<<static_cast<unsigned>(desc->B * desc->H_q), kD, 0, s>>>(
-      a.partial, out, signs_dev, status_dev, splits, a.hadamard);
-  return launch_status();
+  fill_args(a, desc, layer, q, packed, bits_dev, offsets_dev, signs_dev, scratch, status_dev,
+            splits, bps);
+  return launch_decode(a, desc, out, static_cast<cudaStream_t>(stream));
 }

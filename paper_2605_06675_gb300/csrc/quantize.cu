@@ -26,10 +26,17 @@ namespace rq {
 namespace {
 
 constexpr int kThreads = 128;
+// CTAs per SM the quantizer's register budget is sized for
+#ifndef RQ_QUANT_MIN_BLOCKS
+#define RQ_QUANT_MIN_BLOCKS 8
+#endif
 constexpr int kX16Stride = kD + 8;      // u16 per staged row (272 B: spreads banks)
 constexpr int kCStride = kD + 4;        // code tile [t][c], bytes per row
 constexpr int kCTStride = kTile + 4;    // transposed code tile [c][t], bytes per row
-constexpr int kCodeBytes = 4608;        // max(32 * 132, 128 * 36)
+constexpr int kCodeBytes = 4624;        // max(32 * 132, 128 * 36 + 4 * 4)
+// row c of the transposed tile starts at ct_row(c): rows 32 apart are skewed
+// by one bank so the four channel groups of a token store without conflicts
+__host__ __device__ constexpr int ct_row(int c) { return c * kCTStride + 4 * (c >> 5); }
 constexpr int kOutWords = 128 * 9;      // codes image (128 b words) + meta image (128 words)
 
 struct TileSmem {
@@ -256,7 +263,7 @@ __device__ __forceinline__ void pack_codes(const uint8_t* codes, uint32_t* out) 
       } else {            // V: channel 16 mt + gid + 8 (k&1), token 16 ks + 2 tig + 8 (k>>1)
         const int c = 16 * (4 * (q & 1) + f) + gid + 8 * (k & 1);
         const int t = 16 * (q >> 1) + 2 * tig + 8 * (k >> 1);
-        p[k] = *reinterpret_cast<const uint16_t*>(codes + c * kCTStride + t);
+        p[k] = *reinterpret_cast<const uint16_t*>(codes + ct_row(c) + t);
       }
     }
     place_fragment<B>(w, f, p);
@@ -290,16 +297,26 @@ __device__ __forceinline__ void put_meta_half(uint32_t* meta, int word, int half
 // its (scale, zero) into the meta image, at the positions of the packed block
 // format; codes are stored as they are produced (no code array stays live).
 __device__ __forceinline__ void quantize_store_group(TileSmem& sm, int kind, int grouping, int b,
-                                                     const float (&v)[kG], const GroupParams& g) {
+                                                     const float (&v)[kG], float mx,
+                                                     const GroupParams& g) {
   const int tau = threadIdx.x;
   uint32_t* meta = sm.out + 128 * b;
   const float2 nz = make_float2(-g.zf, -g.zf);
   const float2 iv = make_float2(g.inv, g.inv);
   const uint32_t L = (1u << b) - 1u;
+  // (v - zero) * inv is monotone in v, so the group max gives the largest
+  // code; when no group of the warp exceeds L the upper clamp is skipped
+  // (the saturating conversion already clamps at 0 and 255)
+  const uint32_t cmax = cvt_rni_sat_u8(__fmul_rn(__fsub_rn(mx, g.zf), g.inv));
+  const bool clamp = __any_sync(0xffffffffu, cmax > L);
   auto code2 = [&](int i, uint32_t& c0, uint32_t& c1) {
     const float2 t = __fmul2_rn(__fadd2_rn(make_float2(v[i], v[i + 1]), nz), iv);
-    c0 = min(cvt_rni_sat_u8(t.x), L);
-    c1 = min(cvt_rni_sat_u8(t.y), L);
+    c0 = cvt_rni_sat_u8(t.x);
+    c1 = cvt_rni_sat_u8(t.y);
+    if (clamp) {
+      c0 = min(c0, L);
+      c1 = min(c1, L);
+    }
   };
   if (grouping == RQ_PER_CHANNEL) {              // group = channel tau, tokens 0..31
     const int ch = tau;
@@ -320,7 +337,7 @@ __device__ __forceinline__ void quantize_store_group(TileSmem& sm, int kind, int
         uint32_t c0, c1, c2, c3;
         code2(t, c0, c1);
         code2(t + 2, c2, c3);
-        *reinterpret_cast<uint32_t*>(&sm.codes[ch * kCTStride + t]) =
+        *reinterpret_cast<uint32_t*>(&sm.codes[ct_row(ch) + t]) =
             c0 | (c1 << 8) | (c2 << 16) | (c3 << 24);
       }
       const int word = 16 * (ch & 7) + 2 * (ch >> 4) + ((ch >> 3) & 1);
@@ -346,8 +363,8 @@ __device__ __forceinline__ void quantize_store_group(TileSmem& sm, int kind, int
       for (int i = 0; i < kG; i += 2) {
         uint32_t c0, c1;
         code2(i, c0, c1);
-        sm.codes[(32 * G + i) * kCTStride + t] = static_cast<uint8_t>(c0);
-        sm.codes[(32 * G + i + 1) * kCTStride + t] = static_cast<uint8_t>(c1);
+        sm.codes[ct_row(32 * G + i) + t] = static_cast<uint8_t>(c0);
+        sm.codes[ct_row(32 * G + i + 1) + t] = static_cast<uint8_t>(c1);
       }
       const int p = t >> 1;
       const int word = 16 * (p & 3) + 4 * (p >> 2) + G;
@@ -357,30 +374,30 @@ __device__ __forceinline__ void quantize_store_group(TileSmem& sm, int kind, int
   }
 }
 
+// Tile position: block j of stream sk = (batch * H + h) * 2 + kind. A CTA
+// walks tiles blockIdx.x, blockIdx.x + gridDim.x, ...; the position is
+// advanced by carrying (no division in the loop).
 struct TileRef {
-  int j, kind, h, batch;
-  long long bh;
+  int j, sk;
 };
 
-__device__ __forceinline__ TileRef decode_tile(const QuantArgs& a, long long tile) {
-  TileRef r;
-  r.j = static_cast<int>(tile % a.nblk);
-  const long long sk = tile / a.nblk;              // (batch * H + h) * 2 + kind
-  r.kind = static_cast<int>(sk & 1);
-  r.bh = sk >> 1;
-  r.h = static_cast<int>(r.bh % a.H);
-  r.batch = static_cast<int>(r.bh / a.H);
-  return r;
+__device__ __forceinline__ void advance(TileRef& r, int dj, int dsk, int nblk) {
+  r.j += dj;
+  r.sk += dsk;
+  if (r.j >= nblk) {
+    r.j -= nblk;
+    r.sk += 1;
+  }
 }
 
 template <typename T>
 __device__ __forceinline__ const T* quant_tile_base(const QuantArgs& a, const TileRef& r) {
-  const T* base = static_cast<const T*>(r.kind ? a.v : a.k);
-  return base + (r.bh * a.S + static_cast<long long>(kTile) * r.j) * kD;
+  const T* base = static_cast<const T*>((r.sk & 1) ? a.v : a.k);
+  return base + (static_cast<long long>(r.sk >> 1) * a.S + static_cast<long long>(kTile) * r.j) * kD;
 }
 
 template <typename T>
-__global__ void __launch_bounds__(kThreads, 8) quantize_pack_kernel(QuantArgs a) {
+__global__ void __launch_bounds__(kThreads, RQ_QUANT_MIN_BLOCKS) quantize_pack_kernel(QuantArgs a) {
   extern __shared__ __align__(16) unsigned char smem_raw[];
   TileSmem& sm = *reinterpret_cast<TileSmem*>(smem_raw);
   float* x32 = reinterpret_cast<float*>(smem_raw + sizeof(TileSmem));
@@ -391,23 +408,27 @@ __global__ void __launch_bounds__(kThreads, 8) quantize_pack_kernel(QuantArgs a)
   __syncthreads();
   const bool had = a.hadamard != 0;
 
-  TileRef r = decode_tile(a, tile);
-  int grouping = r.kind ? a.vg : a.kg;
+  const int nblk = a.nblk;
+  const int dsk = static_cast<int>(stride / nblk), dj = static_cast<int>(stride % nblk);
+  TileRef r{static_cast<int>(tile % nblk), static_cast<int>(tile / nblk)};
+  int grouping = (r.sk & 1) ? a.vg : a.kg;
   bool row_mode = grouping == RQ_PER_TOKEN || had;
   uint4 ld[4];
   load_tile<T>(quant_tile_base<T>(a, r), row_mode, ld);
 
   for (; tile < a.ntiles; tile += stride) {
-    const int b = a.bits[(a.layer * a.H + r.h) * 2 + r.kind];
+    const TileRef cur = r;
+    const int kind = cur.sk & 1;
+    const int bh = cur.sk >> 1;
+    const int h = bh % a.H;
+    const int b = a.bits[(a.layer * a.H + h) * 2 + kind];
     float v[kG];
     group_values<T>(ld, row_mode, grouping, had, sm, x32, v);
     // the next tile's loads fly while this one is quantized and packed
-    const TileRef cur = r;
     const int cur_grouping = grouping;
-    const long long next = tile + stride;
-    if (next < a.ntiles) {
-      r = decode_tile(a, next);
-      grouping = r.kind ? a.vg : a.kg;
+    if (tile + stride < a.ntiles) {
+      advance(r, dj, dsk, nblk);
+      grouping = (r.sk & 1) ? a.vg : a.kg;
       row_mode = grouping == RQ_PER_TOKEN || had;
       load_tile<T>(quant_tile_base<T>(a, r), row_mode, ld);
     }
@@ -421,13 +442,13 @@ __global__ void __launch_bounds__(kThreads, 8) quantize_pack_kernel(QuantArgs a)
     group_minmax(v, mn, mx, finite);
     const GroupParams g = group_params(mn, mx, finite, b);
     if (g.bad) set_status(a.status, RQ_STATUS_NUMERIC);
-    quantize_store_group(sm, cur.kind, cur_grouping, b, v, g);
+    quantize_store_group(sm, kind, cur_grouping, b, v, mx, g);
     __syncthreads();
-    if (cur.kind == 0) pack_dispatch<0>(b, sm.codes, sm.out);
+    if (kind == 0) pack_dispatch<0>(b, sm.codes, sm.out);
     else pack_dispatch<1>(b, sm.codes, sm.out);
     __syncthreads();
-    const uint64_t off =
-        a.offsets[((static_cast<long long>(a.layer) * a.B + cur.batch) * a.H + cur.h) * 2 + cur.kind];
+    // offsets[layer][batch][h][kind] = offsets[layer * B * H * 2 + sk]
+    const uint64_t off = a.offsets[static_cast<long long>(a.layer) * a.B * a.H * 2 + cur.sk];
     uint4* dst = reinterpret_cast<uint4*>(a.packed + off + static_cast<uint64_t>(cur.j) * 512u * (b + 1));
     const uint4* src = reinterpret_cast<const uint4*>(sm.out);
     for (int i = threadIdx.x; i < 32 * (b + 1); i += kThreads) dst[i] = src[i];
