@@ -189,18 +189,21 @@ __device__ __forceinline__ void frag_codes(const uint32_t (&w)[4 * BW], int f, u
     else if (s == 2) X = __funnelshift_r(w[base + 1], w[base + 2], 16);
     else X = w[base + 2] >> 8;
     const uint32_t W = (X & 0xFFFFu) | ((X << 4) & 0xFFFF0000u);
+    // OR the fp16 magic in once; each field is then one single-mask AND
+    // (the magic's bits and the fields' bits do not overlap)
+    const uint32_t Wm = W | kMagic, Zm = (W >> 3) | kMagic;
     const uint32_t mul[3] = {0x3C003C00u, 0x30003000u, 0x24002400u};   // 8^-k
     const uint32_t add[3] = {0xE400E400u, 0xD800D800u, 0xCC00CC00u};   // -1024 8^-k
 #pragma unroll
-    for (int k = 0; k < 3; ++k) c[k] = hfma2u((W & (0x00070007u << (3 * k))) | kMagic, mul[k], add[k]);
-    c[3] = hfma2u(((W >> 3) & 0x01C001C0u) | kMagic, 0x24002400u, 0xCC00CC00u);
+    for (int k = 0; k < 3; ++k) c[k] = hfma2u(Wm & (kMagic | (0x00070007u << (3 * k))), mul[k], add[k]);
+    c[3] = hfma2u(Zm & (kMagic | 0x01C001C0u), 0x24002400u, 0xCC00CC00u);
   } else if constexpr (BW == 4) {
     // one word: low half nibbles a0 a2 a4 a6, high half a1 a3 a5 a7
-    const uint32_t X = w[f], Y = X >> 8;
-    c[0] = hsub2u((X & 0x000F000Fu) | kMagic, kMagic);
-    c[1] = hfma2u((X & 0x00F000F0u) | kMagic, 0x2C002C00u, 0xD400D400u);   // /16 - 64
-    c[2] = hsub2u((Y & 0x000F000Fu) | kMagic, kMagic);
-    c[3] = hfma2u((Y & 0x00F000F0u) | kMagic, 0x2C002C00u, 0xD400D400u);
+    const uint32_t Xm = w[f] | kMagic, Ym = (w[f] >> 8) | kMagic;
+    c[0] = hsub2u(Xm & (kMagic | 0x000F000Fu), kMagic);
+    c[1] = hfma2u(Xm & (kMagic | 0x00F000F0u), 0x2C002C00u, 0xD400D400u);   // /16 - 64
+    c[2] = hsub2u(Ym & (kMagic | 0x000F000Fu), kMagic);
+    c[3] = hfma2u(Ym & (kMagic | 0x00F000F0u), 0x2C002C00u, 0xD400D400u);
   } else if constexpr (BW == 8) {
     // two words: bytes a0 a2 a4 a6 | a1 a3 a5 a7
     const uint32_t X0 = w[2 * f], X1 = w[2 * f + 1];
@@ -246,13 +249,18 @@ __device__ __forceinline__ void qk_block(const uint8_t* img, int lane, const uin
       const uint2 z2 = *reinterpret_cast<const uint2*>(meta + 256 + 4 * (16 * tig + 2 * ks));
       qs2[ks][0] = h2u(__hmul2(u2h(qb[ks][0]), u2h(s2.x)));
       qs2[ks][1] = h2u(__hmul2(u2h(qb[ks][1]), u2h(s2.y)));
-      const uint32_t az[4] = {z2.x, z2.x, z2.y, z2.y};
+      // z repeats in every token row, so rows gid + 8 are left zero and
+      // rows gid (zb[0], zb[1]) serve both
+      const uint32_t az[4] = {z2.x, 0u, z2.y, 0u};
       mma16816(zb, az, qb[ks][0], qb[ks][1]);
     }
 #pragma unroll
-    for (int mt = 0; mt < 2; ++mt)
-#pragma unroll
-      for (int r = 0; r < 4; ++r) s[mt][r] = zb[r];
+    for (int mt = 0; mt < 2; ++mt) {
+      s[mt][0] = zb[0];
+      s[mt][1] = zb[1];
+      s[mt][2] = zb[0];
+      s[mt][3] = zb[1];
+    }
 #pragma unroll
     for (int ks = 0; ks < 8; ++ks)
 #pragma unroll
@@ -299,7 +307,7 @@ __device__ __forceinline__ void qk_block(const uint8_t* img, int lane, const uin
 // down every channel row of the group.
 template <int BW, int VG>
 __device__ __forceinline__ void pv_block(const uint8_t* img, int lane, const uint32_t (&pb)[2][2],
-                                         float (&o)[8][4]) {
+                                         float (&o)[8][4], float (&bz)[2][4]) {
   const int gid = lane >> 2, tig = lane & 3;
   uint32_t w[4 * BW];
   lane_words<BW>(img, lane, w);
@@ -321,20 +329,25 @@ __device__ __forceinline__ void pv_block(const uint8_t* img, int lane, const uin
     }
 #pragma unroll
     for (int ks = 0; ks < 2; ++ks) {
+      // zero-points: sum_t z_tG p_tj, the same for every channel of group G;
+      // rows gid of the A operand carry group G, rows gid + 8 group G + 1
+#pragma unroll
+      for (int gp = 0; gp < 2; ++gp) {
+        const uint32_t az[4] = {mz[4 * (2 * ks) + 2 * gp], mz[4 * (2 * ks) + 2 * gp + 1],
+                                mz[4 * (2 * ks + 1) + 2 * gp], mz[4 * (2 * ks + 1) + 2 * gp + 1]};
+        mma16816(bz[gp], az, pb[ks][0], pb[ks][1]);
+      }
 #pragma unroll
       for (int G = 0; G < 4; ++G) {
         // B fragment rows: tokens 16 ks + 2 tig (+1) and + 8  ->  pair words j = 2 ks, 2 ks + 1
         const uint32_t b0 = h2u(__hmul2(u2h(pb[ks][0]), u2h(ms[4 * (2 * ks) + G])));
         const uint32_t b1 = h2u(__hmul2(u2h(pb[ks][1]), u2h(ms[4 * (2 * ks + 1) + G])));
-        const uint32_t az[4] = {mz[4 * (2 * ks) + G], mz[4 * (2 * ks) + G],
-                                mz[4 * (2 * ks + 1) + G], mz[4 * (2 * ks + 1) + G]};
 #pragma unroll
         for (int h = 0; h < 2; ++h) {
           const int mt = 2 * G + h;
           uint32_t c[4];
           frag_codes<BW>(w, 8 * ks + mt, c);
           mma16816(o[mt], c, b0, b1);
-          mma16816(o[mt], az, pb[ks][0], pb[ks][1]);
         }
       }
     }
@@ -373,9 +386,10 @@ __device__ __forceinline__ void qk_dispatch_g(int kg, const uint8_t* img, int la
 
 template <int BW>
 __device__ __forceinline__ void pv_dispatch_g(int vg, const uint8_t* img, int lane,
-                                              const uint32_t (&pb)[2][2], float (&o)[8][4]) {
-  if (vg == RQ_PER_TOKEN) pv_block<BW, RQ_PER_TOKEN>(img, lane, pb, o);
-  else pv_block<BW, RQ_PER_CHANNEL>(img, lane, pb, o);
+                                              const uint32_t (&pb)[2][2], float (&o)[8][4],
+                                              float (&bz)[2][4]) {
+  if (vg == RQ_PER_TOKEN) pv_block<BW, RQ_PER_TOKEN>(img, lane, pb, o, bz);
+  else pv_block<BW, RQ_PER_CHANNEL>(img, lane, pb, o, bz);
 }
 
 __device__ __forceinline__ void qk_dispatch(int bw, int kg, const uint8_t* img, int lane,
@@ -393,16 +407,17 @@ __device__ __forceinline__ void qk_dispatch(int bw, int kg, const uint8_t* img, 
 }
 
 __device__ __forceinline__ void pv_dispatch(int bw, int vg, const uint8_t* img, int lane,
-                                            const uint32_t (&pb)[2][2], float (&o)[8][4]) {
+                                            const uint32_t (&pb)[2][2], float (&o)[8][4],
+                                            float (&bz)[2][4]) {
   switch (bw) {
-    case 1: pv_dispatch_g<1>(vg, img, lane, pb, o); break;
-    case 2: pv_dispatch_g<2>(vg, img, lane, pb, o); break;
-    case 3: pv_dispatch_g<3>(vg, img, lane, pb, o); break;
-    case 4: pv_dispatch_g<4>(vg, img, lane, pb, o); break;
-    case 5: pv_dispatch_g<5>(vg, img, lane, pb, o); break;
-    case 6: pv_dispatch_g<6>(vg, img, lane, pb, o); break;
-    case 7: pv_dispatch_g<7>(vg, img, lane, pb, o); break;
-    default: pv_dispatch_g<8>(vg, img, lane, pb, o); break;
+    case 1: pv_dispatch_g<1>(vg, img, lane, pb, o, bz); break;
+    case 2: pv_dispatch_g<2>(vg, img, lane, pb, o, bz); break;
+    case 3: pv_dispatch_g<3>(vg, img, lane, pb, o, bz); break;
+    case 4: pv_dispatch_g<4>(vg, img, lane, pb, o, bz); break;
+    case 5: pv_dispatch_g<5>(vg, img, lane, pb, o, bz); break;
+    case 6: pv_dispatch_g<6>(vg, img, lane, pb, o, bz); break;
+    case 7: pv_dispatch_g<7>(vg, img, lane, pb, o, bz); break;
+    default: pv_dispatch_g<8>(vg, img, lane, pb, o, bz); break;
   }
 }
 
@@ -449,6 +464,7 @@ struct WarpStream {
 // online-softmax state of one warp: o^T accumulators and per-column max/sum
 struct SoftmaxAcc {
   float o[8][4];
+  float bz[2][4];   // per-token V zero-point sums: rows gid -> groups 0/2, rows gid+8 -> 1/3
   float m0, m1, l0, l1;
 };
 
@@ -477,6 +493,13 @@ __device__ __forceinline__ void softmax_block(float (&s)[2][4], SoftmaxAcc& acc,
       acc.o[mt][1] *= al1;
       acc.o[mt][2] *= al0;
       acc.o[mt][3] *= al1;
+    }
+#pragma unroll
+    for (int gp = 0; gp < 2; ++gp) {
+      acc.bz[gp][0] *= al0;
+      acc.bz[gp][1] *= al1;
+      acc.bz[gp][2] *= al0;
+      acc.bz[gp][3] *= al1;
     }
   }
   float p[2][4];
@@ -553,7 +576,7 @@ __device__ __forceinline__ void blocks_static(const WarpStream& ws, const uint32
     iss = iss + 1 == NS ? 0 : iss + 1;
     cp_async_wait<NS - 1>();
     __syncwarp();
-    pv_block<BV, VG>(ws.ring_ptr + use * R::kSlot, ws.lane, pb, acc.o);
+    pv_block<BV, VG>(ws.ring_ptr + use * R::kSlot, ws.lane, pb, acc.o, acc.bz);
     __syncwarp();
     use = use + 1 == NS ? 0 : use + 1;
   }
@@ -594,7 +617,7 @@ __device__ __forceinline__ void blocks_dyn(const WarpStream& ws, const DynRing& 
     iss = iss + 1 == r.ns ? 0 : iss + 1;
     cp_async_wait_dyn(r.ns - 1);
     __syncwarp();
-    pv_dispatch(r.bV, r.vg, ws.ring_ptr + use * r.slot, ws.lane, pb, acc.o);
+    pv_dispatch(r.bV, r.vg, ws.ring_ptr + use * r.slot, ws.lane, pb, acc.o, acc.bz);
     __syncwarp();
     use = use + 1 == r.ns ? 0 : use + 1;
   }
@@ -692,6 +715,10 @@ __global__ void __launch_bounds__(kThreads) decode_split_kernel(DecodeArgs a) {
   for (int mt = 0; mt < 8; ++mt)
 #pragma unroll
     for (int r = 0; r < 4; ++r) acc.o[mt][r] = 0.0f;
+#pragma unroll
+  for (int gp = 0; gp < 2; ++gp)
+#pragma unroll
+    for (int r = 0; r < 4; ++r) acc.bz[gp][r] = 0.0f;
   acc.m0 = acc.m1 = -INFINITY;
   acc.l0 = acc.l1 = 0.0f;
 
@@ -700,6 +727,19 @@ __global__ void __launch_bounds__(kThreads) decode_split_kernel(DecodeArgs a) {
     RQ_FAST_CASES(RQ_BLK)
 #undef RQ_BLK
     default: blocks_dyn(ws, dr, qb, acc); break;
+  }
+  if (a.vg == RQ_PER_TOKEN) {
+    // group G's zero-point sum: rows gid of bz[G/2] for even G, rows gid+8 for odd G
+#pragma unroll
+    for (int mt = 0; mt < 8; ++mt) {
+      const int G = mt >> 1;
+      const float z0 = (G & 1) ? acc.bz[G >> 1][2] : acc.bz[G >> 1][0];
+      const float z1 = (G & 1) ? acc.bz[G >> 1][3] : acc.bz[G >> 1][1];
+      acc.o[mt][0] += z0;
+      acc.o[mt][1] += z1;
+      acc.o[mt][2] += z0;
+      acc.o[mt][3] += z1;
+    }
   }
   float m0 = acc.m0, m1 = acc.m1, l0 = acc.l0, l1 = acc.l1;
 #pragma unroll
