@@ -60,6 +60,27 @@ def _parse():
 
 
 # --------------------------------------------------------------------------
+# replica timing across ranks (every rank runs the whole path on its own GPU;
+# the job's time is the slowest rank's and its value counts every rank's work)
+# --------------------------------------------------------------------------
+
+def max_over_ranks(x: float, world: int, device) -> float:
+    """Maximum of ``x`` over all ranks of the default process group."""
+    if world <= 1:
+        return x
+    import torch
+    import torch.distributed as dist
+    t = torch.tensor([x], dtype=torch.float64, device=device)
+    dist.all_reduce(t, op=dist.ReduceOp.MAX)
+    return float(t.item())
+
+
+def job_gbs(world: int, bytes_per_rank_step: float, ms_per_step: float) -> float:
+    """Whole-job throughput: every rank's bytes over the slowest rank's time."""
+    return world * bytes_per_rank_step / (ms_per_step * 1e-3) / 1e9
+
+
+# --------------------------------------------------------------------------
 # byte accounting (algorithmic bytes; partials and workspaces excluded)
 # --------------------------------------------------------------------------
 
@@ -251,11 +272,8 @@ def run_ours(args, wl, rank, world, local_rank):
     end.record(stream)
     torch.cuda.synchronize()
     clk = clocks.stop()
-    total_ms = start.elapsed_time(end)
+    total_ms = max_over_ranks(start.elapsed_time(end), world, dev)
     if world > 1:
-        t = torch.tensor([total_ms], dtype=torch.float64, device=dev)
-        dist.all_reduce(t, op=dist.ReduceOp.MAX)
-        total_ms = float(t.item())
         dist.barrier()
 
     calib_ms = statistics.mean(e[0].elapsed_time(e[1]) for e in evs)
@@ -268,7 +286,7 @@ def run_ours(args, wl, rank, world, local_rank):
     cb = calib_bytes(wl, n, T)
     step_bytes = qb + db + cb
     peak, peak_kind = _peaks()
-    value = world * step_bytes / (ms_step * 1e-3) / 1e9
+    value = job_gbs(world, step_bytes, ms_step)
     q_gbs = qb / (quant_ms * 1e-3) / 1e9
     d_gbs = db / (dec_ms * 1e-3) / 1e9
     tok_s = wl.B / (dec_ms * 1e-3)
@@ -387,16 +405,12 @@ def run_e2e(args, wl, path, K, V, Q, OUT, X, w, cap, dev, stream, step_bytes, wo
     for _ in range(steps):
         e2e_step()
     torch.cuda.synchronize()
-    el = time.perf_counter() - t0
-    if world > 1:
-        t = torch.tensor([el], dtype=torch.float64, device=dev)
-        dist.all_reduce(t, op=dist.ReduceOp.MAX)
-        el = float(t.item())
+    el = max_over_ranks(time.perf_counter() - t0, world, dev)
     ms = el / steps * 1e3
     h2d = (hX.numel() * hX.element_size() + sum(t.numel() * t.element_size() for t in hQ)
            + wl.L * layer_bytes)
     d2h = sum(t.numel() * t.element_size() for t in hOut) + path._mse.numel() * 8
-    return {"value": round(world * step_bytes / (ms * 1e-3) / 1e9, 2), "unit": "GB/s",
+    return {"value": round(job_gbs(world, step_bytes, ms), 2), "unit": "GB/s",
             "ms_per_step": round(ms, 3), "h2d_bytes_per_step": int(h2d),
             "d2h_bytes_per_step": int(d2h), "steps": steps,
             "host_staging_layers": n_stage,
