@@ -15,37 +15,44 @@ head_dim 128, bit-width b = bits[layer][head][kind]. It is S/32 blocks, block j
 covering tokens [32j, 32j+32). A block is 512*(b+1) bytes: the codes image
 (128*b uint32 words) followed by the meta image (128 uint32 words).
 
-Codes image: the 32x128 code tile X[t][c] (t = token in block, c = channel) is
-split among 32 "lanes"; lane = 4*gid + tig. Each lane owns 16 "fragments" of 8
-codes, slots e = 0..7:
+Codes image: the 32x128 code tile X[t][c] (t = token in block, c = channel)
+is split among 32 lanes, lane = 4*gid + tig (gid 0..7, tig 0..3). A lane owns
+4 units u = 0..3; a unit is 16 registers psi = 4*x + y (class x 0..3, member
+y 0..3) and a register holds two codes, half h = 0 and h = 1:
 
-  kind K:  gid = t % 8,  tig = (c % 8) // 2,  frag = 2*(c // 16) + (t // 16),
-           e = (c & 1) | ((t >> 3) & 1) << 1 | ((c >> 3) & 1) << 2
-  kind V:  gid = c % 8,  tig = (t % 8) // 2,  frag = 8*(t // 16) + (c // 16),
-           e = (t & 1) | ((c >> 3) & 1) << 1 | ((t >> 3) & 1) << 2
+  kind K, per-channel groups:  t = 8*y + gid,        c = 32*u + 8*tig + 2*x + h
+  kind K, per-token groups:    t = 8*x + gid,        c = 32*u + 8*tig + 2*y + h
+  kind V (either grouping):    t = 8*y + 2*tig + h,  c = 32*u + 4*gid + x
 
-  slot position in the fragment: pos = e // 2 for even e, 4 + e // 2 for odd e
-  (codes a0 a2 a4 a6 first, then a1 a3 a5 a7).
+Each lane has a stream of 4*b words; unit u owns lane words b*u .. b*u + b-1
+(unit word w = 0..b-1). With n = 16 // b code slots per 16-bit half, slot
+(w, k) puts the half-h code at bits [16*h + b*k, +b) of unit word w. When
+b*n < 16 the bits [16*h + b*n, 16*h + 16) of the unit's words are spare; the
+half-h spare stream is those bits of unit words 0, 1, ..., b-1 in order, LSB
+first, and leftover register l puts its half-h code at spare-stream bits
+[b*l, b*l + b). Register psi = 4x + y goes to:
 
-  Each lane has a bit stream of 128*b bits: the code sits, LSB first, at bits
-  [8*b*frag + b*pos, +b). Lane-stream word w (bits [32w, 32w+32)) is stored at
-  block word 128*(w // 4) + 4*lane + (w % 4); i.e. 16-byte piece i = w // 4 of
-  lane L lives at byte 16*(32 i + L).
+  b in {1, 2, 4, 8}:  slot s = x + 4*y, i.e. (w, k) = (s // n, s % n)
+  b = 3:  x=0: (0,0) (1,0) (2,0) leftover 0;  x=1: (0,1) (1,1) (2,1) (1,4)
+          x=2: (0,2) (1,2) (2,2) (2,4);       x=3: (0,3) (1,3) (2,3) (0,4)
+  b = 5:  x=0: (0,0) (1,0) (2,0) (3,0);       x=1: (0,1) (1,1) (2,1) (3,1)
+          x=2: (4,0) (0,2) (1,2) leftover 0;  x=3: (4,1) (2,2) (3,2) (4,2)
+  b = 6:  psi < 12: (psi // 2, psi % 2); psi >= 12: leftover psi - 12
+  b = 7:  psi < 14: (psi // 2, psi % 2); psi >= 14: leftover psi - 14
+
+  (members listed y = 0, 1, 2, 3). Lane-stream word w is stored at block word
+  128*(w // 4) + 4*lane + (w % 4); i.e. 16-byte piece i = w // 4 of lane L
+  lives at byte 16*(32 i + L).
 
 Meta image (128 words, one fp16 pair each, low half first):
 
-  "pair planes" -- K per-channel and V per-token. Words 0..63 hold scale pairs,
-  words 64..127 the zero pairs at the same index. A word holds the values of
-  two groups g0 (low half) and g1 (high half):
-    K per-channel (group = channel c):  pair (c, c+1), c even,
-        index = 16*((c % 8)//2) + 2*(c // 16) + ((c // 8) % 2), half = c % 2
-    V per-token (group = (t, G), G = c // 32): pair (t, t+1), t even,
-        p = t // 2,  index = 16*(p % 4) + 4*(p // 4) + G,  half = t % 2
-
-  "scale-zero words" -- K per-token and V per-channel. Word = (scale, zero)
-  of one group:
-    K per-token (group = (t, G)):   index = 16*(t % 8) + 4*(t // 8) + G
-    V per-channel (group = c):      index = 16*(c % 8) + 2*(c // 16) + (c // 8) % 2
+  K per-channel (group = channel c): word c // 2 holds the scales of
+      channels (c, c+1) (c even), word 64 + c // 2 their zeros.
+  K per-token (group = (t, G), G = c // 32): word 16*(t % 8) + 4*G + t // 8
+      holds (scale, zero).
+  V per-token (group = (t, G)): word 4*(t // 2) + G holds the scales of
+      tokens (t, t+1) (t even), word 64 + 4*(t // 2) + G their zeros.
+  V per-channel (group = channel c): word c holds (scale, zero).
 
 Stream order in a packed buffer (``stream_offsets``): layer, batch, kv-head,
 kind (K=0, V=1); each stream starts where the previous one ends.
@@ -66,43 +73,100 @@ def block_bytes(b: int) -> int:
     return 512 * (b + 1)
 
 
-def code_positions(kind: int, b: int):
-    """For every (t, c) of a block tile: lane and lane-stream bit position.
+# Register psi = 4x + y of a unit -> ("slot", unit word, slot) or ("left", l).
+def register_location(b: int, x: int, y: int):
+    n = 16 // b
+    if b in (1, 2, 4, 8):
+        s = x + 4 * y
+        return ("slot", s // n, s % n)
+    if b == 3:
+        table = {0: [(0, 0), (1, 0), (2, 0), None], 1: [(0, 1), (1, 1), (2, 1), (1, 4)],
+                 2: [(0, 2), (1, 2), (2, 2), (2, 4)], 3: [(0, 3), (1, 3), (2, 3), (0, 4)]}
+        loc = table[x][y]
+        return ("left", 0) if loc is None else ("slot",) + loc
+    if b == 5:
+        table = {0: [(0, 0), (1, 0), (2, 0), (3, 0)], 1: [(0, 1), (1, 1), (2, 1), (3, 1)],
+                 2: [(4, 0), (0, 2), (1, 2), None], 3: [(4, 1), (2, 2), (3, 2), (4, 2)]}
+        loc = table[x][y]
+        return ("left", 0) if loc is None else ("slot",) + loc
+    psi = 4 * x + y
+    main = 12 if b == 6 else 14
+    if psi < main:
+        return ("slot", psi // 2, psi % 2)
+    return ("left", psi - main)
 
-    Returns (lane[32,128], bitpos[32,128]) int64 arrays.
-    """
-    t = np.arange(BLOCK_TOKENS)[:, None] * np.ones((1, HEAD_DIM), dtype=np.int64)
-    c = np.ones((BLOCK_TOKENS, 1), dtype=np.int64) * np.arange(HEAD_DIM)[None, :]
+
+def register_element(kind: int, grouping: int, gid: int, tig: int, u: int, x: int, y: int,
+                     h: int):
+    """(token, channel) of half h of register (x, y) of unit u of lane (gid, tig)."""
+    if kind == KIND_K and grouping == PER_CHANNEL:
+        return 8 * y + gid, 32 * u + 8 * tig + 2 * x + h
     if kind == KIND_K:
-        gid = t % 8
-        tig = (c % 8) // 2
-        frag = 2 * (c // 16) + (t // 16)
-        e = (c & 1) | (((t >> 3) & 1) << 1) | (((c >> 3) & 1) << 2)
-    else:
-        gid = c % 8
-        tig = (t % 8) // 2
-        frag = 8 * (t // 16) + (c // 16)
-        e = (t & 1) | (((c >> 3) & 1) << 1) | (((t >> 3) & 1) << 2)
-    lane = 4 * gid + tig
-    pos = np.where(e % 2 == 0, e // 2, 4 + e // 2)
-    bitpos = 8 * b * frag + b * pos
-    return lane.astype(np.int64), bitpos.astype(np.int64)
+        return 8 * x + gid, 32 * u + 8 * tig + 2 * y + h
+    return 8 * y + 2 * tig + h, 32 * u + 4 * gid + x
+
+
+def code_bit_positions(b: int, u: int, x: int, y: int, h: int):
+    """Lane-stream bit positions of code bits 0..b-1 of half h of register (x, y)."""
+    n = 16 // b
+    spare = 16 - b * n
+    loc = register_location(b, x, y)
+    out = []
+    for k in range(b):
+        if loc[0] == "slot":
+            w, slot = loc[1], loc[2]
+            bit = 16 * h + b * slot + k
+        else:
+            i = b * loc[1] + k                     # spare-stream bit index
+            w = i // spare
+            bit = 16 * h + b * n + i % spare
+        out.append(32 * (b * u + w) + bit)
+    return out
+
+
+_POS_CACHE = {}
+
+
+def code_positions(kind: int, grouping: int, b: int):
+    """For every (t, c) of a block tile: its lane and the lane-stream bit
+    positions of its code bits 0..b-1.
+
+    Returns (lane[32,128], bitpos[32,128,b]) int64 arrays.
+    """
+    key = (kind, grouping, b)
+    if key in _POS_CACHE:
+        return _POS_CACHE[key]
+    lane = np.full((BLOCK_TOKENS, HEAD_DIM), -1, dtype=np.int64)
+    bitpos = np.full((BLOCK_TOKENS, HEAD_DIM, b), -1, dtype=np.int64)
+    for gid in range(8):
+        for tig in range(4):
+            for u in range(4):
+                for x in range(4):
+                    for y in range(4):
+                        for h in range(2):
+                            t, c = register_element(kind, grouping, gid, tig, u, x, y, h)
+                            assert lane[t, c] == -1
+                            lane[t, c] = 4 * gid + tig
+                            bitpos[t, c] = code_bit_positions(b, u, x, y, h)
+    assert (lane >= 0).all()
+    _POS_CACHE[key] = (lane, bitpos)
+    return lane, bitpos
 
 
 def lane_word_to_block_word(lane: np.ndarray, w: np.ndarray) -> np.ndarray:
     return 128 * (w // 4) + 4 * lane + (w % 4)
 
 
-def pack_codes_blocks(tiles: np.ndarray, kind: int, b: int) -> np.ndarray:
+def pack_codes_blocks(tiles: np.ndarray, kind: int, grouping: int, b: int) -> np.ndarray:
     """Pack code tiles [nb, 32, 128] into [nb, 128*b] uint32 words, bit by bit."""
     tiles = np.asarray(tiles).astype(np.int64)
     nb = tiles.shape[0]
     assert tiles.shape[1:] == (BLOCK_TOKENS, HEAD_DIM)
     assert nb == 0 or (tiles.min() >= 0 and tiles.max() < (1 << b))
-    lane, bitpos = code_positions(kind, b)
+    lane, bitpos = code_positions(kind, grouping, b)
     bits = np.zeros((nb, 32, 128 * b), dtype=np.uint8)      # lane bit streams
     for k in range(b):
-        bits[:, lane, bitpos + k] = ((tiles >> k) & 1).astype(np.uint8)
+        bits[:, lane, bitpos[:, :, k]] = ((tiles >> k) & 1).astype(np.uint8)
     lane_words = np.zeros((nb, 32, 4 * b), dtype=np.uint64)
     for j in range(32):
         lane_words |= bits[:, :, j::32].astype(np.uint64) << np.uint64(j)
@@ -113,7 +177,7 @@ def pack_codes_blocks(tiles: np.ndarray, kind: int, b: int) -> np.ndarray:
     return out
 
 
-def unpack_codes_blocks(words: np.ndarray, kind: int, b: int) -> np.ndarray:
+def unpack_codes_blocks(words: np.ndarray, kind: int, grouping: int, b: int) -> np.ndarray:
     """Inverse of ``pack_codes_blocks``: [nb, 128*b] words -> [nb, 32, 128] codes."""
     words = np.asarray(words, dtype=np.uint32)
     nb = words.shape[0]
@@ -124,21 +188,21 @@ def unpack_codes_blocks(words: np.ndarray, kind: int, b: int) -> np.ndarray:
     bits = np.zeros((nb, 32, 128 * b), dtype=np.uint8)
     for j in range(32):
         bits[:, :, j::32] = ((lane_words >> np.uint64(j)) & np.uint64(1)).astype(np.uint8)
-    lane, bitpos = code_positions(kind, b)
+    lane, bitpos = code_positions(kind, grouping, b)
     tile = np.zeros((nb, BLOCK_TOKENS, HEAD_DIM), dtype=np.int64)
     for k in range(b):
-        tile |= bits[:, lane, bitpos + k].astype(np.int64) << k
+        tile |= bits[:, lane, bitpos[:, :, k]].astype(np.int64) << k
     return tile.astype(np.uint8)
 
 
-def pack_codes_block(tile: np.ndarray, kind: int, b: int) -> np.ndarray:
+def pack_codes_block(tile: np.ndarray, kind: int, grouping: int, b: int) -> np.ndarray:
     """Pack a 32x128 code tile into 128*b uint32 words (bit by bit)."""
-    return pack_codes_blocks(np.asarray(tile)[None], kind, b)[0]
+    return pack_codes_blocks(np.asarray(tile)[None], kind, grouping, b)[0]
 
 
-def unpack_codes_block(words: np.ndarray, kind: int, b: int) -> np.ndarray:
+def unpack_codes_block(words: np.ndarray, kind: int, grouping: int, b: int) -> np.ndarray:
     """Inverse of ``pack_codes_block``."""
-    return unpack_codes_blocks(np.asarray(words)[None], kind, b)[0]
+    return unpack_codes_blocks(np.asarray(words)[None], kind, grouping, b)[0]
 
 
 def meta_layout(kind: int, grouping: int) -> str:
@@ -168,18 +232,15 @@ def meta_positions(kind: int, grouping: int):
     """
     if kind == KIND_K and grouping == PER_CHANNEL:
         c, _ = _group_indices(kind, grouping)
-        word = 16 * ((c % 8) // 2) + 2 * (c // 16) + ((c // 8) % 2)
-        return word, c % 2
+        return c // 2, c % 2
     if kind == KIND_V and grouping == PER_TOKEN:
         t, G = _group_indices(kind, grouping)
-        p = t // 2
-        word = 16 * (p % 4) + 4 * (p // 4) + G
-        return word, t % 2
+        return 4 * (t // 2) + G, t % 2
     if kind == KIND_K and grouping == PER_TOKEN:
         t, G = _group_indices(kind, grouping)
-        return 16 * (t % 8) + 4 * (t // 8) + G, None
+        return 16 * (t % 8) + 4 * G + t // 8, None
     c, _ = _group_indices(kind, grouping)
-    return 16 * (c % 8) + 2 * (c // 16) + (c // 8) % 2, None
+    return c, None
 
 
 def pack_meta_blocks(scale: np.ndarray, zero: np.ndarray, kind: int, grouping: int) -> np.ndarray:
@@ -237,7 +298,7 @@ def pack_stream(codes: np.ndarray, scale: np.ndarray, zero: np.ndarray, kind: in
     out = np.zeros((nblk, 128 * (b + 1)), dtype=np.uint32)
     for j0 in range(0, nblk, chunk):
         j1 = min(nblk, j0 + chunk)
-        out[j0:j1, :128 * b] = pack_codes_blocks(tiles[j0:j1], kind, b)
+        out[j0:j1, :128 * b] = pack_codes_blocks(tiles[j0:j1], kind, grouping, b)
         out[j0:j1, 128 * b:] = pack_meta_blocks(sc[j0:j1], ze[j0:j1], kind, grouping)
     return out.reshape(-1)
 
@@ -249,7 +310,7 @@ def unpack_stream(words: np.ndarray, S: int, kind: int, grouping: int, b: int):
     words = np.asarray(words, dtype=np.uint32)
     assert words.shape == (nblk * per,)
     w = words.reshape(nblk, per)
-    codes = unpack_codes_blocks(w[:, :128 * b], kind, b).reshape(S, HEAD_DIM)
+    codes = unpack_codes_blocks(w[:, :128 * b], kind, grouping, b).reshape(S, HEAD_DIM)
     s, z = unpack_meta_blocks(w[:, 128 * b:], kind, grouping)
     if grouping == PER_TOKEN:
         return codes, s.reshape(S, 4), z.reshape(S, 4)

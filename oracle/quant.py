@@ -23,7 +23,10 @@ reading used here (every step in the stated precision, in this order) is:
     sf = fp32(scale), zf = fp32(zero)
     if sf == 0: every code is 0
     else:  inv = fp32_rn(1 / sf)
-           c_j = clamp(rint_half_even(fp32_rn(fp32_rn(v_j - zf) * inv)), 0, L)
+           t_j = fp32_rn(v_j - zf)
+           c_j = clamp(rint_half_even(t_j * inv), 0, L)   (the product t_j * inv
+                 taken exactly: one rounding, to the integer, from the
+                 difference to the code)
     dequantized value  x_hat_j = fp32_rn(fp32_rn(fp32(c_j) * sf) + zf)
 
   A group holding a non-finite value, or whose fp16 scale or zero overflows,
@@ -94,9 +97,10 @@ def quantize_groups(v: np.ndarray, b: int):
         ok = (~bad) & (sf != np.float32(0.0))
         inv = (np.float32(1.0) / np.where(ok, sf, np.float32(1.0))).astype(np.float32)
         d = (vv - zf[..., None]).astype(np.float32)
-        t = (d * inv[..., None]).astype(np.float32)
-        c = np.clip(np.rint(t), np.float32(0.0), L)
-        codes = np.where(ok[..., None], c, np.float32(0.0)).astype(np.uint8)
+        # the product of two fp32 values is exact in fp64 (48 <= 53 bits)
+        t = d.astype(np.float64) * inv[..., None].astype(np.float64)
+        c = np.clip(np.rint(t), 0.0, float(L))
+        codes = np.where(ok[..., None], c, 0.0).astype(np.uint8)
     scale = np.where(bad, np.float16(0.0), scale).astype(np.float16)
     zero = np.where(bad, np.float16(0.0), zero).astype(np.float16)
     return codes, scale, zero, bad

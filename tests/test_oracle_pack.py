@@ -18,62 +18,109 @@ from oracle.quant import PER_CHANNEL, PER_TOKEN
 GOLDEN = os.path.join(os.path.dirname(__file__), "golden")
 
 
-@pytest.mark.parametrize("kind", [pack.KIND_K, pack.KIND_V])
+LAYOUTS = [(pack.KIND_K, PER_CHANNEL), (pack.KIND_K, PER_TOKEN),
+           (pack.KIND_V, PER_TOKEN), (pack.KIND_V, PER_CHANNEL)]
+
+
+@pytest.mark.parametrize("kind,grouping", LAYOUTS)
 @pytest.mark.parametrize("b", range(1, 9))
-def test_code_positions_tile_each_lane(kind, b):
-    lane, bitpos = pack.code_positions(kind, b)
+def test_code_positions_tile_each_lane(kind, grouping, b):
+    lane, bitpos = pack.code_positions(kind, grouping, b)
     used = np.zeros((32, 128 * b), dtype=np.int64)
     for k in range(b):
-        np.add.at(used, (lane, bitpos + k), 1)
+        np.add.at(used, (lane, bitpos[:, :, k]), 1)
     assert (used == 1).all()          # every bit of every lane used exactly once
 
 
-@pytest.mark.parametrize("kind", [pack.KIND_K, pack.KIND_V])
+@pytest.mark.parametrize("kind,grouping", LAYOUTS)
 @pytest.mark.parametrize("b", range(1, 9))
-def test_codes_round_trip(kind, b):
-    rng = np.random.default_rng(b * 7 + kind)
+def test_codes_round_trip(kind, grouping, b):
+    rng = np.random.default_rng(b * 7 + kind + 3 * grouping)
     tile = rng.integers(0, 1 << b, size=(32, 128))
-    words = pack.pack_codes_block(tile, kind, b)
+    words = pack.pack_codes_block(tile, kind, grouping, b)
     assert words.shape == (128 * b,)
-    assert np.array_equal(pack.unpack_codes_block(words, kind, b), tile)
+    assert np.array_equal(pack.unpack_codes_block(words, kind, grouping, b), tile)
 
 
-def test_hand_words_b8_K():
-    # tile X[t][c] = (3t + 5c) mod 256, kind K, b = 8.
-    # Lane 0 (gid 0, tig 0), fragment 0 (c < 16, t < 16) holds t in {0, 8},
-    # c in {0, 1, 8, 9}; slots: pos0 (0,0) pos1 (8,0) pos2 (0,8) pos3 (8,8)
-    # pos4 (0,1) pos5 (8,1) pos6 (0,9) pos7 (8,9); one byte each.
-    # lane word 0 = [0, 24, 40, 64] -> 0x40281800 at block word 0
-    # lane word 1 = [5, 29, 45, 69] -> 0x452D1D05 at block word 1
-    # Lane 5 (gid 1, tig 1), word 0: (1,2) (9,2) (1,10) (9,10) = 13 37 53 77
-    #   -> 0x4D35250D at block word 4*5 = 20
-    # Lane 0, word 4 = fragment 2 (16 <= c < 32) low half:
-    #   (0,16) (8,16) (0,24) (8,24) = 80 104 120 144 -> 0x90786850 at word 128
+def test_hand_words_b8_K_per_channel():
+    # tile X[t][c] = (3t + 5c) mod 256, K per-channel, b = 8 (2 slots per half).
+    # Lane 0 (gid 0, tig 0), unit 0, register (x, y): t = 8y, c = 2x + h;
+    # slot s = x + 4y -> unit word s // 2, slot s % 2 (bits 8k, 16 + 8k).
+    # unit word 0: (x0,y0) c 0,1 -> 0, 5 at slot 0; (x1,y0) c 2,3 -> 10, 15
+    #   at slot 1 -> 0x0F050A00 at block word 0
+    # unit word 1: (x2,y0) c 4,5 -> 20, 25; (x3,y0) c 6,7 -> 30, 35 -> 0x23191E14
+    # unit word 2: (x0,y1) t 8 c 0,1 -> 24, 29; (x1,y1) c 2,3 -> 34, 39 -> 0x271D2218
+    # Lane 5 (gid 1, tig 1), unit word 0: t 1, c 8,9 -> 43, 48; c 10,11 -> 53, 58
+    #   -> 0x3A30352B at block word 4*5 = 20
+    # Lane 0, unit 1 = lane word 8 -> block word 128*2 = 256: t 0, c 32,33 ->
+    #   160, 165; c 34,35 -> 170, 175 -> 0xAFA5AAA0
     t = np.arange(32)[:, None]
     c = np.arange(128)[None, :]
     tile = (3 * t + 5 * c) % 256
-    w = pack.pack_codes_block(tile, pack.KIND_K, 8)
-    assert w[0] == 0x40281800
-    assert w[1] == 0x452D1D05
-    assert w[20] == 0x4D35250D
-    assert w[128] == 0x90786850
+    w = pack.pack_codes_block(tile, pack.KIND_K, PER_CHANNEL, 8)
+    assert w[0] == 0x0F050A00
+    assert w[1] == 0x23191E14
+    assert w[2] == 0x271D2218
+    assert w[20] == 0x3A30352B
+    assert w[256] == 0xAFA5AAA0
 
 
 def test_hand_words_b2_V():
-    # tile X[t][c] = (t + c // 8) mod 4, kind V, b = 2.
-    # Lane 0 (gid 0, tig 0): channels c % 8 == 0, tokens t % 8 in {0, 1}.
-    # Fragment 0 (t < 16, c < 16): pos0 (0,0)=0 pos1 (0,8)=1 pos2 (8,0)=0
-    #   pos3 (8,8)=1 pos4 (1,0)=1 pos5 (1,8)=2 pos6 (9,0)=1 pos7 (9,8)=2
-    #   -> 2-bit fields -> 0x9944
-    # Fragment 1 (16 <= c < 32): pos0 (0,16)=2 pos1 (0,24)=3 pos2 (8,16)=2
-    #   pos3 (8,24)=3 pos4 (1,16)=3 pos5 (1,24)=0 pos6 (9,16)=3 pos7 (9,24)=0
-    #   -> 0x33EE
-    # lane word 0 = 0x9944 | 0x33EE << 16 = 0x33EE9944 at block word 0
+    # tile X[t][c] = (t + t // 8 + c) mod 4, V (per-token), b = 2.
+    # Lane 0 (gid 0, tig 0), unit 0, register (x, y): t = 8y + h, c = x;
+    # slot s = x + 4y -> unit word y // 2, slot x + 4 (y % 2) at bits 2k, 16 + 2k.
+    # unit word 0: half 0: y0 codes x = 0,1,2,3; y1 codes (1 + x) % 4 = 1,2,3,0
+    #   -> 0x39E4; half 1: y0 (1 + x) % 4, y1 (2 + x) % 4 -> 0x4E39
+    #   -> 0x4E3939E4 at block word 0
+    # unit word 1: half 0: y2 (2 + x) % 4, y3 (3 + x) % 4 -> 0x934E;
+    #   half 1: y2 (3 + x) % 4, y3 x % 4 -> 0xE493 -> 0xE493934E at block word 1
     t = np.arange(32)[:, None]
     c = np.arange(128)[None, :]
-    tile = (t + c // 8) % 4
-    w = pack.pack_codes_block(tile, pack.KIND_V, 2)
-    assert w[0] == 0x33EE9944
+    tile = (t + t // 8 + c) % 4
+    w = pack.pack_codes_block(tile, pack.KIND_V, PER_TOKEN, 2)
+    assert w[0] == 0x4E3939E4
+    assert w[1] == 0xE493934E
+
+
+def test_hand_words_b3_K_per_token_with_leftover():
+    # tile X[t][c] = (t // 8 + 3c) mod 8, K per-token, b = 3 (5 slots of 3
+    # bits per half, bit 15 spare). Lane 0, unit 0, register (x, y): t = 8x,
+    # c = 2y + h, code (x + 6y + 3h) % 8. Leftover 0 = (x0, y3): codes 2 (h 0)
+    # and 5 (h 1); its bit k sits at bit 15 / 31 of unit word k.
+    # unit word 0 slots (x0 y0)(x1 y0)(x2 y0)(x3 y0)(x3 y3):
+    #   half 0: 0 1 2 3 5 -> 0x5688 (spare 0); half 1: 3 4 5 6 0 -> 0x0D63 | 0x8000
+    #   -> 0x8D635688
+    # unit word 1 slots (x0 y1)(x1 y1)(x2 y1)(x3 y1)(x1 y3):
+    #   half 0: 6 7 0 1 3 -> 0x323E | 0x8000; half 1: 1 2 3 4 6 -> 0x68D1 (spare 0)
+    #   -> 0x68D1B23E
+    # unit word 2 slots (x0 y2)(x1 y2)(x2 y2)(x3 y2)(x2 y3):
+    #   half 0: 4 5 6 7 4 -> 0x4FAC (spare 0); half 1: 7 0 1 2 7 -> 0x7447 | 0x8000
+    #   -> 0xF4474FAC
+    t = np.arange(32)[:, None]
+    c = np.arange(128)[None, :]
+    tile = (t // 8 + 3 * c) % 8
+    w = pack.pack_codes_block(tile, pack.KIND_K, PER_TOKEN, 3)
+    assert w[0] == 0x8D635688
+    assert w[1] == 0x68D1B23E
+    assert w[2] == 0xF4474FAC
+
+
+def test_hand_words_b6_V_per_channel_leftovers_across_words():
+    # tile X[t][c] = (7t + c) mod 64, V per-channel, b = 6 (2 slots per half,
+    # spare bits 12..15). Lane 0, unit 0, register (x, y): t = 8y + h, c = x.
+    # Registers psi = 4x + y < 12 fill slots (psi // 2, psi % 2); x = 3 are
+    # leftovers l = y, whose 6 bits run along the 4-bit spare nibbles.
+    # unit word 0: slot 0 (x0 y0) 0 / 7, slot 1 (x0 y1) 56 / 63, spare = bits
+    #   0..3 of leftover 0 (x3 y0: 3 / 10): half 0 0x3E00, half 1 0xAFC7
+    # unit word 1: slot 0 (x0 y2) 48 / 55, slot 1 (x0 y3) 40 / 47, spare bits
+    #   12,13 = leftover 0 bits 4,5 (0 / 0), 14,15 = leftover 1 (x3 y1: 59 / 2)
+    #   bits 0,1 (3 / 2): half 0 0xCA30, half 1 0x8BF7
+    t = np.arange(32)[:, None]
+    c = np.arange(128)[None, :]
+    tile = (7 * t + c) % 64
+    w = pack.pack_codes_block(tile, pack.KIND_V, PER_CHANNEL, 6)
+    assert w[0] == 0xAFC73E00
+    assert w[1] == 0x8BF7CA30
 
 
 def _h(x):
@@ -81,36 +128,37 @@ def _h(x):
 
 
 def test_hand_meta_words():
-    # K per-channel, scale_c = c, zero_c = -c - 1 ("pair planes").
+    # K per-channel, scale_c = c, zero_c = -c - 1: word c // 2 = scales of
+    # (c, c+1), word 64 + c // 2 their zeros.
     c = np.arange(128)
     w = pack.pack_meta_block(c.astype(np.float16), (-c - 1).astype(np.float16),
                              pack.KIND_K, PER_CHANNEL)
     assert w[0] == (_h(1) << 16) | _h(0)           # channels (0, 1)
-    assert w[1] == (_h(9) << 16) | _h(8)           # channels (8, 9)
-    assert w[16] == (_h(3) << 16) | _h(2)          # channels (2, 3)
+    assert w[1] == (_h(3) << 16) | _h(2)           # channels (2, 3)
     assert w[64] == (_h(-2) << 16) | _h(-1)        # zeros of channels (0, 1)
-    assert w[0] == 0x3C000000 and w[1] == 0x48804800 and w[64] == 0xC000BC00
-    # V per-token, group (t, G), scale = 4t + G ("pair planes").
+    assert w[0] == 0x3C000000 and w[1] == 0x42004000 and w[64] == 0xC000BC00
+    # V per-token, group (t, G), scale = 4t + G: word 4 (t // 2) + G = scales
+    # of tokens (t, t+1).
     tt = np.repeat(np.arange(32), 4)
     GG = np.tile(np.arange(4), 32)
     s = (4 * tt + GG).astype(np.float16)
     w = pack.pack_meta_block(s, np.zeros(128, np.float16), pack.KIND_V, PER_TOKEN)
     assert w[0] == 0x44000000                       # tokens (0,1), G 0: 0, 4
     assert w[1] == 0x45003C00                       # tokens (0,1), G 1: 1, 5
-    assert w[4] == 0x50805000                       # tokens (8,9), G 0: 32, 36
-    assert w[16] == 0x4A004800                      # tokens (2,3), G 0: 8, 12
-    # K per-token: word = (scale, zero) of group (t, G) at 16(t%8) + 4(t//8) + G.
+    assert w[4] == 0x4A004800                       # tokens (2,3), G 0: 8, 12
+    assert w[16] == 0x50805000                      # tokens (8,9), G 0: 32, 36
+    # K per-token: word = (scale, zero) of group (t, G) at 16(t%8) + 4G + t//8.
     w = pack.pack_meta_block(s, -s, pack.KIND_K, PER_TOKEN)
     assert w[0] == (0x8000 << 16)                    # t = 0, G = 0: scale 0, zero -0
-    assert w[4] == (_h(-32) << 16) | _h(32)          # t = 8, G = 0
+    assert w[1] == (_h(-32) << 16) | _h(32)          # t = 8, G = 0
+    assert w[4] == (_h(-1) << 16) | _h(1)            # t = 0, G = 1
     assert w[16] == (_h(-4) << 16) | _h(4)           # t = 1, G = 0
-    assert w[17] == (_h(-5) << 16) | _h(5)           # t = 1, G = 1
-    # V per-channel: word 16(c%8) + 2(c//16) + (c//8)%2.
+    assert w[17] == (_h(-36) << 16) | _h(36)         # t = 9, G = 0
+    # V per-channel: word c = (scale, zero) of channel c.
     w = pack.pack_meta_block(c.astype(np.float16), (-c - 1).astype(np.float16),
                              pack.KIND_V, PER_CHANNEL)
-    assert w[1] == (_h(-9) << 16) | _h(8)            # c = 8
-    assert w[2] == (_h(-17) << 16) | _h(16)          # c = 16
-    assert w[16] == (_h(-2) << 16) | _h(1)           # c = 1
+    assert w[1] == (_h(-2) << 16) | _h(1)            # c = 1
+    assert w[8] == (_h(-9) << 16) | _h(8)            # c = 8
 
 
 @pytest.mark.parametrize("kind,grouping", [(0, PER_CHANNEL), (0, PER_TOKEN),

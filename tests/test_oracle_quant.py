@@ -177,3 +177,71 @@ def test_rotation_preserves_mse():
     back = r["xhat"].astype(np.float64) @ R.T
     e_orig = np.mean((x.astype(np.float64) - back) ** 2)
     assert abs(e_rot / e_orig - 1.0) < 1e-5
+
+
+def _round_half_even(fr):
+    from fractions import Fraction
+    lo = fr.numerator // fr.denominator
+    rem = fr - lo
+    if rem > Fraction(1, 2) or (rem == Fraction(1, 2) and lo % 2 == 1):
+        return lo + 1
+    return lo
+
+
+@pytest.mark.parametrize("b", (2, 3, 4, 8))
+def test_codes_are_exact_rational_rounding(b):
+    # code = clamp(round_half_even((fp32(v - zf)) * inv), 0, L) with the product
+    # taken exactly: checked with rational arithmetic, element by element.
+    from fractions import Fraction
+    rng = np.random.default_rng(100 + b)
+    x = (rng.standard_normal((40, 32)) * rng.uniform(0.01, 50, (40, 1))).astype(np.float32)
+    codes, scale, zero, bad = quant.quantize_groups(x, b)
+    L = 2 ** b - 1
+    for g in range(x.shape[0]):
+        sf = np.float32(scale[g])
+        zf = np.float32(zero[g])
+        inv = np.float32(1.0) / sf
+        for j in range(32):
+            d = np.float32(np.float32(x[g, j]) - zf)
+            want = min(max(_round_half_even(Fraction(float(d)) * Fraction(float(inv))), 0), L)
+            assert codes[g, j] == want
+
+
+def test_one_rounding_not_two():
+    # A value v whose exact product v * inv lies just below k + 1/2 while its
+    # fp32 rounding is exactly k + 1/2 (k odd): rounding the fp32 product
+    # would give the even neighbour k + 1, the exact product gives k. The
+    # group min 0, max m at b = 8 fixes scale = fp16(m / 255), zero = 0.
+    from fractions import Fraction
+    b = 8
+    found = None
+    for m in range(3, 200):
+        sf = np.float32(np.float16(np.float32(m) / np.float32(255.0)))
+        inv = np.float32(1.0) / sf
+        for k in range(1, 255, 2):
+            half = Fraction(2 * k + 1, 2)
+            v = np.float32(float(half / Fraction(float(inv))))
+            cands = [v]
+            lo = hi = v
+            for _ in range(3):
+                lo = np.nextafter(lo, np.float32(-1e9))
+                hi = np.nextafter(hi, np.float32(1e9))
+                cands += [lo, hi]
+            for cand in cands:
+                exact = Fraction(float(cand)) * Fraction(float(inv))
+                fp32_product = float(np.float32(float(cand) * float(inv)))   # fp64 product is exact
+                if exact < half and fp32_product == k + 0.5 and 0 < cand < m:
+                    found = (m, k, np.float32(cand))
+                    break
+            if found:
+                break
+        if found:
+            break
+    assert found is not None
+    m, k, v = found
+    x = np.zeros((1, 32), dtype=np.float32)
+    x[0, 1] = np.float32(m)
+    x[0, 2] = v
+    codes, scale, zero, _ = quant.quantize_groups(x, b)
+    assert float(zero[0]) == 0.0
+    assert codes[0, 2] == k
