@@ -25,6 +25,7 @@
 #include <algorithm>
 #include <atomic>
 
+#include "format.cuh"
 #include "rq_internal.cuh"
 
 namespace rq {
@@ -50,6 +51,10 @@ rq_status current_sm_count(int* sms) {
 
 namespace {
 
+// CTAs per SM the decoder's register budget is sized for
+#ifndef RQ_DECODE_MIN_BLOCKS
+#define RQ_DECODE_MIN_BLOCKS 3
+#endif
 constexpr int kWarps = 4;
 constexpr int kThreads = 32 * kWarps;
 constexpr int kPart = kD + 2;        // partial record: o[128], m (log2 domain), l
@@ -127,7 +132,7 @@ __device__ __forceinline__ uint4 lds128(const uint8_t* p) {
 
 // ------------------------------------------------------- code extraction ----
 // The lane's 4*BW code words of one block image (16-byte piece i of lane L at
-// byte 16*(32 i + L)).
+// byte 16*(32 i + L)); unit u's words are w[BW u .. BW u + BW - 1].
 template <int BW>
 __device__ __forceinline__ void lane_words(const uint8_t* img, int lane, uint32_t (&w)[4 * BW]) {
 #pragma unroll
@@ -140,16 +145,8 @@ __device__ __forceinline__ void lane_words(const uint8_t* img, int lane, uint32_
   }
 }
 
-template <int BW>
-__device__ __forceinline__ uint32_t lane_code(const uint32_t (&w)[4 * BW], int p) {
-  const int wi = p >> 5, sh = p & 31;
-  uint32_t v = w[wi] >> sh;
-  if (sh + BW > 32) v |= w[wi + 1] << (32 - sh);
-  return v & ((1u << BW) - 1u);
-}
-
 constexpr uint32_t kMagic = 0x64006400u;      // fp16 1024.0 in both halves
-constexpr uint32_t kMagicBytes = 0x64646464u;
+constexpr float kTwo24 = 16777216.0f;         // codes enter the MMA as c * 2^(E - 24)
 
 __device__ __forceinline__ uint32_t hfma2u(uint32_t x, uint32_t m, uint32_t a) {
   return h2u(__hfma2(u2h(x), u2h(m), u2h(a)));
@@ -157,154 +154,117 @@ __device__ __forceinline__ uint32_t hfma2u(uint32_t x, uint32_t m, uint32_t a) {
 __device__ __forceinline__ uint32_t hsub2u(uint32_t x, uint32_t y) {
   return h2u(__hsub2(u2h(x), u2h(y)));
 }
+__device__ __forceinline__ uint32_t hmul2u(uint32_t x, uint32_t y) {
+  return h2u(__hmul2(u2h(x), u2h(y)));
+}
 
-// Fragment f of the lane stream: register k holds the code pair
-// (a_2k, a_2k+1) = (slot k, slot 4+k) as exact fp16 integers.
+// 2^-E in both fp16 halves (E <= 14)
+__host__ __device__ constexpr uint32_t pow2_neg_h2(int E) {
+  return (static_cast<uint32_t>(15 - E) << 10) * 0x00010001u;
+}
+
+// register (x, y) of unit u of the lane's words: c * 2^(E - 24) per half
 template <int BW>
-__device__ __forceinline__ void frag_codes(const uint32_t (&w)[4 * BW], int f, uint32_t (&c)[4]) {
-  if constexpr (BW == 1) {
-    // byte = (a0 a2 a4 a6 | a1 a3 a5 a7) bits; both halves get the byte under 0x64
-    const int bi = f & 3;
-    const uint32_t W = __byte_perm(w[f >> 2], kMagicBytes, 0x4040u | (bi << 8) | bi);
-    // half0 keeps bit k (2^k a), half1 bit 4+k (2^(4+k) a'); scales are exact
-    const uint32_t mul[4] = {0x2C003C00u, 0x28003800u, 0x24003400u, 0x20003000u};
-    const uint32_t add[4] = {0xD400E400u, 0xD000E000u, 0xCC00DC00u, 0xC800D800u};
-#pragma unroll
-    for (int k = 0; k < 4; ++k)
-      c[k] = hfma2u(W & (kMagic | (1u << k) | (1u << (20 + k))), mul[k], add[k]);
-  } else if constexpr (BW == 2) {
-    // 16-bit fragment: low byte (a0 a2 a4 a6) -> half0, high byte -> half1
-    const int lb = 2 * (f & 1);
-    const uint32_t W = __byte_perm(w[f >> 1], kMagicBytes, 0x4040u | ((lb + 1) << 8) | lb);
-    const uint32_t mul[4] = {0x3C003C00u, 0x34003400u, 0x2C002C00u, 0x24002400u};   // 4^-k
-    const uint32_t add[4] = {0xE400E400u, 0xDC00DC00u, 0xD400D400u, 0xCC00CC00u};   // -1024 4^-k
-#pragma unroll
-    for (int k = 0; k < 4; ++k) c[k] = hfma2u(W & (kMagic | (0x00030003u << (2 * k))), mul[k], add[k]);
-  } else if constexpr (BW == 3) {
-    // 24-bit fragment: low 12 bits -> half0, next 12 bits -> half1
-    const int base = 3 * (f >> 2), s = f & 3;
-    uint32_t X;
-    if (s == 0) X = w[base];
-    else if (s == 1) X = __funnelshift_r(w[base], w[base + 1], 24);
-    else if (s == 2) X = __funnelshift_r(w[base + 1], w[base + 2], 16);
-    else X = w[base + 2] >> 8;
-    const uint32_t W = (X & 0xFFFFu) | ((X << 4) & 0xFFFF0000u);
-    // OR the fp16 magic in once; each field is then one single-mask AND
-    // (the magic's bits and the fields' bits do not overlap)
-    const uint32_t Wm = W | kMagic, Zm = (W >> 3) | kMagic;
-    const uint32_t mul[3] = {0x3C003C00u, 0x30003000u, 0x24002400u};   // 8^-k
-    const uint32_t add[3] = {0xE400E400u, 0xD800D800u, 0xCC00CC00u};   // -1024 8^-k
-#pragma unroll
-    for (int k = 0; k < 3; ++k) c[k] = hfma2u(Wm & (kMagic | (0x00070007u << (3 * k))), mul[k], add[k]);
-    c[3] = hfma2u(Zm & (kMagic | 0x01C001C0u), 0x24002400u, 0xCC00CC00u);
-  } else if constexpr (BW == 4) {
-    // one word: low half nibbles a0 a2 a4 a6, high half a1 a3 a5 a7
-    const uint32_t Xm = w[f] | kMagic, Ym = (w[f] >> 8) | kMagic;
-    c[0] = hsub2u(Xm & (kMagic | 0x000F000Fu), kMagic);
-    c[1] = hfma2u(Xm & (kMagic | 0x00F000F0u), 0x2C002C00u, 0xD400D400u);   // /16 - 64
-    c[2] = hsub2u(Ym & (kMagic | 0x000F000Fu), kMagic);
-    c[3] = hfma2u(Ym & (kMagic | 0x00F000F0u), 0x2C002C00u, 0xD400D400u);
-  } else if constexpr (BW == 8) {
-    // two words: bytes a0 a2 a4 a6 | a1 a3 a5 a7
-    const uint32_t X0 = w[2 * f], X1 = w[2 * f + 1];
-    const uint32_t Y0 = __byte_perm(X0, X1, 0x5140u);   // a0 a1 a2 a3
-    const uint32_t Y1 = __byte_perm(X0, X1, 0x7362u);   // a4 a5 a6 a7
-    c[0] = hsub2u(__byte_perm(Y0, kMagicBytes, 0x4140u), kMagic);
-    c[1] = hsub2u(__byte_perm(Y0, kMagicBytes, 0x4342u), kMagic);
-    c[2] = hsub2u(__byte_perm(Y1, kMagicBytes, 0x4140u), kMagic);
-    c[3] = hsub2u(__byte_perm(Y1, kMagicBytes, 0x4342u), kMagic);
-  } else {
-    const int base = 8 * BW * f;
-#pragma unroll
-    for (int k = 0; k < 4; ++k) {
-      const uint32_t lo = lane_code<BW>(w, base + BW * k);
-      const uint32_t hi = lane_code<BW>(w, base + BW * (4 + k));
-      c[k] = hsub2u(lo | (hi << 16) | kMagic, kMagic);
-    }
-  }
+__device__ __forceinline__ uint32_t reg(const uint32_t (&w)[4 * BW], int u, int x, int y) {
+  return fmt::extract<BW>(w + BW * u, x, y);
+}
+
+// dequantized pair s * c + z from an extracted register (layouts whose scale
+// cannot be folded): the subnormal c * 2^E under the 1024 exponent, minus
+// 1024 (exact), times m = s * 2^-E plus z (one rounding)
+__device__ __forceinline__ uint32_t dequant(uint32_t sub, uint32_t m, uint32_t z2) {
+  return hfma2u(hsub2u(sub | kMagic, kMagic), m, z2);
 }
 
 // ------------------------------------------------------------ block math ----
-
+// Lane (gid, tig) reads units u = 0..3 of its K words: unit u holds channels
+// 32 u + 8 tig + (0..7) of tokens gid + 8 (0..3); the k-steps 2u and 2u + 1
+// of the scores MMA are its channel pairs x = 0, 1 and 2, 3 (format.cuh).
+//
 // scores^T[mt] (tokens 16 mt + gid (+8), heads 2 tig (+1)) of one K block image.
 // Per-channel keys: k_hat[t][c] = code s_c + z_c, so
 //   scores[t][j] = sum_c code[t][c] (q_jc s_c) + sum_c z_c q_jc:
-// the scale is folded into q (one fp16x2 multiply per q pair) and the
-// zero-point term, the same for every token, comes from MMAs whose A operand
-// repeats z in every row and initialises the accumulators. The codes enter
-// the MMA as exact fp16 integers.
+// the scale (and the code's 2^-E) is folded into q, one fp16x2 multiply per
+// q pair; the zero-point term, the same for every token, comes from MMAs
+// whose A operand carries z in rows gid. Codes enter the tensor cores as
+// exact fp16 subnormals c 2^(E - 24); the accumulator is scaled by 2^24.
 template <int BW, int KG>
-__device__ __forceinline__ void qk_block(const uint8_t* img, int lane, const uint32_t (&qb)[8][2],
-                                         float (&s)[2][4]) {
+__device__ __forceinline__ void qk_block(const uint8_t* img, int lane, const uint32_t (&qb)[4][4],
+                                         const uint32_t (&qf)[4][4], float (&s)[2][4]) {
   const int gid = lane >> 2, tig = lane & 3;
   uint32_t w[4 * BW];
   lane_words<BW>(img, lane, w);
   const uint8_t* meta = img + 512 * BW;
+#pragma unroll
+  for (int mt = 0; mt < 2; ++mt)
+#pragma unroll
+    for (int r = 0; r < 4; ++r) s[mt][r] = 0.0f;
   if constexpr (KG == RQ_PER_CHANNEL) {
-    uint32_t qs2[8][2];
     float zb[4] = {0.0f, 0.0f, 0.0f, 0.0f};
 #pragma unroll
-    for (int ks = 0; ks < 8; ++ks) {   // channel pairs 16 ks + 8 h + 2 tig: words 16 tig + 2 ks + h
-      const uint2 s2 = *reinterpret_cast<const uint2*>(meta + 4 * (16 * tig + 2 * ks));
-      const uint2 z2 = *reinterpret_cast<const uint2*>(meta + 256 + 4 * (16 * tig + 2 * ks));
-      qs2[ks][0] = h2u(__hmul2(u2h(qb[ks][0]), u2h(s2.x)));
-      qs2[ks][1] = h2u(__hmul2(u2h(qb[ks][1]), u2h(s2.y)));
-      // z repeats in every token row, so rows gid + 8 are left zero and
-      // rows gid (zb[0], zb[1]) serve both
-      const uint32_t az[4] = {z2.x, 0u, z2.y, 0u};
-      mma16816(zb, az, qb[ks][0], qb[ks][1]);
+    for (int u = 0; u < 4; ++u) {
+      // scale / zero pairs of channels 32u + 8tig + 2x: words 16u + 4tig + x
+      const uint4 S = lds128(meta + 4 * (16 * u + 4 * tig));
+      const uint4 Z = lds128(meta + 256 + 4 * (16 * u + 4 * tig));
+      const uint32_t S2[4] = {S.x, S.y, S.z, S.w}, Z2[4] = {Z.x, Z.y, Z.z, Z.w};
+#pragma unroll
+      for (int xs = 0; xs < 2; ++xs) {
+        const uint32_t b0 = hmul2u(qf[u][2 * xs], S2[2 * xs]);
+        const uint32_t b1 = hmul2u(qf[u][2 * xs + 1], S2[2 * xs + 1]);
+        const uint32_t az[4] = {Z2[2 * xs], 0u, Z2[2 * xs + 1], 0u};
+        mma16816(zb, az, qb[u][2 * xs], qb[u][2 * xs + 1]);
+#pragma unroll
+        for (int mt = 0; mt < 2; ++mt) {
+          const uint32_t a[4] = {reg<BW>(w, u, 2 * xs, 2 * mt), reg<BW>(w, u, 2 * xs, 2 * mt + 1),
+                                 reg<BW>(w, u, 2 * xs + 1, 2 * mt), reg<BW>(w, u, 2 * xs + 1, 2 * mt + 1)};
+          mma16816(s[mt], a, b0, b1);
+        }
+      }
     }
 #pragma unroll
     for (int mt = 0; mt < 2; ++mt) {
-      s[mt][0] = zb[0];
-      s[mt][1] = zb[1];
-      s[mt][2] = zb[0];
-      s[mt][3] = zb[1];
+      s[mt][0] = __fmaf_rn(s[mt][0], kTwo24, zb[0]);
+      s[mt][1] = __fmaf_rn(s[mt][1], kTwo24, zb[1]);
+      s[mt][2] = __fmaf_rn(s[mt][2], kTwo24, zb[0]);
+      s[mt][3] = __fmaf_rn(s[mt][3], kTwo24, zb[1]);
     }
-#pragma unroll
-    for (int ks = 0; ks < 8; ++ks)
-#pragma unroll
-      for (int mt = 0; mt < 2; ++mt) {
-        uint32_t c[4];
-        frag_codes<BW>(w, 2 * ks + mt, c);
-        mma16816(s[mt], c, qs2[ks][0], qs2[ks][1]);
-      }
   } else {                    // per-token keys: dequantize in registers
-    uint32_t sz[16];          // (scale, zero) of groups (gid + 8m, G): words 16 gid ..
 #pragma unroll
-    for (int i = 0; i < 4; ++i) {
-      const uint4 u = lds128(meta + 64 * gid + 16 * i);
-      sz[4 * i] = u.x;
-      sz[4 * i + 1] = u.y;
-      sz[4 * i + 2] = u.z;
-      sz[4 * i + 3] = u.w;
-    }
+    for (int u = 0; u < 4; ++u) {
+      // (scale, zero) of tokens 8x + gid, group u: words 16 gid + 4u + x
+      const uint4 SZ = lds128(meta + 4 * (16 * gid + 4 * u));
+      const uint32_t sz[4] = {SZ.x, SZ.y, SZ.z, SZ.w};
+      uint32_t m[4], z2[4];
 #pragma unroll
-    for (int mt = 0; mt < 2; ++mt)
-#pragma unroll
-      for (int r = 0; r < 4; ++r) s[mt][r] = 0.0f;
-#pragma unroll
-    for (int ks = 0; ks < 8; ++ks)
-#pragma unroll
-      for (int mt = 0; mt < 2; ++mt) {
-        uint32_t c[4], a[4];
-        frag_codes<BW>(w, 2 * ks + mt, c);
-#pragma unroll
-        for (int k = 0; k < 4; ++k) {     // token 16 mt + gid + 8 (k&1), group ks/2
-          const __half2 szh = u2h(sz[4 * (2 * mt + (k & 1)) + (ks >> 1)]);
-          a[k] = hfma2u(c[k], h2u(__low2half2(szh)), h2u(__high2half2(szh)));
-        }
-        mma16816(s[mt], a, qb[ks][0], qb[ks][1]);
+      for (int x = 0; x < 4; ++x) {
+        const __half2 h = u2h(sz[x]);
+        m[x] = hmul2u(h2u(__low2half2(h)), pow2_neg_h2(fmt::exponent(BW, x)));
+        z2[x] = h2u(__high2half2(h));
       }
+#pragma unroll
+      for (int xs = 0; xs < 2; ++xs)
+#pragma unroll
+        for (int mt = 0; mt < 2; ++mt) {
+          // register (x = token 2mt + r, y = pair 2xs + h)
+          const uint32_t a[4] = {
+              dequant(reg<BW>(w, u, 2 * mt, 2 * xs), m[2 * mt], z2[2 * mt]),
+              dequant(reg<BW>(w, u, 2 * mt + 1, 2 * xs), m[2 * mt + 1], z2[2 * mt + 1]),
+              dequant(reg<BW>(w, u, 2 * mt, 2 * xs + 1), m[2 * mt], z2[2 * mt]),
+              dequant(reg<BW>(w, u, 2 * mt + 1, 2 * xs + 1), m[2 * mt + 1], z2[2 * mt + 1])};
+          mma16816(s[mt], a, qb[u][2 * xs], qb[u][2 * xs + 1]);
+        }
+    }
   }
 }
 
-// o^T[mt] (channels 16 mt + gid (+8), heads 2 tig (+1)) += V_hat^T . P^T of one V block image.
-// Per-token values: v_hat[t][c] = code s_tG + z_tG (G = c / 32), so
+// o^T[mt] (channel rows 16 mt + gid (+8), heads 2 tig (+1)) += V_hat^T . P^T of
+// one V block image. Unit u = channel group G holds channels 32u + 4gid + x
+// (rows of m-tiles 2u, 2u + 1) of tokens 8y + 2tig + (0, 1).
+// Per-token values: v_hat[t][c] = code s_tG + z_tG, so
 //   o[c][j] += sum_t code[t][c] (p_tj s_tG) + sum_t z_tG p_tj:
-// the scale is folded into P^T per channel group (one fp16x2 multiply per
-// pair) and the zero-point term comes from MMAs whose A operand repeats z_tG
-// down every channel row of the group.
+// the scale is folded into P^T per group (one fp16x2 multiply per pair), the
+// zero-point term comes from MMAs whose A operand repeats z_tG in every row
+// of the group, and the codes' 2^(E - 24) is undone on the output rows.
 template <int BW, int VG>
 __device__ __forceinline__ void pv_block(const uint8_t* img, int lane, const uint32_t (&pb)[2][2],
                                          float (&o)[8][4], float (&bz)[2][4]) {
@@ -313,75 +273,77 @@ __device__ __forceinline__ void pv_block(const uint8_t* img, int lane, const uin
   lane_words<BW>(img, lane, w);
   const uint8_t* meta = img + 512 * BW;
   if constexpr (VG == RQ_PER_TOKEN) {
-    uint32_t ms[16], mz[16];  // token pairs (tig + 4j) x group G: words 16 tig + 4 j + G
+    uint32_t ms[4][4], mz[4][4];  // [token pair y][group G]: words 16y + 4tig + G
 #pragma unroll
-    for (int i = 0; i < 4; ++i) {
-      const uint4 u = lds128(meta + 64 * tig + 16 * i);
-      const uint4 z = lds128(meta + 256 + 64 * tig + 16 * i);
-      ms[4 * i] = u.x;
-      ms[4 * i + 1] = u.y;
-      ms[4 * i + 2] = u.z;
-      ms[4 * i + 3] = u.w;
-      mz[4 * i] = z.x;
-      mz[4 * i + 1] = z.y;
-      mz[4 * i + 2] = z.z;
-      mz[4 * i + 3] = z.w;
+    for (int y = 0; y < 4; ++y) {
+      const uint4 S = lds128(meta + 4 * (16 * y + 4 * tig));
+      const uint4 Z = lds128(meta + 256 + 4 * (16 * y + 4 * tig));
+      ms[y][0] = S.x;
+      ms[y][1] = S.y;
+      ms[y][2] = S.z;
+      ms[y][3] = S.w;
+      mz[y][0] = Z.x;
+      mz[y][1] = Z.y;
+      mz[y][2] = Z.z;
+      mz[y][3] = Z.w;
     }
 #pragma unroll
     for (int ks = 0; ks < 2; ++ks) {
-      // zero-points: sum_t z_tG p_tj, the same for every channel of group G;
-      // rows gid of the A operand carry group G, rows gid + 8 group G + 1
+      // zero-points: rows gid of the A operand carry group 2gp, rows gid + 8
+      // group 2gp + 1; columns are token pairs 2ks (k 2tig..) and 2ks + 1
 #pragma unroll
       for (int gp = 0; gp < 2; ++gp) {
-        const uint32_t az[4] = {mz[4 * (2 * ks) + 2 * gp], mz[4 * (2 * ks) + 2 * gp + 1],
-                                mz[4 * (2 * ks + 1) + 2 * gp], mz[4 * (2 * ks + 1) + 2 * gp + 1]};
+        const uint32_t az[4] = {mz[2 * ks][2 * gp], mz[2 * ks][2 * gp + 1],
+                                mz[2 * ks + 1][2 * gp], mz[2 * ks + 1][2 * gp + 1]};
         mma16816(bz[gp], az, pb[ks][0], pb[ks][1]);
       }
 #pragma unroll
       for (int G = 0; G < 4; ++G) {
-        // B fragment rows: tokens 16 ks + 2 tig (+1) and + 8  ->  pair words j = 2 ks, 2 ks + 1
-        const uint32_t b0 = h2u(__hmul2(u2h(pb[ks][0]), u2h(ms[4 * (2 * ks) + G])));
-        const uint32_t b1 = h2u(__hmul2(u2h(pb[ks][1]), u2h(ms[4 * (2 * ks + 1) + G])));
+        const uint32_t b0 = hmul2u(pb[ks][0], ms[2 * ks][G]);
+        const uint32_t b1 = hmul2u(pb[ks][1], ms[2 * ks + 1][G]);
 #pragma unroll
-        for (int h = 0; h < 2; ++h) {
-          const int mt = 2 * G + h;
-          uint32_t c[4];
-          frag_codes<BW>(w, 8 * ks + mt, c);
-          mma16816(o[mt], c, b0, b1);
+        for (int mh = 0; mh < 2; ++mh) {
+          // register (x = row 2mh + r, y = token pair 2ks + h)
+          const uint32_t a[4] = {reg<BW>(w, G, 2 * mh, 2 * ks), reg<BW>(w, G, 2 * mh + 1, 2 * ks),
+                                 reg<BW>(w, G, 2 * mh, 2 * ks + 1), reg<BW>(w, G, 2 * mh + 1, 2 * ks + 1)};
+          mma16816(o[2 * G + mh], a, b0, b1);
         }
       }
     }
   } else {                    // per-channel values: dequantize in registers
-    uint32_t ms[16];          // (scale, zero) of channels 16 mt + gid + 8 h: words 16 gid ..
 #pragma unroll
-    for (int i = 0; i < 4; ++i) {
-      const uint4 u = lds128(meta + 64 * gid + 16 * i);
-      ms[4 * i] = u.x;
-      ms[4 * i + 1] = u.y;
-      ms[4 * i + 2] = u.z;
-      ms[4 * i + 3] = u.w;
-    }
+    for (int u = 0; u < 4; ++u) {
+      // (scale, zero) of channels 32u + 4gid + x: words 32u + 4gid + x
+      const uint4 SZ = lds128(meta + 4 * (32 * u + 4 * gid));
+      const uint32_t sz[4] = {SZ.x, SZ.y, SZ.z, SZ.w};
+      uint32_t m[4], z2[4];
 #pragma unroll
-    for (int ks = 0; ks < 2; ++ks)
-#pragma unroll
-      for (int mt = 0; mt < 8; ++mt) {
-        uint32_t c[4], a[4];
-        frag_codes<BW>(w, 8 * ks + mt, c);
-#pragma unroll
-        for (int k = 0; k < 4; ++k) {     // channel 16 mt + gid + 8 (k&1)
-          const __half2 szh = u2h(ms[2 * mt + (k & 1)]);
-          a[k] = hfma2u(c[k], h2u(__low2half2(szh)), h2u(__high2half2(szh)));
-        }
-        mma16816(o[mt], a, pb[ks][0], pb[ks][1]);
+      for (int x = 0; x < 4; ++x) {
+        const __half2 h = u2h(sz[x]);
+        m[x] = hmul2u(h2u(__low2half2(h)), pow2_neg_h2(fmt::exponent(BW, x)));
+        z2[x] = h2u(__high2half2(h));
       }
+#pragma unroll
+      for (int ks = 0; ks < 2; ++ks)
+#pragma unroll
+        for (int mh = 0; mh < 2; ++mh) {
+          const uint32_t a[4] = {
+              dequant(reg<BW>(w, u, 2 * mh, 2 * ks), m[2 * mh], z2[2 * mh]),
+              dequant(reg<BW>(w, u, 2 * mh + 1, 2 * ks), m[2 * mh + 1], z2[2 * mh + 1]),
+              dequant(reg<BW>(w, u, 2 * mh, 2 * ks + 1), m[2 * mh], z2[2 * mh]),
+              dequant(reg<BW>(w, u, 2 * mh + 1, 2 * ks + 1), m[2 * mh + 1], z2[2 * mh + 1])};
+          mma16816(o[2 * u + mh], a, pb[ks][0], pb[ks][1]);
+        }
+    }
   }
 }
 
 template <int BW>
 __device__ __forceinline__ void qk_dispatch_g(int kg, const uint8_t* img, int lane,
-                                              const uint32_t (&qb)[8][2], float (&s)[2][4]) {
-  if (kg == RQ_PER_CHANNEL) qk_block<BW, RQ_PER_CHANNEL>(img, lane, qb, s);
-  else qk_block<BW, RQ_PER_TOKEN>(img, lane, qb, s);
+                                              const uint32_t (&qb)[4][4], const uint32_t (&qf)[4][4],
+                                              float (&s)[2][4]) {
+  if (kg == RQ_PER_CHANNEL) qk_block<BW, RQ_PER_CHANNEL>(img, lane, qb, qf, s);
+  else qk_block<BW, RQ_PER_TOKEN>(img, lane, qb, qf, s);
 }
 
 template <int BW>
@@ -393,16 +355,17 @@ __device__ __forceinline__ void pv_dispatch_g(int vg, const uint8_t* img, int la
 }
 
 __device__ __forceinline__ void qk_dispatch(int bw, int kg, const uint8_t* img, int lane,
-                                            const uint32_t (&qb)[8][2], float (&s)[2][4]) {
+                                            const uint32_t (&qb)[4][4], const uint32_t (&qf)[4][4],
+                                            float (&s)[2][4]) {
   switch (bw) {
-    case 1: qk_dispatch_g<1>(kg, img, lane, qb, s); break;
-    case 2: qk_dispatch_g<2>(kg, img, lane, qb, s); break;
-    case 3: qk_dispatch_g<3>(kg, img, lane, qb, s); break;
-    case 4: qk_dispatch_g<4>(kg, img, lane, qb, s); break;
-    case 5: qk_dispatch_g<5>(kg, img, lane, qb, s); break;
-    case 6: qk_dispatch_g<6>(kg, img, lane, qb, s); break;
-    case 7: qk_dispatch_g<7>(kg, img, lane, qb, s); break;
-    default: qk_dispatch_g<8>(kg, img, lane, qb, s); break;
+    case 1: qk_dispatch_g<1>(kg, img, lane, qb, qf, s); break;
+    case 2: qk_dispatch_g<2>(kg, img, lane, qb, qf, s); break;
+    case 3: qk_dispatch_g<3>(kg, img, lane, qb, qf, s); break;
+    case 4: qk_dispatch_g<4>(kg, img, lane, qb, qf, s); break;
+    case 5: qk_dispatch_g<5>(kg, img, lane, qb, qf, s); break;
+    case 6: qk_dispatch_g<6>(kg, img, lane, qb, qf, s); break;
+    case 7: qk_dispatch_g<7>(kg, img, lane, qb, qf, s); break;
+    default: qk_dispatch_g<8>(kg, img, lane, qb, qf, s); break;
   }
 }
 
@@ -556,8 +519,8 @@ __device__ __forceinline__ void prologue_static(const WarpStream& ws) {
 }
 
 template <int BK, int KG, int BV, int VG>
-__device__ __forceinline__ void blocks_static(const WarpStream& ws, const uint32_t (&qb)[8][2],
-                                              SoftmaxAcc& acc) {
+__device__ __forceinline__ void blocks_static(const WarpStream& ws, const uint32_t (&qb)[4][4],
+                                              const uint32_t (&qf)[4][4], SoftmaxAcc& acc) {
   using R = Ring<BK, BV>;
   constexpr int NS = R::kSlots;
   int use = 0, iss = NS - 1;          // slot of the next entry to use / to issue
@@ -567,7 +530,7 @@ __device__ __forceinline__ void blocks_static(const WarpStream& ws, const uint32
     cp_async_wait<NS - 1>();
     __syncwarp();
     float s[2][4];
-    qk_block<BK, KG>(ws.ring_ptr + use * R::kSlot, ws.lane, qb, s);
+    qk_block<BK, KG>(ws.ring_ptr + use * R::kSlot, ws.lane, qb, qf, s);
     __syncwarp();
     use = use + 1 == NS ? 0 : use + 1;
     uint32_t pb[2][2];
@@ -600,7 +563,8 @@ __device__ __forceinline__ void prologue_dyn(const WarpStream& ws, const DynRing
 }
 
 __device__ __forceinline__ void blocks_dyn(const WarpStream& ws, const DynRing& r,
-                                           const uint32_t (&qb)[8][2], SoftmaxAcc& acc) {
+                                           const uint32_t (&qb)[4][4], const uint32_t (&qf)[4][4],
+                                           SoftmaxAcc& acc) {
   int use = 0, iss = r.ns - 1;
   for (int i = 0; i < ws.nb; ++i) {
     issue_dyn(ws, r, 2 * i + r.ns - 1, iss);
@@ -608,7 +572,7 @@ __device__ __forceinline__ void blocks_dyn(const WarpStream& ws, const DynRing& 
     cp_async_wait_dyn(r.ns - 1);
     __syncwarp();
     float s[2][4];
-    qk_dispatch(r.bK, r.kg, ws.ring_ptr + use * r.slot, ws.lane, qb, s);
+    qk_dispatch(r.bK, r.kg, ws.ring_ptr + use * r.slot, ws.lane, qb, qf, s);
     __syncwarp();
     use = use + 1 == r.ns ? 0 : use + 1;
     uint32_t pb[2][2];
@@ -638,7 +602,7 @@ __device__ __forceinline__ int fast_key(int bK, int bV, int kg, int vg) {
   X(8, 4, 2) X(9, 4, 3) X(10, 4, 4) X(11, 4, 8) X(12, 8, 2) X(13, 8, 3) X(14, 8, 4) X(15, 8, 8)
 
 template <typename T>
-__global__ void __launch_bounds__(kThreads) decode_split_kernel(DecodeArgs a) {
+__global__ void __launch_bounds__(kThreads, RQ_DECODE_MIN_BLOCKS) decode_split_kernel(DecodeArgs a) {
   extern __shared__ __align__(16) unsigned char smem_raw[];
   float* qs = reinterpret_cast<float*>(smem_raw);                  // [8][128]
   uint8_t* rings = smem_raw + kQBytes;
@@ -700,15 +664,22 @@ __global__ void __launch_bounds__(kThreads) decode_split_kernel(DecodeArgs a) {
   }
   __syncthreads();
   if (a.hadamard) fwht_smem(qs, kMaxHeads);
-  // softmax scale 1/sqrt(128) and log2(e) folded into q (scores in log2 units)
+  // softmax scale 1/sqrt(128) and log2(e) folded into q (scores in log2 units).
+  // K unit u, pair x of lane (gid, tig) is channels 32u + 8tig + 2x (+1);
+  // qf carries the per-channel-key codes' 2^-E(x) as well.
   const float qscale = kLog2e * kInvSqrt128 * (a.hadamard ? kInvSqrt128 : 1.0f);
-  uint32_t qb[8][2];
+  uint32_t qb[4][4], qf[4][4];
+  uint32_t ef[4];
 #pragma unroll
-  for (int ks = 0; ks < 8; ++ks) {
-    const float* qr = qs + gid * kD + 16 * ks + 2 * tig;
-    qb[ks][0] = pack_f16x2(qr[0] * qscale, qr[1] * qscale);
-    qb[ks][1] = pack_f16x2(qr[8] * qscale, qr[9] * qscale);
-  }
+  for (int x = 0; x < 4; ++x) ef[x] = pow2_neg_h2(a.kg == RQ_PER_CHANNEL && valid ? fmt::exponent(bK, x) : 0);
+#pragma unroll
+  for (int u = 0; u < 4; ++u)
+#pragma unroll
+    for (int x = 0; x < 4; ++x) {
+      const float* qr = qs + gid * kD + 32 * u + 8 * tig + 2 * x;
+      qb[u][x] = pack_f16x2(qr[0] * qscale, qr[1] * qscale);
+      qf[u][x] = hmul2u(qb[u][x], ef[x]);
+    }
 
   SoftmaxAcc acc;
 #pragma unroll
@@ -723,22 +694,28 @@ __global__ void __launch_bounds__(kThreads) decode_split_kernel(DecodeArgs a) {
   acc.l0 = acc.l1 = 0.0f;
 
   switch (key) {
-#define RQ_BLK(k, BK, BV) case k: blocks_static<BK, RQ_PER_CHANNEL, BV, RQ_PER_TOKEN>(ws, qb, acc); break;
+#define RQ_BLK(k, BK, BV) case k: blocks_static<BK, RQ_PER_CHANNEL, BV, RQ_PER_TOKEN>(ws, qb, qf, acc); break;
     RQ_FAST_CASES(RQ_BLK)
 #undef RQ_BLK
-    default: blocks_dyn(ws, dr, qb, acc); break;
+    default: blocks_dyn(ws, dr, qb, qf, acc); break;
   }
-  if (a.vg == RQ_PER_TOKEN) {
-    // group G's zero-point sum: rows gid of bz[G/2] for even G, rows gid+8 for odd G
+  if (a.vg == RQ_PER_TOKEN && valid) {
+    // rows of m-tile mt are classes x = 2 (mt & 1) + r of unit mt / 2: undo
+    // their codes' 2^(E(x) - 24), then add group G's zero-point sum (rows gid
+    // of bz[G / 2] for even G, rows gid + 8 for odd G)
+    float rf[4];
+#pragma unroll
+    for (int x = 0; x < 4; ++x) rf[x] = __int_as_float((127 + 24 - fmt::exponent(bV, x)) << 23);   // 2^(24 - E)
 #pragma unroll
     for (int mt = 0; mt < 8; ++mt) {
       const int G = mt >> 1;
       const float z0 = (G & 1) ? acc.bz[G >> 1][2] : acc.bz[G >> 1][0];
       const float z1 = (G & 1) ? acc.bz[G >> 1][3] : acc.bz[G >> 1][1];
-      acc.o[mt][0] += z0;
-      acc.o[mt][1] += z1;
-      acc.o[mt][2] += z0;
-      acc.o[mt][3] += z1;
+      const float f0 = rf[2 * (mt & 1)], f1 = rf[2 * (mt & 1) + 1];
+      acc.o[mt][0] = __fmaf_rn(acc.o[mt][0], f0, z0);
+      acc.o[mt][1] = __fmaf_rn(acc.o[mt][1], f0, z1);
+      acc.o[mt][2] = __fmaf_rn(acc.o[mt][2], f1, z0);
+      acc.o[mt][3] = __fmaf_rn(acc.o[mt][3], f1, z1);
     }
   }
   float m0 = acc.m0, m1 = acc.m1, l0 = acc.l0, l1 = acc.l1;
@@ -753,12 +730,14 @@ __global__ void __launch_bounds__(kThreads) decode_split_kernel(DecodeArgs a) {
   float* red_o = reinterpret_cast<float*>(rings);   // [warp][head][channel]
 #pragma unroll
   for (int mt = 0; mt < 8; ++mt) {
+    // row r of m-tile mt is channel 32 (mt / 2) + 4 gid + 2 (mt & 1) + r
     float* r0 = red_o + (warp * kMaxHeads + 2 * tig) * kD;
     float* r1 = r0 + kD;
-    r0[16 * mt + gid] = acc.o[mt][0];
-    r1[16 * mt + gid] = acc.o[mt][1];
-    r0[16 * mt + gid + 8] = acc.o[mt][2];
-    r1[16 * mt + gid + 8] = acc.o[mt][3];
+    const int ch = 32 * (mt >> 1) + 4 * gid + 2 * (mt & 1);
+    r0[ch] = acc.o[mt][0];
+    r1[ch] = acc.o[mt][1];
+    r0[ch + 1] = acc.o[mt][2];
+    r1[ch + 1] = acc.o[mt][3];
   }
   if (gid == 0) {
     red_m[warp][2 * tig] = m0;

@@ -8,18 +8,23 @@
 // rotation (QuaRot, App. W "QuaRot kernel"); the sweep measures the MSE at
 // every b for the fit of D(b) = alpha beta^-b (Alg. 1 stage 2, Sec. 3.4).
 //
-// One CTA of 128 threads owns one 32-token x 128-channel tile (one packed
-// block) at a time; its 128 groups of 32 map one-to-one onto threads and a
-// group's 32 values live in that thread's registers:
-//   per-token group  (t, G): thread 4t + G loads its 64 bytes straight from
-//                    global memory (the 4 groups of a token sit in 4
-//                    neighbouring lanes, so the Hadamard butterflies across
-//                    groups are two warp shuffles);
-//   per-channel group c:    the tile is staged in shared memory as raw 16-bit
-//                    values and thread c reads its column.
-// The next tile's loads are in flight while the current one is processed.
+// quantize_pack_kernel: persistent CTAs of 128 threads; a CTA owns one
+// 32-token x 128-channel tile (one packed block) at a time, staged raw in
+// shared memory by cp.async one tile ahead. Per tile:
+//   phase 1, one group per thread: min / max with NaN-propagating fp16x2 or
+//     bf16x2 compares on the raw values, the group's fp16 scale and zero
+//     (its meta words go straight to global memory) and (-zero, 1/scale)
+//     into a shared table;
+//   phase 2, one unit of the packed format (16 two-code registers of one
+//     decoder lane, format.cuh) per thread: code = low bits of
+//     RN(fp32(v - zero) * inv + 1.5 * 2^23) (fp32x2 add + fma), two codes
+//     per register by one byte permute, OR-ed into the unit's words, stored
+//     with vector stores. Codes never pass through shared memory.
+// Phase 1 flags a tile whose codes could leave [0, L], or that holds a
+// degenerate group; such a tile takes the clamping variant of phase 2.
 #include <algorithm>
 
+#include "format.cuh"
 #include "rq_internal.cuh"
 
 namespace rq {
@@ -30,23 +35,21 @@ constexpr int kThreads = 128;
 #ifndef RQ_QUANT_MIN_BLOCKS
 #define RQ_QUANT_MIN_BLOCKS 8
 #endif
-constexpr int kX16Stride = kD + 8;      // u16 per staged row (272 B: spreads banks)
-constexpr int kCStride = kD + 4;        // code tile [t][c], bytes per row
-constexpr int kCTStride = kTile + 4;    // transposed code tile [c][t], bytes per row
-constexpr int kCodeBytes = 4624;        // max(32 * 132, 128 * 36 + 4 * 4)
-// row c of the transposed tile starts at ct_row(c): rows 32 apart are skewed
-// by one bank so the four channel groups of a token store without conflicts
-__host__ __device__ constexpr int ct_row(int c) { return c * kCTStride + 4 * (c >> 5); }
-constexpr int kOutWords = 128 * 9;      // codes image (128 b words) + meta image (128 words)
+// staged tile row: 256 bytes of values + 64 bytes, so that rows 1 apart land
+// 16 banks apart (conflict-free 16-byte reads of neighbouring tokens)
+constexpr int kRowBytes = 320;
+constexpr int kTileBytes = kTile * kRowBytes;
+constexpr int kX32S = kD + 4;           // rotated fp32 row (floats)
 
-struct TileSmem {
-  uint16_t x16[kTile * kX16Stride];     // raw staged tile (column mode)
-  uint8_t codes[kCodeBytes];            // code tile (K: [t][c], V: [c][t])
-  uint32_t out[kOutWords];              // packed block image
+enum { kModeKC = 0, kModeKT = 1, kModeVT = 2, kModeVC = 3 };
+
+struct QSmem {
+  uint8_t tile[2][kTileBytes];
+  float nz[kD];                 // -zero of every group (channel c, or 32 G + t)
+  float inv[kD];                // 1 / scale (0 for a group without codes)
+  uint2 xchg[kThreads];         // per-channel min/max of half the tokens
   int8_t signs[kD];
 };
-// a rotated per-channel tile needs the rotated fp32 values in shared memory
-constexpr int kX32Floats = kTile * (kD + 1);
 
 struct QuantArgs {
   const void* k;
@@ -69,6 +72,8 @@ struct CalibArgs {
   long long ntiles;
 };
 
+// ------------------------------------------------------------- helpers ----
+
 __device__ __forceinline__ float fmin_nan(float a, float b) {
   float r;
   asm("min.NaN.f32 %0, %1, %2;" : "=f"(r) : "f"(a), "f"(b));
@@ -79,300 +84,65 @@ __device__ __forceinline__ float fmax_nan(float a, float b) {
   asm("max.NaN.f32 %0, %1, %2;" : "=f"(r) : "f"(a), "f"(b));
   return r;
 }
-// round to nearest even and saturate to [0, 255] in one conversion
-__device__ __forceinline__ uint32_t cvt_rni_sat_u8(float x) {
+
+// NaN-propagating min / max of two packed 16-bit pairs
+template <typename T>
+__device__ __forceinline__ uint32_t min2_nan(uint32_t a, uint32_t b);
+template <typename T>
+__device__ __forceinline__ uint32_t max2_nan(uint32_t a, uint32_t b);
+template <>
+__device__ __forceinline__ uint32_t min2_nan<__nv_bfloat16>(uint32_t a, uint32_t b) {
   uint32_t r;
-  asm("cvt.rni.sat.u8.f32 %0, %1;" : "=r"(r) : "f"(x));
+  asm("min.NaN.bf16x2 %0, %1, %2;" : "=r"(r) : "r"(a), "r"(b));
+  return r;
+}
+template <>
+__device__ __forceinline__ uint32_t max2_nan<__nv_bfloat16>(uint32_t a, uint32_t b) {
+  uint32_t r;
+  asm("max.NaN.bf16x2 %0, %1, %2;" : "=r"(r) : "r"(a), "r"(b));
+  return r;
+}
+template <>
+__device__ __forceinline__ uint32_t min2_nan<__half>(uint32_t a, uint32_t b) {
+  uint32_t r;
+  asm("min.NaN.f16x2 %0, %1, %2;" : "=r"(r) : "r"(a), "r"(b));
+  return r;
+}
+template <>
+__device__ __forceinline__ uint32_t max2_nan<__half>(uint32_t a, uint32_t b) {
+  uint32_t r;
+  asm("max.NaN.f16x2 %0, %1, %2;" : "=r"(r) : "r"(a), "r"(b));
   return r;
 }
 
-// ------------------------------------------------------------- loading ----
-
-// Row mode (per-token groups, or any rotated tile): thread 4t + G holds the
-// 64 bytes of token t, channels 32G..32G+31. Column mode: thread tau holds
-// 16-byte chunks tau + 128 i of the tile (coalesced).
+// the low / high 16-bit value of a packed pair as fp32 (exact)
 template <typename T>
-__device__ __forceinline__ void load_tile(const T* tile_base, bool row_mode, uint4 (&ld)[4]) {
-  const uint4* src = row_mode
-      ? reinterpret_cast<const uint4*>(tile_base + (threadIdx.x >> 2) * kD + 32 * (threadIdx.x & 3))
-      : reinterpret_cast<const uint4*>(tile_base) + threadIdx.x;
-  const int stride = row_mode ? 1 : kThreads;
-#pragma unroll
-  for (int i = 0; i < 4; ++i) ld[i] = ldg_stream(src + i * stride);
-}
-
-// The 32 values of this thread's group, in the quantizer's domain, in
-// registers (rotated when `hadamard`). Ends with every thread's group ready;
-// contains __syncthreads (call uniformly).
+__device__ __forceinline__ float lo_f32(uint32_t w);
 template <typename T>
-__device__ __forceinline__ void group_values(const uint4 (&ld)[4], bool row_mode, int grouping,
-                                             bool hadamard, TileSmem& sm, float* x32,
-                                             float (&v)[kG]) {
-  const int tau = threadIdx.x;
-  if (row_mode) {
-#pragma unroll
-    for (int i = 0; i < 4; ++i) {
-      float f[8];
-      unpack8<T>(ld[i], f);
-#pragma unroll
-      for (int e = 0; e < 8; ++e) v[8 * i + e] = f[e];
-    }
-    if (hadamard) {
-      const int G = tau & 3;
-#pragma unroll
-      for (int i = 0; i < kG; ++i)
-        if (sm.signs[32 * G + i] < 0) v[i] = -v[i];
-      // butterflies of stride 1..16 inside the group, in order
-#pragma unroll
-      for (int h = 1; h < kG; h <<= 1) {
-#pragma unroll
-        for (int i = 0; i < kG; ++i) {
-          if (i & h) continue;
-          const float a = v[i], b = v[i + h];
-          v[i] = __fadd_rn(a, b);
-          v[i + h] = __fsub_rn(a, b);
-        }
-      }
-      // strides 32 and 64 pair this group with the lanes holding G^1, G^2;
-      // the lower channel gets a + b, the upper a - b (a = lower's value)
-#pragma unroll
-      for (int s = 1; s <= 2; s <<= 1) {
-        const bool upper = (G & s) != 0;
-#pragma unroll
-        for (int i = 0; i < kG; ++i) {
-          const float o = __shfl_xor_sync(0xffffffffu, v[i], s);
-          v[i] = upper ? __fsub_rn(o, v[i]) : __fadd_rn(v[i], o);
-        }
-      }
-#pragma unroll
-      for (int i = 0; i < kG; ++i) v[i] = __fmul_rn(v[i], kInvSqrt128);
-      if (grouping == RQ_PER_CHANNEL) {       // regroup the rotated tile by column
-        const int t = tau >> 2;
-#pragma unroll
-        for (int i = 0; i < kG; ++i) x32[t * (kD + 1) + 32 * G + i] = v[i];
-        __syncthreads();
-#pragma unroll
-        for (int i = 0; i < kG; ++i) v[i] = x32[i * (kD + 1) + tau];
-      }
-    }
-  } else {
-#pragma unroll
-    for (int i = 0; i < 4; ++i) {
-      const int ch = tau + kThreads * i;
-      *reinterpret_cast<uint4*>(&sm.x16[(ch >> 4) * kX16Stride + (ch & 15) * 8]) = ld[i];
-    }
-    __syncthreads();
-#pragma unroll
-    for (int i = 0; i < kG; ++i) {
-      const uint16_t raw = sm.x16[i * kX16Stride + tau];
-      v[i] = to_f32<T>(*reinterpret_cast<const T*>(&raw));
-    }
-  }
+__device__ __forceinline__ float hi_f32(uint32_t w);
+template <>
+__device__ __forceinline__ float lo_f32<__nv_bfloat16>(uint32_t w) { return __uint_as_float(w << 16); }
+template <>
+__device__ __forceinline__ float hi_f32<__nv_bfloat16>(uint32_t w) {
+  return __uint_as_float(w & 0xFFFF0000u);
+}
+template <>
+__device__ __forceinline__ float lo_f32<__half>(uint32_t w) {
+  return __half2float(__ushort_as_half(static_cast<unsigned short>(w & 0xFFFFu)));
+}
+template <>
+__device__ __forceinline__ float hi_f32<__half>(uint32_t w) {
+  return __half2float(__ushort_as_half(static_cast<unsigned short>(w >> 16)));
 }
 
-// min / max of the group; NaN propagates so a non-finite group is detected
-__device__ __forceinline__ void group_minmax(const float (&v)[kG], float& mn, float& mx,
-                                             bool& finite) {
-  float lo[16], hi[16];
-#pragma unroll
-  for (int i = 0; i < 16; ++i) {
-    lo[i] = fmin_nan(v[2 * i], v[2 * i + 1]);
-    hi[i] = fmax_nan(v[2 * i], v[2 * i + 1]);
-  }
-#pragma unroll
-  for (int w = 8; w >= 1; w >>= 1)
-#pragma unroll
-    for (int i = 0; i < w; ++i) {
-      lo[i] = fmin_nan(lo[i], lo[i + w]);
-      hi[i] = fmax_nan(hi[i], hi[i + w]);
-    }
-  mn = __fadd_rn(lo[0], 0.0f);   // -0 -> +0
-  mx = __fadd_rn(hi[0], 0.0f);
-  finite = isfinite(mn) && isfinite(mx);
+__device__ __forceinline__ uint32_t smem_u32(const void* p) {
+  return static_cast<uint32_t>(__cvta_generic_to_shared(p));
 }
-
-// codes c_i = clamp(rint((v_i - zero) * inv), 0, L); a group without codes
-// (bad, or scale 0) has inv = 0 and yields 0 everywhere
-__device__ __forceinline__ void group_codes(const float (&v)[kG], const GroupParams& g, int b,
-                                            uint32_t (&c)[kG]) {
-  const float2 nz = make_float2(-g.zf, -g.zf);
-  const float2 iv = make_float2(g.inv, g.inv);
-  const uint32_t L = (1u << b) - 1u;
-#pragma unroll
-  for (int i = 0; i < kG; i += 2) {
-    const float2 t = __fmul2_rn(__fadd2_rn(make_float2(v[i], v[i + 1]), nz), iv);
-    c[i] = min(cvt_rni_sat_u8(t.x), L);
-    c[i + 1] = min(cvt_rni_sat_u8(t.y), L);
-  }
+__device__ __forceinline__ void cp_async16(uint32_t dst, const void* src) {
+  asm volatile("cp.async.cg.shared.global [%0], [%1], 16;\n" ::"r"(dst), "l"(src));
 }
-
-// ------------------------------------------------------------- packing ----
-
-// Fragment slot layout (the packed block format): fragment phi of lane L
-// holds 8 codes in slots a0 a2 a4 a6 a1 a3 a5 a7, b bits each, LSB first.
-// Pair k = (a_2k, a_2k+1) sits at adjacent bytes of the code tile (K: same
-// token, channels c and c+1; V: same channel, tokens t and t+1, transposed tile).
-template <int B>
-__device__ __forceinline__ void put_bits(uint32_t (&w)[B], int pos, uint32_t x) {
-  const int wi = pos >> 5, sh = pos & 31;
-  w[wi] |= x << sh;
-  if (sh + B > 32) w[wi + 1] |= x >> (32 - sh);
-}
-
-template <int B>
-__device__ __forceinline__ void place_fragment(uint32_t (&w)[B], int f, const uint32_t (&p)[4]) {
-  if constexpr (B == 2) {          // p << 2k puts lo at 2k and hi at 8 + 2k
-    const uint32_t frag = p[0] | (p[1] << 2) | (p[2] << 4) | (p[3] << 6);
-    w[f >> 1] |= frag << (16 * (f & 1));
-  } else if constexpr (B == 4) {   // spread bytes to half-words, then << 4k
-    uint32_t frag = 0;
-#pragma unroll
-    for (int k = 0; k < 4; ++k) frag |= __byte_perm(p[k], 0u, 0x4140) << (4 * k);
-    w[f] = frag;
-  } else if constexpr (B == 8) {   // lo bytes -> word 2f, hi bytes -> word 2f+1
-    const uint32_t a = __byte_perm(p[0], p[1], 0x5140);
-    const uint32_t b = __byte_perm(p[2], p[3], 0x5140);
-    w[2 * f] = __byte_perm(a, b, 0x5410);
-    w[2 * f + 1] = __byte_perm(a, b, 0x7632);
-  } else {
-#pragma unroll
-    for (int k = 0; k < 4; ++k) {
-      put_bits<B>(w, 8 * B * f + B * k, p[k] & 0xFFu);
-      put_bits<B>(w, 8 * B * f + 4 * B + B * k, p[k] >> 8);
-    }
-  }
-}
-
-// Thread (lane L = tau % 32, quarter q = tau / 32) writes lane-stream words
-// [B q, B q + B) of lane L: fragments 4q .. 4q+3.
-template <int KIND, int B>
-__device__ __forceinline__ void pack_codes(const uint8_t* codes, uint32_t* out) {
-  const int L = threadIdx.x & 31, q = threadIdx.x >> 5, gid = L >> 2, tig = L & 3;
-  uint32_t w[B];
-#pragma unroll
-  for (int i = 0; i < B; ++i) w[i] = 0;
-#pragma unroll
-  for (int f = 0; f < 4; ++f) {
-    uint32_t p[4];
-#pragma unroll
-    for (int k = 0; k < 4; ++k) {
-      if (KIND == 0) {    // K: token 16 mt + gid + 8 (k&1), channel 16 ks + 2 tig + 8 (k>>1)
-        const int t = 16 * (f & 1) + gid + 8 * (k & 1);
-        const int c = 16 * (2 * q + (f >> 1)) + 2 * tig + 8 * (k >> 1);
-        p[k] = *reinterpret_cast<const uint16_t*>(codes + t * kCStride + c);
-      } else {            // V: channel 16 mt + gid + 8 (k&1), token 16 ks + 2 tig + 8 (k>>1)
-        const int c = 16 * (4 * (q & 1) + f) + gid + 8 * (k & 1);
-        const int t = 16 * (q >> 1) + 2 * tig + 8 * (k >> 1);
-        p[k] = *reinterpret_cast<const uint16_t*>(codes + ct_row(c) + t);
-      }
-    }
-    place_fragment<B>(w, f, p);
-  }
-#pragma unroll
-  for (int i = 0; i < B; ++i) {
-    const int ws = B * q + i;
-    out[128 * (ws >> 2) + 4 * L + (ws & 3)] = w[i];
-  }
-}
-
-template <int KIND>
-__device__ __forceinline__ void pack_dispatch(int b, const uint8_t* codes, uint32_t* out) {
-  switch (b) {
-    case 1: pack_codes<KIND, 1>(codes, out); break;
-    case 2: pack_codes<KIND, 2>(codes, out); break;
-    case 3: pack_codes<KIND, 3>(codes, out); break;
-    case 4: pack_codes<KIND, 4>(codes, out); break;
-    case 5: pack_codes<KIND, 5>(codes, out); break;
-    case 6: pack_codes<KIND, 6>(codes, out); break;
-    case 7: pack_codes<KIND, 7>(codes, out); break;
-    default: pack_codes<KIND, 8>(codes, out); break;
-  }
-}
-
-__device__ __forceinline__ void put_meta_half(uint32_t* meta, int word, int half, __half x) {
-  reinterpret_cast<__half*>(meta)[2 * word + half] = x;
-}
-
-// Quantize this thread's group and write its codes into the code tile and
-// its (scale, zero) into the meta image, at the positions of the packed block
-// format; codes are stored as they are produced (no code array stays live).
-__device__ __forceinline__ void quantize_store_group(TileSmem& sm, int kind, int grouping, int b,
-                                                     const float (&v)[kG], float mx,
-                                                     const GroupParams& g) {
-  const int tau = threadIdx.x;
-  uint32_t* meta = sm.out + 128 * b;
-  const float2 nz = make_float2(-g.zf, -g.zf);
-  const float2 iv = make_float2(g.inv, g.inv);
-  const uint32_t L = (1u << b) - 1u;
-  // (v - zero) * inv is monotone in v, so the group max gives the largest
-  // code; when no group of the warp exceeds L the upper clamp is skipped
-  // (the saturating conversion already clamps at 0 and 255)
-  const uint32_t cmax = cvt_rni_sat_u8(__fmul_rn(__fsub_rn(mx, g.zf), g.inv));
-  const bool clamp = __any_sync(0xffffffffu, cmax > L);
-  auto code2 = [&](int i, uint32_t& c0, uint32_t& c1) {
-    const float2 t = __fmul2_rn(__fadd2_rn(make_float2(v[i], v[i + 1]), nz), iv);
-    c0 = cvt_rni_sat_u8(t.x);
-    c1 = cvt_rni_sat_u8(t.y);
-    if (clamp) {
-      c0 = min(c0, L);
-      c1 = min(c1, L);
-    }
-  };
-  if (grouping == RQ_PER_CHANNEL) {              // group = channel tau, tokens 0..31
-    const int ch = tau;
-    if (kind == 0) {
-#pragma unroll
-      for (int t = 0; t < kG; t += 2) {
-        uint32_t c0, c1;
-        code2(t, c0, c1);
-        sm.codes[t * kCStride + ch] = static_cast<uint8_t>(c0);
-        sm.codes[(t + 1) * kCStride + ch] = static_cast<uint8_t>(c1);
-      }
-      const int word = 16 * ((ch & 7) >> 1) + 2 * (ch >> 4) + ((ch >> 3) & 1);
-      put_meta_half(meta, word, ch & 1, g.scale);
-      put_meta_half(meta, 64 + word, ch & 1, g.zero);
-    } else {
-#pragma unroll
-      for (int t = 0; t < kG; t += 4) {
-        uint32_t c0, c1, c2, c3;
-        code2(t, c0, c1);
-        code2(t + 2, c2, c3);
-        *reinterpret_cast<uint32_t*>(&sm.codes[ct_row(ch) + t]) =
-            c0 | (c1 << 8) | (c2 << 16) | (c3 << 24);
-      }
-      const int word = 16 * (ch & 7) + 2 * (ch >> 4) + ((ch >> 3) & 1);
-      put_meta_half(meta, word, 0, g.scale);
-      put_meta_half(meta, word, 1, g.zero);
-    }
-  } else {                                        // group = (token t, channels 32G..)
-    const int t = tau >> 2, G = tau & 3;
-    if (kind == 0) {
-#pragma unroll
-      for (int i = 0; i < kG; i += 4) {
-        uint32_t c0, c1, c2, c3;
-        code2(i, c0, c1);
-        code2(i + 2, c2, c3);
-        *reinterpret_cast<uint32_t*>(&sm.codes[t * kCStride + 32 * G + i]) =
-            c0 | (c1 << 8) | (c2 << 16) | (c3 << 24);
-      }
-      const int word = 16 * (t & 7) + 4 * (t >> 3) + G;
-      put_meta_half(meta, word, 0, g.scale);
-      put_meta_half(meta, word, 1, g.zero);
-    } else {
-#pragma unroll
-      for (int i = 0; i < kG; i += 2) {
-        uint32_t c0, c1;
-        code2(i, c0, c1);
-        sm.codes[ct_row(32 * G + i) + t] = static_cast<uint8_t>(c0);
-        sm.codes[ct_row(32 * G + i + 1) + t] = static_cast<uint8_t>(c1);
-      }
-      const int p = t >> 1;
-      const int word = 16 * (p & 3) + 4 * (p >> 2) + G;
-      put_meta_half(meta, word, t & 1, g.scale);
-      put_meta_half(meta, 64 + word, t & 1, g.zero);
-    }
-  }
-}
+__device__ __forceinline__ void cp_async_commit() { asm volatile("cp.async.commit_group;\n" ::); }
+__device__ __forceinline__ void cp_async_wait_all() { asm volatile("cp.async.wait_group 0;\n" ::); }
 
 // Tile position: block j of stream sk = (batch * H + h) * 2 + kind. A CTA
 // walks tiles blockIdx.x, blockIdx.x + gridDim.x, ...; the position is
@@ -396,63 +166,468 @@ __device__ __forceinline__ const T* quant_tile_base(const QuantArgs& a, const Ti
   return base + (static_cast<long long>(r.sk >> 1) * a.S + static_cast<long long>(kTile) * r.j) * kD;
 }
 
+// the 8 KB tile into a staging buffer: thread tau copies 16-byte chunks
+// tau + 128 i (row = chunk / 16)
+__device__ __forceinline__ void issue_tile(uint8_t* buf, const void* src) {
+  const uint32_t dst = smem_u32(buf);
+  const uint8_t* s = static_cast<const uint8_t*>(src);
+#pragma unroll
+  for (int i = 0; i < 4; ++i) {
+    const int ch = threadIdx.x + kThreads * i;
+    cp_async16(dst + (ch >> 4) * kRowBytes + 16 * (ch & 15), s + 16 * ch);
+  }
+}
+
+// ------------------------------------------------------------- phase 1 ----
+
+struct GroupOut {
+  bool slow, bad;
+};
+
+// Scale/zero of one group: meta words to global memory (packed format),
+// (-zero, 1/scale) to the table. `slow`: no codes (bad or zero range) or
+// codes that could fall outside [0, L] (they are monotone in v, so the
+// group's min and max bound them).
+__device__ __forceinline__ GroupOut finish_group(int kind, int grouping, int t, int G, int c,
+                                                 float mn, float mx, bool finite, int b,
+                                                 uint8_t* meta, QSmem& sm) {
+  const GroupParams g = group_params(mn, mx, finite, b);
+  const uint32_t sb = __half_as_ushort(g.scale), zb = __half_as_ushort(g.zero);
+  uint16_t* m16 = reinterpret_cast<uint16_t*>(meta);
+  uint32_t* m32 = reinterpret_cast<uint32_t*>(meta);
+  int slot;
+  if (grouping == RQ_PER_CHANNEL) {
+    slot = c;
+    if (kind == 0) {                          // scale / zero pairs of channels (c, c^1)
+      m16[c] = static_cast<uint16_t>(sb);
+      m16[128 + c] = static_cast<uint16_t>(zb);
+    } else {
+      m32[c] = sb | (zb << 16);
+    }
+  } else {
+    slot = 32 * G + t;
+    if (kind == 0) {
+      m32[16 * (t & 7) + 4 * G + (t >> 3)] = sb | (zb << 16);
+    } else {                                  // scale / zero pairs of tokens (t, t^1)
+      const int i = 2 * (4 * (t >> 1) + G) + (t & 1);
+      m16[i] = static_cast<uint16_t>(sb);
+      m16[128 + i] = static_cast<uint16_t>(zb);
+    }
+  }
+  sm.nz[slot] = -g.zf;
+  sm.inv[slot] = g.inv;
+  GroupOut o;
+  o.bad = g.bad;
+  if (!g.ok) {
+    o.slow = true;
+    return o;
+  }
+  const float L = static_cast<float>((1 << b) - 1);
+  const float um = __fmaf_rn(__fsub_rn(mn, g.zf), g.inv, kRoundMagic);
+  const float uM = __fmaf_rn(__fsub_rn(mx, g.zf), g.inv, kRoundMagic);
+  o.slow = um < kRoundMagic || uM > kRoundMagic + L;
+  return o;
+}
+
+// Per-channel groups on the raw tile: thread (pair p, token half hv) takes
+// channels 2p, 2p+1 over tokens 16 hv .. 16 hv + 15, the two halves meet
+// through shared memory, and the thread finishes channel 2p + hv.
 template <typename T>
+__device__ __forceinline__ GroupOut phase1_cols(const uint8_t* tile, int kind, int b,
+                                                uint8_t* meta, QSmem& sm) {
+  const int tau = threadIdx.x, p = tau & 63, hv = tau >> 6;
+  const uint8_t* col = tile + 4 * p + hv * 16 * kRowBytes;
+  uint32_t mn2 = *reinterpret_cast<const uint32_t*>(col), mx2 = mn2;
+#pragma unroll
+  for (int i = 1; i < 16; ++i) {
+    const uint32_t x = *reinterpret_cast<const uint32_t*>(col + i * kRowBytes);
+    mn2 = min2_nan<T>(mn2, x);
+    mx2 = max2_nan<T>(mx2, x);
+  }
+  sm.xchg[tau] = make_uint2(mn2, mx2);
+  __syncthreads();
+  const uint2 o = sm.xchg[tau ^ 64];
+  mn2 = min2_nan<T>(mn2, o.x);
+  mx2 = max2_nan<T>(mx2, o.y);
+  float mn = hv ? hi_f32<T>(mn2) : lo_f32<T>(mn2);
+  float mx = hv ? hi_f32<T>(mx2) : lo_f32<T>(mx2);
+  const bool finite = isfinite(mn) && isfinite(mx);
+  mn = __fadd_rn(mn, 0.0f);     // -0 -> +0
+  mx = __fadd_rn(mx, 0.0f);
+  return finish_group(kind, RQ_PER_CHANNEL, 0, 0, 2 * p + hv, mn, mx, finite, b, meta, sm);
+}
+
+// Per-token groups on the raw tile: thread 4 t + G takes token t, channels
+// 32 G .. 32 G + 31 (four 16-byte reads, started at a rotating chunk so the
+// eight threads of a read phase hit distinct banks).
+template <typename T>
+__device__ __forceinline__ GroupOut phase1_rows(const uint8_t* tile, int kind, int b,
+                                                uint8_t* meta, QSmem& sm) {
+  const int tau = threadIdx.x, t = tau >> 2, G = tau & 3;
+  const uint8_t* row = tile + t * kRowBytes + 64 * G;
+  uint32_t w[16];
+#pragma unroll
+  for (int i = 0; i < 4; ++i) {
+    const uint4 u = *reinterpret_cast<const uint4*>(row + 16 * ((i + (t >> 1)) & 3));
+    w[4 * i] = u.x;
+    w[4 * i + 1] = u.y;
+    w[4 * i + 2] = u.z;
+    w[4 * i + 3] = u.w;
+  }
+  uint32_t lo[8], hi[8];
+#pragma unroll
+  for (int i = 0; i < 8; ++i) {
+    lo[i] = min2_nan<T>(w[2 * i], w[2 * i + 1]);
+    hi[i] = max2_nan<T>(w[2 * i], w[2 * i + 1]);
+  }
+#pragma unroll
+  for (int s = 4; s >= 1; s >>= 1)
+#pragma unroll
+    for (int i = 0; i < s; ++i) {
+      lo[i] = min2_nan<T>(lo[i], lo[i + s]);
+      hi[i] = max2_nan<T>(hi[i], hi[i + s]);
+    }
+  float mn = fmin_nan(lo_f32<T>(lo[0]), hi_f32<T>(lo[0]));
+  float mx = fmax_nan(lo_f32<T>(hi[0]), hi_f32<T>(hi[0]));
+  const bool finite = isfinite(mn) && isfinite(mx);
+  mn = __fadd_rn(mn, 0.0f);
+  mx = __fadd_rn(mx, 0.0f);
+  return finish_group(kind, RQ_PER_TOKEN, t, G, 0, mn, mx, finite, b, meta, sm);
+}
+
+// min / max of 32 fp32 values; NaN propagates
+__device__ __forceinline__ void minmax32(const float (&v)[kG], float& mn, float& mx) {
+  float lo[16], hi[16];
+#pragma unroll
+  for (int i = 0; i < 16; ++i) {
+    lo[i] = fmin_nan(v[2 * i], v[2 * i + 1]);
+    hi[i] = fmax_nan(v[2 * i], v[2 * i + 1]);
+  }
+#pragma unroll
+  for (int w = 8; w >= 1; w >>= 1)
+#pragma unroll
+    for (int i = 0; i < w; ++i) {
+      lo[i] = fmin_nan(lo[i], lo[i + w]);
+      hi[i] = fmax_nan(hi[i], hi[i + w]);
+    }
+  mn = lo[0];
+  mx = hi[0];
+}
+
+// y = FWHT(x * sigma) / sqrt(128) of token t's channels 32 G .. 32 G + 31
+// held by thread 4 t + G: butterflies of stride 1..16 in registers, strides
+// 32 and 64 with the lanes holding G ^ 1, G ^ 2 (the lower channel of a
+// pair takes a + b, the upper a - b), in that order.
+__device__ __forceinline__ void rotate_group(float (&v)[kG], int G, const int8_t* signs) {
+#pragma unroll
+  for (int i = 0; i < kG; ++i)
+    if (signs[32 * G + i] < 0) v[i] = -v[i];
+#pragma unroll
+  for (int h = 1; h < kG; h <<= 1) {
+#pragma unroll
+    for (int i = 0; i < kG; ++i) {
+      if (i & h) continue;
+      const float a = v[i], b = v[i + h];
+      v[i] = __fadd_rn(a, b);
+      v[i + h] = __fsub_rn(a, b);
+    }
+  }
+#pragma unroll
+  for (int s = 1; s <= 2; s <<= 1) {
+    const bool upper = (G & s) != 0;
+#pragma unroll
+    for (int i = 0; i < kG; ++i) {
+      const float o = __shfl_xor_sync(0xffffffffu, v[i], s);
+      v[i] = upper ? __fsub_rn(o, v[i]) : __fadd_rn(v[i], o);
+    }
+  }
+#pragma unroll
+  for (int i = 0; i < kG; ++i) v[i] = __fmul_rn(v[i], kInvSqrt128);
+}
+
+// Rotated tiles: every thread rotates one 32-channel quarter of a token and
+// writes it to the fp32 tile x32; groups are then formed on x32.
+template <typename T>
+__device__ __forceinline__ GroupOut phase1_rotated(const uint8_t* tile, float* x32, int kind,
+                                                   int grouping, int b, uint8_t* meta,
+                                                   QSmem& sm) {
+  const int tau = threadIdx.x, t = tau >> 2, G = tau & 3;
+  float v[kG];
+  const uint8_t* row = tile + t * kRowBytes + 64 * G;
+#pragma unroll
+  for (int i = 0; i < 4; ++i) {
+    const uint4 u = *reinterpret_cast<const uint4*>(row + 16 * i);
+    const uint32_t w[4] = {u.x, u.y, u.z, u.w};
+#pragma unroll
+    for (int e = 0; e < 4; ++e) {
+      v[8 * i + 2 * e] = lo_f32<T>(w[e]);
+      v[8 * i + 2 * e + 1] = hi_f32<T>(w[e]);
+    }
+  }
+  rotate_group(v, G, sm.signs);
+  float* xr = x32 + t * kX32S + 32 * G;
+#pragma unroll
+  for (int i = 0; i < kG; i += 4)
+    *reinterpret_cast<float4*>(xr + i) = make_float4(v[i], v[i + 1], v[i + 2], v[i + 3]);
+  if (grouping == RQ_PER_TOKEN) {
+    float mn, mx;
+    minmax32(v, mn, mx);
+    const bool finite = isfinite(mn) && isfinite(mx);
+    return finish_group(kind, RQ_PER_TOKEN, t, G, 0, __fadd_rn(mn, 0.0f), __fadd_rn(mx, 0.0f),
+                        finite, b, meta, sm);
+  }
+  __syncthreads();
+  const int p = tau & 63, hv = tau >> 6;
+  const float* col = x32 + 16 * hv * kX32S + 2 * p;
+  float2 lo = *reinterpret_cast<const float2*>(col), hi = lo;
+#pragma unroll
+  for (int i = 1; i < 16; ++i) {
+    const float2 x = *reinterpret_cast<const float2*>(col + i * kX32S);
+    lo = make_float2(fmin_nan(lo.x, x.x), fmin_nan(lo.y, x.y));
+    hi = make_float2(fmax_nan(hi.x, x.x), fmax_nan(hi.y, x.y));
+  }
+  const float mnh = hv ? lo.y : lo.x, mxh = hv ? hi.y : hi.x;
+  sm.xchg[tau] = make_uint2(__float_as_uint(hv ? lo.x : lo.y), __float_as_uint(hv ? hi.x : hi.y));
+  __syncthreads();
+  // the partner (other token half) left this thread's channel in xchg
+  const uint2 o = sm.xchg[tau ^ 64];
+  const float mn = fmin_nan(mnh, __uint_as_float(o.x));
+  const float mx = fmax_nan(mxh, __uint_as_float(o.y));
+  const bool finite = isfinite(mn) && isfinite(mx);
+  return finish_group(kind, RQ_PER_CHANNEL, 0, 0, 2 * p + hv, __fadd_rn(mn, 0.0f),
+                      __fadd_rn(mx, 0.0f), finite, b, meta, sm);
+}
+
+// ------------------------------------------------------------- phase 2 ----
+
+// four channel pairs (c .. c + 7) of token t as fp32 pairs
+template <typename T, bool F32>
+__device__ __forceinline__ void load_pairs(const uint8_t* tile, const float* x32, int t, int c,
+                                           float2 (&v)[4]) {
+  if constexpr (F32) {
+    const float4 a = *reinterpret_cast<const float4*>(x32 + t * kX32S + c);
+    const float4 b = *reinterpret_cast<const float4*>(x32 + t * kX32S + c + 4);
+    v[0] = make_float2(a.x, a.y);
+    v[1] = make_float2(a.z, a.w);
+    v[2] = make_float2(b.x, b.y);
+    v[3] = make_float2(b.z, b.w);
+  } else {
+    const uint4 u = *reinterpret_cast<const uint4*>(tile + t * kRowBytes + 2 * c);
+    v[0] = make_float2(lo_f32<T>(u.x), hi_f32<T>(u.x));
+    v[1] = make_float2(lo_f32<T>(u.y), hi_f32<T>(u.y));
+    v[2] = make_float2(lo_f32<T>(u.z), hi_f32<T>(u.z));
+    v[3] = make_float2(lo_f32<T>(u.w), hi_f32<T>(u.w));
+  }
+}
+
+// four channels (c .. c + 3) of token t as fp32
+template <typename T, bool F32>
+__device__ __forceinline__ void load_quad(const uint8_t* tile, const float* x32, int t, int c,
+                                          float (&v)[4]) {
+  if constexpr (F32) {
+    const float4 a = *reinterpret_cast<const float4*>(x32 + t * kX32S + c);
+    v[0] = a.x;
+    v[1] = a.y;
+    v[2] = a.z;
+    v[3] = a.w;
+  } else {
+    const uint2 u = *reinterpret_cast<const uint2*>(tile + t * kRowBytes + 2 * c);
+    v[0] = lo_f32<T>(u.x);
+    v[1] = hi_f32<T>(u.x);
+    v[2] = lo_f32<T>(u.y);
+    v[3] = hi_f32<T>(u.y);
+  }
+}
+
+// codes of register (x, y) from its two values: RN(fp32(v - zero) * inv +
+// magic) has the code in its low byte (and 0 in the next) when in range
+template <int B, bool CLAMP>
+__device__ __forceinline__ void emit(uint32_t (&uw)[B], int x, int y, float2 v, float2 nz,
+                                     float2 iv) {
+  const float2 d = __fadd2_rn(v, nz);
+  float2 q = __ffma2_rn(d, iv, make_float2(kRoundMagic, kRoundMagic));
+  if constexpr (CLAMP) {
+    constexpr float top = kRoundMagic + static_cast<float>((1 << B) - 1);
+    q.x = fminf(fmaxf(q.x, kRoundMagic), top);
+    q.y = fminf(fmaxf(q.y, kRoundMagic), top);
+  }
+  fmt::place<B>(uw, x, y, __byte_perm(__float_as_uint(q.x), __float_as_uint(q.y), 0x5410u));
+}
+
+// Thread -> (lane gid/tig of the packed format, unit u). K: warp = unit,
+// lane = format lane. V: a half warp is (gid 0..7) x (two units), so the
+// 8-byte reads of one token row hit 16 distinct bank pairs.
+template <int MODE, typename T, int B, bool CLAMP, bool F32>
+__device__ __forceinline__ void phase2(const uint8_t* tile, const float* x32, const QSmem& sm,
+                                       uint32_t* blk) {
+  const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+  int gid, tig, u;
+  if (MODE == kModeKC || MODE == kModeKT) {
+    gid = lane >> 2;
+    tig = lane & 3;
+    u = warp;
+  } else {
+    gid = lane & 7;
+    u = 2 * (warp & 1) + ((lane >> 3) & 1);
+    tig = 2 * (warp >> 1) + (lane >> 4);
+  }
+  uint32_t uw[B];
+#pragma unroll
+  for (int i = 0; i < B; ++i) uw[i] = 0u;
+
+  if constexpr (MODE == kModeKC) {
+    // channels 32u + 8tig + 2x + h, token 8y + gid; group = channel
+    const int c = 32 * u + 8 * tig;
+    const float4 z0 = *reinterpret_cast<const float4*>(sm.nz + c);
+    const float4 z1 = *reinterpret_cast<const float4*>(sm.nz + c + 4);
+    const float4 i0 = *reinterpret_cast<const float4*>(sm.inv + c);
+    const float4 i1 = *reinterpret_cast<const float4*>(sm.inv + c + 4);
+    const float2 nz[4] = {make_float2(z0.x, z0.y), make_float2(z0.z, z0.w),
+                          make_float2(z1.x, z1.y), make_float2(z1.z, z1.w)};
+    const float2 iv[4] = {make_float2(i0.x, i0.y), make_float2(i0.z, i0.w),
+                          make_float2(i1.x, i1.y), make_float2(i1.z, i1.w)};
+#pragma unroll
+    for (int y = 0; y < 4; ++y) {
+      float2 v[4];
+      load_pairs<T, F32>(tile, x32, 8 * y + gid, c, v);
+#pragma unroll
+      for (int x = 0; x < 4; ++x) emit<B, CLAMP>(uw, x, y, v[x], nz[x], iv[x]);
+    }
+  } else if constexpr (MODE == kModeKT) {
+    // token 8x + gid, channels 32u + 8tig + 2y + h; group = (token, G = u)
+    const int c = 32 * u + 8 * tig;
+#pragma unroll
+    for (int x = 0; x < 4; ++x) {
+      const int t = 8 * x + gid;
+      const float z = sm.nz[32 * u + t], i = sm.inv[32 * u + t];
+      float2 v[4];
+      load_pairs<T, F32>(tile, x32, t, c, v);
+#pragma unroll
+      for (int y = 0; y < 4; ++y) emit<B, CLAMP>(uw, x, y, v[y], make_float2(z, z), make_float2(i, i));
+    }
+  } else {
+    // channel 32u + 4gid + x, tokens 8y + 2tig + h
+    const int c = 32 * u + 4 * gid;
+    float4 zc, ic;
+    if constexpr (MODE == kModeVC) {
+      zc = *reinterpret_cast<const float4*>(sm.nz + c);
+      ic = *reinterpret_cast<const float4*>(sm.inv + c);
+    }
+#pragma unroll
+    for (int y = 0; y < 4; ++y) {
+      const int t = 8 * y + 2 * tig;
+      float a[4], b[4];
+      load_quad<T, F32>(tile, x32, t, c, a);
+      load_quad<T, F32>(tile, x32, t + 1, c, b);
+      if constexpr (MODE == kModeVT) {
+        const float2 nz = *reinterpret_cast<const float2*>(sm.nz + 32 * u + t);
+        const float2 iv = *reinterpret_cast<const float2*>(sm.inv + 32 * u + t);
+#pragma unroll
+        for (int x = 0; x < 4; ++x) emit<B, CLAMP>(uw, x, y, make_float2(a[x], b[x]), nz, iv);
+      } else {
+        const float zz[4] = {zc.x, zc.y, zc.z, zc.w}, ii[4] = {ic.x, ic.y, ic.z, ic.w};
+#pragma unroll
+        for (int x = 0; x < 4; ++x)
+          emit<B, CLAMP>(uw, x, y, make_float2(a[x], b[x]), make_float2(zz[x], zz[x]),
+                         make_float2(ii[x], ii[x]));
+      }
+    }
+  }
+
+  // lane word w = B u + i of lane L lives at block word 128 (w / 4) + 4 L + w % 4
+  const int L = 4 * gid + tig;
+  if constexpr (B == 2) {
+    const int w = 2 * u;
+    *reinterpret_cast<uint2*>(blk + 128 * (w >> 2) + 4 * L + (w & 3)) = make_uint2(uw[0], uw[1]);
+  } else if constexpr (B == 4) {
+    *reinterpret_cast<uint4*>(blk + 128 * u + 4 * L) = make_uint4(uw[0], uw[1], uw[2], uw[3]);
+  } else if constexpr (B == 8) {
+    *reinterpret_cast<uint4*>(blk + 128 * (2 * u) + 4 * L) = make_uint4(uw[0], uw[1], uw[2], uw[3]);
+    *reinterpret_cast<uint4*>(blk + 128 * (2 * u + 1) + 4 * L) = make_uint4(uw[4], uw[5], uw[6], uw[7]);
+  } else {
+#pragma unroll
+    for (int i = 0; i < B; ++i) {
+      const int w = B * u + i;
+      blk[128 * (w >> 2) + 4 * L + (w & 3)] = uw[i];
+    }
+  }
+}
+
+template <typename T, bool CLAMP, bool F32>
+__device__ __forceinline__ void phase2_dispatch(int mode, int b, const uint8_t* tile,
+                                                const float* x32, const QSmem& sm, uint32_t* blk) {
+#define RQ_P2_WIDTHS(MODE)                                                          \
+  switch (b) {                                                                      \
+    case 1: phase2<MODE, T, 1, CLAMP, F32>(tile, x32, sm, blk); break;              \
+    case 2: phase2<MODE, T, 2, CLAMP, F32>(tile, x32, sm, blk); break;              \
+    case 3: phase2<MODE, T, 3, CLAMP, F32>(tile, x32, sm, blk); break;              \
+    case 4: phase2<MODE, T, 4, CLAMP, F32>(tile, x32, sm, blk); break;              \
+    case 5: phase2<MODE, T, 5, CLAMP, F32>(tile, x32, sm, blk); break;              \
+    case 6: phase2<MODE, T, 6, CLAMP, F32>(tile, x32, sm, blk); break;              \
+    case 7: phase2<MODE, T, 7, CLAMP, F32>(tile, x32, sm, blk); break;              \
+    default: phase2<MODE, T, 8, CLAMP, F32>(tile, x32, sm, blk); break;             \
+  }
+  switch (mode) {
+    case kModeKC: RQ_P2_WIDTHS(kModeKC) break;
+    case kModeKT: RQ_P2_WIDTHS(kModeKT) break;
+    case kModeVT: RQ_P2_WIDTHS(kModeVT) break;
+    default: RQ_P2_WIDTHS(kModeVC) break;
+  }
+#undef RQ_P2_WIDTHS
+}
+
+template <typename T, bool HAD>
 __global__ void __launch_bounds__(kThreads, RQ_QUANT_MIN_BLOCKS) quantize_pack_kernel(QuantArgs a) {
   extern __shared__ __align__(16) unsigned char smem_raw[];
-  TileSmem& sm = *reinterpret_cast<TileSmem*>(smem_raw);
-  float* x32 = reinterpret_cast<float*>(smem_raw + sizeof(TileSmem));
+  QSmem& sm = *reinterpret_cast<QSmem*>(smem_raw);
+  float* x32 = HAD ? reinterpret_cast<float*>(smem_raw + sizeof(QSmem)) : nullptr;
   const long long stride = gridDim.x;
   long long tile = blockIdx.x;
   if (tile >= a.ntiles) return;
-  if (threadIdx.x < kD) sm.signs[threadIdx.x] = a.signs ? a.signs[threadIdx.x] : int8_t(1);
-  __syncthreads();
-  const bool had = a.hadamard != 0;
+  if (HAD && threadIdx.x < kD) sm.signs[threadIdx.x] = a.signs ? a.signs[threadIdx.x] : int8_t(1);
 
   const int nblk = a.nblk;
   const int dsk = static_cast<int>(stride / nblk), dj = static_cast<int>(stride % nblk);
   TileRef r{static_cast<int>(tile % nblk), static_cast<int>(tile / nblk)};
-  int grouping = (r.sk & 1) ? a.vg : a.kg;
-  bool row_mode = grouping == RQ_PER_TOKEN || had;
-  uint4 ld[4];
-  load_tile<T>(quant_tile_base<T>(a, r), row_mode, ld);
+  issue_tile(sm.tile[0], quant_tile_base<T>(a, r));
+  cp_async_commit();
 
-  for (; tile < a.ntiles; tile += stride) {
+  for (int it = 0; tile < a.ntiles; tile += stride, ++it) {
     const TileRef cur = r;
-    const int kind = cur.sk & 1;
-    const int bh = cur.sk >> 1;
-    const int h = bh % a.H;
-    const int b = a.bits[(a.layer * a.H + h) * 2 + kind];
-    float v[kG];
-    group_values<T>(ld, row_mode, grouping, had, sm, x32, v);
-    // the next tile's loads fly while this one is quantized and packed
-    const int cur_grouping = grouping;
+    const uint8_t* buf = sm.tile[it & 1];
+    cp_async_wait_all();
+    __syncthreads();             // tile visible; every thread is past the previous tile
     if (tile + stride < a.ntiles) {
       advance(r, dj, dsk, nblk);
-      grouping = (r.sk & 1) ? a.vg : a.kg;
-      row_mode = grouping == RQ_PER_TOKEN || had;
-      load_tile<T>(quant_tile_base<T>(a, r), row_mode, ld);
+      issue_tile(sm.tile[(it + 1) & 1], quant_tile_base<T>(a, r));
     }
+    cp_async_commit();
+
+    const int kind = cur.sk & 1;
+    const int h = (cur.sk >> 1) % a.H;
+    const int b = a.bits[(a.layer * a.H + h) * 2 + kind];
     if (b < 1 || b > 8) {
       if (threadIdx.x == 0) set_status(a.status, RQ_STATUS_BAD_BITS);
-      __syncthreads();
       continue;
     }
-    float mn, mx;
-    bool finite;
-    group_minmax(v, mn, mx, finite);
-    const GroupParams g = group_params(mn, mx, finite, b);
-    if (g.bad) set_status(a.status, RQ_STATUS_NUMERIC);
-    quantize_store_group(sm, kind, cur_grouping, b, v, mx, g);
-    __syncthreads();
-    if (kind == 0) pack_dispatch<0>(b, sm.codes, sm.out);
-    else pack_dispatch<1>(b, sm.codes, sm.out);
-    __syncthreads();
+    const int grouping = kind ? a.vg : a.kg;
     // offsets[layer][batch][h][kind] = offsets[layer * B * H * 2 + sk]
     const uint64_t off = a.offsets[static_cast<long long>(a.layer) * a.B * a.H * 2 + cur.sk];
-    uint4* dst = reinterpret_cast<uint4*>(a.packed + off + static_cast<uint64_t>(cur.j) * 512u * (b + 1));
-    const uint4* src = reinterpret_cast<const uint4*>(sm.out);
-    for (int i = threadIdx.x; i < 32 * (b + 1); i += kThreads) dst[i] = src[i];
-    __syncthreads();
+    uint8_t* blk = a.packed + off + static_cast<uint64_t>(cur.j) * 512u * (b + 1);
+    uint8_t* meta = blk + 512 * b;
+
+    GroupOut g;
+    if constexpr (HAD) g = phase1_rotated<T>(buf, x32, kind, grouping, b, meta, sm);
+    else if (grouping == RQ_PER_CHANNEL) g = phase1_cols<T>(buf, kind, b, meta, sm);
+    else g = phase1_rows<T>(buf, kind, b, meta, sm);
+    if (g.bad) set_status(a.status, RQ_STATUS_NUMERIC);
+    const bool slow = __syncthreads_or(g.slow) != 0;
+
+    const int mode = kind == 0 ? (grouping == RQ_PER_CHANNEL ? kModeKC : kModeKT)
+                               : (grouping == RQ_PER_TOKEN ? kModeVT : kModeVC);
+    uint32_t* blk32 = reinterpret_cast<uint32_t*>(blk);
+    if (slow) phase2_dispatch<T, true, HAD>(mode, b, buf, x32, sm, blk32);
+    else phase2_dispatch<T, false, HAD>(mode, b, buf, x32, sm, blk32);
   }
 }
 
@@ -461,14 +636,73 @@ __global__ void __launch_bounds__(kThreads, RQ_QUANT_MIN_BLOCKS) quantize_pack_k
 // (y - y_hat)^2 with y_hat = fp32(fp32(c * scale) + zero). A group's 32
 // squared errors are summed in fp32 (two interleaved partial sums, fixed
 // order) and the per-group sums in fp64; per-tile partials are reduced in a
-// fixed order (deterministic).
+// fixed order (deterministic). One group per thread: per-token groups are
+// loaded as rows (thread 4 t + G), per-channel groups as columns of the
+// tile staged in shared memory.
+
+struct CalibSmem {
+  uint16_t x16[kTile * (kD + 8)];       // raw tile (column mode), rows 272 bytes apart
+  int8_t signs[kD];
+  double red[kThreads / 32][8];
+};
+constexpr int kX16Stride = kD + 8;
+
+template <typename T>
+__device__ __forceinline__ void calib_load(const T* tile_base, bool row_mode, uint4 (&ld)[4]) {
+  const uint4* src = row_mode
+      ? reinterpret_cast<const uint4*>(tile_base + (threadIdx.x >> 2) * kD + 32 * (threadIdx.x & 3))
+      : reinterpret_cast<const uint4*>(tile_base) + threadIdx.x;
+  const int stride = row_mode ? 1 : kThreads;
+#pragma unroll
+  for (int i = 0; i < 4; ++i) ld[i] = ldg_stream(src + i * stride);
+}
+
+// The 32 values of this thread's group in the quantizer's domain (rotated
+// when `hadamard`); contains __syncthreads (call uniformly).
+template <typename T>
+__device__ __forceinline__ void calib_group_values(const uint4 (&ld)[4], bool row_mode,
+                                                   int grouping, bool hadamard, CalibSmem& sm,
+                                                   float* x32, float (&v)[kG]) {
+  const int tau = threadIdx.x;
+  if (row_mode) {
+#pragma unroll
+    for (int i = 0; i < 4; ++i) {
+      float f[8];
+      unpack8<T>(ld[i], f);
+#pragma unroll
+      for (int e = 0; e < 8; ++e) v[8 * i + e] = f[e];
+    }
+    if (hadamard) {
+      rotate_group(v, tau & 3, sm.signs);
+      if (grouping == RQ_PER_CHANNEL) {       // regroup the rotated tile by column
+        const int t = tau >> 2, G = tau & 3;
+#pragma unroll
+        for (int i = 0; i < kG; ++i) x32[t * (kD + 1) + 32 * G + i] = v[i];
+        __syncthreads();
+#pragma unroll
+        for (int i = 0; i < kG; ++i) v[i] = x32[i * (kD + 1) + tau];
+      }
+    }
+  } else {
+#pragma unroll
+    for (int i = 0; i < 4; ++i) {
+      const int ch = tau + kThreads * i;
+      *reinterpret_cast<uint4*>(&sm.x16[(ch >> 4) * kX16Stride + (ch & 15) * 8]) = ld[i];
+    }
+    __syncthreads();
+#pragma unroll
+    for (int i = 0; i < kG; ++i) {
+      const uint16_t raw = sm.x16[i * kX16Stride + tau];
+      v[i] = to_f32<T>(*reinterpret_cast<const T*>(&raw));
+    }
+  }
+}
 
 template <typename T>
 __global__ void __launch_bounds__(kThreads) calib_sweep_kernel(CalibArgs a) {
   extern __shared__ __align__(16) unsigned char smem_raw[];
-  TileSmem& sm = *reinterpret_cast<TileSmem*>(smem_raw);
-  float* x32 = reinterpret_cast<float*>(smem_raw + sizeof(TileSmem));
-  __shared__ double red[kThreads / 32][8];
+  CalibSmem& sm = *reinterpret_cast<CalibSmem*>(smem_raw);
+  float* x32 = reinterpret_cast<float*>(smem_raw + sizeof(CalibSmem));
   const long long stride = gridDim.x;
   long long tile = blockIdx.x;
   if (tile >= a.ntiles) return;
@@ -481,32 +715,35 @@ __global__ void __launch_bounds__(kThreads) calib_sweep_kernel(CalibArgs a) {
   int grouping = (static_cast<int>(tile / a.ntile) & 1) ? a.vg : a.kg;
   bool row_mode = grouping == RQ_PER_TOKEN || had;
   uint4 ld[4];
-  load_tile<T>(xbase + tile * kTile * kD, row_mode, ld);
+  calib_load<T>(xbase + tile * kTile * kD, row_mode, ld);
   for (; tile < a.ntiles; tile += stride) {
     float v[kG];
-    group_values<T>(ld, row_mode, grouping, had, sm, x32, v);
+    calib_group_values<T>(ld, row_mode, grouping, had, sm, x32, v);
     const long long next = tile + stride;
     if (next < a.ntiles) {
       grouping = (static_cast<int>(next / a.ntile) & 1) ? a.vg : a.kg;
       row_mode = grouping == RQ_PER_TOKEN || had;
-      load_tile<T>(xbase + next * kTile * kD, row_mode, ld);
+      calib_load<T>(xbase + next * kTile * kD, row_mode, ld);
     }
     float mn, mx;
-    bool finite;
-    group_minmax(v, mn, mx, finite);
+    minmax32(v, mn, mx);
+    const bool finite = isfinite(mn) && isfinite(mx);
+    mn = __fadd_rn(mn, 0.0f);
+    mx = __fadd_rn(mx, 0.0f);
     double acc[8];
 #pragma unroll
     for (int b = 1; b <= 8; ++b) {
       const GroupParams g = group_params(mn, mx, finite, b);
       if (b == 1 && g.bad) set_status(a.status, RQ_STATUS_NUMERIC);
-      uint32_t c[kG];
-      group_codes(v, g, b, c);
+      const float L = static_cast<float>((1 << b) - 1);
       const float2 sf = make_float2(g.sf, g.sf), zf = make_float2(g.zf, g.zf);
       float2 s2 = make_float2(0.0f, 0.0f);
 #pragma unroll
       for (int i = 0; i < kG; i += 2) {
-        const float2 xh = __fadd2_rn(
-            __fmul2_rn(make_float2(static_cast<float>(c[i]), static_cast<float>(c[i + 1])), sf), zf);
+        // code = clamp(rint(fp32(v - zero) * inv)), one rounding of the product
+        const float c0 = round_magic_clamped(__fsub_rn(v[i], g.zf), g.inv, L) - kRoundMagic;
+        const float c1 = round_magic_clamped(__fsub_rn(v[i + 1], g.zf), g.inv, L) - kRoundMagic;
+        const float2 xh = __fadd2_rn(__fmul2_rn(make_float2(c0, c1), sf), zf);
         const float2 e = __fadd2_rn(make_float2(v[i], v[i + 1]), make_float2(-xh.x, -xh.y));
         s2 = __ffma2_rn(e, e, s2);
       }
@@ -517,13 +754,13 @@ __global__ void __launch_bounds__(kThreads) calib_sweep_kernel(CalibArgs a) {
       double t = acc[k];
 #pragma unroll
       for (int o = 16; o >= 1; o >>= 1) t = __dadd_rn(t, __shfl_xor_sync(0xffffffffu, t, o));
-      if (lane == 0) red[warp][k] = t;
+      if (lane == 0) sm.red[warp][k] = t;
     }
     __syncthreads();
     if (threadIdx.x < 8) {
-      double t = red[0][threadIdx.x];
+      double t = sm.red[0][threadIdx.x];
 #pragma unroll
-      for (int w = 1; w < kThreads / 32; ++w) t = __dadd_rn(t, red[w][threadIdx.x]);
+      for (int w = 1; w < kThreads / 32; ++w) t = __dadd_rn(t, sm.red[w][threadIdx.x]);
       a.partial[tile * 8 + threadIdx.x] = t;
     }
     __syncthreads();
@@ -557,9 +794,13 @@ rq_status launch_persistent(Kern kern, const Args& a, size_t smem, cudaStream_t 
   return launch_status();
 }
 
-size_t tile_smem_bytes(bool hadamard, int kg, int vg) {
+size_t quant_smem_bytes(bool hadamard) {
+  return sizeof(QSmem) + (hadamard ? kTile * kX32S * sizeof(float) : 0);
+}
+
+size_t calib_smem_bytes(bool hadamard, int kg, int vg) {
   const bool x32 = hadamard && (kg == RQ_PER_CHANNEL || vg == RQ_PER_CHANNEL);
-  return sizeof(TileSmem) + (x32 ? kX32Floats * sizeof(float) : 0);
+  return sizeof(CalibSmem) + (x32 ? kTile * (kD + 1) * sizeof(float) : 0);
 }
 
 }  // namespace
@@ -597,9 +838,12 @@ extern "C" rq_status rq_quantize_pack(const rq_cache_desc* desc, int32_t layer, 
   a.ntiles = static_cast<long long>(desc->B) * desc->H_kv * 2 * a.nblk;
   if (a.ntiles == 0) return RQ_OK;
   cudaStream_t st = static_cast<cudaStream_t>(stream);
-  const size_t smem = tile_smem_bytes(a.hadamard != 0, a.kg, a.vg);
-  return desc->dtype == RQ_F16 ? launch_persistent(quantize_pack_kernel<__half>, a, smem, st)
-                               : launch_persistent(quantize_pack_kernel<__nv_bfloat16>, a, smem, st);
+  const size_t smem = quant_smem_bytes(a.hadamard != 0);
+  if (desc->dtype == RQ_F16)
+    return a.hadamard ? launch_persistent(quantize_pack_kernel<__half, true>, a, smem, st)
+                      : launch_persistent(quantize_pack_kernel<__half, false>, a, smem, st);
+  return a.hadamard ? launch_persistent(quantize_pack_kernel<__nv_bfloat16, true>, a, smem, st)
+                    : launch_persistent(quantize_pack_kernel<__nv_bfloat16, false>, a, smem, st);
 }
 
 extern "C" size_t rq_calibrate_workspace_bytes(int32_t n, int32_t T) {
@@ -635,7 +879,7 @@ extern "C" rq_status rq_calibrate_distortion(const void* x, int32_t dtype, int32
   a.hadamard = hadamard ? 1 : 0;
   a.ntiles = static_cast<long long>(n) * a.ntile;
   cudaStream_t st = static_cast<cudaStream_t>(stream);
-  const size_t smem = tile_smem_bytes(a.hadamard != 0, a.kg, a.vg);
+  const size_t smem = calib_smem_bytes(a.hadamard != 0, a.kg, a.vg);
   const rq_status s = dtype == RQ_F16
                           ? launch_persistent(calib_sweep_kernel<__half>, a, smem, st)
                           : launch_persistent(calib_sweep_kernel<__nv_bfloat16>, a, smem, st);

@@ -90,11 +90,15 @@ __device__ __forceinline__ GroupParams group_params(float mn, float mx, bool fin
   return g;
 }
 
-// code = clamp(rint((v - zero) * inv), 0, L), fp32, round half to even
-__device__ __forceinline__ int quant_code(float v, const GroupParams& g, int b) {
-  if (!g.ok) return 0;
-  const int c = __float2int_rn(__fmul_rn(__fsub_rn(v, g.zf), g.inv));
-  return min(max(c, 0), (1 << b) - 1);
+// 1.5 * 2^23: RN(t * inv + kRoundMagic) = kRoundMagic + rint_half_even(t * inv)
+// (exact product, one rounding) for |t * inv| < 2^22, so the code is the low
+// bits of the result; out-of-range values are clamped to [magic, magic + L]
+// (NaN from a bad group clamps to magic: code 0).
+constexpr float kRoundMagic = 12582912.0f;
+
+__device__ __forceinline__ float round_magic_clamped(float t, float inv, float L) {
+  const float u = __fmaf_rn(t, inv, kRoundMagic);
+  return fminf(fmaxf(u, kRoundMagic), kRoundMagic + L);
 }
 
 }  // namespace rq
