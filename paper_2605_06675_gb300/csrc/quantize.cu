@@ -144,28 +144,6 @@ __device__ __forceinline__ void cp_async16(uint32_t dst, const void* src) {
 __device__ __forceinline__ void cp_async_commit() { asm volatile("cp.async.commit_group;\n" ::); }
 __device__ __forceinline__ void cp_async_wait_all() { asm volatile("cp.async.wait_group 0;\n" ::); }
 
-// Tile position: block j of stream sk = (batch * H + h) * 2 + kind. A CTA
-// walks tiles blockIdx.x, blockIdx.x + gridDim.x, ...; the position is
-// advanced by carrying (no division in the loop).
-struct TileRef {
-  int j, sk;
-};
-
-__device__ __forceinline__ void advance(TileRef& r, int dj, int dsk, int nblk) {
-  r.j += dj;
-  r.sk += dsk;
-  if (r.j >= nblk) {
-    r.j -= nblk;
-    r.sk += 1;
-  }
-}
-
-template <typename T>
-__device__ __forceinline__ const T* quant_tile_base(const QuantArgs& a, const TileRef& r) {
-  const T* base = static_cast<const T*>((r.sk & 1) ? a.v : a.k);
-  return base + (static_cast<long long>(r.sk >> 1) * a.S + static_cast<long long>(kTile) * r.j) * kD;
-}
-
 // the 8 KB tile into a staging buffer: thread tau copies 16-byte chunks
 // tau + 128 i (row = chunk / 16)
 __device__ __forceinline__ void issue_tile(uint8_t* buf, const void* src) {
@@ -576,58 +554,87 @@ __device__ __forceinline__ void phase2_dispatch(int mode, int b, const uint8_t* 
 #undef RQ_P2_WIDTHS
 }
 
+// Per-stream constants of the tiles a CTA walks (recomputed only when the
+// walk crosses into the next stream).
+struct StreamState {
+  const uint8_t* src;     // first tile of the stream (raw values)
+  uint8_t* dst;           // first packed block of the stream
+  int b, kind, grouping, blk_bytes;
+};
+
+template <typename T>
+__device__ __forceinline__ StreamState stream_state(const QuantArgs& a, int sk) {
+  StreamState st;
+  st.kind = sk & 1;
+  const int h = (sk >> 1) % a.H;
+  st.b = a.bits[(a.layer * a.H + h) * 2 + st.kind];
+  st.grouping = st.kind ? a.vg : a.kg;
+  st.src = reinterpret_cast<const uint8_t*>(static_cast<const T*>(st.kind ? a.v : a.k) +
+                                            static_cast<long long>(sk >> 1) * a.S * kD);
+  // offsets[layer][batch][h][kind] = offsets[layer * B * H * 2 + sk]
+  st.dst = a.packed + a.offsets[static_cast<long long>(a.layer) * a.B * a.H * 2 + sk];
+  st.blk_bytes = 512 * (st.b + 1);
+  return st;
+}
+
+// A CTA owns a contiguous range of tiles (block j of stream sk = (batch * H
+// + h) * 2 + kind, tile index sk * nblk + j), so consecutive tiles share
+// their stream's constants.
 template <typename T, bool HAD>
 __global__ void __launch_bounds__(kThreads, RQ_QUANT_MIN_BLOCKS) quantize_pack_kernel(QuantArgs a) {
   extern __shared__ __align__(16) unsigned char smem_raw[];
   QSmem& sm = *reinterpret_cast<QSmem*>(smem_raw);
   float* x32 = HAD ? reinterpret_cast<float*>(smem_raw + sizeof(QSmem)) : nullptr;
-  const long long stride = gridDim.x;
-  long long tile = blockIdx.x;
-  if (tile >= a.ntiles) return;
+  const long long t0 = a.ntiles * blockIdx.x / gridDim.x;
+  const long long t1 = a.ntiles * (blockIdx.x + 1) / gridDim.x;
+  if (t0 >= t1) return;
   if (HAD && threadIdx.x < kD) sm.signs[threadIdx.x] = a.signs ? a.signs[threadIdx.x] : int8_t(1);
 
   const int nblk = a.nblk;
-  const int dsk = static_cast<int>(stride / nblk), dj = static_cast<int>(stride % nblk);
-  TileRef r{static_cast<int>(tile % nblk), static_cast<int>(tile / nblk)};
-  issue_tile(sm.tile[0], quant_tile_base<T>(a, r));
+  constexpr int kTileSrcBytes = kTile * kD * static_cast<int>(sizeof(T));
+  int sk = static_cast<int>(t0 / nblk), j = static_cast<int>(t0 % nblk);
+  StreamState cur = stream_state<T>(a, sk);
+  StreamState nxt = cur;
+  int nj = j;
+  issue_tile(sm.tile[0], cur.src + static_cast<long long>(j) * kTileSrcBytes);
   cp_async_commit();
 
-  for (int it = 0; tile < a.ntiles; tile += stride, ++it) {
-    const TileRef cur = r;
+  for (long long t = t0; t < t1; ++t) {
+    const int it = static_cast<int>(t - t0);
     const uint8_t* buf = sm.tile[it & 1];
     cp_async_wait_all();
     __syncthreads();             // tile visible; every thread is past the previous tile
-    if (tile + stride < a.ntiles) {
-      advance(r, dj, dsk, nblk);
-      issue_tile(sm.tile[(it + 1) & 1], quant_tile_base<T>(a, r));
+    if (t + 1 < t1) {
+      if (++nj == nblk) {
+        nj = 0;
+        nxt = stream_state<T>(a, ++sk);
+      }
+      issue_tile(sm.tile[(it + 1) & 1], nxt.src + static_cast<long long>(nj) * kTileSrcBytes);
     }
     cp_async_commit();
 
-    const int kind = cur.sk & 1;
-    const int h = (cur.sk >> 1) % a.H;
-    const int b = a.bits[(a.layer * a.H + h) * 2 + kind];
-    if (b < 1 || b > 8) {
-      if (threadIdx.x == 0) set_status(a.status, RQ_STATUS_BAD_BITS);
-      continue;
+    const int b = cur.b;
+    if (b >= 1 && b <= 8) {
+      uint8_t* blk = cur.dst + static_cast<long long>(j) * cur.blk_bytes;
+      uint8_t* meta = blk + 512 * b;
+      const int kind = cur.kind, grouping = cur.grouping;
+      GroupOut g;
+      if constexpr (HAD) g = phase1_rotated<T>(buf, x32, kind, grouping, b, meta, sm);
+      else if (grouping == RQ_PER_CHANNEL) g = phase1_cols<T>(buf, kind, b, meta, sm);
+      else g = phase1_rows<T>(buf, kind, b, meta, sm);
+      if (g.bad) set_status(a.status, RQ_STATUS_NUMERIC);
+      const bool slow = __syncthreads_or(g.slow) != 0;
+
+      const int mode = kind == 0 ? (grouping == RQ_PER_CHANNEL ? kModeKC : kModeKT)
+                                 : (grouping == RQ_PER_TOKEN ? kModeVT : kModeVC);
+      uint32_t* blk32 = reinterpret_cast<uint32_t*>(blk);
+      if (slow) phase2_dispatch<T, true, HAD>(mode, b, buf, x32, sm, blk32);
+      else phase2_dispatch<T, false, HAD>(mode, b, buf, x32, sm, blk32);
+    } else if (threadIdx.x == 0) {
+      set_status(a.status, RQ_STATUS_BAD_BITS);
     }
-    const int grouping = kind ? a.vg : a.kg;
-    // offsets[layer][batch][h][kind] = offsets[layer * B * H * 2 + sk]
-    const uint64_t off = a.offsets[static_cast<long long>(a.layer) * a.B * a.H * 2 + cur.sk];
-    uint8_t* blk = a.packed + off + static_cast<uint64_t>(cur.j) * 512u * (b + 1);
-    uint8_t* meta = blk + 512 * b;
-
-    GroupOut g;
-    if constexpr (HAD) g = phase1_rotated<T>(buf, x32, kind, grouping, b, meta, sm);
-    else if (grouping == RQ_PER_CHANNEL) g = phase1_cols<T>(buf, kind, b, meta, sm);
-    else g = phase1_rows<T>(buf, kind, b, meta, sm);
-    if (g.bad) set_status(a.status, RQ_STATUS_NUMERIC);
-    const bool slow = __syncthreads_or(g.slow) != 0;
-
-    const int mode = kind == 0 ? (grouping == RQ_PER_CHANNEL ? kModeKC : kModeKT)
-                               : (grouping == RQ_PER_TOKEN ? kModeVT : kModeVC);
-    uint32_t* blk32 = reinterpret_cast<uint32_t*>(blk);
-    if (slow) phase2_dispatch<T, true, HAD>(mode, b, buf, x32, sm, blk32);
-    else phase2_dispatch<T, false, HAD>(mode, b, buf, x32, sm, blk32);
+    j = nj;
+    cur = nxt;
   }
 }
 
