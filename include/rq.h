@@ -171,7 +171,8 @@ rq_status rq_quantize_pack(const rq_cache_desc* desc, int32_t layer, const void*
                            const uint64_t* offsets_dev, void* packed, uint32_t* status_dev,
                            void* stream);
 
-/* Workspace rq_decode_attention needs on the current device (split-K partials). */
+/* Workspace rq_decode_attention needs on the current device (the split-K
+ * partial records). */
 rq_status rq_decode_workspace_bytes(const rq_cache_desc* desc, size_t* bytes);
 
 /* Decode attention of one query per (batch, query head) over all S cached
@@ -179,9 +180,12 @@ rq_status rq_decode_workspace_bytes(const rq_cache_desc* desc, size_t* bytes);
  * (App. W "Kernel fusion"): out[b][j] = sum_t softmax_t(q_j . k_hat_t / sqrt(128)) v_hat_t
  * with k_hat, v_hat the dequantized cache of kv head j / (H_q / H_kv); with
  * desc->hadamard the rotated cache is used as Q(XR)R^T (App. W "QuaRot kernel").
- * Split-K over the sequence with a log-sum-exp merge.
+ * Split-K over the sequence, then a log-sum-exp merge kernel launched as a
+ * programmatic dependent of the split kernel (it overlaps the split grid's
+ * tail and waits for it before reading).
  * q: device [B][H_q][128] of desc->dtype; out: device fp32 [B][H_q][128];
- * ws: device workspace of at least rq_decode_workspace_bytes.
+ * ws: device workspace of at least rq_decode_workspace_bytes, 16-byte
+ * aligned, contents arbitrary on entry; one call at a time per workspace.
  * Errors: RQ_ERR_INVALID_ARG, RQ_ERR_SHAPE (S == 0, S % 32, GQA > 8),
  * RQ_ERR_ALIGNMENT, RQ_ERR_WORKSPACE, RQ_ERR_CUDA. */
 rq_status rq_decode_attention(const rq_cache_desc* desc, int32_t layer, const void* q,
@@ -198,9 +202,9 @@ rq_status rq_decode_attention(const rq_cache_desc* desc, int32_t layer, const vo
  * split-K partials live in a fixed device array inside librq of
  * RQ_STATIC_SCRATCH_BYTES bytes, reserved on every GPU that loads the
  * library until the process exits. It calls no cudaMalloc/cudaFree.
- *  - Limit: B * H_q * splits * 130 * 4 bytes must fit in RQ_STATIC_SCRATCH_BYTES
- *    (splits as chosen for rq_decode_workspace_bytes); larger shapes return
- *    RQ_ERR_WORKSPACE before anything is launched.
+ *  - Limit: the rq_decode_workspace_bytes of the shape must fit in
+ *    RQ_STATIC_SCRATCH_BYTES; larger shapes return RQ_ERR_WORKSPACE before
+ *    anything is launched.
  *  - The first call on a device looks up the array's device address
  *    (cudaGetSymbolAddress) with that device current; make that first call
  *    before any stream capture.

@@ -53,16 +53,16 @@ namespace {
 
 // CTAs per SM the decoder's register budget is sized for
 #ifndef RQ_DECODE_MIN_BLOCKS
-#define RQ_DECODE_MIN_BLOCKS 3
+#define RQ_DECODE_MIN_BLOCKS 4
 #endif
 constexpr int kWarps = 4;
 constexpr int kThreads = 32 * kWarps;
-constexpr int kPart = kD + 2;        // partial record: o[128], m (log2 domain), l
+constexpr int kPart = kD + 4;        // partial record: o[128], m (log2 domain), l, 2 pad (16-byte rows)
 constexpr int kMaxHeads = 8;         // MMA n
-constexpr int kRingBytes = 12800;    // per-warp ring of shared-memory slots
+constexpr int kRingBytes = 11264;    // per-warp ring of shared-memory slots
 constexpr int kMaxSlots = 8;
 constexpr int kQBytes = kMaxHeads * kD * 4;
-constexpr int kSmemBytes = kQBytes + kWarps * kRingBytes;   // 55296: 4 CTAs per SM
+constexpr int kSmemBytes = kQBytes + kWarps * kRingBytes;   // 49152: 4 CTAs per SM
 static_assert(kWarps * kMaxHeads * kD * 4 <= kWarps * kRingBytes, "merge buffer aliases rings");
 
 struct DecodeArgs {
@@ -71,7 +71,7 @@ struct DecodeArgs {
   const uint8_t* bits;
   const uint64_t* offsets;
   const int8_t* signs;
-  float* partial;
+  float* partial;            // [B][H_q][splits][132]
   uint32_t* status;
   int layer, B, H, Hq, g, nblk, splits, bps, kg, vg, hadamard;
 };
@@ -188,9 +188,11 @@ __device__ __forceinline__ uint32_t dequant(uint32_t sub, uint32_t m, uint32_t z
 // q pair; the zero-point term, the same for every token, comes from MMAs
 // whose A operand carries z in rows gid. Codes enter the tensor cores as
 // exact fp16 subnormals c 2^(E - 24); the accumulator is scaled by 2^24.
+// q operands of lane L for unit u: qtab + 16 (32 u + L) holds q pairs x = 0..3
+// (channels 32u + 8tig + 2x), qtab + 2048 + the same with 2^-E(x) folded in.
 template <int BW, int KG>
-__device__ __forceinline__ void qk_block(const uint8_t* img, int lane, const uint32_t (&qb)[4][4],
-                                         const uint32_t (&qf)[4][4], float (&s)[2][4]) {
+__device__ __forceinline__ void qk_block(const uint8_t* img, int lane, const uint8_t* qtab,
+                                         float (&s)[2][4]) {
   const int gid = lane >> 2, tig = lane & 3;
   uint32_t w[4 * BW];
   lane_words<BW>(img, lane, w);
@@ -206,13 +208,16 @@ __device__ __forceinline__ void qk_block(const uint8_t* img, int lane, const uin
       // scale / zero pairs of channels 32u + 8tig + 2x: words 16u + 4tig + x
       const uint4 S = lds128(meta + 4 * (16 * u + 4 * tig));
       const uint4 Z = lds128(meta + 256 + 4 * (16 * u + 4 * tig));
+      const uint4 QB = lds128(qtab + 16 * (32 * u + lane));
+      const uint4 QF = lds128(qtab + 2048 + 16 * (32 * u + lane));
       const uint32_t S2[4] = {S.x, S.y, S.z, S.w}, Z2[4] = {Z.x, Z.y, Z.z, Z.w};
+      const uint32_t qb[4] = {QB.x, QB.y, QB.z, QB.w}, qf[4] = {QF.x, QF.y, QF.z, QF.w};
 #pragma unroll
       for (int xs = 0; xs < 2; ++xs) {
-        const uint32_t b0 = hmul2u(qf[u][2 * xs], S2[2 * xs]);
-        const uint32_t b1 = hmul2u(qf[u][2 * xs + 1], S2[2 * xs + 1]);
+        const uint32_t b0 = hmul2u(qf[2 * xs], S2[2 * xs]);
+        const uint32_t b1 = hmul2u(qf[2 * xs + 1], S2[2 * xs + 1]);
         const uint32_t az[4] = {Z2[2 * xs], 0u, Z2[2 * xs + 1], 0u};
-        mma16816(zb, az, qb[u][2 * xs], qb[u][2 * xs + 1]);
+        mma16816(zb, az, qb[2 * xs], qb[2 * xs + 1]);
 #pragma unroll
         for (int mt = 0; mt < 2; ++mt) {
           const uint32_t a[4] = {reg<BW>(w, u, 2 * xs, 2 * mt), reg<BW>(w, u, 2 * xs, 2 * mt + 1),
@@ -233,6 +238,8 @@ __device__ __forceinline__ void qk_block(const uint8_t* img, int lane, const uin
     for (int u = 0; u < 4; ++u) {
       // (scale, zero) of tokens 8x + gid, group u: words 16 gid + 4u + x
       const uint4 SZ = lds128(meta + 4 * (16 * gid + 4 * u));
+      const uint4 QB = lds128(qtab + 16 * (32 * u + lane));
+      const uint32_t qb[4] = {QB.x, QB.y, QB.z, QB.w};
       const uint32_t sz[4] = {SZ.x, SZ.y, SZ.z, SZ.w};
       uint32_t m[4], z2[4];
 #pragma unroll
@@ -251,7 +258,7 @@ __device__ __forceinline__ void qk_block(const uint8_t* img, int lane, const uin
               dequant(reg<BW>(w, u, 2 * mt + 1, 2 * xs), m[2 * mt + 1], z2[2 * mt + 1]),
               dequant(reg<BW>(w, u, 2 * mt, 2 * xs + 1), m[2 * mt], z2[2 * mt]),
               dequant(reg<BW>(w, u, 2 * mt + 1, 2 * xs + 1), m[2 * mt + 1], z2[2 * mt + 1])};
-          mma16816(s[mt], a, qb[u][2 * xs], qb[u][2 * xs + 1]);
+          mma16816(s[mt], a, qb[2 * xs], qb[2 * xs + 1]);
         }
     }
   }
@@ -273,30 +280,28 @@ __device__ __forceinline__ void pv_block(const uint8_t* img, int lane, const uin
   lane_words<BW>(img, lane, w);
   const uint8_t* meta = img + 512 * BW;
   if constexpr (VG == RQ_PER_TOKEN) {
-    uint32_t ms[4][4], mz[4][4];  // [token pair y][group G]: words 16y + 4tig + G
+    // zero-points: rows gid of the A operand carry group 2gp, rows gid + 8
+    // group 2gp + 1; columns are token pairs 2ks (k 2tig..) and 2ks + 1.
+    // Zero pairs of token pair y, groups 0..3: words 64 + 16y + 4tig + G.
+#pragma unroll
+    for (int ks = 0; ks < 2; ++ks) {
+      const uint4 Z0 = lds128(meta + 256 + 4 * (16 * (2 * ks) + 4 * tig));
+      const uint4 Z1 = lds128(meta + 256 + 4 * (16 * (2 * ks + 1) + 4 * tig));
+      const uint32_t az0[4] = {Z0.x, Z0.y, Z1.x, Z1.y}, az1[4] = {Z0.z, Z0.w, Z1.z, Z1.w};
+      mma16816(bz[0], az0, pb[ks][0], pb[ks][1]);
+      mma16816(bz[1], az1, pb[ks][0], pb[ks][1]);
+    }
+    uint32_t ms[4][4];        // scale pairs [token pair y][group G]: words 16y + 4tig + G
 #pragma unroll
     for (int y = 0; y < 4; ++y) {
       const uint4 S = lds128(meta + 4 * (16 * y + 4 * tig));
-      const uint4 Z = lds128(meta + 256 + 4 * (16 * y + 4 * tig));
       ms[y][0] = S.x;
       ms[y][1] = S.y;
       ms[y][2] = S.z;
       ms[y][3] = S.w;
-      mz[y][0] = Z.x;
-      mz[y][1] = Z.y;
-      mz[y][2] = Z.z;
-      mz[y][3] = Z.w;
     }
 #pragma unroll
-    for (int ks = 0; ks < 2; ++ks) {
-      // zero-points: rows gid of the A operand carry group 2gp, rows gid + 8
-      // group 2gp + 1; columns are token pairs 2ks (k 2tig..) and 2ks + 1
-#pragma unroll
-      for (int gp = 0; gp < 2; ++gp) {
-        const uint32_t az[4] = {mz[2 * ks][2 * gp], mz[2 * ks][2 * gp + 1],
-                                mz[2 * ks + 1][2 * gp], mz[2 * ks + 1][2 * gp + 1]};
-        mma16816(bz[gp], az, pb[ks][0], pb[ks][1]);
-      }
+    for (int ks = 0; ks < 2; ++ks)
 #pragma unroll
       for (int G = 0; G < 4; ++G) {
         const uint32_t b0 = hmul2u(pb[ks][0], ms[2 * ks][G]);
@@ -309,7 +314,6 @@ __device__ __forceinline__ void pv_block(const uint8_t* img, int lane, const uin
           mma16816(o[2 * G + mh], a, b0, b1);
         }
       }
-    }
   } else {                    // per-channel values: dequantize in registers
 #pragma unroll
     for (int u = 0; u < 4; ++u) {
@@ -340,10 +344,9 @@ __device__ __forceinline__ void pv_block(const uint8_t* img, int lane, const uin
 
 template <int BW>
 __device__ __forceinline__ void qk_dispatch_g(int kg, const uint8_t* img, int lane,
-                                              const uint32_t (&qb)[4][4], const uint32_t (&qf)[4][4],
-                                              float (&s)[2][4]) {
-  if (kg == RQ_PER_CHANNEL) qk_block<BW, RQ_PER_CHANNEL>(img, lane, qb, qf, s);
-  else qk_block<BW, RQ_PER_TOKEN>(img, lane, qb, qf, s);
+                                              const uint8_t* qtab, float (&s)[2][4]) {
+  if (kg == RQ_PER_CHANNEL) qk_block<BW, RQ_PER_CHANNEL>(img, lane, qtab, s);
+  else qk_block<BW, RQ_PER_TOKEN>(img, lane, qtab, s);
 }
 
 template <int BW>
@@ -355,17 +358,16 @@ __device__ __forceinline__ void pv_dispatch_g(int vg, const uint8_t* img, int la
 }
 
 __device__ __forceinline__ void qk_dispatch(int bw, int kg, const uint8_t* img, int lane,
-                                            const uint32_t (&qb)[4][4], const uint32_t (&qf)[4][4],
-                                            float (&s)[2][4]) {
+                                            const uint8_t* qtab, float (&s)[2][4]) {
   switch (bw) {
-    case 1: qk_dispatch_g<1>(kg, img, lane, qb, qf, s); break;
-    case 2: qk_dispatch_g<2>(kg, img, lane, qb, qf, s); break;
-    case 3: qk_dispatch_g<3>(kg, img, lane, qb, qf, s); break;
-    case 4: qk_dispatch_g<4>(kg, img, lane, qb, qf, s); break;
-    case 5: qk_dispatch_g<5>(kg, img, lane, qb, qf, s); break;
-    case 6: qk_dispatch_g<6>(kg, img, lane, qb, qf, s); break;
-    case 7: qk_dispatch_g<7>(kg, img, lane, qb, qf, s); break;
-    default: qk_dispatch_g<8>(kg, img, lane, qb, qf, s); break;
+    case 1: qk_dispatch_g<1>(kg, img, lane, qtab, s); break;
+    case 2: qk_dispatch_g<2>(kg, img, lane, qtab, s); break;
+    case 3: qk_dispatch_g<3>(kg, img, lane, qtab, s); break;
+    case 4: qk_dispatch_g<4>(kg, img, lane, qtab, s); break;
+    case 5: qk_dispatch_g<5>(kg, img, lane, qtab, s); break;
+    case 6: qk_dispatch_g<6>(kg, img, lane, qtab, s); break;
+    case 7: qk_dispatch_g<7>(kg, img, lane, qtab, s); break;
+    default: qk_dispatch_g<8>(kg, img, lane, qtab, s); break;
   }
 }
 
@@ -519,8 +521,8 @@ __device__ __forceinline__ void prologue_static(const WarpStream& ws) {
 }
 
 template <int BK, int KG, int BV, int VG>
-__device__ __forceinline__ void blocks_static(const WarpStream& ws, const uint32_t (&qb)[4][4],
-                                              const uint32_t (&qf)[4][4], SoftmaxAcc& acc) {
+__device__ __forceinline__ void blocks_static(const WarpStream& ws, const uint8_t* qtab,
+                                              SoftmaxAcc& acc) {
   using R = Ring<BK, BV>;
   constexpr int NS = R::kSlots;
   int use = 0, iss = NS - 1;          // slot of the next entry to use / to issue
@@ -530,7 +532,7 @@ __device__ __forceinline__ void blocks_static(const WarpStream& ws, const uint32
     cp_async_wait<NS - 1>();
     __syncwarp();
     float s[2][4];
-    qk_block<BK, KG>(ws.ring_ptr + use * R::kSlot, ws.lane, qb, qf, s);
+    qk_block<BK, KG>(ws.ring_ptr + use * R::kSlot, ws.lane, qtab, s);
     __syncwarp();
     use = use + 1 == NS ? 0 : use + 1;
     uint32_t pb[2][2];
@@ -563,8 +565,7 @@ __device__ __forceinline__ void prologue_dyn(const WarpStream& ws, const DynRing
 }
 
 __device__ __forceinline__ void blocks_dyn(const WarpStream& ws, const DynRing& r,
-                                           const uint32_t (&qb)[4][4], const uint32_t (&qf)[4][4],
-                                           SoftmaxAcc& acc) {
+                                           const uint8_t* qtab, SoftmaxAcc& acc) {
   int use = 0, iss = r.ns - 1;
   for (int i = 0; i < ws.nb; ++i) {
     issue_dyn(ws, r, 2 * i + r.ns - 1, iss);
@@ -572,7 +573,7 @@ __device__ __forceinline__ void blocks_dyn(const WarpStream& ws, const DynRing& 
     cp_async_wait_dyn(r.ns - 1);
     __syncwarp();
     float s[2][4];
-    qk_dispatch(r.bK, r.kg, ws.ring_ptr + use * r.slot, ws.lane, qb, qf, s);
+    qk_dispatch(r.bK, r.kg, ws.ring_ptr + use * r.slot, ws.lane, qtab, s);
     __syncwarp();
     use = use + 1 == r.ns ? 0 : use + 1;
     uint32_t pb[2][2];
@@ -672,14 +673,27 @@ __global__ void __launch_bounds__(kThreads, RQ_DECODE_MIN_BLOCKS) decode_split_k
   uint32_t ef[4];
 #pragma unroll
   for (int x = 0; x < 4; ++x) ef[x] = pow2_neg_h2(a.kg == RQ_PER_CHANNEL && valid ? fmt::exponent(bK, x) : 0);
+  if (warp == 0) {
 #pragma unroll
-  for (int u = 0; u < 4; ++u)
+    for (int u = 0; u < 4; ++u)
 #pragma unroll
-    for (int x = 0; x < 4; ++x) {
-      const float* qr = qs + gid * kD + 32 * u + 8 * tig + 2 * x;
-      qb[u][x] = pack_f16x2(qr[0] * qscale, qr[1] * qscale);
-      qf[u][x] = hmul2u(qb[u][x], ef[x]);
+      for (int x = 0; x < 4; ++x) {
+        const float* qr = qs + gid * kD + 32 * u + 8 * tig + 2 * x;
+        qb[u][x] = pack_f16x2(qr[0] * qscale, qr[1] * qscale);
+        qf[u][x] = hmul2u(qb[u][x], ef[x]);
+      }
+  }
+  __syncthreads();                  // qs is read; its space becomes the q operand table
+  uint8_t* qtab = smem_raw;
+  if (warp == 0) {
+#pragma unroll
+    for (int u = 0; u < 4; ++u) {
+      *reinterpret_cast<uint4*>(qtab + 16 * (32 * u + lane)) = make_uint4(qb[u][0], qb[u][1], qb[u][2], qb[u][3]);
+      *reinterpret_cast<uint4*>(qtab + 2048 + 16 * (32 * u + lane)) =
+          make_uint4(qf[u][0], qf[u][1], qf[u][2], qf[u][3]);
     }
+  }
+  __syncthreads();
 
   SoftmaxAcc acc;
 #pragma unroll
@@ -694,11 +708,13 @@ __global__ void __launch_bounds__(kThreads, RQ_DECODE_MIN_BLOCKS) decode_split_k
   acc.l0 = acc.l1 = 0.0f;
 
   switch (key) {
-#define RQ_BLK(k, BK, BV) case k: blocks_static<BK, RQ_PER_CHANNEL, BV, RQ_PER_TOKEN>(ws, qb, qf, acc); break;
+#define RQ_BLK(k, BK, BV) case k: blocks_static<BK, RQ_PER_CHANNEL, BV, RQ_PER_TOKEN>(ws, qtab, acc); break;
     RQ_FAST_CASES(RQ_BLK)
 #undef RQ_BLK
-    default: blocks_dyn(ws, dr, qb, qf, acc); break;
+    default: blocks_dyn(ws, dr, qtab, acc); break;
   }
+  // the merge kernel may be scheduled now; it waits for this grid to finish
+  asm volatile("griddepcontrol.launch_dependents;\n" ::: "memory");
   if (a.vg == RQ_PER_TOKEN && valid) {
     // rows of m-tile mt are classes x = 2 (mt & 1) + r of unit mt / 2: undo
     // their codes' 2^(E(x) - 24), then add group G's zero-point sum (rows gid
@@ -766,41 +782,155 @@ __global__ void __launch_bounds__(kThreads, RQ_DECODE_MIN_BLOCKS) decode_split_k
       dst[kD + 1] = lsum;
     }
   }
+
 }
 
-// out[row] = sum_s 2^(m_s - M) o_s / sum_s 2^(m_s - M) l_s, rotated back
-// (o R^T = FWHT(o) / sqrt(128) * signs) for a Hadamard cache.
-__global__ void __launch_bounds__(kD) decode_combine_kernel(const float* partial, float* out,
-                                                           const int8_t* signs, uint32_t* status,
-                                                           int splits, int hadamard) {
-  __shared__ float y[kD];
-  const long long row = blockIdx.x;
-  const int d = threadIdx.x;
-  const float* p = partial + row * splits * kPart;
-  float M = -INFINITY;
-  for (int s = 0; s < splits; ++s) M = fmaxf(M, p[s * kPart + kD]);
-  float L = 0.0f, acc = 0.0f;
-  if (M != -INFINITY) {
-    for (int s = 0; s < splits; ++s) {
-      const float ms = p[s * kPart + kD];
-      const float sc = (ms == -INFINITY) ? 0.0f : exp2f(ms - M);
-      L += sc * p[s * kPart + kD + 1];
-      acc += sc * p[s * kPart + d];
+// ------------------------------------------------------------ split merge ----
+// out_n = sum_s 2^(m_ns - M_n) o_ns / sum_s 2^(m_ns - M_n) l_ns for the g
+// query rows n of one (batch, kv head), rotated back (o R^T =
+// FWHT(o) / sqrt(128) * signs) for a Hadamard cache. A CTA owns one (batch,
+// kv head) and 128 / CQ channels of its rows (the whole row when CQ = 1, as
+// the rotation needs). It is launched as a programmatic dependent of the
+// split kernel and waits for it on entry. Records are pulled into shared
+// memory with cp.async, a chunk of splits at a time (one round trip per
+// chunk), and merged there with a running max per row.
+constexpr int kMergeSmem = 64 * 1024;
+
+template <int CQ>
+__global__ void __launch_bounds__(kThreads) decode_merge_kernel(const float* partial, float* out,
+                                                                const int8_t* signs,
+                                                                uint32_t* status, int Hq, int H,
+                                                                int g, int splits, int hadamard) {
+  asm volatile("griddepcontrol.wait;\n" ::: "memory");
+  constexpr int CW = kD / CQ;          // channels of this CTA
+  constexpr int CH = CW / 4;           // 16-byte pieces of a record's o slice
+  constexpr int SLOT = CH + 1;         // pieces per (row, split): o slice, then (m, l, pad)
+  constexpr int PAIRS = kMaxHeads * CW / kThreads;   // (row, channel) pairs per thread, at most
+  extern __shared__ float4 msm[];
+  __shared__ float wgt[kMaxHeads][64];
+  __shared__ float run_m[kMaxHeads], run_l[kMaxHeads], run_scale[kMaxHeads];
+  __shared__ float y[kMaxHeads * kD];
+  const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
+  const int batch = blockIdx.x / H, h = blockIdx.x % H, part = blockIdx.y;
+  const long long row0 = static_cast<long long>(batch) * Hq + h * g;
+  const long long rstride = static_cast<long long>(splits) * kPart;
+  const float* p = partial + row0 * rstride + part * CW;     // o slice of row 0, split 0
+  const float* pml = partial + row0 * rstride + kD;           // (m, l) of row 0, split 0
+  // splits per chunk: shared budget, and at most 64 (one weight per lane pair)
+  const int cs_max = min(64, kMergeSmem / (g * SLOT * 16));
+  if (tid < kMaxHeads) {
+    run_m[tid] = -INFINITY;
+    run_l[tid] = 0.0f;
+  }
+  float acc[PAIRS];
+#pragma unroll
+  for (int k = 0; k < PAIRS; ++k) acc[k] = 0.0f;
+  const uint32_t sbase = static_cast<uint32_t>(__cvta_generic_to_shared(msm));
+
+  for (int c0 = 0; c0 < splits; c0 += cs_max) {
+    const int cs = min(cs_max, splits - c0);
+    // piece (n, s, i): i < CH the o slice, i == CH (m, l, pad, pad)
+    const int npieces = g * cs * SLOT;
+    for (int x = tid; x < npieces; x += kThreads) {
+      const int i = x % SLOT, ns = x / SLOT, n = ns / cs, sl = ns % cs;
+      const float* src = (i < CH ? p + 4 * i : pml) + n * rstride + static_cast<long long>(c0 + sl) * kPart;
+      asm volatile("cp.async.cg.shared.global [%0], [%1], 16;\n" ::"r"(sbase + 16 * x), "l"(src));
+    }
+    asm volatile("cp.async.commit_group;\n" ::);
+    asm volatile("cp.async.wait_group 0;\n" ::);
+    __syncthreads();
+    // warp w: rows w, w + 4; lanes over the chunk's splits (two per lane)
+#pragma unroll
+    for (int k = 0; k < 2; ++k) {
+      const int n = warp + kWarps * k;
+      if (n < g) {
+        float mv[2], lv[2], mx = -INFINITY;
+#pragma unroll
+        for (int r = 0; r < 2; ++r) {
+          const int sl = lane + 32 * r;
+          mv[r] = -INFINITY;
+          lv[r] = 0.0f;
+          if (sl < cs) {
+            const float4 ml = msm[(n * cs + sl) * SLOT + CH];
+            mv[r] = ml.x;
+            lv[r] = ml.y;
+          }
+          mx = fmaxf(mx, mv[r]);
+        }
+#pragma unroll
+        for (int off = 16; off >= 1; off >>= 1) mx = fmaxf(mx, __shfl_xor_sync(0xffffffffu, mx, off));
+        const float mold = run_m[n];
+        const float mnew = fmaxf(mold, mx);
+        float l = 0.0f;
+#pragma unroll
+        for (int r = 0; r < 2; ++r) {
+          const int sl = lane + 32 * r;
+          const float wv = (mv[r] == -INFINITY) ? 0.0f : exp2f(mv[r] - mnew);
+          if (sl < cs) wgt[n][sl] = wv;
+          l += wv * lv[r];
+        }
+#pragma unroll
+        for (int off = 16; off >= 1; off >>= 1) l += __shfl_xor_sync(0xffffffffu, l, off);
+        __syncwarp();
+        if (lane == 0) {
+          const float sc = (mold == -INFINITY) ? 0.0f : exp2f(mold - mnew);
+          run_scale[n] = sc;
+          run_l[n] = run_l[n] * sc + l;
+          run_m[n] = mnew;
+        }
+      }
+    }
+    __syncthreads();
+#pragma unroll
+    for (int k = 0; k < PAIRS; ++k) {
+      const int pi = tid + kThreads * k, n = pi / CW, c = pi % CW;
+      if (n < g) {
+        float a = acc[k] * run_scale[n];
+        const float* o = reinterpret_cast<const float*>(msm + n * cs * SLOT) + c;
+        const float* wn = wgt[n];
+#pragma unroll 4
+        for (int sl = 0; sl < cs; ++sl) a += wn[sl] * o[sl * SLOT * 4];
+        acc[k] = a;
+      }
+    }
+    __syncthreads();
+  }
+#pragma unroll
+  for (int k = 0; k < PAIRS; ++k) {
+    const int pi = tid + kThreads * k, n = pi / CW, c = pi % CW;
+    if (n < g) {
+      const float L = run_l[n];
+      float v = L > 0.0f ? acc[k] / L : 0.0f;
+      if (!(L > 0.0f) || !isfinite(v)) {
+        set_status(status, RQ_STATUS_NUMERIC);
+        if (!isfinite(v)) v = 0.0f;
+      }
+      acc[k] = v;
     }
   }
-  float r = L > 0.0f ? acc / L : 0.0f;
-  if (!(L > 0.0f) || !isfinite(r)) {
-    if (d == 0) set_status(status, RQ_STATUS_NUMERIC);
-    if (!isfinite(r)) r = 0.0f;
-  }
-  if (hadamard) {
-    y[d] = r;
+  if (CQ == 1 && hadamard) {
+#pragma unroll
+    for (int k = 0; k < PAIRS; ++k) {
+      const int pi = tid + kThreads * k;
+      if (pi / CW < g) y[pi] = acc[k];
+    }
     __syncthreads();
-    fwht_smem(y, 1);
-    r = y[d] * kInvSqrt128;
-    if (signs && signs[d] < 0) r = -r;
+    fwht_smem(y, g);
+#pragma unroll
+    for (int k = 0; k < PAIRS; ++k) {
+      const int pi = tid + kThreads * k, c = pi % CW;
+      if (pi / CW < g) {
+        float v = y[pi] * kInvSqrt128;
+        if (signs && signs[c] < 0) v = -v;
+        acc[k] = v;
+      }
+    }
   }
-  out[row * kD + d] = r;
+#pragma unroll
+  for (int k = 0; k < PAIRS; ++k) {
+    const int pi = tid + kThreads * k, n = pi / CW, c = pi % CW;
+    if (n < g) out[(row0 + n) * kD + part * CW + c] = acc[k];
+  }
 }
 
 void decode_plan(const rq_cache_desc* desc, int sms, int* splits, int* bps) {
@@ -827,15 +957,20 @@ rq_status check_desc(const rq_cache_desc* desc) {
   return RQ_OK;
 }
 
+// Workspace: the split records [B][H_q][splits][132] fp32.
+size_t workspace_bytes(const rq_cache_desc* desc, int splits) {
+  return static_cast<size_t>(desc->B) * desc->H_q * splits * kPart * sizeof(float);
+}
+
 void fill_args(DecodeArgs& a, const rq_cache_desc* desc, int32_t layer, const void* q,
                const void* packed, const uint8_t* bits_dev, const uint64_t* offsets_dev,
-               const int8_t* signs_dev, float* partial, uint32_t* status_dev, int splits, int bps) {
+               const int8_t* signs_dev, void* ws, uint32_t* status_dev, int splits, int bps) {
   a.q = q;
   a.packed = static_cast<const uint8_t*>(packed);
   a.bits = bits_dev;
   a.offsets = offsets_dev;
   a.signs = signs_dev;
-  a.partial = partial;
+  a.partial = static_cast<float*>(ws);
   a.status = status_dev;
   a.layer = layer;
   a.B = desc->B;
@@ -850,25 +985,43 @@ void fill_args(DecodeArgs& a, const rq_cache_desc* desc, int32_t layer, const vo
   a.hadamard = desc->hadamard ? 1 : 0;
 }
 
-// split kernel + combine kernel on `stream`
-rq_status launch_decode(const DecodeArgs& a, const rq_cache_desc* desc, float* out,
-                        cudaStream_t s) {
+template <typename T>
+rq_status launch_split(const DecodeArgs& a, const dim3& grid, cudaStream_t s) {
+  auto kern = decode_split_kernel<T>;
+  if (cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, kSmemBytes) != cudaSuccess ||
+      cudaFuncSetAttribute(kern, cudaFuncAttributePreferredSharedMemoryCarveout,
+                           cudaSharedmemCarveoutMaxShared) != cudaSuccess)
+    return RQ_ERR_CUDA;
+  kern<<<grid, kThreads, kSmemBytes, s>>>(a);
+  return launch_status();
+}
+
+// split kernel, then the merge kernel as its programmatic dependent
+rq_status launch_decode(const DecodeArgs& a, const rq_cache_desc* desc, float* out, cudaStream_t s) {
   const dim3 grid(static_cast<unsigned>(a.splits), static_cast<unsigned>(desc->H_kv),
                   static_cast<unsigned>(desc->B));
-  if (desc->dtype == RQ_F16) {
-    if (cudaFuncSetAttribute(decode_split_kernel<__half>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                             kSmemBytes) != cudaSuccess)
-      return RQ_ERR_CUDA;
-    decode_split_kernel<__half><<<grid, kThreads, kSmemBytes, s>>>(a);
-  } else {
-    if (cudaFuncSetAttribute(decode_split_kernel<__nv_bfloat16>,
-                             cudaFuncAttributeMaxDynamicSharedMemorySize, kSmemBytes) != cudaSuccess)
-      return RQ_ERR_CUDA;
-    decode_split_kernel<__nv_bfloat16><<<grid, kThreads, kSmemBytes, s>>>(a);
-  }
-  if (launch_status() != RQ_OK) return RQ_ERR_CUDA;
-  decode_combine_kernel<<<static_cast<unsigned>(desc->B * desc->H_q), kD, 0, s>>>(
-      a.partial, out, a.signs, a.status, a.splits, a.hadamard);
+  const rq_status st = desc->dtype == RQ_F16 ? launch_split<__half>(a, grid, s)
+                                             : launch_split<__nv_bfloat16>(a, grid, s);
+  if (st != RQ_OK) return st;
+  // a whole row per CTA for a rotated cache (the rotation mixes channels),
+  // a quarter of the channels otherwise (four times the CTAs)
+  const int cq = a.hadamard ? 1 : 4;
+  cudaLaunchConfig_t cfg = {};
+  cfg.gridDim = dim3(static_cast<unsigned>(desc->B * desc->H_kv), static_cast<unsigned>(cq));
+  cfg.blockDim = dim3(kThreads);
+  cfg.dynamicSmemBytes = kMergeSmem;
+  cfg.stream = s;
+  cudaLaunchAttribute attr[1];
+  attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+  attr[0].val.programmaticStreamSerializationAllowed = 1;
+  cfg.attrs = attr;
+  cfg.numAttrs = 1;
+  auto kern = a.hadamard ? decode_merge_kernel<1> : decode_merge_kernel<4>;
+  if (cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, kMergeSmem) != cudaSuccess)
+    return RQ_ERR_CUDA;
+  if (cudaLaunchKernelEx(&cfg, kern, static_cast<const float*>(a.partial), out, a.signs, a.status,
+                         a.Hq, a.H, a.g, a.splits, a.hadamard) != cudaSuccess)
+    return RQ_ERR_CUDA;
   return launch_status();
 }
 
@@ -884,7 +1037,7 @@ extern "C" rq_status rq_decode_workspace_bytes(const rq_cache_desc* desc, size_t
   if (current_sm_count(&sms) != RQ_OK) return RQ_ERR_CUDA;
   int splits = 1, bps = 1;
   decode_plan(desc, sms, &splits, &bps);
-  *bytes = static_cast<size_t>(desc->B) * desc->H_q * splits * kPart * sizeof(float);
+  *bytes = workspace_bytes(desc, splits);
   return RQ_OK;
 }
 
@@ -906,11 +1059,9 @@ extern "C" rq_status rq_decode_attention(const rq_cache_desc* desc, int32_t laye
   if (current_sm_count(&sms) != RQ_OK) return RQ_ERR_CUDA;
   int splits = 1, bps = 1;
   decode_plan(desc, sms, &splits, &bps);
-  const size_t need = static_cast<size_t>(desc->B) * desc->H_q * splits * kPart * sizeof(float);
-  if (ws_bytes < need) return RQ_ERR_WORKSPACE;
+  if (ws_bytes < workspace_bytes(desc, splits)) return RQ_ERR_WORKSPACE;
   DecodeArgs a;
-  fill_args(a, desc, layer, q, packed, bits_dev, offsets_dev, signs_dev, static_cast<float*>(ws),
-            status_dev, splits, bps);
+  fill_args(a, desc, layer, q, packed, bits_dev, offsets_dev, signs_dev, ws, status_dev, splits, bps);
   return launch_decode(a, desc, out, static_cast<cudaStream_t>(stream));
 }
 
@@ -967,12 +1118,11 @@ extern "C" rq_status rq_decode_attention_static(const rq_cache_desc* desc, int32
   if (current_sm_count(&sms) != RQ_OK) return RQ_ERR_CUDA;
   int splits = 1, bps = 1;
   decode_plan(desc, sms, &splits, &bps);
-  const size_t need = static_cast<size_t>(desc->B) * desc->H_q * splits * kPart * sizeof(float);
-  if (need > RQ_STATIC_SCRATCH_BYTES) return RQ_ERR_WORKSPACE;
+  if (workspace_bytes(desc, splits) > RQ_STATIC_SCRATCH_BYTES) return RQ_ERR_WORKSPACE;
   float* scratch = nullptr;
   if (static_scratch_ptr(&scratch) != RQ_OK) return RQ_ERR_CUDA;
   DecodeArgs a;
-  fill_args(a, desc, layer, q, packed, bits_dev, offsets_dev, signs_dev, scratch, status_dev,
-            splits, bps);
+  fill_args(a, desc, layer, q, packed, bits_dev, offsets_dev, signs_dev, scratch, status_dev, splits,
+            bps);
   return launch_decode(a, desc, out, static_cast<cudaStream_t>(stream));
 }
