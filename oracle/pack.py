@@ -46,12 +46,15 @@ first, and leftover register l puts its half-h code at spare-stream bits
 
 Meta image (128 words, one fp16 pair each, low half first):
 
-  K per-channel (group = channel c): word c // 2 holds the scales of
-      channels (c, c+1) (c even), word 64 + c // 2 their zeros.
+  K per-channel (group = channel c): for the channel pair P = c // 2,
+      word 2P holds the zeros of channels (2P, 2P+1), word 2P + 1 their
+      scales.
   K per-token (group = (t, G), G = c // 32): word 16*(t % 8) + 4*G + t // 8
       holds (scale, zero).
-  V per-token (group = (t, G)): word 4*(t // 2) + G holds the scales of
-      tokens (t, t+1) (t even), word 64 + 4*(t // 2) + G their zeros.
+  V per-token (group = (t, G)): for the token pair Q = t // 2, word 4Q + G
+      holds the scales of tokens (2Q, 2Q+1), and word
+      64 + 32*(Q >> 3) + 8*(Q & 3) + 4*(G >> 1) + 2*((Q >> 2) & 1) + (G & 1)
+      their zeros.
   V per-channel (group = channel c): word c holds (scale, zero).
 
 Stream order in a packed buffer (``stream_offsets``): layer, batch, kv-head,
@@ -227,15 +230,19 @@ def _group_indices(kind: int, grouping: int):
 def meta_positions(kind: int, grouping: int):
     """For every group of a block (``to_groups`` order): (word index, half).
 
-    For "pairs" layouts the scale goes to ``word``, the zero to ``64 + word``,
-    both in ``half``. For "sz" layouts ``half`` is None: scale low, zero high.
+    For "pairs" layouts ``word`` is a pair (scale word, zero word) and both
+    values go to ``half``. For "sz" layouts ``half`` is None: scale low, zero
+    high in the one word.
     """
     if kind == KIND_K and grouping == PER_CHANNEL:
         c, _ = _group_indices(kind, grouping)
-        return c // 2, c % 2
+        P = c // 2
+        return (2 * P + 1, 2 * P), c % 2
     if kind == KIND_V and grouping == PER_TOKEN:
         t, G = _group_indices(kind, grouping)
-        return 4 * (t // 2) + G, t % 2
+        Q = t // 2
+        zw = 64 + 32 * (Q >> 3) + 8 * (Q & 3) + 4 * (G >> 1) + 2 * ((Q >> 2) & 1) + (G & 1)
+        return (4 * Q + G, zw), t % 2
     if kind == KIND_K and grouping == PER_TOKEN:
         t, G = _group_indices(kind, grouping)
         return 16 * (t % 8) + 4 * G + t // 8, None
@@ -253,11 +260,12 @@ def pack_meta_blocks(scale: np.ndarray, zero: np.ndarray, kind: int, grouping: i
     if half is None:
         out[:, word] = s | (z << np.uint32(16))
     else:
+        sw, zw = word
         # two groups share a word: one pass per half so no index repeats
         for h in (0, 1):
             m = half == h
-            out[:, word[m]] |= s[:, m] << np.uint32(16 * h)
-            out[:, 64 + word[m]] |= z[:, m] << np.uint32(16 * h)
+            out[:, sw[m]] |= s[:, m] << np.uint32(16 * h)
+            out[:, zw[m]] |= z[:, m] << np.uint32(16 * h)
     return out
 
 
@@ -273,9 +281,10 @@ def unpack_meta_blocks(words: np.ndarray, kind: int, grouping: int):
         s = (words[:, word] & 0xFFFF).astype(np.uint16)
         z = (words[:, word] >> 16).astype(np.uint16)
     else:
+        sw, zw = word
         sh = (16 * half).astype(np.uint32)
-        s = ((words[:, word] >> sh) & 0xFFFF).astype(np.uint16)
-        z = ((words[:, 64 + word] >> sh) & 0xFFFF).astype(np.uint16)
+        s = ((words[:, sw] >> sh) & 0xFFFF).astype(np.uint16)
+        z = ((words[:, zw] >> sh) & 0xFFFF).astype(np.uint16)
     return s.view(np.float16), z.view(np.float16)
 
 

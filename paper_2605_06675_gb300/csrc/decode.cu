@@ -205,18 +205,20 @@ __device__ __forceinline__ void qk_block(const uint8_t* img, int lane, const uin
     float zb[4] = {0.0f, 0.0f, 0.0f, 0.0f};
 #pragma unroll
     for (int u = 0; u < 4; ++u) {
-      // scale / zero pairs of channels 32u + 8tig + 2x: words 16u + 4tig + x
-      const uint4 S = lds128(meta + 4 * (16 * u + 4 * tig));
-      const uint4 Z = lds128(meta + 256 + 4 * (16 * u + 4 * tig));
+      // channel pairs P = 16u + 4tig + x: zeros at word 2P, scales at 2P + 1,
+      // so each 16-byte read {z(x), s(x), z(x+1), s(x+1)} is the A operand of
+      // a zero-point MMA (rows gid take z; rows gid + 8 take s and are unused)
+      const uint4 MZ0 = lds128(meta + 4 * (32 * u + 8 * tig));
+      const uint4 MZ1 = lds128(meta + 4 * (32 * u + 8 * tig + 4));
       const uint4 QB = lds128(qtab + 16 * (32 * u + lane));
       const uint4 QF = lds128(qtab + 2048 + 16 * (32 * u + lane));
-      const uint32_t S2[4] = {S.x, S.y, S.z, S.w}, Z2[4] = {Z.x, Z.y, Z.z, Z.w};
       const uint32_t qb[4] = {QB.x, QB.y, QB.z, QB.w}, qf[4] = {QF.x, QF.y, QF.z, QF.w};
 #pragma unroll
       for (int xs = 0; xs < 2; ++xs) {
-        const uint32_t b0 = hmul2u(qf[2 * xs], S2[2 * xs]);
-        const uint32_t b1 = hmul2u(qf[2 * xs + 1], S2[2 * xs + 1]);
-        const uint32_t az[4] = {Z2[2 * xs], 0u, Z2[2 * xs + 1], 0u};
+        const uint4 MZ = xs ? MZ1 : MZ0;
+        const uint32_t b0 = hmul2u(qf[2 * xs], MZ.y);
+        const uint32_t b1 = hmul2u(qf[2 * xs + 1], MZ.w);
+        const uint32_t az[4] = {MZ.x, MZ.y, MZ.z, MZ.w};
         mma16816(zb, az, qb[2 * xs], qb[2 * xs + 1]);
 #pragma unroll
         for (int mt = 0; mt < 2; ++mt) {
@@ -282,15 +284,17 @@ __device__ __forceinline__ void pv_block(const uint8_t* img, int lane, const uin
   if constexpr (VG == RQ_PER_TOKEN) {
     // zero-points: rows gid of the A operand carry group 2gp, rows gid + 8
     // group 2gp + 1; columns are token pairs 2ks (k 2tig..) and 2ks + 1.
-    // Zero pairs of token pair y, groups 0..3: words 64 + 16y + 4tig + G.
+    // Zero pairs are stored so that each 16-byte read is an A operand:
+    // words 64 + 32ks + 8tig + 4gp + {0..3} = z of (token pair 2ks, group
+    // 2gp), (2ks, 2gp+1), (2ks+1, 2gp), (2ks+1, 2gp+1).
 #pragma unroll
-    for (int ks = 0; ks < 2; ++ks) {
-      const uint4 Z0 = lds128(meta + 256 + 4 * (16 * (2 * ks) + 4 * tig));
-      const uint4 Z1 = lds128(meta + 256 + 4 * (16 * (2 * ks + 1) + 4 * tig));
-      const uint32_t az0[4] = {Z0.x, Z0.y, Z1.x, Z1.y}, az1[4] = {Z0.z, Z0.w, Z1.z, Z1.w};
-      mma16816(bz[0], az0, pb[ks][0], pb[ks][1]);
-      mma16816(bz[1], az1, pb[ks][0], pb[ks][1]);
-    }
+    for (int ks = 0; ks < 2; ++ks)
+#pragma unroll
+      for (int gp = 0; gp < 2; ++gp) {
+        const uint4 Z = lds128(meta + 4 * (64 + 32 * ks + 8 * tig + 4 * gp));
+        const uint32_t az[4] = {Z.x, Z.y, Z.z, Z.w};
+        mma16816(bz[gp], az, pb[ks][0], pb[ks][1]);
+      }
     uint32_t ms[4][4];        // scale pairs [token pair y][group G]: words 16y + 4tig + G
 #pragma unroll
     for (int y = 0; y < 4; ++y) {

@@ -176,9 +176,10 @@ __device__ __forceinline__ GroupOut finish_group(int kind, int grouping, int t, 
   int slot;
   if (grouping == RQ_PER_CHANNEL) {
     slot = c;
-    if (kind == 0) {                          // scale / zero pairs of channels (c, c^1)
-      m16[c] = static_cast<uint16_t>(sb);
-      m16[128 + c] = static_cast<uint16_t>(zb);
+    if (kind == 0) {                          // pair P = c / 2: zeros at word 2P, scales at 2P + 1
+      const int P = c >> 1, hh = c & 1;
+      m16[4 * P + 2 + hh] = static_cast<uint16_t>(sb);
+      m16[4 * P + hh] = static_cast<uint16_t>(zb);
     } else {
       m32[c] = sb | (zb << 16);
     }
@@ -187,9 +188,10 @@ __device__ __forceinline__ GroupOut finish_group(int kind, int grouping, int t, 
     if (kind == 0) {
       m32[16 * (t & 7) + 4 * G + (t >> 3)] = sb | (zb << 16);
     } else {                                  // scale / zero pairs of tokens (t, t^1)
-      const int i = 2 * (4 * (t >> 1) + G) + (t & 1);
-      m16[i] = static_cast<uint16_t>(sb);
-      m16[128 + i] = static_cast<uint16_t>(zb);
+      const int Q = t >> 1;
+      const int zw = 64 + 32 * (Q >> 3) + 8 * (Q & 3) + 4 * (G >> 1) + 2 * ((Q >> 2) & 1) + (G & 1);
+      m16[2 * (4 * Q + G) + (t & 1)] = static_cast<uint16_t>(sb);
+      m16[2 * zw + (t & 1)] = static_cast<uint16_t>(zb);
     }
   }
   sm.nz[slot] = -g.zf;

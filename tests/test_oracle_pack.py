@@ -128,25 +128,34 @@ def _h(x):
 
 
 def test_hand_meta_words():
-    # K per-channel, scale_c = c, zero_c = -c - 1: word c // 2 = scales of
-    # (c, c+1), word 64 + c // 2 their zeros.
+    # K per-channel, scale_c = c, zero_c = -c - 1: for the channel pair P,
+    # word 2P = zeros of (2P, 2P+1), word 2P + 1 = their scales.
     c = np.arange(128)
     w = pack.pack_meta_block(c.astype(np.float16), (-c - 1).astype(np.float16),
                              pack.KIND_K, PER_CHANNEL)
-    assert w[0] == (_h(1) << 16) | _h(0)           # channels (0, 1)
-    assert w[1] == (_h(3) << 16) | _h(2)           # channels (2, 3)
-    assert w[64] == (_h(-2) << 16) | _h(-1)        # zeros of channels (0, 1)
-    assert w[0] == 0x3C000000 and w[1] == 0x42004000 and w[64] == 0xC000BC00
-    # V per-token, group (t, G), scale = 4t + G: word 4 (t // 2) + G = scales
-    # of tokens (t, t+1).
+    assert w[1] == (_h(1) << 16) | _h(0)           # scales of channels (0, 1)
+    assert w[3] == (_h(3) << 16) | _h(2)           # scales of channels (2, 3)
+    assert w[0] == (_h(-2) << 16) | _h(-1)         # zeros of channels (0, 1)
+    assert w[1] == 0x3C000000 and w[3] == 0x42004000 and w[0] == 0xC000BC00
+    # V per-token, group (t, G), scale = 4t + G, zero = -(4t + G): word 4Q + G
+    # = scales of tokens (2Q, 2Q+1); zeros at 64 + 32(Q>>3) + 8(Q&3) + 4(G>>1)
+    # + 2((Q>>2)&1) + (G&1).
     tt = np.repeat(np.arange(32), 4)
     GG = np.tile(np.arange(4), 32)
     s = (4 * tt + GG).astype(np.float16)
-    w = pack.pack_meta_block(s, np.zeros(128, np.float16), pack.KIND_V, PER_TOKEN)
+    w = pack.pack_meta_block(s, -s, pack.KIND_V, PER_TOKEN)
     assert w[0] == 0x44000000                       # tokens (0,1), G 0: 0, 4
     assert w[1] == 0x45003C00                       # tokens (0,1), G 1: 1, 5
     assert w[4] == 0x4A004800                       # tokens (2,3), G 0: 8, 12
     assert w[16] == 0x50805000                      # tokens (8,9), G 0: 32, 36
+    # zeros: Q = 0, G = 0 -> word 64; Q = 0, G = 1 -> 65; Q = 4 (tokens 8, 9),
+    # G = 0 -> 64 + 2 = 66; Q = 1 (tokens 2, 3), G = 2 -> 64 + 8 + 4 = 76;
+    # Q = 8 (tokens 16, 17), G = 3 -> 64 + 32 + 4 + 1 = 101 (zeros -67, -71)
+    assert w[64] == (_h(-4) << 16) | 0x8000          # -0 and -4
+    assert w[65] == (_h(-5) << 16) | _h(-1)
+    assert w[66] == (_h(-36) << 16) | _h(-32)
+    assert w[76] == (_h(-14) << 16) | _h(-10)
+    assert w[101] == (_h(-71) << 16) | _h(-67)
     # K per-token: word = (scale, zero) of group (t, G) at 16(t%8) + 4G + t//8.
     w = pack.pack_meta_block(s, -s, pack.KIND_K, PER_TOKEN)
     assert w[0] == (0x8000 << 16)                    # t = 0, G = 0: scale 0, zero -0
@@ -175,7 +184,9 @@ def test_meta_round_trip(kind, grouping):
     if half is None:
         assert sorted(word.tolist()) == list(range(128))
     else:
-        assert sorted((2 * word + half).tolist()) == list(range(128))
+        sw, zw = word
+        slots = np.concatenate([2 * sw + half, 2 * zw + half])
+        assert sorted(slots.tolist()) == list(range(256))
 
 
 def test_stream_round_trip():
