@@ -190,9 +190,11 @@ __device__ __forceinline__ uint32_t dequant(uint32_t sub, uint32_t m, uint32_t z
 // exact fp16 subnormals c 2^(E - 24); the accumulator is scaled by 2^24.
 // q operands of lane L for unit u: qtab + 16 (32 u + L) holds q pairs x = 0..3
 // (channels 32u + 8tig + 2x), qtab + 2048 + the same with 2^-E(x) folded in.
+// s is returned relative to the running max (ms0, ms1: the max of heads
+// 2tig, 2tig + 1, 0 while unset).
 template <int BW, int KG>
 __device__ __forceinline__ void qk_block(const uint8_t* img, int lane, const uint8_t* qtab,
-                                         float (&s)[2][4]) {
+                                         float ms0, float ms1, float (&s)[2][4]) {
   const int gid = lane >> 2, tig = lane & 3;
   uint32_t w[4 * BW];
   lane_words<BW>(img, lane, w);
@@ -228,12 +230,13 @@ __device__ __forceinline__ void qk_block(const uint8_t* img, int lane, const uin
         }
       }
     }
+    const float c0 = zb[0] - ms0, c1 = zb[1] - ms1;
 #pragma unroll
     for (int mt = 0; mt < 2; ++mt) {
-      s[mt][0] = __fmaf_rn(s[mt][0], kTwo24, zb[0]);
-      s[mt][1] = __fmaf_rn(s[mt][1], kTwo24, zb[1]);
-      s[mt][2] = __fmaf_rn(s[mt][2], kTwo24, zb[0]);
-      s[mt][3] = __fmaf_rn(s[mt][3], kTwo24, zb[1]);
+      s[mt][0] = __fmaf_rn(s[mt][0], kTwo24, c0);
+      s[mt][1] = __fmaf_rn(s[mt][1], kTwo24, c1);
+      s[mt][2] = __fmaf_rn(s[mt][2], kTwo24, c0);
+      s[mt][3] = __fmaf_rn(s[mt][3], kTwo24, c1);
     }
   } else {                    // per-token keys: dequantize in registers
 #pragma unroll
@@ -262,6 +265,13 @@ __device__ __forceinline__ void qk_block(const uint8_t* img, int lane, const uin
               dequant(reg<BW>(w, u, 2 * mt + 1, 2 * xs + 1), m[2 * mt + 1], z2[2 * mt + 1])};
           mma16816(s[mt], a, qb[2 * xs], qb[2 * xs + 1]);
         }
+    }
+#pragma unroll
+    for (int mt = 0; mt < 2; ++mt) {
+      s[mt][0] -= ms0;
+      s[mt][1] -= ms1;
+      s[mt][2] -= ms0;
+      s[mt][3] -= ms1;
     }
   }
 }
@@ -348,9 +358,10 @@ __device__ __forceinline__ void pv_block(const uint8_t* img, int lane, const uin
 
 template <int BW>
 __device__ __forceinline__ void qk_dispatch_g(int kg, const uint8_t* img, int lane,
-                                              const uint8_t* qtab, float (&s)[2][4]) {
-  if (kg == RQ_PER_CHANNEL) qk_block<BW, RQ_PER_CHANNEL>(img, lane, qtab, s);
-  else qk_block<BW, RQ_PER_TOKEN>(img, lane, qtab, s);
+                                              const uint8_t* qtab, float ms0, float ms1,
+                                              float (&s)[2][4]) {
+  if (kg == RQ_PER_CHANNEL) qk_block<BW, RQ_PER_CHANNEL>(img, lane, qtab, ms0, ms1, s);
+  else qk_block<BW, RQ_PER_TOKEN>(img, lane, qtab, ms0, ms1, s);
 }
 
 template <int BW>
@@ -362,16 +373,17 @@ __device__ __forceinline__ void pv_dispatch_g(int vg, const uint8_t* img, int la
 }
 
 __device__ __forceinline__ void qk_dispatch(int bw, int kg, const uint8_t* img, int lane,
-                                            const uint8_t* qtab, float (&s)[2][4]) {
+                                            const uint8_t* qtab, float ms0, float ms1,
+                                            float (&s)[2][4]) {
   switch (bw) {
-    case 1: qk_dispatch_g<1>(kg, img, lane, qtab, s); break;
-    case 2: qk_dispatch_g<2>(kg, img, lane, qtab, s); break;
-    case 3: qk_dispatch_g<3>(kg, img, lane, qtab, s); break;
-    case 4: qk_dispatch_g<4>(kg, img, lane, qtab, s); break;
-    case 5: qk_dispatch_g<5>(kg, img, lane, qtab, s); break;
-    case 6: qk_dispatch_g<6>(kg, img, lane, qtab, s); break;
-    case 7: qk_dispatch_g<7>(kg, img, lane, qtab, s); break;
-    default: qk_dispatch_g<8>(kg, img, lane, qtab, s); break;
+    case 1: qk_dispatch_g<1>(kg, img, lane, qtab, ms0, ms1, s); break;
+    case 2: qk_dispatch_g<2>(kg, img, lane, qtab, ms0, ms1, s); break;
+    case 3: qk_dispatch_g<3>(kg, img, lane, qtab, ms0, ms1, s); break;
+    case 4: qk_dispatch_g<4>(kg, img, lane, qtab, ms0, ms1, s); break;
+    case 5: qk_dispatch_g<5>(kg, img, lane, qtab, ms0, ms1, s); break;
+    case 6: qk_dispatch_g<6>(kg, img, lane, qtab, ms0, ms1, s); break;
+    case 7: qk_dispatch_g<7>(kg, img, lane, qtab, ms0, ms1, s); break;
+    default: qk_dispatch_g<8>(kg, img, lane, qtab, ms0, ms1, s); break;
   }
 }
 
@@ -442,18 +454,42 @@ struct SoftmaxAcc {
 // exceeds it by more than 8, so p <= 2^8 and rescaling is rare.
 __device__ __forceinline__ void softmax_block(float (&s)[2][4], SoftmaxAcc& acc,
                                               uint32_t (&pb)[2][2]) {
+  // s holds score - running max (log2 units). Each lane checks its own
+  // values; only when one exceeds the bound is the column max reduced across
+  // the lanes and the running max moved (rare), so p <= 2^8 always.
   float bm0 = fmaxf(fmaxf(s[0][0], s[0][2]), fmaxf(s[1][0], s[1][2]));
   float bm1 = fmaxf(fmaxf(s[0][1], s[0][3]), fmaxf(s[1][1], s[1][3]));
+  const bool first = acc.m0 == -INFINITY;      // the warp's first block: set the max
+  if (__any_sync(0xffffffffu, first || bm0 > 8.0f || bm1 > 8.0f)) {
 #pragma unroll
-  for (int off = 4; off <= 16; off <<= 1) {
-    bm0 = fmaxf(bm0, __shfl_xor_sync(0xffffffffu, bm0, off));
-    bm1 = fmaxf(bm1, __shfl_xor_sync(0xffffffffu, bm1, off));
-  }
-  if (__any_sync(0xffffffffu, bm0 > acc.m0 + 8.0f || bm1 > acc.m1 + 8.0f)) {
-    const float nm0 = fmaxf(acc.m0, bm0), nm1 = fmaxf(acc.m1, bm1);
-    const float al0 = fast_exp2(acc.m0 - nm0), al1 = fast_exp2(acc.m1 - nm1);
-    acc.m0 = nm0;
-    acc.m1 = nm1;
+    for (int off = 4; off <= 16; off <<= 1) {
+      bm0 = fmaxf(bm0, __shfl_xor_sync(0xffffffffu, bm0, off));
+      bm1 = fmaxf(bm1, __shfl_xor_sync(0xffffffffu, bm1, off));
+    }
+    // first block: max = block max (s holds raw scores); later: the max moves
+    // up by d = max(block max - m, 0) and the state is scaled by 2^-d
+    float d0, d1, al0, al1;
+    if (first) {
+      d0 = bm0;
+      d1 = bm1;
+      al0 = al1 = 0.0f;
+      acc.m0 = bm0;
+      acc.m1 = bm1;
+    } else {
+      d0 = fmaxf(bm0, 0.0f);
+      d1 = fmaxf(bm1, 0.0f);
+      al0 = fast_exp2(-d0);
+      al1 = fast_exp2(-d1);
+      acc.m0 += d0;
+      acc.m1 += d1;
+    }
+#pragma unroll
+    for (int mt = 0; mt < 2; ++mt) {
+      s[mt][0] -= d0;
+      s[mt][1] -= d1;
+      s[mt][2] -= d0;
+      s[mt][3] -= d1;
+    }
     acc.l0 *= al0;
     acc.l1 *= al1;
 #pragma unroll
@@ -473,12 +509,9 @@ __device__ __forceinline__ void softmax_block(float (&s)[2][4], SoftmaxAcc& acc,
   }
   float p[2][4];
 #pragma unroll
-  for (int mt = 0; mt < 2; ++mt) {
-    p[mt][0] = fast_exp2(s[mt][0] - acc.m0);
-    p[mt][1] = fast_exp2(s[mt][1] - acc.m1);
-    p[mt][2] = fast_exp2(s[mt][2] - acc.m0);
-    p[mt][3] = fast_exp2(s[mt][3] - acc.m1);
-  }
+  for (int mt = 0; mt < 2; ++mt)
+#pragma unroll
+    for (int r = 0; r < 4; ++r) p[mt][r] = fast_exp2(s[mt][r]);
   acc.l0 += (p[0][0] + p[0][2]) + (p[1][0] + p[1][2]);
   acc.l1 += (p[0][1] + p[0][3]) + (p[1][1] + p[1][3]);
 #pragma unroll
@@ -536,7 +569,8 @@ __device__ __forceinline__ void blocks_static(const WarpStream& ws, const uint8_
     cp_async_wait<NS - 1>();
     __syncwarp();
     float s[2][4];
-    qk_block<BK, KG>(ws.ring_ptr + use * R::kSlot, ws.lane, qtab, s);
+    qk_block<BK, KG>(ws.ring_ptr + use * R::kSlot, ws.lane, qtab, acc.m0 == -INFINITY ? 0.0f : acc.m0,
+                     acc.m1 == -INFINITY ? 0.0f : acc.m1, s);
     __syncwarp();
     use = use + 1 == NS ? 0 : use + 1;
     uint32_t pb[2][2];
@@ -577,7 +611,8 @@ __device__ __forceinline__ void blocks_dyn(const WarpStream& ws, const DynRing& 
     cp_async_wait_dyn(r.ns - 1);
     __syncwarp();
     float s[2][4];
-    qk_dispatch(r.bK, r.kg, ws.ring_ptr + use * r.slot, ws.lane, qtab, s);
+    qk_dispatch(r.bK, r.kg, ws.ring_ptr + use * r.slot, ws.lane, qtab,
+                acc.m0 == -INFINITY ? 0.0f : acc.m0, acc.m1 == -INFINITY ? 0.0f : acc.m1, s);
     __syncwarp();
     use = use + 1 == r.ns ? 0 : use + 1;
     uint32_t pb[2][2];
