@@ -9,19 +9,21 @@
 //
 // Design (sm_103a): one CTA = (split of the sequence, kv head, batch), four
 // warps, each warp walking its own 32-token blocks. Per block a warp runs
-//   scores^T[32 tok x 8 heads] = K_hat[32 x 128] . q^T      (16 x mma m16n8k16)
+//   scores^T[32 tok x 8 heads] = K_hat[32 x 128] . q^T      (mma m16n8k16)
 //   online softmax in fp32 (log2 domain), P^T via movmatrix.trans
-//   o^T[128 x 8 heads]       += V_hat^T[128 x 32] . P^T    (16 x mma m16n8k16)
+//   o^T[128 x 8 heads]       += V_hat^T[128 x 32] . P^T    (mma m16n8k16)
 // The GQA group (g <= 8 query heads) is the MMA n dimension, so it is never
 // padded to 16. Each warp streams its K and V block images through its own
 // ring of shared-memory slots with cp.async, several entries ahead of use.
-// Codes are read in the MMA-fragment order the quantizer wrote and turned into
-// exact fp16 integers with the fp16-1024 exponent trick (a code placed in the
-// mantissa of 1024, scaled by a power of two, removed with one fp16x2 FMA).
-// For the KIVI layouts (per-channel keys, per-token values) the group scale
-// is folded into the small MMA operand (q or P) and the zero-points are added
-// by extra MMAs, so the codes enter the tensor cores undequantized; the other
-// layouts dequantize in registers with one fp16x2 FMA (scale, zero).
+// Codes are stored in the MMA-fragment order of format.cuh: one AND of a
+// word yields a register's two codes as exact fp16 subnormals c * 2^(E - 24)
+// that enter the tensor cores undequantized. For the KIVI layouts
+// (per-channel keys, per-token values) the group scales and 2^-E are folded
+// into the small operand (q or P) or the output rows, and the zero-points are
+// added by extra MMAs whose A operand is the meta image as read; the other
+// layouts dequantize in registers (fp16 1024 exponent, one fp16x2 FMA).
+// Split records are merged by decode_merge_kernel, a programmatic dependent
+// launch of the split kernel.
 #include <algorithm>
 #include <atomic>
 
