@@ -80,7 +80,9 @@ template <int B>
 __device__ __forceinline__ void place(uint32_t (&uw)[B], int x, int y, uint32_t P) {
   const Loc l = location(B, x, y);
   if (l.left < 0) {
-    uw[l.w] |= P << (B * l.k);
+    // the slot's bits are still zero, so adding the shifted pair sets them
+    // (one multiply-add instead of a shift and an OR)
+    uw[l.w] += P * (1u << (B * l.k));
   } else if constexpr (spare(B) > 0) {
     constexpr int n = 16 / B, r = spare(B);
 #pragma unroll
