@@ -974,15 +974,50 @@ __global__ void __launch_bounds__(kThreads) decode_merge_kernel(const float* par
   }
 }
 
-void decode_plan(const rq_cache_desc* desc, int sms, int* splits, int* bps) {
+// Resident split-kernel CTAs per SM on the current device (cached per device).
+rq_status split_ctas_per_sm(int* per_sm) {
+  static std::atomic<int> cache[64];
+  int dev = 0;
+  if (cudaGetDevice(&dev) != cudaSuccess) return RQ_ERR_CUDA;
+  if (dev >= 0 && dev < 64) {
+    const int c = cache[dev].load(std::memory_order_relaxed);
+    if (c > 0) {
+      *per_sm = c;
+      return RQ_OK;
+    }
+  }
+  auto kern = decode_split_kernel<__nv_bfloat16>;
+  if (cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, kSmemBytes) != cudaSuccess ||
+      cudaFuncSetAttribute(kern, cudaFuncAttributePreferredSharedMemoryCarveout,
+                           cudaSharedmemCarveoutMaxShared) != cudaSuccess)
+    return RQ_ERR_CUDA;
+  int v = 0;
+  if (cudaOccupancyMaxActiveBlocksPerMultiprocessor(&v, kern, kThreads, kSmemBytes) != cudaSuccess)
+    return RQ_ERR_CUDA;
+  v = std::max(v, 1);
+  if (dev >= 0 && dev < 64) cache[dev].store(v, std::memory_order_relaxed);
+  *per_sm = v;
+  return RQ_OK;
+}
+
+// Splits of the sequence per (batch, kv head): as many as fit in one wave of
+// resident CTAs (slots = SMs x CTAs per SM), so every CTA streams a long run
+// of blocks and none waits for a second wave; at least one.
+void decode_plan(const rq_cache_desc* desc, int slots, int* splits, int* bps) {
   const int nblk = desc->S / kTile;
   const long long units = static_cast<long long>(desc->B) * desc->H_kv;
-  const long long target = static_cast<long long>(sms) * 16;
-  long long sp = units > 0 ? (target + units - 1) / units : 1;
+  long long sp = units > 0 ? slots / units : 1;
   sp = std::max<long long>(1, std::min<long long>(sp, nblk));
   const int b = static_cast<int>((nblk + sp - 1) / sp);
   *bps = std::max(b, 1);
   *splits = std::max(1, (nblk + *bps - 1) / *bps);
+}
+
+rq_status decode_slots(int* slots) {
+  int sms = 0, per_sm = 0;
+  if (current_sm_count(&sms) != RQ_OK || split_ctas_per_sm(&per_sm) != RQ_OK) return RQ_ERR_CUDA;
+  *slots = sms * per_sm;
+  return RQ_OK;
 }
 
 rq_status check_desc(const rq_cache_desc* desc) {
@@ -1074,10 +1109,10 @@ extern "C" rq_status rq_decode_workspace_bytes(const rq_cache_desc* desc, size_t
   if (!bytes) return RQ_ERR_INVALID_ARG;
   const rq_status st = check_desc(desc);
   if (st != RQ_OK) return st;
-  int sms = 0;
-  if (current_sm_count(&sms) != RQ_OK) return RQ_ERR_CUDA;
+  int slots = 0;
+  if (decode_slots(&slots) != RQ_OK) return RQ_ERR_CUDA;
   int splits = 1, bps = 1;
-  decode_plan(desc, sms, &splits, &bps);
+  decode_plan(desc, slots, &splits, &bps);
   *bytes = workspace_bytes(desc, splits);
   return RQ_OK;
 }
@@ -1096,10 +1131,10 @@ extern "C" rq_status rq_decode_attention(const rq_cache_desc* desc, int32_t laye
       (reinterpret_cast<uintptr_t>(out) & 3u))
     return RQ_ERR_ALIGNMENT;
   if (desc->B == 0) return RQ_OK;
-  int sms = 0;
-  if (current_sm_count(&sms) != RQ_OK) return RQ_ERR_CUDA;
+  int slots = 0;
+  if (decode_slots(&slots) != RQ_OK) return RQ_ERR_CUDA;
   int splits = 1, bps = 1;
-  decode_plan(desc, sms, &splits, &bps);
+  decode_plan(desc, slots, &splits, &bps);
   if (ws_bytes < workspace_bytes(desc, splits)) return RQ_ERR_WORKSPACE;
   DecodeArgs a;
   fill_args(a, desc, layer, q, packed, bits_dev, offsets_dev, signs_dev, ws, status_dev, splits, bps);
@@ -1155,10 +1190,10 @@ extern "C" rq_status rq_decode_attention_static(const rq_cache_desc* desc, int32
       (reinterpret_cast<uintptr_t>(out) & 3u))
     return RQ_ERR_ALIGNMENT;
   if (desc->B == 0) return RQ_OK;
-  int sms = 0;
-  if (current_sm_count(&sms) != RQ_OK) return RQ_ERR_CUDA;
+  int slots = 0;
+  if (decode_slots(&slots) != RQ_OK) return RQ_ERR_CUDA;
   int splits = 1, bps = 1;
-  decode_plan(desc, sms, &splits, &bps);
+  decode_plan(desc, slots, &splits, &bps);
   if (workspace_bytes(desc, splits) > RQ_STATIC_SCRATCH_BYTES) return RQ_ERR_WORKSPACE;
   float* scratch = nullptr;
   if (static_scratch_ptr(&scratch) != RQ_OK) return RQ_ERR_CUDA;
