@@ -165,8 +165,20 @@ class ClockSampler:
 # were taken on)
 # --------------------------------------------------------------------------
 
-def recorded_traffic(kernel: str, workload: str):
+def kernel_source_hash(name: str) -> str:
+    """sha256[:16] of a kernel's translation unit together with the headers it
+    includes (format.cuh, rq_internal.cuh, rq.h), so a record goes stale when
+    any of them changes."""
     import hashlib
+    csrc = os.path.join(ROOT, "paper_2605_06675_gb300", "csrc")
+    h = hashlib.sha256()
+    for path in (os.path.join(csrc, name), os.path.join(csrc, "format.cuh"),
+                 os.path.join(csrc, "rq_internal.cuh"), os.path.join(ROOT, "include", "rq.h")):
+        h.update(open(path, "rb").read())
+    return h.hexdigest()[:16]
+
+
+def recorded_traffic(kernel: str, workload: str):
     path = os.path.join(ROOT, "profiles", "traffic.txt")
     if not os.path.exists(path):
         return None
@@ -176,10 +188,8 @@ def recorded_traffic(kernel: str, workload: str):
         parts = line.split()
         if len(parts) < 4 or parts[0] != kernel or parts[1] != workload:
             continue
-        src = os.path.join(ROOT, "paper_2605_06675_gb300", "csrc", parts[3].split(":")[0])
-        want = parts[3].split(":")[1]
-        have = hashlib.sha256(open(src, "rb").read()).hexdigest()[:16]
-        return float(parts[2]) if have == want else None
+        src, want = parts[3].split(":")
+        return float(parts[2]) if kernel_source_hash(src) == want else None
     return None
 
 
