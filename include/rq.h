@@ -220,6 +220,48 @@ rq_status rq_decode_attention_static(const rq_cache_desc* desc, int32_t layer, c
                                      const uint64_t* offsets_dev, const int8_t* signs_dev,
                                      float* out, uint32_t* status_dev, void* stream);
 
+/* ---- Decode-time append (KIVI-style residual window) ----------------------
+ * The paper allocates bits per head uniformly over token positions (appendix
+ * "Scope and Extensions", "Design choices"), so a token appended during
+ * decoding is stored at its head's widths like every other. Per-channel key
+ * groups span 32 tokens, so the open block of every stream stays unquantized
+ * in a residual window of 32 tokens (the KIVI residual, Sec. 2) until it is
+ * full; it is then quantized and packed exactly as rq_quantize_pack packs
+ * that block. desc->S is the cache's capacity in tokens (a multiple of 32);
+ * the packed buffer and offsets are those of rq_packed_layout(desc). */
+
+/* Bytes of the residual windows of a cache: [L][B][H_kv][2][32][128] values of
+ * desc->dtype, K then V per (layer, batch, kv head); token t sits in slot
+ * t % 32. 0 for an invalid descriptor. */
+size_t rq_residual_bytes(const rq_cache_desc* desc);
+
+/* Append the token at position pos (0 <= pos < desc->S, the same position for
+ * every batch row) of one layer: k_new, v_new: device [B][H_kv][128] of
+ * desc->dtype (16-byte aligned) are written to slot pos % 32 of the layer's
+ * residual windows (device, rq_residual_bytes, 16-byte aligned). When
+ * pos % 32 == 31 the windows are full and block pos / 32 of every stream of
+ * the layer is quantized (and rotated with desc->hadamard) and packed into
+ * `packed` at the widths of bits_dev; the windows are then free for the next
+ * block. signs_dev, status_dev as in rq_quantize_pack.
+ * Errors: RQ_ERR_INVALID_ARG (null pointers, layer or pos out of range),
+ * RQ_ERR_SHAPE, RQ_ERR_ALIGNMENT, RQ_ERR_CUDA. */
+rq_status rq_append(const rq_cache_desc* desc, int32_t layer, int32_t pos, const void* k_new,
+                    const void* v_new, void* residual, const int8_t* signs_dev,
+                    const uint8_t* bits_dev, const uint64_t* offsets_dev, void* packed,
+                    uint32_t* status_dev, void* stream);
+
+/* Decode attention over the first n_tokens (1 <= n_tokens <= desc->S) of one
+ * layer: tokens below 32 * (n_tokens / 32) from the packed blocks, the last
+ * n_tokens % 32 from the residual windows (unquantized; slots 0..). Otherwise
+ * as rq_decode_attention (same workspace size, ws of
+ * rq_decode_workspace_bytes(desc)); residual may be NULL when
+ * n_tokens % 32 == 0. */
+rq_status rq_decode_attention_len(const rq_cache_desc* desc, int32_t layer, int32_t n_tokens,
+                                  const void* q, const void* packed, const uint8_t* bits_dev,
+                                  const uint64_t* offsets_dev, const int8_t* signs_dev,
+                                  const void* residual, float* out, void* ws, size_t ws_bytes,
+                                  uint32_t* status_dev, void* stream);
+
 #ifdef __cplusplus
 }
 #endif

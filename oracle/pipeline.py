@@ -69,3 +69,32 @@ def attend_layer(q, qlayer, batches=None, heads=None):
             qs = q[bb, h * g:(h + 1) * g]
             out[bb, h * g:(h + 1) * g] = decode_attention(qs, kh, vh)
     return out
+
+
+def attend_with_residual(q, qlayer, k_res, v_res, batches=None, heads=None):
+    """Decode attention over a packed prefix plus unquantized residual tokens
+    (decode-time append: the open 32-token block stays unquantized, as in
+    KIVI's residual, Sec. 2; allocation is uniform over positions, appendix
+    "Scope and Extensions").
+
+    q [B][H_q][128]; ``qlayer``: ``quantize_layer`` output of the packed prefix
+    (empty dict when no block is packed yet); k_res, v_res [B][H_kv][R][128]
+    the residual tokens in the original domain (R may be 0). Returns out
+    [B][H_q][128] float32.
+    """
+    q = np.asarray(q, dtype=np.float32)
+    k_res = np.asarray(k_res, dtype=np.float64)
+    v_res = np.asarray(v_res, dtype=np.float64)
+    B, Hq, d = q.shape
+    Hkv = k_res.shape[1]
+    g = Hq // Hkv
+    out = np.zeros((B, Hq, d), dtype=np.float32)
+    for bb in (range(B) if batches is None else batches):
+        for h in (range(Hkv) if heads is None else heads):
+            kh, vh = k_res[bb, h], v_res[bb, h]
+            if (bb, h, 0) in qlayer:
+                kh = np.concatenate([qlayer[(bb, h, 0)]["xhat"], kh], axis=0)
+                vh = np.concatenate([qlayer[(bb, h, 1)]["xhat"], vh], axis=0)
+            out[bb, h * g:(h + 1) * g] = decode_attention(q[bb, h * g:(h + 1) * g], kh[None],
+                                                          vh[None])
+    return out

@@ -192,11 +192,12 @@ __device__ __forceinline__ uint32_t dequant(uint32_t sub, uint32_t m, uint32_t z
 // exact fp16 subnormals c 2^(E - 24); the accumulator is scaled by 2^24.
 // q operands of lane L for unit u: qtab + 16 (32 u + L) holds q pairs x = 0..3
 // (channels 32u + 8tig + 2x), qtab + 2048 + the same with 2^-E(x) folded in.
-// s is returned relative to the running max (ms0, ms1: the max of heads
-// 2tig, 2tig + 1, 0 while unset).
+// s is returned in log2 units (q . k times qsc = log2(e) / sqrt(128), applied
+// here in fp32 so q enters the MMAs unscaled) relative to the running max
+// (ms0, ms1: the max of heads 2tig, 2tig + 1, 0 while unset).
 template <int BW, int KG>
 __device__ __forceinline__ void qk_block(const uint8_t* img, int lane, const uint8_t* qtab,
-                                         float ms0, float ms1, float (&s)[2][4]) {
+                                         float qsc, float ms0, float ms1, float (&s)[2][4]) {
   const int gid = lane >> 2, tig = lane & 3;
   uint32_t w[4 * BW];
   lane_words<BW>(img, lane, w);
@@ -220,8 +221,12 @@ __device__ __forceinline__ void qk_block(const uint8_t* img, int lane, const uin
 #pragma unroll
       for (int xs = 0; xs < 2; ++xs) {
         const uint4 MZ = xs ? MZ1 : MZ0;
+        // q s 2^-E as an fp16 pair sum hi + lo: lo = fp16(q s 2^-E - hi) is
+        // the exact remainder (one fp16 FMA), so the products keep ~22 bits
         const uint32_t b0 = hmul2u(qf[2 * xs], MZ.y);
         const uint32_t b1 = hmul2u(qf[2 * xs + 1], MZ.w);
+        const uint32_t l0 = hfma2u(qf[2 * xs], MZ.y, b0 ^ 0x80008000u);
+        const uint32_t l1 = hfma2u(qf[2 * xs + 1], MZ.w, b1 ^ 0x80008000u);
         const uint32_t az[4] = {MZ.x, MZ.y, MZ.z, MZ.w};
         mma16816(zb, az, qb[2 * xs], qb[2 * xs + 1]);
 #pragma unroll
@@ -229,16 +234,18 @@ __device__ __forceinline__ void qk_block(const uint8_t* img, int lane, const uin
           const uint32_t a[4] = {reg<BW>(w, u, 2 * xs, 2 * mt), reg<BW>(w, u, 2 * xs, 2 * mt + 1),
                                  reg<BW>(w, u, 2 * xs + 1, 2 * mt), reg<BW>(w, u, 2 * xs + 1, 2 * mt + 1)};
           mma16816(s[mt], a, b0, b1);
+          mma16816(s[mt], a, l0, l1);
         }
       }
     }
-    const float c0 = zb[0] - ms0, c1 = zb[1] - ms1;
+    const float c0 = __fmaf_rn(zb[0], qsc, -ms0), c1 = __fmaf_rn(zb[1], qsc, -ms1);
+    const float f = kTwo24 * qsc;
 #pragma unroll
     for (int mt = 0; mt < 2; ++mt) {
-      s[mt][0] = __fmaf_rn(s[mt][0], kTwo24, c0);
-      s[mt][1] = __fmaf_rn(s[mt][1], kTwo24, c1);
-      s[mt][2] = __fmaf_rn(s[mt][2], kTwo24, c0);
-      s[mt][3] = __fmaf_rn(s[mt][3], kTwo24, c1);
+      s[mt][0] = __fmaf_rn(s[mt][0], f, c0);
+      s[mt][1] = __fmaf_rn(s[mt][1], f, c1);
+      s[mt][2] = __fmaf_rn(s[mt][2], f, c0);
+      s[mt][3] = __fmaf_rn(s[mt][3], f, c1);
     }
   } else {                    // per-token keys: dequantize in registers
 #pragma unroll
@@ -270,10 +277,10 @@ __device__ __forceinline__ void qk_block(const uint8_t* img, int lane, const uin
     }
 #pragma unroll
     for (int mt = 0; mt < 2; ++mt) {
-      s[mt][0] -= ms0;
-      s[mt][1] -= ms1;
-      s[mt][2] -= ms0;
-      s[mt][3] -= ms1;
+      s[mt][0] = __fmaf_rn(s[mt][0], qsc, -ms0);
+      s[mt][1] = __fmaf_rn(s[mt][1], qsc, -ms1);
+      s[mt][2] = __fmaf_rn(s[mt][2], qsc, -ms0);
+      s[mt][3] = __fmaf_rn(s[mt][3], qsc, -ms1);
     }
   }
 }
@@ -360,10 +367,10 @@ __device__ __forceinline__ void pv_block(const uint8_t* img, int lane, const uin
 
 template <int BW>
 __device__ __forceinline__ void qk_dispatch_g(int kg, const uint8_t* img, int lane,
-                                              const uint8_t* qtab, float ms0, float ms1,
+                                              const uint8_t* qtab, float qsc, float ms0, float ms1,
                                               float (&s)[2][4]) {
-  if (kg == RQ_PER_CHANNEL) qk_block<BW, RQ_PER_CHANNEL>(img, lane, qtab, ms0, ms1, s);
-  else qk_block<BW, RQ_PER_TOKEN>(img, lane, qtab, ms0, ms1, s);
+  if (kg == RQ_PER_CHANNEL) qk_block<BW, RQ_PER_CHANNEL>(img, lane, qtab, qsc, ms0, ms1, s);
+  else qk_block<BW, RQ_PER_TOKEN>(img, lane, qtab, qsc, ms0, ms1, s);
 }
 
 template <int BW>
@@ -375,17 +382,17 @@ __device__ __forceinline__ void pv_dispatch_g(int vg, const uint8_t* img, int la
 }
 
 __device__ __forceinline__ void qk_dispatch(int bw, int kg, const uint8_t* img, int lane,
-                                            const uint8_t* qtab, float ms0, float ms1,
+                                            const uint8_t* qtab, float qsc, float ms0, float ms1,
                                             float (&s)[2][4]) {
   switch (bw) {
-    case 1: qk_dispatch_g<1>(kg, img, lane, qtab, ms0, ms1, s); break;
-    case 2: qk_dispatch_g<2>(kg, img, lane, qtab, ms0, ms1, s); break;
-    case 3: qk_dispatch_g<3>(kg, img, lane, qtab, ms0, ms1, s); break;
-    case 4: qk_dispatch_g<4>(kg, img, lane, qtab, ms0, ms1, s); break;
-    case 5: qk_dispatch_g<5>(kg, img, lane, qtab, ms0, ms1, s); break;
-    case 6: qk_dispatch_g<6>(kg, img, lane, qtab, ms0, ms1, s); break;
-    case 7: qk_dispatch_g<7>(kg, img, lane, qtab, ms0, ms1, s); break;
-    default: qk_dispatch_g<8>(kg, img, lane, qtab, ms0, ms1, s); break;
+    case 1: qk_dispatch_g<1>(kg, img, lane, qtab, qsc, ms0, ms1, s); break;
+    case 2: qk_dispatch_g<2>(kg, img, lane, qtab, qsc, ms0, ms1, s); break;
+    case 3: qk_dispatch_g<3>(kg, img, lane, qtab, qsc, ms0, ms1, s); break;
+    case 4: qk_dispatch_g<4>(kg, img, lane, qtab, qsc, ms0, ms1, s); break;
+    case 5: qk_dispatch_g<5>(kg, img, lane, qtab, qsc, ms0, ms1, s); break;
+    case 6: qk_dispatch_g<6>(kg, img, lane, qtab, qsc, ms0, ms1, s); break;
+    case 7: qk_dispatch_g<7>(kg, img, lane, qtab, qsc, ms0, ms1, s); break;
+    default: qk_dispatch_g<8>(kg, img, lane, qtab, qsc, ms0, ms1, s); break;
   }
 }
 
@@ -560,7 +567,7 @@ __device__ __forceinline__ void prologue_static(const WarpStream& ws) {
 }
 
 template <int BK, int KG, int BV, int VG>
-__device__ __forceinline__ void blocks_static(const WarpStream& ws, const uint8_t* qtab,
+__device__ __forceinline__ void blocks_static(const WarpStream& ws, const uint8_t* qtab, float qsc,
                                               SoftmaxAcc& acc) {
   using R = Ring<BK, BV>;
   constexpr int NS = R::kSlots;
@@ -571,8 +578,8 @@ __device__ __forceinline__ void blocks_static(const WarpStream& ws, const uint8_
     cp_async_wait<NS - 1>();
     __syncwarp();
     float s[2][4];
-    qk_block<BK, KG>(ws.ring_ptr + use * R::kSlot, ws.lane, qtab, acc.m0 == -INFINITY ? 0.0f : acc.m0,
-                     acc.m1 == -INFINITY ? 0.0f : acc.m1, s);
+    qk_block<BK, KG>(ws.ring_ptr + use * R::kSlot, ws.lane, qtab, qsc,
+                     acc.m0 == -INFINITY ? 0.0f : acc.m0, acc.m1 == -INFINITY ? 0.0f : acc.m1, s);
     __syncwarp();
     use = use + 1 == NS ? 0 : use + 1;
     uint32_t pb[2][2];
@@ -605,7 +612,7 @@ __device__ __forceinline__ void prologue_dyn(const WarpStream& ws, const DynRing
 }
 
 __device__ __forceinline__ void blocks_dyn(const WarpStream& ws, const DynRing& r,
-                                           const uint8_t* qtab, SoftmaxAcc& acc) {
+                                           const uint8_t* qtab, float qsc, SoftmaxAcc& acc) {
   int use = 0, iss = r.ns - 1;
   for (int i = 0; i < ws.nb; ++i) {
     issue_dyn(ws, r, 2 * i + r.ns - 1, iss);
@@ -613,7 +620,7 @@ __device__ __forceinline__ void blocks_dyn(const WarpStream& ws, const DynRing& 
     cp_async_wait_dyn(r.ns - 1);
     __syncwarp();
     float s[2][4];
-    qk_dispatch(r.bK, r.kg, ws.ring_ptr + use * r.slot, ws.lane, qtab,
+    qk_dispatch(r.bK, r.kg, ws.ring_ptr + use * r.slot, ws.lane, qtab, qsc,
                 acc.m0 == -INFINITY ? 0.0f : acc.m0, acc.m1 == -INFINITY ? 0.0f : acc.m1, s);
     __syncwarp();
     use = use + 1 == r.ns ? 0 : use + 1;
@@ -706,10 +713,15 @@ __global__ void __launch_bounds__(kThreads, RQ_DECODE_MIN_BLOCKS) decode_split_k
   }
   __syncthreads();
   if (a.hadamard) fwht_smem(qs, kMaxHeads);
-  // softmax scale 1/sqrt(128) and log2(e) folded into q (scores in log2 units).
+  // q enters the MMAs scaled by a power of two only (no rounding beyond its
+  // fp16 conversion); the rest of the softmax scale 1/sqrt(128) * log2(e) is
+  // applied to the fp32 scores (log2 units).
   // K unit u, pair x of lane (gid, tig) is channels 32u + 8tig + 2x (+1);
   // qf carries the per-channel-key codes' 2^-E(x) as well.
-  const float qscale = kLog2e * kInvSqrt128 * (a.hadamard ? kInvSqrt128 : 1.0f);
+  // q is scaled by a power of two only (exact: headroom for q . scale in
+  // fp16), the rest of the softmax scale is applied in fp32
+  const float qpow = a.hadamard ? 0.015625f : 0.125f;
+  const float qscale = kLog2e * kInvSqrt128 * (a.hadamard ? kInvSqrt128 : 1.0f) / qpow;
   uint32_t qb[4][4], qf[4][4];
   uint32_t ef[4];
 #pragma unroll
@@ -720,7 +732,7 @@ __global__ void __launch_bounds__(kThreads, RQ_DECODE_MIN_BLOCKS) decode_split_k
 #pragma unroll
       for (int x = 0; x < 4; ++x) {
         const float* qr = qs + gid * kD + 32 * u + 8 * tig + 2 * x;
-        qb[u][x] = pack_f16x2(qr[0] * qscale, qr[1] * qscale);
+        qb[u][x] = pack_f16x2(qr[0] * qpow, qr[1] * qpow);
         qf[u][x] = hmul2u(qb[u][x], ef[x]);
       }
   }
@@ -749,10 +761,10 @@ __global__ void __launch_bounds__(kThreads, RQ_DECODE_MIN_BLOCKS) decode_split_k
   acc.l0 = acc.l1 = 0.0f;
 
   switch (key) {
-#define RQ_BLK(k, BK, BV) case k: blocks_static<BK, RQ_PER_CHANNEL, BV, RQ_PER_TOKEN>(ws, qtab, acc); break;
+#define RQ_BLK(k, BK, BV) case k: blocks_static<BK, RQ_PER_CHANNEL, BV, RQ_PER_TOKEN>(ws, qtab, qscale, acc); break;
     RQ_FAST_CASES(RQ_BLK)
 #undef RQ_BLK
-    default: blocks_dyn(ws, dr, qtab, acc); break;
+    default: blocks_dyn(ws, dr, qtab, qscale, acc); break;
   }
   // the merge kernel may be scheduled now; it waits for this grid to finish
   asm volatile("griddepcontrol.launch_dependents;\n" ::: "memory");
@@ -837,11 +849,80 @@ __global__ void __launch_bounds__(kThreads, RQ_DECODE_MIN_BLOCKS) decode_split_k
 // chunk), and merged there with a running max per row.
 constexpr int kMergeSmem = 64 * 1024;
 
-template <int CQ>
+// The unquantized residual tokens (decode-time append) of one (batch, kv
+// head): their exact fp32 attention record (m, l, o) for the g query rows
+// starts the running merge. Scores use the unrotated q and keys (a rotation
+// leaves dot products unchanged); the value sum is rotated into the cache's
+// domain when the cache is rotated. Whole CTA; sm: 64 KB of shared memory.
+template <int CQ, typename T>
+__device__ __forceinline__ void residual_record(const T* q, const T* res, int R, int g,
+                                                const int8_t* signs, int hadamard, int part,
+                                                float* sm, float* y, float* run_m, float* run_l,
+                                                float (&acc)[kMaxHeads * (kD / CQ) / kThreads]) {
+  constexpr int CW = kD / CQ;
+  constexpr int PAIRS = kMaxHeads * CW / kThreads;
+  const int tid = threadIdx.x;
+  float* qf = sm;                                  // [g][128], scaled to log2 units
+  float* kr = qf + kMaxHeads * kD;                 // [32][129]
+  float* vr = kr + kTile * (kD + 1);               // [32][128]
+  float* sc = vr + kTile * kD;                     // [g][32]
+  const float qscale = kLog2e * kInvSqrt128;
+  for (int n = 0; n < g; ++n) qf[n * kD + tid] = to_f32<T>(q[n * kD + tid]) * qscale;
+  for (int t = 0; t < R; ++t) {
+    kr[t * (kD + 1) + tid] = to_f32<T>(res[t * kD + tid]);
+    vr[t * kD + tid] = to_f32<T>(res[(kTile + t) * kD + tid]);
+  }
+  __syncthreads();
+  for (int idx = tid; idx < g * R; idx += kThreads) {
+    const int n = idx / R, t = idx % R;
+    float sdot = 0.0f;
+    for (int c = 0; c < kD; ++c) sdot = __fmaf_rn(qf[n * kD + c], kr[t * (kD + 1) + c], sdot);
+    sc[n * kTile + t] = sdot;
+  }
+  __syncthreads();
+#pragma unroll
+  for (int k = 0; k < PAIRS; ++k) {
+    const int pi = tid + kThreads * k, n = pi / CW, c = pi % CW;
+    if (n < g) {
+      float m = -INFINITY;
+      for (int t = 0; t < R; ++t) m = fmaxf(m, sc[n * kTile + t]);
+      float l = 0.0f, o = 0.0f;
+      for (int t = 0; t < R; ++t) {
+        const float p = exp2f(sc[n * kTile + t] - m);
+        l += p;
+        o = __fmaf_rn(p, vr[t * kD + part * CW + c], o);
+      }
+      acc[k] = o;
+      if (c == 0) {
+        run_m[n] = m;
+        run_l[n] = l;
+      }
+    }
+  }
+  if (CQ == 1 && hadamard) {                       // o R = FWHT(o * signs) / sqrt(128)
+#pragma unroll
+    for (int k = 0; k < PAIRS; ++k) {
+      const int pi = tid + kThreads * k, c = pi % CW;
+      if (pi / CW < g) y[pi] = (signs && signs[c] < 0) ? -acc[k] : acc[k];
+    }
+    __syncthreads();
+    fwht_smem(y, g);
+#pragma unroll
+    for (int k = 0; k < PAIRS; ++k) {
+      const int pi = tid + kThreads * k;
+      if (pi / CW < g) acc[k] = y[pi] * kInvSqrt128;
+    }
+  }
+  __syncthreads();
+}
+
+template <int CQ, typename T>
 __global__ void __launch_bounds__(kThreads) decode_merge_kernel(const float* partial, float* out,
                                                                 const int8_t* signs,
                                                                 uint32_t* status, int Hq, int H,
-                                                                int g, int splits, int hadamard) {
+                                                                int g, int splits, int hadamard,
+                                                                const T* q, const T* residual,
+                                                                int R) {
   asm volatile("griddepcontrol.wait;\n" ::: "memory");
   constexpr int CW = kD / CQ;          // channels of this CTA
   constexpr int CH = CW / 4;           // 16-byte pieces of a record's o slice
@@ -866,6 +947,11 @@ __global__ void __launch_bounds__(kThreads) decode_merge_kernel(const float* par
   float acc[PAIRS];
 #pragma unroll
   for (int k = 0; k < PAIRS; ++k) acc[k] = 0.0f;
+  __syncthreads();
+  if (R > 0)
+    residual_record<CQ, T>(q + row0 * kD, residual + (static_cast<long long>(batch) * H + h) * 2 * kTile * kD,
+                           R, g, signs, hadamard, part, reinterpret_cast<float*>(msm), y, run_m, run_l,
+                           acc);
   const uint32_t sbase = static_cast<uint32_t>(__cvta_generic_to_shared(msm));
 
   for (int c0 = 0; c0 < splits; c0 += cs_max) {
@@ -1003,8 +1089,15 @@ rq_status split_ctas_per_sm(int* per_sm) {
 // Splits of the sequence per (batch, kv head): as many as fit in one wave of
 // resident CTAs (slots = SMs x CTAs per SM), so every CTA streams a long run
 // of blocks and none waits for a second wave; at least one.
-void decode_plan(const rq_cache_desc* desc, int slots, int* splits, int* bps) {
-  const int nblk = desc->S / kTile;
+// nblk: the packed blocks attended (<= the capacity's); splits <= the
+// capacity's split bound (max_splits), which sizes the workspace.
+int max_splits(const rq_cache_desc* desc, int slots) {
+  const long long units = static_cast<long long>(desc->B) * desc->H_kv;
+  const long long sp = units > 0 ? slots / units : 1;
+  return static_cast<int>(std::max<long long>(1, std::min<long long>(sp, desc->S / kTile)));
+}
+
+void decode_plan(const rq_cache_desc* desc, int nblk, int slots, int* splits, int* bps) {
   const long long units = static_cast<long long>(desc->B) * desc->H_kv;
   long long sp = units > 0 ? slots / units : 1;
   sp = std::max<long long>(1, std::min<long long>(sp, nblk));
@@ -1073,12 +1166,9 @@ rq_status launch_split(const DecodeArgs& a, const dim3& grid, cudaStream_t s) {
 }
 
 // split kernel, then the merge kernel as its programmatic dependent
-rq_status launch_decode(const DecodeArgs& a, const rq_cache_desc* desc, float* out, cudaStream_t s) {
-  const dim3 grid(static_cast<unsigned>(a.splits), static_cast<unsigned>(desc->H_kv),
-                  static_cast<unsigned>(desc->B));
-  const rq_status st = desc->dtype == RQ_F16 ? launch_split<__half>(a, grid, s)
-                                             : launch_split<__nv_bfloat16>(a, grid, s);
-  if (st != RQ_OK) return st;
+template <typename T>
+rq_status launch_merge(const DecodeArgs& a, const rq_cache_desc* desc, float* out,
+                       const void* res_layer, int R, cudaStream_t s) {
   // a whole row per CTA for a rotated cache (the rotation mixes channels),
   // a quarter of the channels otherwise (four times the CTAs)
   const int cq = a.hadamard ? 1 : 4;
@@ -1092,13 +1182,26 @@ rq_status launch_decode(const DecodeArgs& a, const rq_cache_desc* desc, float* o
   attr[0].val.programmaticStreamSerializationAllowed = 1;
   cfg.attrs = attr;
   cfg.numAttrs = 1;
-  auto kern = a.hadamard ? decode_merge_kernel<1> : decode_merge_kernel<4>;
+  auto kern = a.hadamard ? decode_merge_kernel<1, T> : decode_merge_kernel<4, T>;
   if (cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, kMergeSmem) != cudaSuccess)
     return RQ_ERR_CUDA;
   if (cudaLaunchKernelEx(&cfg, kern, static_cast<const float*>(a.partial), out, a.signs, a.status,
-                         a.Hq, a.H, a.g, a.splits, a.hadamard) != cudaSuccess)
+                         a.Hq, a.H, a.g, a.splits, a.hadamard, static_cast<const T*>(a.q),
+                         static_cast<const T*>(res_layer), R) != cudaSuccess)
     return RQ_ERR_CUDA;
   return launch_status();
+}
+
+// split kernel, then the merge kernel as its programmatic dependent
+rq_status launch_decode(const DecodeArgs& a, const rq_cache_desc* desc, float* out, cudaStream_t s,
+                        const void* res_layer = nullptr, int R = 0) {
+  const dim3 grid(static_cast<unsigned>(a.splits), static_cast<unsigned>(desc->H_kv),
+                  static_cast<unsigned>(desc->B));
+  const bool f16 = desc->dtype == RQ_F16;
+  const rq_status st = f16 ? launch_split<__half>(a, grid, s) : launch_split<__nv_bfloat16>(a, grid, s);
+  if (st != RQ_OK) return st;
+  return f16 ? launch_merge<__half>(a, desc, out, res_layer, R, s)
+             : launch_merge<__nv_bfloat16>(a, desc, out, res_layer, R, s);
 }
 
 }  // namespace
@@ -1111,9 +1214,7 @@ extern "C" rq_status rq_decode_workspace_bytes(const rq_cache_desc* desc, size_t
   if (st != RQ_OK) return st;
   int slots = 0;
   if (decode_slots(&slots) != RQ_OK) return RQ_ERR_CUDA;
-  int splits = 1, bps = 1;
-  decode_plan(desc, slots, &splits, &bps);
-  *bytes = workspace_bytes(desc, splits);
+  *bytes = workspace_bytes(desc, max_splits(desc, slots));
   return RQ_OK;
 }
 
@@ -1134,7 +1235,7 @@ extern "C" rq_status rq_decode_attention(const rq_cache_desc* desc, int32_t laye
   int slots = 0;
   if (decode_slots(&slots) != RQ_OK) return RQ_ERR_CUDA;
   int splits = 1, bps = 1;
-  decode_plan(desc, slots, &splits, &bps);
+  decode_plan(desc, desc->S / kTile, slots, &splits, &bps);
   if (ws_bytes < workspace_bytes(desc, splits)) return RQ_ERR_WORKSPACE;
   DecodeArgs a;
   fill_args(a, desc, layer, q, packed, bits_dev, offsets_dev, signs_dev, ws, status_dev, splits, bps);
@@ -1193,7 +1294,7 @@ extern "C" rq_status rq_decode_attention_static(const rq_cache_desc* desc, int32
   int slots = 0;
   if (decode_slots(&slots) != RQ_OK) return RQ_ERR_CUDA;
   int splits = 1, bps = 1;
-  decode_plan(desc, slots, &splits, &bps);
+  decode_plan(desc, desc->S / kTile, slots, &splits, &bps);
   if (workspace_bytes(desc, splits) > RQ_STATIC_SCRATCH_BYTES) return RQ_ERR_WORKSPACE;
   float* scratch = nullptr;
   if (static_scratch_ptr(&scratch) != RQ_OK) return RQ_ERR_CUDA;
@@ -1201,4 +1302,39 @@ extern "C" rq_status rq_decode_attention_static(const rq_cache_desc* desc, int32
   fill_args(a, desc, layer, q, packed, bits_dev, offsets_dev, signs_dev, scratch, status_dev, splits,
             bps);
   return launch_decode(a, desc, out, static_cast<cudaStream_t>(stream));
+}
+
+// ------------------------------------------------- decode over n_tokens ----
+extern "C" rq_status rq_decode_attention_len(const rq_cache_desc* desc, int32_t layer,
+                                             int32_t n_tokens, const void* q, const void* packed,
+                                             const uint8_t* bits_dev, const uint64_t* offsets_dev,
+                                             const int8_t* signs_dev, const void* residual,
+                                             float* out, void* ws, size_t ws_bytes,
+                                             uint32_t* status_dev, void* stream) {
+  using namespace rq;
+  const rq_status st = check_desc(desc);
+  if (st != RQ_OK) return st;
+  if (!q || !packed || !bits_dev || !offsets_dev || !out || !ws) return RQ_ERR_INVALID_ARG;
+  if (layer < 0 || layer >= desc->L || n_tokens < 1 || n_tokens > desc->S) return RQ_ERR_INVALID_ARG;
+  const int R = n_tokens % kTile;
+  if (R > 0 && !residual) return RQ_ERR_INVALID_ARG;
+  if (!aligned16(packed) || !aligned16(ws) || (R > 0 && !aligned16(residual)) ||
+      (reinterpret_cast<uintptr_t>(q) & 1u) || (reinterpret_cast<uintptr_t>(out) & 3u))
+    return RQ_ERR_ALIGNMENT;
+  if (desc->B == 0) return RQ_OK;
+  int slots = 0;
+  if (decode_slots(&slots) != RQ_OK) return RQ_ERR_CUDA;
+  int splits = 1, bps = 1;
+  const int nblk = n_tokens / kTile;
+  decode_plan(desc, nblk, slots, &splits, &bps);
+  if (ws_bytes < workspace_bytes(desc, splits)) return RQ_ERR_WORKSPACE;
+  DecodeArgs a;
+  fill_args(a, desc, layer, q, packed, bits_dev, offsets_dev, signs_dev, ws, status_dev, splits, bps);
+  a.nblk = nblk;
+  // this layer's residual windows: [B][H][2][32][128] values of the cache dtype
+  const void* res_layer =
+      R > 0 ? static_cast<const uint8_t*>(residual) +
+                  static_cast<size_t>(layer) * desc->B * desc->H_kv * 2 * kTile * kD * 2
+            : nullptr;
+  return launch_decode(a, desc, out, static_cast<cudaStream_t>(stream), res_layer, R);
 }

@@ -60,6 +60,7 @@ struct QuantArgs {
   uint8_t* packed;
   uint32_t* status;
   int layer, B, H, S, nblk, kg, vg, hadamard;
+  int j_dst0;                // packed block index of each stream's first tile
   long long ntiles;
 };
 
@@ -574,8 +575,9 @@ __device__ __forceinline__ StreamState stream_state(const QuantArgs& a, int sk) 
   st.src = reinterpret_cast<const uint8_t*>(static_cast<const T*>(st.kind ? a.v : a.k) +
                                             static_cast<long long>(sk >> 1) * a.S * kD);
   // offsets[layer][batch][h][kind] = offsets[layer * B * H * 2 + sk]
-  st.dst = a.packed + a.offsets[static_cast<long long>(a.layer) * a.B * a.H * 2 + sk];
   st.blk_bytes = 512 * (st.b + 1);
+  st.dst = a.packed + a.offsets[static_cast<long long>(a.layer) * a.B * a.H * 2 + sk] +
+           static_cast<long long>(a.j_dst0) * st.blk_bytes;
   return st;
 }
 
@@ -844,6 +846,7 @@ extern "C" rq_status rq_quantize_pack(const rq_cache_desc* desc, int32_t layer, 
   a.kg = desc->k_grouping;
   a.vg = desc->v_grouping;
   a.hadamard = desc->hadamard ? 1 : 0;
+  a.j_dst0 = 0;
   a.ntiles = static_cast<long long>(desc->B) * desc->H_kv * 2 * a.nblk;
   if (a.ntiles == 0) return RQ_OK;
   cudaStream_t st = static_cast<cudaStream_t>(stream);
@@ -896,4 +899,88 @@ extern "C" rq_status rq_calibrate_distortion(const void* x, int32_t dtype, int32
   calib_finalize_kernel<<<(n * 8 + 127) / 128, 128, 0, st>>>(a.partial, mse_dev, n, a.ntile,
                                                               static_cast<double>(T) * kD);
   return launch_status();
+}
+
+// ---------------------------------------------------------- decode append ----
+// Residual windows: [L][B][H][2][32][128] values, K then V per (layer, batch,
+// kv head); token t in slot t % 32. One CTA of 32 threads per (batch, head):
+// threads 0..15 copy the new key's 16-byte chunks, 16..31 the value's.
+namespace rq {
+namespace {
+
+__global__ void append_token_kernel(const uint4* k_new, const uint4* v_new, uint4* residual_layer,
+                                    int slot) {
+  const int bh = blockIdx.x, t = threadIdx.x, kind = t >> 4, ch = t & 15;
+  const uint4* src = (kind ? v_new : k_new) + bh * 16 + ch;
+  // 16-byte chunks: a token row is 16, a window 32 * 16, a (batch, head) 2 windows
+  residual_layer[(bh * 2 + kind) * 32 * 16 + slot * 16 + ch] = *src;
+}
+
+size_t residual_layer_elems(const rq_cache_desc* desc) {
+  return static_cast<size_t>(desc->B) * desc->H_kv * 2 * kTile * kD;
+}
+
+}  // namespace
+}  // namespace rq
+
+extern "C" size_t rq_residual_bytes(const rq_cache_desc* desc) {
+  using namespace rq;
+  if (!desc || desc->L <= 0 || desc->B < 0 || desc->H_kv <= 0) return 0;
+  if (desc->dtype != RQ_F16 && desc->dtype != RQ_BF16) return 0;
+  return static_cast<size_t>(desc->L) * residual_layer_elems(desc) * 2;
+}
+
+extern "C" rq_status rq_append(const rq_cache_desc* desc, int32_t layer, int32_t pos,
+                               const void* k_new, const void* v_new, void* residual,
+                               const int8_t* signs_dev, const uint8_t* bits_dev,
+                               const uint64_t* offsets_dev, void* packed, uint32_t* status_dev,
+                               void* stream) {
+  using namespace rq;
+  if (!desc || !k_new || !v_new || !residual || !bits_dev || !offsets_dev || !packed)
+    return RQ_ERR_INVALID_ARG;
+  if (desc->L <= 0 || desc->B < 0 || desc->H_kv <= 0 || desc->S < 0) return RQ_ERR_INVALID_ARG;
+  if (layer < 0 || layer >= desc->L || pos < 0 || pos >= desc->S) return RQ_ERR_INVALID_ARG;
+  if (desc->dtype != RQ_F16 && desc->dtype != RQ_BF16) return RQ_ERR_INVALID_ARG;
+  for (int g : {desc->k_grouping, desc->v_grouping})
+    if (g != RQ_PER_TOKEN && g != RQ_PER_CHANNEL) return RQ_ERR_INVALID_ARG;
+  if (desc->d != kD || desc->group != kG || desc->S % kTile != 0) return RQ_ERR_SHAPE;
+  if (!aligned16(k_new) || !aligned16(v_new) || !aligned16(residual) || !aligned16(packed))
+    return RQ_ERR_ALIGNMENT;
+  if (desc->B == 0) return RQ_OK;
+  cudaStream_t st = static_cast<cudaStream_t>(stream);
+  const size_t layer_bytes = residual_layer_elems(desc) * 2;
+  uint8_t* res_layer = static_cast<uint8_t*>(residual) + static_cast<size_t>(layer) * layer_bytes;
+  const int slot = pos % kTile;
+  append_token_kernel<<<static_cast<unsigned>(desc->B * desc->H_kv), 32, 0, st>>>(
+      static_cast<const uint4*>(k_new), static_cast<const uint4*>(v_new),
+      reinterpret_cast<uint4*>(res_layer), slot);
+  if (launch_status() != RQ_OK) return RQ_ERR_CUDA;
+  if (slot != kTile - 1) return RQ_OK;
+  // the windows are full: quantize + pack them as block pos / 32 of every
+  // stream (a stream's source is its window: K at +0, V at +32 tokens, the
+  // next (batch, head) 64 tokens on)
+  QuantArgs a;
+  a.k = res_layer;
+  a.v = res_layer + static_cast<size_t>(kTile) * kD * 2;
+  a.signs = signs_dev;
+  a.bits = bits_dev;
+  a.offsets = offsets_dev;
+  a.packed = static_cast<uint8_t*>(packed);
+  a.status = status_dev;
+  a.layer = layer;
+  a.B = desc->B;
+  a.H = desc->H_kv;
+  a.S = 2 * kTile;
+  a.nblk = 1;
+  a.kg = desc->k_grouping;
+  a.vg = desc->v_grouping;
+  a.hadamard = desc->hadamard ? 1 : 0;
+  a.j_dst0 = pos / kTile;
+  a.ntiles = static_cast<long long>(desc->B) * desc->H_kv * 2;
+  const size_t smem = quant_smem_bytes(a.hadamard != 0);
+  if (desc->dtype == RQ_F16)
+    return a.hadamard ? launch_persistent(quantize_pack_kernel<__half, true>, a, smem, st)
+                      : launch_persistent(quantize_pack_kernel<__half, false>, a, smem, st);
+  return a.hadamard ? launch_persistent(quantize_pack_kernel<__nv_bfloat16, true>, a, smem, st)
+                    : launch_persistent(quantize_pack_kernel<__nv_bfloat16, false>, a, smem, st);
 }

@@ -84,6 +84,25 @@ class PackedKVPath:
         rq.rq_decode_attention(self.desc, layer, q, self.packed, self.bits, self.offsets,
                                self.signs, out, ws, self.status, stream)
 
+    # ---- decode-time append ---------------------------------------------------
+    def residual(self) -> torch.Tensor:
+        """The residual windows [L][B][H][2][32][128] (allocated on first use)."""
+        if getattr(self, "_residual", None) is None:
+            n = rq.rq_residual_bytes(self.desc)
+            self._residual = torch.zeros(max(n, 16), dtype=torch.uint8, device=self.device)
+        return self._residual
+
+    def append(self, layer: int, pos: int, k_new: torch.Tensor, v_new: torch.Tensor, stream=None):
+        rq.rq_append(self.desc, layer, pos, k_new, v_new, self.residual(), self.signs, self.bits,
+                     self.offsets, self.packed, self.status, stream)
+
+    def decode_len(self, layer: int, n_tokens: int, q: torch.Tensor, out: torch.Tensor,
+                   stream=None):
+        ws = self.decode_workspace()
+        rq.rq_decode_attention_len(self.desc, layer, n_tokens, q, self.packed, self.bits,
+                                   self.offsets, self.signs, self.residual(), out, ws,
+                                   self.status, stream)
+
     def stream_bytes(self, layer: int, batch: int, head: int, kind: int) -> torch.Tensor:
         """The packed bytes of one stream (a view into the packed buffer)."""
         off = int(self.offsets_host[layer, batch, head, kind])

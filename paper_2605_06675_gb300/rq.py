@@ -32,7 +32,8 @@ STATUS_NAMES = {0: "RQ_OK", 1: "RQ_ERR_INVALID_ARG", 2: "RQ_ERR_INFEASIBLE", 3: 
 EXPORTS = ["rq_status_string", "rq_abi_version", "rq_fit_distortion", "rq_alloc",
            "rq_alloc_continuous", "rq_packed_layout", "rq_calibrate_workspace_bytes",
            "rq_calibrate_distortion", "rq_quantize_pack", "rq_decode_workspace_bytes",
-           "rq_decode_attention", "rq_decode_attention_static"]
+           "rq_decode_attention", "rq_decode_attention_static", "rq_residual_bytes",
+           "rq_append", "rq_decode_attention_len"]
 
 
 class RQError(RuntimeError):
@@ -74,6 +75,10 @@ def lib() -> ctypes.CDLL:
             "rq_decode_workspace_bytes": ([_P, _P], _I),
             "rq_decode_attention": ([_P, _I, _P, _P, _P, _P, _P, _P, _P, _SZ, _P, _P], _I),
             "rq_decode_attention_static": ([_P, _I, _P, _P, _P, _P, _P, _P, _P, _P], _I),
+            "rq_residual_bytes": ([_P], _SZ),
+            "rq_append": ([_P, _I, _I, _P, _P, _P, _P, _P, _P, _P, _P, _P], _I),
+            "rq_decode_attention_len": ([_P, _I, _I, _P, _P, _P, _P, _P, _P, _P, _P, _SZ, _P, _P],
+                                        _I),
         }
         for name, (args, res) in sig.items():
             f = getattr(L, name)
@@ -235,3 +240,26 @@ def rq_decode_attention_static(desc, layer, q, packed, bits_dev, offsets_dev, si
     _check("rq_decode_attention_static", lib().rq_decode_attention_static(
         ctypes.byref(desc), layer, _dp(q), _dp(packed), _dp(bits_dev), _dp(offsets_dev),
         _dp(signs), _dp(out), _dp(status), _stream(stream)))
+
+
+def rq_residual_bytes(desc) -> int:
+    return int(lib().rq_residual_bytes(ctypes.byref(desc)))
+
+
+def rq_append(desc, layer, pos, k_new, v_new, residual, signs, bits_dev, offsets_dev, packed,
+              status=None, stream=None):
+    """Append token ``pos`` (k_new, v_new: CUDA [B][H_kv][128]) of one layer to
+    the residual windows; a full window is quantized into block pos // 32."""
+    _check("rq_append", lib().rq_append(
+        ctypes.byref(desc), layer, pos, _dp(k_new), _dp(v_new), _dp(residual), _dp(signs),
+        _dp(bits_dev), _dp(offsets_dev), _dp(packed), _dp(status), _stream(stream)))
+
+
+def rq_decode_attention_len(desc, layer, n_tokens, q, packed, bits_dev, offsets_dev, signs,
+                            residual, out, ws, status=None, stream=None):
+    """Decode attention over the first ``n_tokens`` tokens: packed blocks plus
+    the residual window's last n_tokens % 32 tokens."""
+    _check("rq_decode_attention_len", lib().rq_decode_attention_len(
+        ctypes.byref(desc), layer, n_tokens, _dp(q), _dp(packed), _dp(bits_dev),
+        _dp(offsets_dev), _dp(signs), _dp(residual), _dp(out), _dp(ws),
+        ws.numel() * ws.element_size(), _dp(status), _stream(stream)))

@@ -85,3 +85,25 @@ def test_rotated_pipeline_close_to_plain_attention():
     out = pipeline.attend_layer(q, ql)
     ref = decode_attention(q[0], k[0].astype(np.float64), v[0].astype(np.float64))
     assert np.abs(out[0] - ref).max() < 0.02
+
+
+def test_residual_attention_reduces_to_its_parts():
+    # with no residual token it is the packed-cache attention; with no packed
+    # block it is exact attention over the raw tokens
+    from oracle import pipeline as opipe
+    rng = np.random.default_rng(12)
+    B, H, Hq, S = 1, 2, 4, 64
+    k = rng.standard_normal((B, H, S, 128)).astype(np.float32)
+    v = rng.standard_normal((B, H, S, 128)).astype(np.float32)
+    q = rng.standard_normal((B, Hq, 128)).astype(np.float32)
+    bits = np.array([[2, 3], [4, 2]])
+    ol = opipe.quantize_layer(k, v, bits, 1, 0)
+    empty = np.zeros((B, H, 0, 128), np.float32)
+    assert np.array_equal(opipe.attend_with_residual(q, ol, empty, empty), opipe.attend_layer(q, ol))
+    got = opipe.attend_with_residual(q, {}, k[:, :, :20], v[:, :, :20])
+    for h in range(H):
+        for j in range(2):
+            s = (k[0, h, :20].astype(np.float64) @ q[0, 2 * h + j]) / np.sqrt(128)
+            p = np.exp(s - s.max())
+            want = (p @ v[0, h, :20].astype(np.float64)) / p.sum()
+            assert np.allclose(got[0, 2 * h + j], want, rtol=1e-6, atol=1e-6)
