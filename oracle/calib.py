@@ -34,7 +34,7 @@ from .quant import quantize_stream
 
 
 def distortion_sweep(x: np.ndarray, groupings, hadamard: bool = False, signs=None,
-                     bits=range(1, 9)) -> np.ndarray:
+                     bits=range(1, 9), symmetric: bool = False) -> np.ndarray:
     """x [n][T][128] (fp16/bf16 values as fp32); groupings[n] in {PER_TOKEN, PER_CHANNEL}.
 
     Returns mse [n][len(bits)] float64.
@@ -45,7 +45,7 @@ def distortion_sweep(x: np.ndarray, groupings, hadamard: bool = False, signs=Non
     out = np.zeros((n, len(bits)), dtype=np.float64)
     for i in range(n):
         for k, b in enumerate(bits):
-            r = quantize_stream(x[i], int(groupings[i]), b, signs, hadamard)
+            r = quantize_stream(x[i], int(groupings[i]), b, signs, hadamard, symmetric)
             err = r["y"].astype(np.float64) - r["xhat"].astype(np.float64)
             out[i, k] = float(np.sum(err * err)) / err.size
     return out

@@ -18,7 +18,7 @@ from .quant import quantize_stream
 
 
 def quantize_layer(k, v, bits, k_grouping, v_grouping, hadamard=False, signs=None,
-                   streams=None):
+                   streams=None, symmetric=False):
     """Quantize and pack one layer.
 
     bits [H][2]. ``streams`` optionally restricts work to a list of
@@ -36,7 +36,7 @@ def quantize_layer(k, v, bits, k_grouping, v_grouping, hadamard=False, signs=Non
     for bb, h in streams:
         for kind, x, grouping in ((pack.KIND_K, k, k_grouping), (pack.KIND_V, v, v_grouping)):
             b = int(bits[h, kind])
-            r = quantize_stream(x[bb, h], grouping, b, signs, hadamard)
+            r = quantize_stream(x[bb, h], grouping, b, signs, hadamard, symmetric)
             words = pack.pack_stream(r["codes"], r["scale"], r["zero"], kind, grouping, b)
             xhat = r["xhat"].astype(np.float64)
             if hadamard:

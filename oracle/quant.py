@@ -32,6 +32,23 @@ reading used here (every step in the stated precision, in this order) is:
   A group holding a non-finite value, or whose fp16 scale or zero overflows,
   is a numeric failure: codes 0, scale 0, zero 0, and the failure is reported.
 
+Symmetric variant. The paper's one printed symmetric quantizer is the absmax
+form of App. W ("TurboQuant kernel"): x_hat = round(x M / a) a / M with
+a = max |x| and M = 2^(b-1) - 1 (levels q a / M, q = -M..M, zero among
+them); KIVI's keys (Sec. 2, "per-channel symmetric") and QuaRot's / RTN's
+per-token quantizer (Sec. 4.1; App. M, Table 16) are read as this same form over the
+same groups of 32. Stored as an asymmetric group (code c = q + M, so one
+decoder serves both), in the same precision steps as above:
+    a   = max |v|                                  (exact)
+    M   = 2^(b-1) - 1
+    if M == 0 (b = 1): the only level is 0: codes 0, scale 0, zero 0
+    s32 = fp32_rn(a / M),  scale = fp16_rn(s32)
+    zero = fp16_rn(-M * sf)       (M * sf is exact in fp32: 7 + 11 bits)
+    codes as above from the stored scale and zero, clamped to 0..2M
+    (code 2^b - 1 is never used)
+so level c sits at fp16(c sf + zf) ~ (c - M) sf, off the exact symmetric grid
+only by the fp16 rounding of zero (at most 2^-12 |zero|).
+
 Rotation (QuaRot reading of "Hadamard" / "random orthogonal R"):
   y = FWHT(x * sigma) * fp32_rn(1/sqrt(128)), in fp32, butterfly stages with
   stride 1, 2, 4, ..., 64 in that order; each stage maps the pair (i, i+h),
@@ -73,11 +90,12 @@ def hadamard_rotate(x: np.ndarray, signs: np.ndarray | None) -> np.ndarray:
     return (y * INV_SQRT_128_F32).astype(np.float32)
 
 
-def quantize_groups(v: np.ndarray, b: int):
+def quantize_groups(v: np.ndarray, b: int, symmetric: bool = False):
     """Quantize groups along the last axis (length 32) at b bits.
 
     Returns (codes uint8, scale float16, zero float16, bad bool), the last
-    three with the group shape (last axis removed).
+    three with the group shape (last axis removed). ``symmetric``: the absmax
+    form (levels q max|v| / M, q = -M..M, stored as code q + M).
     """
     assert 1 <= b <= 8
     v = canonical(v)
@@ -87,10 +105,18 @@ def quantize_groups(v: np.ndarray, b: int):
         vv = np.where(finite[..., None], v, np.float32(0.0))
         mn = vv.min(axis=-1)
         mx = vv.max(axis=-1)
-        L = np.float32(2 ** b - 1)
-        s32 = ((mx - mn).astype(np.float32) / L).astype(np.float32)
-        scale = s32.astype(np.float16)
-        zero = mn.astype(np.float16)
+        if symmetric:
+            M = np.float32(2 ** (b - 1) - 1)
+            L = np.float32(2.0 * M)                       # the largest code
+            a = np.maximum(np.abs(mn), np.abs(mx)).astype(np.float32)
+            s32 = (a / np.float32(max(M, 1.0))).astype(np.float32) * np.float32(M > 0)
+            scale = s32.astype(np.float16)
+            zero = (-M * scale.astype(np.float32)).astype(np.float32).astype(np.float16)
+        else:
+            L = np.float32(2 ** b - 1)
+            s32 = ((mx - mn).astype(np.float32) / L).astype(np.float32)
+            scale = s32.astype(np.float16)
+            zero = mn.astype(np.float16)
         bad = (~finite) | (~np.isfinite(scale)) | (~np.isfinite(zero))
         sf = scale.astype(np.float32)
         zf = zero.astype(np.float32)
@@ -138,7 +164,7 @@ def from_groups(g: np.ndarray, grouping: int) -> np.ndarray:
 
 
 def quantize_stream(x: np.ndarray, grouping: int, b: int, signs: np.ndarray | None = None,
-                    hadamard: bool = False):
+                    hadamard: bool = False, symmetric: bool = False):
     """Quantize one (batch, head, K/V) stream x[S, 128].
 
     Returns dict with the quantizer-domain values ``y`` [S,128] (rotated when
@@ -149,7 +175,7 @@ def quantize_stream(x: np.ndarray, grouping: int, b: int, signs: np.ndarray | No
     y = hadamard_rotate(x, signs) if hadamard else x.astype(np.float32)
     y = canonical(y)
     g = to_groups(y, grouping)
-    codes, scale, zero, bad = quantize_groups(g, b)
+    codes, scale, zero, bad = quantize_groups(g, b, symmetric)
     xhat = dequantize_groups(codes, scale, zero)
     return {
         "y": y,

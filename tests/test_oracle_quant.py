@@ -245,3 +245,101 @@ def test_one_rounding_not_two():
     codes, scale, zero, _ = quant.quantize_groups(x, b)
     assert float(zero[0]) == 0.0
     assert codes[0, 2] == k
+
+
+def test_symmetric_levels_are_exact():
+    # b = 3 (M = 3), a = 3 * 2^-2: levels q / 4, q = -3..3 (scale 2^-2 and
+    # zero -3/4 both exact in fp16), code q + 3; a group drawn from the levels
+    # with +a present reconstructs exactly, and its min does not matter
+    rng = np.random.default_rng(21)
+    lv = np.arange(-3, 4, dtype=np.float32) / 4
+    x = lv[rng.integers(0, 7, size=(50, 32))]
+    x[:, 0] = 0.75
+    x[:, 1] = 0.25
+    x[x < -0.5] = 0.0
+    codes, scale, zero, bad = quant.quantize_groups(x, 3, symmetric=True)
+    assert (scale == 0.25).all() and (zero == -0.75).all() and not bad.any()
+    assert np.array_equal(codes.astype(np.float32), 4 * x + 3)
+    assert np.array_equal(quant.dequantize_groups(codes, scale, zero), x)
+    assert codes.max() <= 6                       # code 2^b - 1 is never used
+
+
+def test_symmetric_matches_printed_absmax_formula():
+    # round(x M / a) a / M (App. W, "TurboQuant kernel") in exact arithmetic,
+    # when a / M is a power of two (scale and zero exact in fp16) and no value
+    # sits on a rounding tie
+    rng = np.random.default_rng(22)
+    for b in range(2, 9):
+        M = 2 ** (b - 1) - 1
+        for e in (-6, 0, 3):
+            a = M * 2.0 ** e
+            x = rng.uniform(-a, a, size=(64, 32))
+            x[:, 5] = -a if b % 2 else a
+            x = x.astype(np.float16).astype(np.float32)
+            u = x.astype(np.float64) * M / a
+            keep = np.abs(u - np.floor(u) - 0.5) > 1e-9
+            codes, scale, zero, bad = quant.quantize_groups(x, b, symmetric=True)
+            assert not bad.any() and (scale == 2.0 ** e).all()
+            want = np.round(u) * a / M
+            got = quant.dequantize_groups(codes, scale, zero).astype(np.float64)
+            assert np.array_equal(got[keep], want[keep]), (b, e)
+            assert np.array_equal((codes.astype(np.int64) - M)[keep], np.round(u).astype(np.int64)[keep])
+
+
+def test_symmetric_one_bit_has_the_single_level_zero():
+    # M = 2^0 - 1 = 0: the absmax form has one level, 0
+    x = np.random.default_rng(23).standard_normal((40, 32)).astype(np.float32)
+    codes, scale, zero, bad = quant.quantize_groups(x, 1, symmetric=True)
+    assert not bad.any() and (codes == 0).all() and (scale == 0).all() and (zero == 0).all()
+    assert (quant.dequantize_groups(codes, scale, zero) == 0).all()
+
+
+@pytest.mark.parametrize("b", range(2, 9))
+def test_symmetric_codes_are_nearest_level(b):
+    # brute force over every code: the chosen level is the nearest one of the
+    # 2M + 1 stored levels (up to the fp32 rounding of x - zero near a tie)
+    rng = np.random.default_rng(40 + b)
+    x = (rng.standard_normal((256, 32)) * np.exp(rng.uniform(-4, 4, (256, 1)))).astype(np.float32)
+    codes, scale, zero, bad = quant.quantize_groups(x, b, symmetric=True)
+    assert not bad.any()
+    M = 2 ** (b - 1) - 1
+    sf = scale.astype(np.float64)[:, None, None]
+    zf = zero.astype(np.float64)[:, None, None]
+    levels = np.arange(2 * M + 1)[None, None, :] * sf + zf
+    dist = np.abs(x.astype(np.float64)[..., None] - levels)
+    best = dist.min(axis=-1)
+    mine = np.take_along_axis(dist, codes[..., None].astype(np.int64), axis=-1)[..., 0]
+    a = np.abs(x).max(axis=-1, keepdims=True).astype(np.float64)
+    assert (mine <= best + 2.0 ** -22 * a).all()      # the fp32 rounding of x - zero
+    # mirror symmetry of the levels about 0, up to the fp16 rounding of zero
+    assert (np.abs(zf[..., 0] + M * sf[..., 0]) <= 2.0 ** -11 * np.abs(zf[..., 0])).all()
+
+
+@pytest.mark.parametrize("b", range(2, 9))
+def test_symmetric_error_bound(b):
+    # |x - x_hat| <= s / 2 + the fp16 rounding of zero, s = max|x| / M
+    rng = np.random.default_rng(30 + b)
+    x = rng.standard_normal((1024, 32)).astype(np.float32) * 2.0
+    codes, scale, zero, bad = quant.quantize_groups(x, b, symmetric=True)
+    xhat = quant.dequantize_groups(codes, scale, zero).astype(np.float64)
+    M = 2 ** (b - 1) - 1
+    sf = scale.astype(np.float64)[:, None]
+    zslack = np.abs(zero.astype(np.float64)[:, None] + M * sf)
+    a = np.abs(x).max(axis=1, keepdims=True).astype(np.float64)
+    assert (np.abs(x - xhat) <= sf / 2 + zslack + 1e-6 * a).all()
+    assert (np.abs(sf - a / M) <= 2.0 ** -11 * a / M).all()
+
+
+def test_symmetric_costs_one_level():
+    # the absmax form spends one code (2M + 1 = 2^b - 1 levels over a range
+    # 2a >= max - min), so on the same data its MSE is never far below the
+    # min-max form's and, for zero-mean data, about (2^b - 1)^2 / (2^b - 2)^2
+    # times it: a different beta, the point of a per-quantizer calibration
+    rng = np.random.default_rng(24)
+    x = rng.standard_normal((4096, 32)).astype(np.float32)
+    for b in (3, 4, 6):
+        ms = []
+        for sym in (False, True):
+            c, s, z, _ = quant.quantize_groups(x, b, symmetric=sym)
+            ms.append(((quant.dequantize_groups(c, s, z) - x) ** 2).mean())
+        assert ms[1] > ms[0]
