@@ -39,7 +39,7 @@
 extern "C" {
 #endif
 
-#define RQ_ABI_VERSION 1
+#define RQ_ABI_VERSION 2
 #define RQ_HEAD_DIM 128
 #define RQ_GROUP 32
 #define RQ_MAX_GQA 8
@@ -65,6 +65,20 @@ typedef enum { RQ_F16 = 0, RQ_BF16 = 1 } rq_dtype;
  * Sec. 2 "KV cache quantization", App. W "KIVI kernel". */
 typedef enum { RQ_PER_TOKEN = 0, RQ_PER_CHANNEL = 1 } rq_grouping;
 
+/* Per-group quantizer of a kind (keys or values), groups of 32 either way.
+ * RQ_MINMAX: asymmetric min-max, scale = fp16(fp32(max - min) / (2^b - 1)),
+ *   zero = fp16(min), codes 0 .. 2^b - 1 (KIVI values, Sec. 2).
+ * RQ_ABSMAX: the symmetric absmax form of App. W ("TurboQuant kernel"),
+ *   x_hat = round(x M / a) a / M, a = max |x|, M = 2^(b-1) - 1 (KIVI's
+ *   "per-channel symmetric" keys, Sec. 2; QuaRot / RTN per-token symmetric,
+ *   Sec. 4.1, Table 16). Stored like a min-max group: scale = fp16(a / M),
+ *   zero = fp16(0 - M * scale), codes q + M in 0 .. 2M; b = 1 (M = 0) has
+ *   the single level 0 (scale 0, zero 0, codes 0).
+ * Codes are c = clamp(rint((x - zero) * (1/scale)), 0, c_max) in fp32 with
+ * one rounding of the product, from the stored fp16 scale and zero, for
+ * both; the decoder reads both the same way (x_hat = c * scale + zero). */
+typedef enum { RQ_MINMAX = 0, RQ_ABSMAX = 1 } rq_quantizer;
+
 /* allocation flags */
 #define RQ_CAP_5X 1u /* w_i <- min(w_i, 5 * mean w) first (App. W "Mitigation") */
 
@@ -81,6 +95,8 @@ typedef struct {
   int32_t v_grouping; /* rq_grouping of values */
   int32_t hadamard;   /* 1: rotate K and V per token by R = diag(signs) H / sqrt(128)
                          before quantizing (QuaRot, App. W "QuaRot kernel") */
+  int32_t k_quantizer; /* rq_quantizer of keys */
+  int32_t v_quantizer; /* rq_quantizer of values */
 } rq_cache_desc;
 
 const char* rq_status_string(rq_status s);
@@ -141,11 +157,13 @@ size_t rq_calibrate_workspace_bytes(int32_t n, int32_t T);
 
 /* Distortion sweep (Alg. 1 stage 2; Sec. 3.4 "Distortion calibration"):
  * for every component i and b = 1..8, quantize-dequantize every group with
- * the asymmetric min-max quantizer (after the per-token Hadamard rotation
- * when `hadamard`) and store mse_dev[i][b-1] = mean over the component's
- * T*128 elements of (y - y_hat)^2 in the quantizer's domain, fp64.
+ * the kind's quantizer (after the per-token Hadamard rotation when
+ * `hadamard`) and store mse_dev[i][b-1] = mean over the component's T*128
+ * elements of (y - y_hat)^2 in the quantizer's domain, fp64. Each quantizer
+ * gets its own curve and so its own fitted beta (Sec. 3.4, Sec. 4.3, App. C).
  * x: device [n][T][128] of `dtype`; component i is a key (grouping
- * k_grouping) when i is even, a value (v_grouping) when odd.
+ * k_grouping, quantizer k_quantizer) when i is even, a value (v_grouping,
+ * v_quantizer) when odd.
  * signs_dev: device int8 [128] of +-1 (NULL = all +1; used when hadamard).
  * ws: device workspace of rq_calibrate_workspace_bytes(n, T) bytes.
  * Deterministic (fixed reduction order).
@@ -153,13 +171,15 @@ size_t rq_calibrate_workspace_bytes(int32_t n, int32_t T);
  * RQ_ERR_WORKSPACE, RQ_ERR_CUDA. */
 rq_status rq_calibrate_distortion(const void* x, int32_t dtype, int32_t n, int32_t T,
                                   int32_t k_grouping, int32_t v_grouping, int32_t hadamard,
+                                  int32_t k_quantizer, int32_t v_quantizer,
                                   const int8_t* signs_dev, double* mse_dev, void* ws,
                                   size_t ws_bytes, uint32_t* status_dev, void* stream);
 
 /* Quantize and pack one layer (the quantizer kernel indexing the per-head
  * table, App. M / App. U): for every (batch, kv head, kind) stream, every
- * group gets scale = fp16(fp32(max - min) / (2^b - 1)), zero = fp16(min),
- * codes c = clamp(rint((x - zero) * (1/scale)), 0, 2^b - 1) (fp32), written
+ * group gets the scale, zero and codes of the kind's rq_quantizer, e.g.
+ * for min-max scale = fp16(fp32(max - min) / (2^b - 1)), zero = fp16(min),
+ * codes c = clamp(rint((x - zero) * (1/scale)), 0, 2^b - 1) in fp32, written
  * to packed + offsets[layer][batch][head][kind] in the block format of
  * rq_packed_layout. k, v: device [B][H_kv][S][128] of desc->dtype (16-byte
  * aligned). bits_dev: device [L][H_kv][2]; offsets_dev: device copy of the

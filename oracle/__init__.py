@@ -9,9 +9,10 @@ pre/post-processing.
 Everything here is plain, slow and written to be checked against the paper by
 eye (RateQuant, arXiv 2605.06675):
 
-* ``quant``     -- group-wise asymmetric min-max quantizer and the randomized
-                   Hadamard pre-rotation (Sec. 4.1 "Base quantizers",
-                   App. W "Quantizer Implementation").
+* ``quant``     -- group-wise asymmetric min-max quantizer, its symmetric
+                   absmax variant, and the randomized Hadamard pre-rotation
+                   (Sec. 4.1 "Base quantizers", App. W "Quantizer
+                   Implementation").
 * ``pack``      -- the packed block format (codes + fp16 scale/zero); the paper
                    leaves storage unspecified, the format is this library's.
 * ``calib``     -- distortion sweep D_i(b) and the log-linear fit of

@@ -34,18 +34,20 @@ from .quant import quantize_stream
 
 
 def distortion_sweep(x: np.ndarray, groupings, hadamard: bool = False, signs=None,
-                     bits=range(1, 9), symmetric: bool = False) -> np.ndarray:
-    """x [n][T][128] (fp16/bf16 values as fp32); groupings[n] in {PER_TOKEN, PER_CHANNEL}.
+                     bits=range(1, 9), symmetric=False) -> np.ndarray:
+    """x [n][T][128] (fp16/bf16 values as fp32); groupings[n] in {PER_TOKEN, PER_CHANNEL};
+    ``symmetric``: one bool, or one per component (absmax instead of min-max).
 
     Returns mse [n][len(bits)] float64.
     """
     x = np.asarray(x, dtype=np.float32)
     n = x.shape[0]
     bits = list(bits)
+    sym = np.broadcast_to(np.asarray(symmetric, dtype=bool), (n,))
     out = np.zeros((n, len(bits)), dtype=np.float64)
     for i in range(n):
         for k, b in enumerate(bits):
-            r = quantize_stream(x[i], int(groupings[i]), b, signs, hadamard, symmetric)
+            r = quantize_stream(x[i], int(groupings[i]), b, signs, hadamard, bool(sym[i]))
             err = r["y"].astype(np.float64) - r["xhat"].astype(np.float64)
             out[i, k] = float(np.sum(err * err)) / err.size
     return out

@@ -1,4 +1,5 @@
-"""Group-wise asymmetric min-max quantizer and Hadamard pre-rotation (oracle).
+"""Group-wise min-max (asymmetric) and absmax (symmetric) quantizers and the
+Hadamard pre-rotation (oracle).
 
 TEST INFRASTRUCTURE ONLY -- see ``oracle/__init__.py``.
 
@@ -43,7 +44,8 @@ decoder serves both), in the same precision steps as above:
     M   = 2^(b-1) - 1
     if M == 0 (b = 1): the only level is 0: codes 0, scale 0, zero 0
     s32 = fp32_rn(a / M),  scale = fp16_rn(s32)
-    zero = fp16_rn(-M * sf)       (M * sf is exact in fp32: 7 + 11 bits)
+    zero = fp16_rn(0 - M * sf)    (M * sf is exact in fp32: 7 + 11 bits;
+                                   0 - 0 = +0, so a zero scale stores +0)
     codes as above from the stored scale and zero, clamped to 0..2M
     (code 2^b - 1 is never used)
 so level c sits at fp16(c sf + zf) ~ (c - M) sf, off the exact symmetric grid
@@ -111,7 +113,7 @@ def quantize_groups(v: np.ndarray, b: int, symmetric: bool = False):
             a = np.maximum(np.abs(mn), np.abs(mx)).astype(np.float32)
             s32 = (a / np.float32(max(M, 1.0))).astype(np.float32) * np.float32(M > 0)
             scale = s32.astype(np.float16)
-            zero = (-M * scale.astype(np.float32)).astype(np.float32).astype(np.float16)
+            zero = (np.float32(0.0) - M * scale.astype(np.float32)).astype(np.float16)
         else:
             L = np.float32(2 ** b - 1)
             s32 = ((mx - mn).astype(np.float32) / L).astype(np.float32)

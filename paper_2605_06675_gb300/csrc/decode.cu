@@ -1024,7 +1024,7 @@ __global__ void __launch_bounds__(kThreads) decode_merge_kernel(const float* par
   }
 #pragma unroll
   for (int k = 0; k < PAIRS; ++k) {
-    const int pi = tid + kThreads * k, n = pi / CW, c = pi % CW;
+    const int n = (tid + kThreads * k) / CW;
     if (n < g) {
       const float L = run_l[n];
       float v = L > 0.0f ? acc[k] / L : 0.0f;
@@ -1120,6 +1120,8 @@ rq_status check_desc(const rq_cache_desc* desc) {
   if (desc->dtype != RQ_F16 && desc->dtype != RQ_BF16) return RQ_ERR_INVALID_ARG;
   for (int g : {desc->k_grouping, desc->v_grouping})
     if (g != RQ_PER_TOKEN && g != RQ_PER_CHANNEL) return RQ_ERR_INVALID_ARG;
+  for (int qz : {desc->k_quantizer, desc->v_quantizer})
+    if (qz != RQ_MINMAX && qz != RQ_ABSMAX) return RQ_ERR_INVALID_ARG;
   if (desc->d != kD || desc->group != kG || desc->S % kTile != 0 || desc->S == 0)
     return RQ_ERR_SHAPE;
   if (desc->H_q % desc->H_kv != 0 || desc->H_q / desc->H_kv > kMaxHeads) return RQ_ERR_SHAPE;

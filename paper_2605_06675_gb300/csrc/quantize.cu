@@ -20,7 +20,7 @@
 //     RN(fp32(v - zero) * inv + 1.5 * 2^23) (fp32x2 add + fma), two codes
 //     per register by one byte permute, OR-ed into the unit's words, stored
 //     with vector stores. Codes never pass through shared memory.
-// Phase 1 flags a tile whose codes could leave [0, L], or that holds a
+// Phase 1 flags a tile whose codes could leave [0, largest code], or that holds a
 // degenerate group; such a tile takes the clamping variant of phase 2.
 #include <algorithm>
 
@@ -43,13 +43,24 @@ constexpr int kX32S = kD + 4;           // rotated fp32 row (floats)
 
 enum { kModeKC = 0, kModeKT = 1, kModeVT = 2, kModeVC = 3 };
 
-struct QSmem {
+// 16-byte multiple: the rotated fp32 tile follows it (float4 accesses)
+struct alignas(16) QSmem {
   uint8_t tile[2][kTileBytes];
   float nz[kD];                 // -zero of every group (channel c, or 32 G + t)
   float inv[kD];                // 1 / scale (0 for a group without codes)
   uint2 xchg[kThreads];         // per-channel min/max of half the tokens
+  float top;                    // magic + the largest code of the tile's quantizer
   int8_t signs[kD];
 };
+
+static_assert(sizeof(QSmem) % 16 == 0, "the rotated tile after QSmem must stay 16-byte aligned");
+
+// sm.top, read where it is used (a volatile load from a fixed shared address,
+// so the clamping variant keeps no register for it)
+__device__ __forceinline__ float clamp_top() {
+  extern __shared__ __align__(16) unsigned char smem_raw[];
+  return *reinterpret_cast<volatile const float*>(smem_raw + offsetof(QSmem, top));
+}
 
 struct QuantArgs {
   const void* k;
@@ -60,6 +71,7 @@ struct QuantArgs {
   uint8_t* packed;
   uint32_t* status;
   int layer, B, H, S, nblk, kg, vg, hadamard;
+  int kq, vq;                // rq_quantizer of keys / values
   int j_dst0;                // packed block index of each stream's first tile
   long long ntiles;
 };
@@ -70,6 +82,7 @@ struct CalibArgs {
   double* partial;           // [n][T/32][8]
   uint32_t* status;
   int n, T, ntile, kg, vg, hadamard;
+  int kq, vq;                // rq_quantizer of keys / values
   long long ntiles;
 };
 
@@ -163,14 +176,21 @@ struct GroupOut {
   bool slow, bad;
 };
 
+// quantizer of a tile at b bits: absmax when SYM, else min-max
+template <bool SYM>
+struct TileQ {
+  int b;
+};
+
 // Scale/zero of one group: meta words to global memory (packed format),
 // (-zero, 1/scale) to the table. `slow`: no codes (bad or zero range) or
-// codes that could fall outside [0, L] (they are monotone in v, so the
+// codes that could fall outside [0, cmax] (they are monotone in v, so the
 // group's min and max bound them).
+template <bool SYM>
 __device__ __forceinline__ GroupOut finish_group(int kind, int grouping, int t, int G, int c,
-                                                 float mn, float mx, bool finite, int b,
+                                                 float mn, float mx, bool finite, TileQ<SYM> q,
                                                  uint8_t* meta, QSmem& sm) {
-  const GroupParams g = group_params(mn, mx, finite, b);
+  const GroupParams g = group_params(mn, mx, finite, q.b, SYM);
   const uint32_t sb = __half_as_ushort(g.scale), zb = __half_as_ushort(g.zero);
   uint16_t* m16 = reinterpret_cast<uint16_t*>(meta);
   uint32_t* m32 = reinterpret_cast<uint32_t*>(meta);
@@ -203,18 +223,17 @@ __device__ __forceinline__ GroupOut finish_group(int kind, int grouping, int t, 
     o.slow = true;
     return o;
   }
-  const float L = static_cast<float>((1 << b) - 1);
   const float um = __fmaf_rn(__fsub_rn(mn, g.zf), g.inv, kRoundMagic);
   const float uM = __fmaf_rn(__fsub_rn(mx, g.zf), g.inv, kRoundMagic);
-  o.slow = um < kRoundMagic || uM > kRoundMagic + L;
+  o.slow = um < kRoundMagic || uM > kRoundMagic + g.cmax;
   return o;
 }
 
 // Per-channel groups on the raw tile: thread (pair p, token half hv) takes
 // channels 2p, 2p+1 over tokens 16 hv .. 16 hv + 15, the two halves meet
 // through shared memory, and the thread finishes channel 2p + hv.
-template <typename T>
-__device__ __forceinline__ GroupOut phase1_cols(const uint8_t* tile, int kind, int b,
+template <typename T, bool SYM>
+__device__ __forceinline__ GroupOut phase1_cols(const uint8_t* tile, int kind, TileQ<SYM> q,
                                                 uint8_t* meta, QSmem& sm) {
   const int tau = threadIdx.x, p = tau & 63, hv = tau >> 6;
   const uint8_t* col = tile + 4 * p + hv * 16 * kRowBytes;
@@ -235,14 +254,14 @@ __device__ __forceinline__ GroupOut phase1_cols(const uint8_t* tile, int kind, i
   const bool finite = isfinite(mn) && isfinite(mx);
   mn = __fadd_rn(mn, 0.0f);     // -0 -> +0
   mx = __fadd_rn(mx, 0.0f);
-  return finish_group(kind, RQ_PER_CHANNEL, 0, 0, 2 * p + hv, mn, mx, finite, b, meta, sm);
+  return finish_group(kind, RQ_PER_CHANNEL, 0, 0, 2 * p + hv, mn, mx, finite, q, meta, sm);
 }
 
 // Per-token groups on the raw tile: thread 4 t + G takes token t, channels
 // 32 G .. 32 G + 31 (four 16-byte reads, started at a rotating chunk so the
 // eight threads of a read phase hit distinct banks).
-template <typename T>
-__device__ __forceinline__ GroupOut phase1_rows(const uint8_t* tile, int kind, int b,
+template <typename T, bool SYM>
+__device__ __forceinline__ GroupOut phase1_rows(const uint8_t* tile, int kind, TileQ<SYM> q,
                                                 uint8_t* meta, QSmem& sm) {
   const int tau = threadIdx.x, t = tau >> 2, G = tau & 3;
   const uint8_t* row = tile + t * kRowBytes + 64 * G;
@@ -273,7 +292,7 @@ __device__ __forceinline__ GroupOut phase1_rows(const uint8_t* tile, int kind, i
   const bool finite = isfinite(mn) && isfinite(mx);
   mn = __fadd_rn(mn, 0.0f);
   mx = __fadd_rn(mx, 0.0f);
-  return finish_group(kind, RQ_PER_TOKEN, t, G, 0, mn, mx, finite, b, meta, sm);
+  return finish_group(kind, RQ_PER_TOKEN, t, G, 0, mn, mx, finite, q, meta, sm);
 }
 
 // min / max of 32 fp32 values; NaN propagates
@@ -328,9 +347,9 @@ __device__ __forceinline__ void rotate_group(float (&v)[kG], int G, const int8_t
 
 // Rotated tiles: every thread rotates one 32-channel quarter of a token and
 // writes it to the fp32 tile x32; groups are then formed on x32.
-template <typename T>
+template <typename T, bool SYM>
 __device__ __forceinline__ GroupOut phase1_rotated(const uint8_t* tile, float* x32, int kind,
-                                                   int grouping, int b, uint8_t* meta,
+                                                   int grouping, TileQ<SYM> q, uint8_t* meta,
                                                    QSmem& sm) {
   const int tau = threadIdx.x, t = tau >> 2, G = tau & 3;
   float v[kG];
@@ -355,7 +374,7 @@ __device__ __forceinline__ GroupOut phase1_rotated(const uint8_t* tile, float* x
     minmax32(v, mn, mx);
     const bool finite = isfinite(mn) && isfinite(mx);
     return finish_group(kind, RQ_PER_TOKEN, t, G, 0, __fadd_rn(mn, 0.0f), __fadd_rn(mx, 0.0f),
-                        finite, b, meta, sm);
+                        finite, q, meta, sm);
   }
   __syncthreads();
   const int p = tau & 63, hv = tau >> 6;
@@ -376,7 +395,16 @@ __device__ __forceinline__ GroupOut phase1_rotated(const uint8_t* tile, float* x
   const float mx = fmax_nan(mxh, __uint_as_float(o.y));
   const bool finite = isfinite(mn) && isfinite(mx);
   return finish_group(kind, RQ_PER_CHANNEL, 0, 0, 2 * p + hv, __fadd_rn(mn, 0.0f),
-                      __fadd_rn(mx, 0.0f), finite, b, meta, sm);
+                      __fadd_rn(mx, 0.0f), finite, q, meta, sm);
+}
+
+template <typename T, bool HAD, bool SYM>
+__device__ __forceinline__ GroupOut phase1(const uint8_t* tile, float* x32, int kind, int grouping,
+                                           int b, uint8_t* meta, QSmem& sm) {
+  const TileQ<SYM> q{b};
+  if constexpr (HAD) return phase1_rotated<T>(tile, x32, kind, grouping, q, meta, sm);
+  else if (grouping == RQ_PER_CHANNEL) return phase1_cols<T>(tile, kind, q, meta, sm);
+  else return phase1_rows<T>(tile, kind, q, meta, sm);
 }
 
 // ------------------------------------------------------------- phase 2 ----
@@ -428,9 +456,8 @@ __device__ __forceinline__ void emit(uint32_t (&uw)[B], int x, int y, float2 v, 
   const float2 d = __fadd2_rn(v, nz);
   float2 q = __ffma2_rn(d, iv, make_float2(kRoundMagic, kRoundMagic));
   if constexpr (CLAMP) {
-    constexpr float top = kRoundMagic + static_cast<float>((1 << B) - 1);
-    q.x = fminf(fmaxf(q.x, kRoundMagic), top);
-    q.y = fminf(fmaxf(q.y, kRoundMagic), top);
+    q.x = fminf(fmaxf(q.x, kRoundMagic), clamp_top());
+    q.y = fminf(fmaxf(q.y, kRoundMagic), clamp_top());
   }
   fmt::place<B>(uw, x, y, __byte_perm(__float_as_uint(q.x), __float_as_uint(q.y), 0x5410u));
 }
@@ -623,9 +650,11 @@ __global__ void __launch_bounds__(kThreads, RQ_QUANT_MIN_BLOCKS) quantize_pack_k
       uint8_t* meta = blk + 512 * b;
       const int kind = cur.kind, grouping = cur.grouping;
       GroupOut g;
-      if constexpr (HAD) g = phase1_rotated<T>(buf, x32, kind, grouping, b, meta, sm);
-      else if (grouping == RQ_PER_CHANNEL) g = phase1_cols<T>(buf, kind, b, meta, sm);
-      else g = phase1_rows<T>(buf, kind, b, meta, sm);
+      const bool sym = (kind ? a.vq : a.kq) == RQ_ABSMAX;   // kernel parameters, no register
+      if (threadIdx.x == 0)        // read by phase 2, after the barrier below
+        sm.top = kRoundMagic + static_cast<float>(sym ? (1 << b) - 2 : (1 << b) - 1);
+      if (sym) g = phase1<T, HAD, true>(buf, x32, kind, grouping, b, meta, sm);
+      else g = phase1<T, HAD, false>(buf, x32, kind, grouping, b, meta, sm);
       if (g.bad) set_status(a.status, RQ_STATUS_NUMERIC);
       const bool slow = __syncthreads_or(g.slow) != 0;
 
@@ -724,6 +753,7 @@ __global__ void __launch_bounds__(kThreads) calib_sweep_kernel(CalibArgs a) {
   const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
 
   int grouping = (static_cast<int>(tile / a.ntile) & 1) ? a.vg : a.kg;
+  bool sym = ((static_cast<int>(tile / a.ntile) & 1) ? a.vq : a.kq) == RQ_ABSMAX;
   bool row_mode = grouping == RQ_PER_TOKEN || had;
   uint4 ld[4];
   calib_load<T>(xbase + tile * kTile * kD, row_mode, ld);
@@ -731,7 +761,9 @@ __global__ void __launch_bounds__(kThreads) calib_sweep_kernel(CalibArgs a) {
     float v[kG];
     calib_group_values<T>(ld, row_mode, grouping, had, sm, x32, v);
     const long long next = tile + stride;
+    const bool sym_now = sym;
     if (next < a.ntiles) {
+      sym = ((static_cast<int>(next / a.ntile) & 1) ? a.vq : a.kq) == RQ_ABSMAX;
       grouping = (static_cast<int>(next / a.ntile) & 1) ? a.vg : a.kg;
       row_mode = grouping == RQ_PER_TOKEN || had;
       calib_load<T>(xbase + next * kTile * kD, row_mode, ld);
@@ -744,16 +776,15 @@ __global__ void __launch_bounds__(kThreads) calib_sweep_kernel(CalibArgs a) {
     double acc[8];
 #pragma unroll
     for (int b = 1; b <= 8; ++b) {
-      const GroupParams g = group_params(mn, mx, finite, b);
+      const GroupParams g = group_params(mn, mx, finite, b, sym_now);
       if (b == 1 && g.bad) set_status(a.status, RQ_STATUS_NUMERIC);
-      const float L = static_cast<float>((1 << b) - 1);
       const float2 sf = make_float2(g.sf, g.sf), zf = make_float2(g.zf, g.zf);
       float2 s2 = make_float2(0.0f, 0.0f);
 #pragma unroll
       for (int i = 0; i < kG; i += 2) {
         // code = clamp(rint(fp32(v - zero) * inv)), one rounding of the product
-        const float c0 = round_magic_clamped(__fsub_rn(v[i], g.zf), g.inv, L) - kRoundMagic;
-        const float c1 = round_magic_clamped(__fsub_rn(v[i + 1], g.zf), g.inv, L) - kRoundMagic;
+        const float c0 = round_magic_clamped(__fsub_rn(v[i], g.zf), g.inv, g.cmax) - kRoundMagic;
+        const float c1 = round_magic_clamped(__fsub_rn(v[i + 1], g.zf), g.inv, g.cmax) - kRoundMagic;
         const float2 xh = __fadd2_rn(__fmul2_rn(make_float2(c0, c1), sf), zf);
         const float2 e = __fadd2_rn(make_float2(v[i], v[i + 1]), make_float2(-xh.x, -xh.y));
         s2 = __ffma2_rn(e, e, s2);
@@ -828,6 +859,8 @@ extern "C" rq_status rq_quantize_pack(const rq_cache_desc* desc, int32_t layer, 
   if (desc->dtype != RQ_F16 && desc->dtype != RQ_BF16) return RQ_ERR_INVALID_ARG;
   for (int g : {desc->k_grouping, desc->v_grouping})
     if (g != RQ_PER_TOKEN && g != RQ_PER_CHANNEL) return RQ_ERR_INVALID_ARG;
+  for (int qz : {desc->k_quantizer, desc->v_quantizer})
+    if (qz != RQ_MINMAX && qz != RQ_ABSMAX) return RQ_ERR_INVALID_ARG;
   if (desc->d != kD || desc->group != kG || desc->S % kTile != 0) return RQ_ERR_SHAPE;
   if (!aligned16(k) || !aligned16(v) || !aligned16(packed)) return RQ_ERR_ALIGNMENT;
   QuantArgs a;
@@ -845,6 +878,8 @@ extern "C" rq_status rq_quantize_pack(const rq_cache_desc* desc, int32_t layer, 
   a.nblk = desc->S / kTile;
   a.kg = desc->k_grouping;
   a.vg = desc->v_grouping;
+  a.kq = desc->k_quantizer;
+  a.vq = desc->v_quantizer;
   a.hadamard = desc->hadamard ? 1 : 0;
   a.j_dst0 = 0;
   a.ntiles = static_cast<long long>(desc->B) * desc->H_kv * 2 * a.nblk;
@@ -866,7 +901,8 @@ extern "C" size_t rq_calibrate_workspace_bytes(int32_t n, int32_t T) {
 
 extern "C" rq_status rq_calibrate_distortion(const void* x, int32_t dtype, int32_t n, int32_t T,
                                              int32_t k_grouping, int32_t v_grouping,
-                                             int32_t hadamard, const int8_t* signs_dev,
+                                             int32_t hadamard, int32_t k_quantizer,
+                                             int32_t v_quantizer, const int8_t* signs_dev,
                                              double* mse_dev, void* ws, size_t ws_bytes,
                                              uint32_t* status_dev, void* stream) {
   using namespace rq;
@@ -874,6 +910,8 @@ extern "C" rq_status rq_calibrate_distortion(const void* x, int32_t dtype, int32
   if (dtype != RQ_F16 && dtype != RQ_BF16) return RQ_ERR_INVALID_ARG;
   for (int g : {k_grouping, v_grouping})
     if (g != RQ_PER_TOKEN && g != RQ_PER_CHANNEL) return RQ_ERR_INVALID_ARG;
+  for (int qz : {k_quantizer, v_quantizer})
+    if (qz != RQ_MINMAX && qz != RQ_ABSMAX) return RQ_ERR_INVALID_ARG;
   if (T % kTile != 0) return RQ_ERR_SHAPE;
   if (!aligned16(x) || !aligned16(ws) || (reinterpret_cast<uintptr_t>(mse_dev) & 7u))
     return RQ_ERR_ALIGNMENT;
@@ -888,6 +926,8 @@ extern "C" rq_status rq_calibrate_distortion(const void* x, int32_t dtype, int32
   a.ntile = T / kTile;
   a.kg = k_grouping;
   a.vg = v_grouping;
+  a.kq = k_quantizer;
+  a.vq = v_quantizer;
   a.hadamard = hadamard ? 1 : 0;
   a.ntiles = static_cast<long long>(n) * a.ntile;
   cudaStream_t st = static_cast<cudaStream_t>(stream);
@@ -943,6 +983,8 @@ extern "C" rq_status rq_append(const rq_cache_desc* desc, int32_t layer, int32_t
   if (desc->dtype != RQ_F16 && desc->dtype != RQ_BF16) return RQ_ERR_INVALID_ARG;
   for (int g : {desc->k_grouping, desc->v_grouping})
     if (g != RQ_PER_TOKEN && g != RQ_PER_CHANNEL) return RQ_ERR_INVALID_ARG;
+  for (int qz : {desc->k_quantizer, desc->v_quantizer})
+    if (qz != RQ_MINMAX && qz != RQ_ABSMAX) return RQ_ERR_INVALID_ARG;
   if (desc->d != kD || desc->group != kG || desc->S % kTile != 0) return RQ_ERR_SHAPE;
   if (!aligned16(k_new) || !aligned16(v_new) || !aligned16(residual) || !aligned16(packed))
     return RQ_ERR_ALIGNMENT;
@@ -974,6 +1016,8 @@ extern "C" rq_status rq_append(const rq_cache_desc* desc, int32_t layer, int32_t
   a.nblk = 1;
   a.kg = desc->k_grouping;
   a.vg = desc->v_grouping;
+  a.kq = desc->k_quantizer;
+  a.vq = desc->v_quantizer;
   a.hadamard = desc->hadamard ? 1 : 0;
   a.j_dst0 = pos / kTile;
   a.ntiles = static_cast<long long>(desc->B) * desc->H_kv * 2;

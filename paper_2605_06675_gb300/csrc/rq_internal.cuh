@@ -59,24 +59,35 @@ __device__ __forceinline__ void set_status(uint32_t* status, uint32_t bits) {
   if (status) atomicOr(status, bits);
 }
 
-// Quantizer parameters of one group (every step rounded as stated):
-//   s32 = fp32(mx - mn) / L, scale = fp16(s32), zero = fp16(mn),
+// Quantizer parameters of one group (every step rounded as stated).
+//   min-max:  s32 = fp32(mx - mn) / L, scale = fp16(s32), zero = fp16(mn),
+//             codes 0 .. L = 2^b - 1;
+//   absmax (sym): a = max(|mn|, |mx|), M = 2^(b-1) - 1, s32 = a / M (0 when
+//             M = 0), scale = fp16(s32), zero = fp16(0 - M * fp32(scale))
+//             (the product is exact), codes 0 .. 2M;
 //   inv = 1 / fp32(scale); a group is "bad" when it held a non-finite value
 //   or scale/zero overflowed fp16 (then codes, scale and zero are all 0).
 struct GroupParams {
   __half scale, zero;
   float sf, zf, inv;
-  bool ok;   // codes are computed (not bad and scale != 0)
+  float cmax;  // largest code
+  bool ok;     // codes are computed (not bad and scale != 0)
   bool bad;
 };
 
-__device__ __forceinline__ GroupParams group_params(float mn, float mx, bool finite, int b) {
+__device__ __forceinline__ GroupParams group_params(float mn, float mx, bool finite, int b,
+                                                    bool sym) {
   GroupParams g;
+  // one division for both forms: (mx - mn) / L, or a / M (0 when M = 0)
+  const float M = static_cast<float>((1 << (b - 1)) - 1);
   const float L = static_cast<float>((1 << b) - 1);
-  const float s32 = __fdiv_rn(__fsub_rn(mx, mn), L);
-  g.scale = __float2half_rn(s32);
-  g.zero = __float2half_rn(mn);
+  const float a = fmaxf(fabsf(mn), fabsf(mx));
+  const float num = sym ? (M > 0.0f ? a : 0.0f) : __fsub_rn(mx, mn);
+  const float den = sym ? fmaxf(M, 1.0f) : L;
+  g.scale = __float2half_rn(__fdiv_rn(num, den));
   g.sf = __half2float(g.scale);
+  g.zero = __float2half_rn(sym ? __fsub_rn(0.0f, __fmul_rn(M, g.sf)) : mn);
+  g.cmax = sym ? 2.0f * M : L;
   g.zf = __half2float(g.zero);
   g.bad = !finite || !isfinite(g.sf) || !isfinite(g.zf);
   g.ok = !g.bad && g.sf != 0.0f;
@@ -92,13 +103,13 @@ __device__ __forceinline__ GroupParams group_params(float mn, float mx, bool fin
 
 // 1.5 * 2^23: RN(t * inv + kRoundMagic) = kRoundMagic + rint_half_even(t * inv)
 // (exact product, one rounding) for |t * inv| < 2^22, so the code is the low
-// bits of the result; out-of-range values are clamped to [magic, magic + L]
+// bits of the result; out-of-range values are clamped to [magic, magic + cmax]
 // (NaN from a bad group clamps to magic: code 0).
 constexpr float kRoundMagic = 12582912.0f;
 
-__device__ __forceinline__ float round_magic_clamped(float t, float inv, float L) {
+__device__ __forceinline__ float round_magic_clamped(float t, float inv, float cmax) {
   const float u = __fmaf_rn(t, inv, kRoundMagic);
-  return fminf(fmaxf(u, kRoundMagic), kRoundMagic + L);
+  return fminf(fmaxf(u, kRoundMagic), kRoundMagic + cmax);
 }
 
 }  // namespace rq

@@ -22,7 +22,7 @@ class PackedKVPath:
         self.device = torch.device(device)
         self.dtype = {"float16": torch.float16, "bfloat16": torch.bfloat16}[wl.dtype]
         self.desc = rq.make_desc(wl.L, wl.B, wl.H_kv, wl.H_q, wl.S, self.dtype, wl.k_grouping,
-                                 wl.v_grouping, wl.hadamard)
+                                 wl.v_grouping, wl.hadamard, wl.k_quantizer, wl.v_quantizer)
         self.signs = signs.to(self.device) if (wl.hadamard and signs is not None) else None
         self.status = torch.zeros(1, dtype=torch.int32, device=self.device)
         self.bits = None
@@ -43,7 +43,8 @@ class PackedKVPath:
         if self._mse is None or self._mse.shape[0] != n:
             self._mse = torch.empty((n, 8), dtype=torch.float64, device=self.device)
         rq.rq_calibrate_distortion(x, self.wl.k_grouping, self.wl.v_grouping, self.wl.hadamard,
-                                   self.signs, self._mse, self._calib_ws, self.status, stream)
+                                   self.signs, self._mse, self._calib_ws, self.status, stream,
+                                   self.wl.k_quantizer, self.wl.v_quantizer)
         return self._mse
 
     # ---- a2 + a3: fit and allocate (host) ------------------------------------

@@ -18,6 +18,7 @@ LIB_PATH = os.path.join(_HERE, "librq.so")
 RQ_OK = 0
 RQ_F16, RQ_BF16 = 0, 1
 RQ_PER_TOKEN, RQ_PER_CHANNEL = 0, 1
+RQ_MINMAX, RQ_ABSMAX = 0, 1
 RQ_CAP_5X = 1
 RQ_STATUS_NUMERIC = 1
 RQ_STATUS_BAD_BITS = 2
@@ -45,7 +46,7 @@ class RQError(RuntimeError):
 class rq_cache_desc(ctypes.Structure):
     _fields_ = [(n, ctypes.c_int32) for n in
                 ("L", "B", "H_kv", "H_q", "S", "d", "group", "dtype", "k_grouping",
-                 "v_grouping", "hadamard")]
+                 "v_grouping", "hadamard", "k_quantizer", "v_quantizer")]
 
 
 _lib = None
@@ -70,7 +71,8 @@ def lib() -> ctypes.CDLL:
             "rq_alloc_continuous": ([_I, _P, _P, _P, _D, _D, _D, _P], _I),
             "rq_packed_layout": ([_P, _P, _P, _P], _I),
             "rq_calibrate_workspace_bytes": ([_I, _I], _SZ),
-            "rq_calibrate_distortion": ([_P, _I, _I, _I, _I, _I, _I, _P, _P, _P, _SZ, _P, _P], _I),
+            "rq_calibrate_distortion": ([_P, _I, _I, _I, _I, _I, _I, _I, _I, _P, _P, _P, _SZ, _P,
+                                         _P], _I),
             "rq_quantize_pack": ([_P, _I, _P, _P, _P, _P, _P, _P, _P, _P], _I),
             "rq_decode_workspace_bytes": ([_P, _P], _I),
             "rq_decode_attention": ([_P, _I, _P, _P, _P, _P, _P, _P, _P, _SZ, _P, _P], _I),
@@ -130,10 +132,11 @@ def torch_dtype_code(dtype) -> int:
     raise ValueError(f"unsupported dtype {dtype}")
 
 
-def make_desc(L, B, H_kv, H_q, S, dtype, k_grouping, v_grouping, hadamard=False) -> rq_cache_desc:
+def make_desc(L, B, H_kv, H_q, S, dtype, k_grouping, v_grouping, hadamard=False,
+              k_quantizer=RQ_MINMAX, v_quantizer=RQ_MINMAX) -> rq_cache_desc:
     code = dtype if isinstance(dtype, int) else torch_dtype_code(dtype)
     return rq_cache_desc(L, B, H_kv, H_q, S, HEAD_DIM, GROUP, code, k_grouping, v_grouping,
-                         1 if hadamard else 0)
+                         1 if hadamard else 0, k_quantizer, v_quantizer)
 
 
 # ------------------------------------------------------------------ host ----
@@ -200,12 +203,12 @@ def rq_calibrate_workspace_bytes(n: int, T: int) -> int:
 
 
 def rq_calibrate_distortion(x, k_grouping, v_grouping, hadamard, signs, mse, ws, status=None,
-                            stream=None):
+                            stream=None, k_quantizer=RQ_MINMAX, v_quantizer=RQ_MINMAX):
     """x: CUDA [n][T][128] fp16/bf16; mse: CUDA float64 [n][8]; ws: CUDA byte buffer."""
     n, T, d = x.shape
     _check("rq_calibrate_distortion", lib().rq_calibrate_distortion(
         _dp(x), torch_dtype_code(x.dtype), n, T, k_grouping, v_grouping, 1 if hadamard else 0,
-        _dp(signs), _dp(mse), _dp(ws), ws.numel() * ws.element_size(), _dp(status),
+        k_quantizer, v_quantizer, _dp(signs), _dp(mse), _dp(ws), ws.numel() * ws.element_size(), _dp(status),
         _stream(stream)))
 
 

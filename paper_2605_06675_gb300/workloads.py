@@ -38,6 +38,8 @@ class Workload:
     value_dist: str            # "gaussian" | "student_t4"
     seed: int
     calib_T: int = 512
+    k_quantizer: int = 0       # rq_quantizer: 0 min-max, 1 absmax (symmetric)
+    v_quantizer: int = 0
 
     @property
     def g(self) -> int:

@@ -37,7 +37,7 @@ def to_np(t: torch.Tensor) -> np.ndarray:
     return t.detach().float().cpu().numpy()
 
 
-def oracle_layer(k, v, bits_layer, kg, vg, hadamard, signs, streams=None):
+def oracle_layer(k, v, bits_layer, kg, vg, hadamard, signs, streams=None, symmetric=False):
     """Oracle quantize+pack of the requested (batch, head) streams of one
     layer; only those slices are copied to the host."""
     sg = None if signs is None else signs.cpu().numpy()
@@ -48,7 +48,8 @@ def oracle_layer(k, v, bits_layer, kg, vg, hadamard, signs, streams=None):
     for bb, h in streams:
         kk = to_np(k[bb:bb + 1, h:h + 1])
         vv = to_np(v[bb:bb + 1, h:h + 1])
-        r = opipe.quantize_layer(kk, vv, np.asarray(bits_layer)[h:h + 1], kg, vg, hadamard, sg)
+        r = opipe.quantize_layer(kk, vv, np.asarray(bits_layer)[h:h + 1], kg, vg, hadamard, sg,
+                                 symmetric=symmetric)
         for kind in (0, 1):
             out[(bb, h, kind)] = r[(0, 0, kind)]
     return out

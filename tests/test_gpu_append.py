@@ -24,17 +24,19 @@ CHECKPOINTS = (1, 17, 31, 32, 33, 64, 95, 96, 100, 128, 159, 160)
 
 
 @pytest.mark.gpu
-@pytest.mark.parametrize("dtype,kg,vg,hadamard,allowed", [
-    ("bfloat16", PER_CHANNEL, PER_TOKEN, False, (2, 3, 4)),
-    ("float16", PER_CHANNEL, PER_TOKEN, False, (2, 3, 4, 8)),
-    ("bfloat16", PER_TOKEN, PER_TOKEN, True, (3, 5, 6, 7)),
-    ("float16", PER_TOKEN, PER_CHANNEL, False, (1, 2, 4)),
+@pytest.mark.parametrize("dtype,kg,vg,hadamard,allowed,kq,vq", [
+    ("bfloat16", PER_CHANNEL, PER_TOKEN, False, (2, 3, 4), 0, 0),
+    ("float16", PER_CHANNEL, PER_TOKEN, False, (2, 3, 4, 8), 0, 0),
+    ("bfloat16", PER_TOKEN, PER_TOKEN, True, (3, 5, 6, 7), 0, 0),
+    ("float16", PER_TOKEN, PER_CHANNEL, False, (1, 2, 4), 0, 0),
+    ("bfloat16", PER_CHANNEL, PER_TOKEN, False, (2, 3, 4, 6), 1, 0),     # KIVI symmetric keys
+    ("bfloat16", PER_TOKEN, PER_TOKEN, True, (2, 4, 5, 8), 1, 1),        # QuaRot symmetric
 ])
-def test_append_then_decode_matches_oracle(dtype, kg, vg, hadamard, allowed):
+def test_append_then_decode_matches_oracle(dtype, kg, vg, hadamard, allowed, kq, vq):
     ensure_built()
     wl = Workload("append", L=2, B=2, H_kv=2, H_q=8, S=160, dtype=dtype, k_grouping=kg,
                   v_grouping=vg, hadamard=hadamard, allowed=allowed, avg_bits=3.0, sigma_lnw=0.5,
-                  value_dist="gaussian", seed=51)
+                  value_dist="gaussian", seed=51, k_quantizer=kq, v_quantizer=vq)
     layer = 1
     signs = synth.hadamard_signs(wl.seed).to(DEV) if hadamard else None
     path = PackedKVPath(wl, DEV, signs)
@@ -54,7 +56,8 @@ def test_append_then_decode_matches_oracle(dtype, kg, vg, hadamard, allowed):
         s_pk = 32 * (n // 32)
         ol = {}
         if s_pk:
-            ol = oracle_layer(k[:, :, :s_pk], v[:, :, :s_pk], bits[layer], kg, vg, hadamard, signs)
+            ol = oracle_layer(k[:, :, :s_pk], v[:, :, :s_pk], bits[layer], kg, vg, hadamard, signs,
+                              symmetric=(kq == 1, vq == 1))
             for (bb, h, kind), r in ol.items():   # the packed prefix, bit for bit
                 words = r["words"].view(np.uint8)
                 got = path.stream_bytes(layer, bb, h, kind)[:words.size].cpu().numpy()

@@ -23,13 +23,18 @@ def rq():
 
 
 def small_wl(L=2, B=2, H=4, g=4, S=96, dtype="float16", kg=PER_CHANNEL, vg=PER_TOKEN,
-             hadamard=False, seed=11, value_dist="gaussian"):
+             hadamard=False, seed=11, value_dist="gaussian", kq=0, vq=0):
     return Workload(f"t{seed}", L=L, B=B, H_kv=H, H_q=H * g, S=S, dtype=dtype, k_grouping=kg,
                     v_grouping=vg, hadamard=hadamard, allowed=tuple(range(1, 9)), avg_bits=4.0,
-                    sigma_lnw=0.5, value_dist=value_dist, seed=seed)
+                    sigma_lnw=0.5, value_dist=value_dist, seed=seed, k_quantizer=kq,
+                    v_quantizer=vq)
 
 
-def run_layers(rq, wl, bits, layers=None, q_seed=0):
+def symmetric_of(wl):
+    return (wl.k_quantizer == 1, wl.v_quantizer == 1)
+
+
+def run_layers(rq, wl, bits, layers=None, q_seed=0, kv_scale=1.0):
     """Quantize every layer and decode; returns (path, {l: (k, v, q, out)})."""
     signs = synth.hadamard_signs(wl.seed) if wl.hadamard else None
     path = PackedKVPath(wl, DEV, signs)
@@ -37,6 +42,8 @@ def run_layers(rq, wl, bits, layers=None, q_seed=0):
     res = {}
     for l in (range(wl.L) if layers is None else layers):
         k, v = synth.kv_layer(wl.B, wl.H_kv, wl.S, wl.dtype, wl.seed, l, wl.value_dist, DEV)
+        if kv_scale != 1.0:
+            k, v = k * kv_scale, v * kv_scale
         q = synth.queries(wl.B, wl.H_q, wl.dtype, wl.seed + q_seed, l, DEV)
         out = torch.empty((wl.B, wl.H_q, 128), dtype=torch.float32, device=DEV)
         path.quantize(l, k, v)
@@ -49,7 +56,7 @@ def run_layers(rq, wl, bits, layers=None, q_seed=0):
 def check_layer(path, wl, l, k, v, q, out, signs, streams=None):
     """Bit-exact packed bytes and attention within TOL for the given streams."""
     ol = oracle_layer(k, v, path.bits_host[l], wl.k_grouping, wl.v_grouping, wl.hadamard,
-                      signs, streams)
+                      signs, streams, symmetric_of(wl))
     for (bb, h, kind), r in ol.items():
         got = path.stream_bytes(l, bb, h, kind).cpu().numpy()
         want = r["words"].view(np.uint8)
@@ -237,3 +244,79 @@ def test_calibration_deterministic(rq):
     a = path.calibrate(x).clone()
     b = path.calibrate(x).clone()
     assert torch.equal(a, b)
+
+
+# ---- symmetric absmax quantizer (App. W "TurboQuant kernel" form) -----------
+# KIVI: per-channel symmetric keys, per-token asymmetric values (Sec. 2);
+# RTN: per-token symmetric (Table 16); QuaRot: rotation + per-token
+# symmetric (Sec. 4.1); and every grouping with both kinds symmetric.
+SYM_CASES = [
+    ("kivi", "float16", PER_CHANNEL, PER_TOKEN, False, 1, 0),
+    ("kivi", "bfloat16", PER_CHANNEL, PER_TOKEN, False, 1, 0),
+    ("rtn", "bfloat16", PER_TOKEN, PER_TOKEN, False, 1, 1),
+    ("quarot", "bfloat16", PER_TOKEN, PER_TOKEN, True, 1, 1),
+    ("quarot", "float16", PER_TOKEN, PER_TOKEN, True, 1, 1),
+    ("vc", "float16", PER_TOKEN, PER_CHANNEL, False, 1, 1),
+    ("kc_vc_mixed", "bfloat16", PER_CHANNEL, PER_CHANNEL, False, 0, 1),
+]
+
+
+@pytest.mark.parametrize("name,dtype,kg,vg,hadamard,kq,vq", SYM_CASES)
+def test_symmetric_all_widths_bit_exact_and_attention(rq, name, dtype, kg, vg, hadamard, kq, vq):
+    wl = small_wl(dtype=dtype, kg=kg, vg=vg, hadamard=hadamard, S=96, seed=61, kq=kq, vq=vq)
+    bits = bits_cycle(wl.L, wl.H_kv, range(1, 9), offset=2)
+    path, res, signs = run_layers(rq, wl, bits)
+    for l, (k, v, q, out) in res.items():
+        check_layer(path, wl, l, k, v, q, out, signs)
+    assert int(path.status.item()) == 0
+
+
+@pytest.mark.parametrize("kq,vq", [(1, 1), (0, 1)])
+def test_symmetric_tiny_values_take_the_clamped_path(rq, kq, vq):
+    # |x| ~ 2^-20: scales fall in the fp16 subnormal range, codes can leave
+    # 0..2M before clamping (the clamped variant of the quantizer)
+    wl = small_wl(L=1, dtype="bfloat16", kg=PER_CHANNEL, vg=PER_TOKEN, S=64, seed=62,
+                  kq=kq, vq=vq)
+    bits = bits_cycle(1, wl.H_kv, range(1, 9), offset=1)
+    path, res, signs = run_layers(rq, wl, bits, kv_scale=2.0 ** -20)
+    check_layer(path, wl, 0, *res[0], signs)
+
+
+@pytest.mark.parametrize("hadamard,kg,vg", [(False, PER_CHANNEL, PER_TOKEN),
+                                            (True, PER_TOKEN, PER_TOKEN),
+                                            (True, PER_CHANNEL, PER_CHANNEL)])
+def test_symmetric_calibration_matches_oracle(rq, hadamard, kg, vg):
+    wl = small_wl(L=2, H=4, S=96, dtype="bfloat16", hadamard=hadamard, seed=63, kg=kg, vg=vg,
+                  kq=1, vq=0 if kg == PER_CHANNEL and not hadamard else 1)
+    x = synth.calibration_sample(wl, T=96, device=DEV)
+    signs = synth.hadamard_signs(wl.seed) if hadamard else None
+    path = PackedKVPath(wl, DEV, signs)
+    mse = path.calibrate(x).cpu().numpy()
+    torch.cuda.synchronize()
+    n = x.shape[0]
+    groupings = [wl.k_grouping if i % 2 == 0 else wl.v_grouping for i in range(n)]
+    sym = [symmetric_of(wl)[i % 2] for i in range(n)]
+    ref = ocalib.distortion_sweep(to_np(x), groupings, hadamard,
+                                  None if signs is None else signs.numpy(), symmetric=sym)
+    rel = np.abs(mse - ref) / np.abs(ref)
+    assert rel.max() < MSE_RTOL, rel.max()
+    assert np.all(np.diff(mse, axis=1) < 0)
+
+
+def test_quantizer_argument_errors(rq):
+    wl = small_wl(L=1, B=1, H=2, g=2, S=64, dtype="bfloat16", seed=64)
+    path = PackedKVPath(wl, DEV)
+    path.set_bits(bits_cycle(1, 2, (2, 3)))
+    k = torch.zeros((1, 2, 64, 128), dtype=torch.bfloat16, device=DEV)
+    for kq, vq in ((2, 0), (0, -1)):
+        bad = rq.make_desc(1, 1, 2, 4, 64, torch.bfloat16, 1, 0, False, kq, vq)
+        with pytest.raises(rq.RQError) as e:
+            rq.rq_quantize_pack(bad, 0, k, k, None, path.bits, path.offsets, path.packed)
+        assert e.value.status == 1
+    x = torch.zeros((2, 64, 128), dtype=torch.bfloat16, device=DEV)
+    mse = torch.empty((2, 8), dtype=torch.float64, device=DEV)
+    ws = torch.empty(rq.rq_calibrate_workspace_bytes(2, 64), dtype=torch.uint8, device=DEV)
+    with pytest.raises(rq.RQError) as e:
+        rq.rq_calibrate_distortion(x, 1, 0, False, None, mse, ws, k_quantizer=3)
+    assert e.value.status == 1
+

@@ -34,7 +34,7 @@ def test_exports_every_header_symbol(rq):
     for name in declared:
         assert hasattr(lib, name), name
     assert sorted(rq.EXPORTS) == declared
-    assert rq.rq_abi_version() == 1
+    assert rq.rq_abi_version() == 2
     assert rq.rq_status_string(3) == "unsupported shape"
 
 

@@ -291,6 +291,7 @@ def test_symmetric_one_bit_has_the_single_level_zero():
     x = np.random.default_rng(23).standard_normal((40, 32)).astype(np.float32)
     codes, scale, zero, bad = quant.quantize_groups(x, 1, symmetric=True)
     assert not bad.any() and (codes == 0).all() and (scale == 0).all() and (zero == 0).all()
+    assert (zero.view(np.uint16) == 0).all()      # +0, not -0: the stored words are exact
     assert (quant.dequantize_groups(codes, scale, zero) == 0).all()
 
 
