@@ -38,6 +38,9 @@ def _peaks():
         return FALLBACK_HBM_GBS, "fallback"
 
 
+QUANTIZERS = ["minmax", "absmax"]       # rq_quantizer values 0, 1
+
+
 def _workloads():
     from paper_2605_06675_gb300 import workloads as W
     return {w.name: w for w in W.ALL}, W.LLAMA3_8B_32K
@@ -52,6 +55,9 @@ def _parse():
     ap.add_argument("--workload", default=None)
     ap.add_argument("--layers", type=int, default=None,
                     help="run only the first N layers (small cases for profiling)")
+    ap.add_argument("--k-quantizer", choices=["minmax", "absmax"], default=None,
+                    help="override the workload's key quantizer (absmax = symmetric)")
+    ap.add_argument("--v-quantizer", choices=["minmax", "absmax"], default=None)
     ap.add_argument("--no-e2e", action="store_true")
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--cpu-leg", action="store_true", help=argparse.SUPPRESS)
@@ -326,7 +332,9 @@ def run_ours(args, wl, rank, world, local_rank):
                    "S": wl.S, "head_dim": 128, "group": 32, "bits_allowed": list(wl.allowed),
                    "avg_bits": wl.avg_bits, "k_grouping": "per_channel" if wl.k_grouping else "per_token",
                    "v_grouping": "per_channel" if wl.v_grouping else "per_token",
-                   "hadamard": wl.hadamard, "calib_tokens": T, "parallelism": f"replicas x{world}",
+                   "hadamard": wl.hadamard, "k_quantizer": QUANTIZERS[wl.k_quantizer],
+                   "v_quantizer": QUANTIZERS[wl.v_quantizer],
+                   "calib_tokens": T, "parallelism": f"replicas x{world}",
                    "l2": "inputs larger than L2 (no flush)"},
         "components": {
             "decode_attention": {"gbs": round(d_gbs, 1), "frac_of_measured_hbm": round(d_gbs / peak, 4),
@@ -456,7 +464,8 @@ def oracle_sample_run(wl, tokens: int, n_calib: int, heads: int = 1, budget_s: f
 
     t0 = time.perf_counter()
     groupings = [wl.k_grouping if i % 2 == 0 else wl.v_grouping for i in range(xs.shape[0])]
-    mse = ocalib.distortion_sweep(xs, groupings, wl.hadamard, signs)
+    sym = [(wl.v_quantizer if i % 2 else wl.k_quantizer) == 1 for i in range(xs.shape[0])]
+    mse = ocalib.distortion_sweep(xs, groupings, wl.hadamard, signs, symmetric=sym)
     mse_all = np.resize(mse, (n, 8))
     a, b, _ = ocalib.fit_distortion(mse_all, 2, 6, 0.96, np.arange(n) % 2)
     oalloc.allocate(w, a, b, wl.avg_bits, wl.allowed_mask)
@@ -478,7 +487,8 @@ def oracle_sample_run(wl, tokens: int, n_calib: int, heads: int = 1, budget_s: f
                           dtype=np.uint8)
             t1 = time.perf_counter()
             ol = opipe.quantize_layer(ks[:, h:h + 1], vs[:, h:h + 1], bl, wl.k_grouping,
-                                      wl.v_grouping, wl.hadamard, signs)
+                                      wl.v_grouping, wl.hadamard, signs,
+                                      symmetric=(wl.k_quantizer == 1, wl.v_quantizer == 1))
             opipe.attend_layer(qs[:, h * wl.g:(h + 1) * wl.g], ol)
             el += time.perf_counter() - t1
             packed = sum(nblk * 512 * (int(x) + 1) for x in bl.reshape(-1))
@@ -507,7 +517,8 @@ def run_cpu_leg_subprocess(wl, tokens=None):
     env["CUDA_VISIBLE_DEVICES"] = ""
     for var in ("RANK", "WORLD_SIZE", "LOCAL_RANK", "MASTER_ADDR", "MASTER_PORT"):
         env.pop(var, None)
-    cmd = [sys.executable, os.path.join(ROOT, "bench.py"), "--cpu-leg", "--workload", wl.name]
+    cmd = [sys.executable, os.path.join(ROOT, "bench.py"), "--cpu-leg", "--workload", wl.name,
+           "--k-quantizer", QUANTIZERS[wl.k_quantizer], "--v-quantizer", QUANTIZERS[wl.v_quantizer]]
     if tokens:
         cmd += ["--cpu-tokens", str(tokens)]
     try:
@@ -552,6 +563,10 @@ def main():
     wl = table[args.workload] if args.workload else default
     if args.layers:
         wl = wl.scaled(L=min(args.layers, wl.L))
+    for kind in ("k", "v"):
+        qz = getattr(args, f"{kind}_quantizer")
+        if qz is not None:
+            wl = wl.scaled(**{f"{kind}_quantizer": QUANTIZERS.index(qz)})
     if args.cpu_leg:
         cpu_leg_main(args, wl)
         return

@@ -22,6 +22,9 @@ eye (RateQuant, arXiv 2605.06675):
                    Alg. 2, Prop. 3), exact DP for non-contiguous bit sets, and
                    continuous reverse waterfilling (Thm. 1 Eq. 2, App. B.1).
 * ``attention`` -- decode attention on the dequantized cache, fp64.
+* ``transfer``  -- cross-quantizer transfer matrix: allocate with one
+                   quantizer's fitted model, score on another's measured
+                   distortion (Sec. 3.4, Fig. 3; App. W Table 25).
 
 Floating point: fp64 everywhere except the quantizer, whose steps are pinned
 to fp32 / fp16 rounding (see ``quant``), because codes, scales and zero-points
