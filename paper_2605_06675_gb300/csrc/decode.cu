@@ -195,9 +195,16 @@ __device__ __forceinline__ uint32_t dequant(uint32_t sub, uint32_t m, uint32_t z
 // s is returned in log2 units (q . k times qsc = log2(e) / sqrt(128), applied
 // here in fp32 so q enters the MMAs unscaled) relative to the running max
 // (ms0, ms1: the max of heads 2tig, 2tig + 1, 0 while unset).
-template <int BW, int KG>
+// q s 2^-E enters as an fp16 sum hi + lo (lo = the exact remainder, one fp16
+// FMA), so the products keep ~22 bits. With g <= 4 query heads (MERGED)
+// the MMA's 8 columns hold hi for heads 0..3 and lo for the same heads in
+// columns 4..7 (lanes gid >= 4 carry q of head gid - 4 and mneg = -1 there,
+// -0 elsewhere), and one shuffle adds the halves; otherwise hi and lo take
+// one MMA each.
+template <int BW, int KG, bool MERGED>
 __device__ __forceinline__ void qk_block(const uint8_t* img, int lane, const uint8_t* qtab,
-                                         float qsc, float ms0, float ms1, float (&s)[2][4]) {
+                                         float qsc, float ms0, float ms1, uint32_t mneg,
+                                         float (&s)[2][4]) {
   const int gid = lane >> 2, tig = lane & 3;
   uint32_t w[4 * BW];
   lane_words<BW>(img, lane, w);
@@ -221,22 +228,40 @@ __device__ __forceinline__ void qk_block(const uint8_t* img, int lane, const uin
 #pragma unroll
       for (int xs = 0; xs < 2; ++xs) {
         const uint4 MZ = xs ? MZ1 : MZ0;
-        // q s 2^-E as an fp16 pair sum hi + lo: lo = fp16(q s 2^-E - hi) is
-        // the exact remainder (one fp16 FMA), so the products keep ~22 bits
-        const uint32_t b0 = hmul2u(qf[2 * xs], MZ.y);
-        const uint32_t b1 = hmul2u(qf[2 * xs + 1], MZ.w);
-        const uint32_t l0 = hfma2u(qf[2 * xs], MZ.y, b0 ^ 0x80008000u);
-        const uint32_t l1 = hfma2u(qf[2 * xs + 1], MZ.w, b1 ^ 0x80008000u);
+        const uint32_t h0 = hmul2u(qf[2 * xs], MZ.y);
+        const uint32_t h1 = hmul2u(qf[2 * xs + 1], MZ.w);
         const uint32_t az[4] = {MZ.x, MZ.y, MZ.z, MZ.w};
         mma16816(zb, az, qb[2 * xs], qb[2 * xs + 1]);
+        if constexpr (MERGED) {
+          // hi lanes: fma(q, s, hi * -0) = hi; lo lanes: fma(q, s, -hi) = lo
+          // (fp16 multiplies, not bitwise ops: they run on the FMA pipe,
+          // which the code extraction leaves idle)
+          const uint32_t b0 = hfma2u(qf[2 * xs], MZ.y, hmul2u(h0, mneg));
+          const uint32_t b1 = hfma2u(qf[2 * xs + 1], MZ.w, hmul2u(h1, mneg));
 #pragma unroll
-        for (int mt = 0; mt < 2; ++mt) {
-          const uint32_t a[4] = {reg<BW>(w, u, 2 * xs, 2 * mt), reg<BW>(w, u, 2 * xs, 2 * mt + 1),
-                                 reg<BW>(w, u, 2 * xs + 1, 2 * mt), reg<BW>(w, u, 2 * xs + 1, 2 * mt + 1)};
-          mma16816(s[mt], a, b0, b1);
-          mma16816(s[mt], a, l0, l1);
+          for (int mt = 0; mt < 2; ++mt) {
+            const uint32_t a[4] = {reg<BW>(w, u, 2 * xs, 2 * mt), reg<BW>(w, u, 2 * xs, 2 * mt + 1),
+                                   reg<BW>(w, u, 2 * xs + 1, 2 * mt), reg<BW>(w, u, 2 * xs + 1, 2 * mt + 1)};
+            mma16816(s[mt], a, b0, b1);
+          }
+        } else {
+          const uint32_t l0 = hfma2u(qf[2 * xs], MZ.y, h0 ^ 0x80008000u);
+          const uint32_t l1 = hfma2u(qf[2 * xs + 1], MZ.w, h1 ^ 0x80008000u);
+#pragma unroll
+          for (int mt = 0; mt < 2; ++mt) {
+            const uint32_t a[4] = {reg<BW>(w, u, 2 * xs, 2 * mt), reg<BW>(w, u, 2 * xs, 2 * mt + 1),
+                                   reg<BW>(w, u, 2 * xs + 1, 2 * mt), reg<BW>(w, u, 2 * xs + 1, 2 * mt + 1)};
+            mma16816(s[mt], a, h0, h1);
+            mma16816(s[mt], a, l0, l1);
+          }
         }
       }
+    }
+    if constexpr (MERGED) {   // columns j and j + 4 of the accumulator: hi + lo
+#pragma unroll
+      for (int mt = 0; mt < 2; ++mt)
+#pragma unroll
+        for (int r = 0; r < 4; ++r) s[mt][r] += __shfl_xor_sync(0xffffffffu, s[mt][r], 2);
     }
     const float c0 = __fmaf_rn(zb[0], qsc, -ms0), c1 = __fmaf_rn(zb[1], qsc, -ms1);
     const float f = kTwo24 * qsc;
@@ -369,8 +394,8 @@ template <int BW>
 __device__ __forceinline__ void qk_dispatch_g(int kg, const uint8_t* img, int lane,
                                               const uint8_t* qtab, float qsc, float ms0, float ms1,
                                               float (&s)[2][4]) {
-  if (kg == RQ_PER_CHANNEL) qk_block<BW, RQ_PER_CHANNEL>(img, lane, qtab, qsc, ms0, ms1, s);
-  else qk_block<BW, RQ_PER_TOKEN>(img, lane, qtab, qsc, ms0, ms1, s);
+  if (kg == RQ_PER_CHANNEL) qk_block<BW, RQ_PER_CHANNEL, false>(img, lane, qtab, qsc, ms0, ms1, 0u, s);
+  else qk_block<BW, RQ_PER_TOKEN, false>(img, lane, qtab, qsc, ms0, ms1, 0u, s);   // mneg unused
 }
 
 template <int BW>
@@ -449,6 +474,8 @@ struct WarpStream {
   uint8_t* ring_ptr;      // this warp's ring of slots
   uint32_t ring;          // its shared-memory address
   int lane, nb;
+  bool merged;            // g <= 4: hi and lo q operands share one MMA
+  uint32_t mneg;          // merged: fp16x2 -1 on the lanes that carry lo (gid >= 4), else -0
 };
 
 // online-softmax state of one warp: o^T accumulators and per-column max/sum
@@ -566,7 +593,7 @@ __device__ __forceinline__ void prologue_static(const WarpStream& ws) {
   for (int e = 0; e < Ring<BK, BV>::kSlots - 1; ++e) issue_static<BK, BV>(ws, e, e);
 }
 
-template <int BK, int KG, int BV, int VG>
+template <int BK, int KG, int BV, int VG, bool MERGED>
 __device__ __forceinline__ void blocks_static(const WarpStream& ws, const uint8_t* qtab, float qsc,
                                               SoftmaxAcc& acc) {
   using R = Ring<BK, BV>;
@@ -578,8 +605,9 @@ __device__ __forceinline__ void blocks_static(const WarpStream& ws, const uint8_
     cp_async_wait<NS - 1>();
     __syncwarp();
     float s[2][4];
-    qk_block<BK, KG>(ws.ring_ptr + use * R::kSlot, ws.lane, qtab, qsc,
-                     acc.m0 == -INFINITY ? 0.0f : acc.m0, acc.m1 == -INFINITY ? 0.0f : acc.m1, s);
+    qk_block<BK, KG, MERGED>(ws.ring_ptr + use * R::kSlot, ws.lane, qtab, qsc,
+                     acc.m0 == -INFINITY ? 0.0f : acc.m0, acc.m1 == -INFINITY ? 0.0f : acc.m1,
+                     ws.mneg, s);
     __syncwarp();
     use = use + 1 == NS ? 0 : use + 1;
     uint32_t pb[2][2];
@@ -689,6 +717,8 @@ __global__ void __launch_bounds__(kThreads, RQ_DECODE_MIN_BLOCKS) decode_split_k
   ws.kwarp = kbase + static_cast<size_t>(blk_first) * dr.sK;
   ws.vwarp = vbase + static_cast<size_t>(blk_first) * dr.sV;
   const int key = valid ? fast_key(bK, bV, a.kg, a.vg) : -1;
+  ws.merged = a.g <= kMaxHeads / 2 && key >= 0;   // the compile-time KIVI paths only
+  ws.mneg = ws.merged && gid >= kMaxHeads / 2 ? 0xBC00BC00u : 0x80008000u;
 
   // start streaming the first entries before the q prologue
   switch (key) {
@@ -727,11 +757,14 @@ __global__ void __launch_bounds__(kThreads, RQ_DECODE_MIN_BLOCKS) decode_split_k
 #pragma unroll
   for (int x = 0; x < 4; ++x) ef[x] = pow2_neg_h2(a.kg == RQ_PER_CHANNEL && valid ? fmt::exponent(bK, x) : 0);
   if (warp == 0) {
+    // merged (g <= 4): columns 4..7 repeat heads 0..3 (they carry lo in the
+    // scores MMA; elsewhere they give duplicate results that are not stored)
+    const int qrow = ws.merged ? (gid & 3) : gid;
 #pragma unroll
     for (int u = 0; u < 4; ++u)
 #pragma unroll
       for (int x = 0; x < 4; ++x) {
-        const float* qr = qs + gid * kD + 32 * u + 8 * tig + 2 * x;
+        const float* qr = qs + qrow * kD + 32 * u + 8 * tig + 2 * x;
         qb[u][x] = pack_f16x2(qr[0] * qpow, qr[1] * qpow);
         qf[u][x] = hmul2u(qb[u][x], ef[x]);
       }
@@ -761,7 +794,11 @@ __global__ void __launch_bounds__(kThreads, RQ_DECODE_MIN_BLOCKS) decode_split_k
   acc.l0 = acc.l1 = 0.0f;
 
   switch (key) {
-#define RQ_BLK(k, BK, BV) case k: blocks_static<BK, RQ_PER_CHANNEL, BV, RQ_PER_TOKEN>(ws, qtab, qscale, acc); break;
+#define RQ_BLK(k, BK, BV)                                                                        \
+  case k:                                                                                        \
+    if (ws.merged) blocks_static<BK, RQ_PER_CHANNEL, BV, RQ_PER_TOKEN, true>(ws, qtab, qscale, acc); \
+    else blocks_static<BK, RQ_PER_CHANNEL, BV, RQ_PER_TOKEN, false>(ws, qtab, qscale, acc);        \
+    break;
     RQ_FAST_CASES(RQ_BLK)
 #undef RQ_BLK
     default: blocks_dyn(ws, dr, qtab, qscale, acc); break;
@@ -835,7 +872,6 @@ __global__ void __launch_bounds__(kThreads, RQ_DECODE_MIN_BLOCKS) decode_split_k
       dst[kD + 1] = lsum;
     }
   }
-
 }
 
 // ------------------------------------------------------------ split merge ----
