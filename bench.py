@@ -172,14 +172,15 @@ class ClockSampler:
 # --------------------------------------------------------------------------
 
 def kernel_source_hash(name: str) -> str:
-    """sha256[:16] of a kernel's translation unit together with the headers it
-    includes (format.cuh, rq_internal.cuh, rq.h), so a record goes stale when
-    any of them changes."""
+    """sha256[:16] of a kernel's translation unit together with the library's
+    headers (every .cuh and rq.h), so a record goes stale when any of them
+    changes."""
     import hashlib
     csrc = os.path.join(ROOT, "paper_2605_06675_gb300", "csrc")
     h = hashlib.sha256()
-    for path in (os.path.join(csrc, name), os.path.join(csrc, "format.cuh"),
-                 os.path.join(csrc, "rq_internal.cuh"), os.path.join(ROOT, "include", "rq.h")):
+    headers = sorted(f for f in os.listdir(csrc) if f.endswith(".cuh"))
+    for path in ([os.path.join(csrc, name)] + [os.path.join(csrc, f) for f in headers] +
+                 [os.path.join(ROOT, "include", "rq.h")]):
         h.update(open(path, "rb").read())
     return h.hexdigest()[:16]
 

@@ -24,7 +24,8 @@ ARCH = ["-gencode", "arch=compute_103a,code=sm_103a"]
 NVCC_FLAGS = ["-O3", "-lineinfo", "-std=c++17", "-Xcompiler", "-fPIC", "-Xcompiler", "-O2",
               "-Xcompiler", "-ffp-contract=off",
               "-prec-div=true", "-prec-sqrt=true", f"-I{INCLUDE}", f"-I{CSRC}"]
-SOURCES = ["host.cpp", "quantize.cu", "decode.cu"]
+SOURCES = ["host.cpp", "quantize.cu", "quantize_k_f16.cu", "quantize_k_f16_rot.cu",
+           "quantize_k_bf16.cu", "quantize_k_bf16_rot.cu", "decode.cu"]
 
 
 def nvcc() -> str:

@@ -75,6 +75,24 @@ struct GroupParams {
   bool bad;
 };
 
+// RN(1 / (2^k - 1)), k = 0..8 (index 0 unused): the divisors of the scale
+static __constant__ float kInvPow2m1[9] = {1.0f,         1.0f / 1.0f,   1.0f / 3.0f,
+                                           1.0f / 7.0f,  1.0f / 15.0f,  1.0f / 31.0f,
+                                           1.0f / 63.0f, 1.0f / 127.0f, 1.0f / 255.0f};
+
+// RN(x / y) for y = 2^k - 1 (k = 1..8) and yi = RN(1 / y): Markstein's
+// correction step, q0 = RN(x yi), r = x - q0 y (exact in one FMA),
+// q = RN(q0 + r yi). Checked equal to IEEE division for every fp32
+// significand of x and each of these divisors (tests/test_lib_host.py);
+// exact scaling by powers of two carries it to every exponent of a normal
+// quotient, and quotients below the fp32 normal range round to fp16 zero
+// either way.
+__device__ __forceinline__ float div_pow2m1(float x, float y, float yi) {
+  const float q0 = __fmul_rn(x, yi);
+  const float r = __fmaf_rn(-q0, y, x);
+  return __fmaf_rn(r, yi, q0);
+}
+
 __device__ __forceinline__ GroupParams group_params(float mn, float mx, bool finite, int b,
                                                     bool sym) {
   GroupParams g;
@@ -84,7 +102,8 @@ __device__ __forceinline__ GroupParams group_params(float mn, float mx, bool fin
   const float a = fmaxf(fabsf(mn), fabsf(mx));
   const float num = sym ? (M > 0.0f ? a : 0.0f) : __fsub_rn(mx, mn);
   const float den = sym ? fmaxf(M, 1.0f) : L;
-  g.scale = __float2half_rn(__fdiv_rn(num, den));
+  const float deni = kInvPow2m1[sym ? (b > 1 ? b - 1 : 1) : b];
+  g.scale = __float2half_rn(div_pow2m1(num, den, deni));
   g.sf = __half2float(g.scale);
   g.zero = __float2half_rn(sym ? __fsub_rn(0.0f, __fmul_rn(M, g.sf)) : mn);
   g.cmax = sym ? 2.0f * M : L;

@@ -130,3 +130,49 @@ def test_packed_layout_matches_oracle(rq):
     bits[0, 0, 0] = 9
     with pytest.raises(rq.RQError):
         rq.rq_packed_layout(desc, bits)
+
+
+DIV_CHECK_C = r"""
+#include <math.h>
+#include <stdint.h>
+#include <stdio.h>
+#include <string.h>
+/* The quantizer's scale division: q0 = RN(x yi), r = RN(x - q0 y) by one fma,
+   q = RN(q0 + r yi), yi = RN(1 / y), against x / y, for every significand of x
+   in [1, 2) and y = 2^k - 1, k = 1..8. */
+int main(void) {
+  long bad = 0;
+  for (int k = 1; k <= 8; ++k) {
+    const float y = (float)((1 << k) - 1), yi = 1.0f / y;
+    for (uint32_t m = 0; m < (1u << 23); ++m) {
+      uint32_t u = (127u << 23) | m;
+      float x;
+      memcpy(&x, &u, 4);
+      const float q0 = x * yi;
+      const float r = fmaf(-q0, y, x);
+      const float q = fmaf(r, yi, q0);
+      if (q != x / y) ++bad;
+    }
+  }
+  printf("%ld\n", bad);
+  return 0;
+}
+"""
+
+
+def test_scale_division_method_is_exact(tmp_path):
+    # The kernels divide the group range by 2^b - 1 (and the absmax by
+    # 2^(b-1) - 1) with a correction step instead of an IEEE division; this
+    # proves it exact for every fp32 significand on an IEEE host (binary32
+    # multiply and fma correctly rounded, no contraction).
+    import shutil
+    import subprocess
+    cc = shutil.which("gcc") or shutil.which("cc")
+    if cc is None:
+        pytest.skip("no C compiler")
+    src = tmp_path / "div.c"
+    src.write_text(DIV_CHECK_C)
+    exe = tmp_path / "div"
+    subprocess.run([cc, "-O2", "-ffp-contract=off", "-o", str(exe), str(src), "-lm"], check=True)
+    out = subprocess.run([str(exe)], capture_output=True, text=True, check=True).stdout
+    assert out.strip() == "0"
