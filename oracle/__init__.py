@@ -22,6 +22,9 @@ eye (RateQuant, arXiv 2605.06675):
                    Alg. 2, Prop. 3), exact DP for non-contiguous bit sets, and
                    continuous reverse waterfilling (Thm. 1 Eq. 2, App. B.1).
 * ``attention`` -- decode attention on the dequantized cache, fp64.
+* ``lloydmax``  -- Lloyd-Max codebook of N(0, 1) (Lloyd iteration + Newton)
+                   and the RMS-normalised group quantizer that uses it
+                   (App. F Table 8; TurboQuant's scalar quantizer, App. W).
 * ``transfer``  -- cross-quantizer transfer matrix: allocate with one
                    quantizer's fitted model, score on another's measured
                    distortion (Sec. 3.4, Fig. 3; App. W Table 25).

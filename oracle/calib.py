@@ -9,7 +9,7 @@ Paper passages followed
 * Alg. 1 stage 2 and Sec. 3.4 "Distortion calibration": measure the MSE at
   b in {2,...,6} and fit by least squares on ln D = ln alpha - b ln beta.
 * App. W "Outlier heads": heads with R^2 < 0.96 use beta = min(beta_fit, beta_bar).
-* App. G Table 8 (Lloyd-Max, d = 128): the exact D(b) column is the pin for
+* App. F Table 8 (Lloyd-Max, d = 128): the exact D(b) column is the pin for
   the fit; the paper reports alpha ~ 1.36, beta ~ 3.48.
 
 Readings where the paper is silent
@@ -36,18 +36,19 @@ from .quant import quantize_stream
 def distortion_sweep(x: np.ndarray, groupings, hadamard: bool = False, signs=None,
                      bits=range(1, 9), symmetric=False) -> np.ndarray:
     """x [n][T][128] (fp16/bf16 values as fp32); groupings[n] in {PER_TOKEN, PER_CHANNEL};
-    ``symmetric``: one bool, or one per component (absmax instead of min-max).
+    ``symmetric``: the quantizer form (``quant.MINMAX`` / ``ABSMAX`` /
+    ``LLOYDMAX``; a bool means min-max / absmax), one, or one per component.
 
     Returns mse [n][len(bits)] float64.
     """
     x = np.asarray(x, dtype=np.float32)
     n = x.shape[0]
     bits = list(bits)
-    sym = np.broadcast_to(np.asarray(symmetric, dtype=bool), (n,))
+    sym = np.broadcast_to(np.asarray(symmetric, dtype=np.int64), (n,))
     out = np.zeros((n, len(bits)), dtype=np.float64)
     for i in range(n):
         for k, b in enumerate(bits):
-            r = quantize_stream(x[i], int(groupings[i]), b, signs, hadamard, bool(sym[i]))
+            r = quantize_stream(x[i], int(groupings[i]), b, signs, hadamard, int(sym[i]))
             err = r["y"].astype(np.float64) - r["xhat"].astype(np.float64)
             out[i, k] = float(np.sum(err * err)) / err.size
     return out

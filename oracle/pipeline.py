@@ -23,7 +23,8 @@ def quantize_layer(k, v, bits, k_grouping, v_grouping, hadamard=False, signs=Non
 
     bits [H][2]. ``streams`` optionally restricts work to a list of
     (batch, head) pairs (for sampled checks at large sizes). ``symmetric``:
-    one bool, or a (keys, values) pair (absmax instead of min-max).
+    the quantizer form (``quant.MINMAX`` / ``ABSMAX`` / ``LLOYDMAX``; a bool
+    means min-max / absmax), one, or a (keys, values) pair.
     Returns {(batch, head, kind): dict(words=uint32[...], xhat=fp64 [S,128]
     in the original domain, bad=bool groups)}.
     """
@@ -33,12 +34,12 @@ def quantize_layer(k, v, bits, k_grouping, v_grouping, hadamard=False, signs=Non
     bits = np.asarray(bits).reshape(H, 2)
     if streams is None:
         streams = [(bb, h) for bb in range(B) for h in range(H)]
-    sym = np.broadcast_to(np.asarray(symmetric, dtype=bool), (2,))
+    sym = np.broadcast_to(np.asarray(symmetric, dtype=np.int64), (2,))
     out = {}
     for bb, h in streams:
         for kind, x, grouping in ((pack.KIND_K, k, k_grouping), (pack.KIND_V, v, v_grouping)):
             b = int(bits[h, kind])
-            r = quantize_stream(x[bb, h], grouping, b, signs, hadamard, bool(sym[kind]))
+            r = quantize_stream(x[bb, h], grouping, b, signs, hadamard, int(sym[kind]))
             words = pack.pack_stream(r["codes"], r["scale"], r["zero"], kind, grouping, b)
             xhat = r["xhat"].astype(np.float64)
             if hadamard:

@@ -165,10 +165,15 @@ def from_groups(g: np.ndarray, grouping: int) -> np.ndarray:
     return g.transpose(0, 2, 1).reshape(nblk * GROUP, HEAD_DIM)
 
 
+MINMAX, ABSMAX, LLOYDMAX = 0, 1, 2      # group quantizer forms
+
+
 def quantize_stream(x: np.ndarray, grouping: int, b: int, signs: np.ndarray | None = None,
-                    hadamard: bool = False, symmetric: bool = False):
+                    hadamard: bool = False, symmetric=False):
     """Quantize one (batch, head, K/V) stream x[S, 128].
 
+    ``symmetric`` selects the group quantizer: False / MINMAX, True / ABSMAX,
+    or LLOYDMAX (the codebook quantizer of ``lloydmax``).
     Returns dict with the quantizer-domain values ``y`` [S,128] (rotated when
     ``hadamard``), ``codes`` [S,128] uint8 (element order), group-shaped
     ``scale``/``zero``/``bad``, and ``xhat`` [S,128] fp32 in the quantizer domain.
@@ -177,8 +182,14 @@ def quantize_stream(x: np.ndarray, grouping: int, b: int, signs: np.ndarray | No
     y = hadamard_rotate(x, signs) if hadamard else x.astype(np.float32)
     y = canonical(y)
     g = to_groups(y, grouping)
-    codes, scale, zero, bad = quantize_groups(g, b, symmetric)
-    xhat = dequantize_groups(codes, scale, zero)
+    form = int(symmetric)
+    if form == LLOYDMAX:
+        from . import lloydmax
+        codes, scale, zero, bad = lloydmax.quantize_groups(g, b)
+        xhat = lloydmax.dequantize_groups(codes, scale, b)
+    else:
+        codes, scale, zero, bad = quantize_groups(g, b, form == ABSMAX)
+        xhat = dequantize_groups(codes, scale, zero)
     return {
         "y": y,
         "codes": from_groups(codes, grouping),

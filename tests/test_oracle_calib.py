@@ -22,7 +22,7 @@ def _table8():
 
 
 def test_table8_fit_reproduces_paper():
-    # Sec. 3.1 / App. G Table 8: fitting the exact Lloyd-Max D(b), b = 1..6,
+    # Sec. 3.1 / App. F Table 8: fitting the exact Lloyd-Max D(b), b = 1..6,
     # gives alpha ~ 1.36, beta ~ 3.48, R^2 > 0.99, and the "Fit" column.
     b, exact, fit, ratio = _table8()
     row = np.zeros(8)
