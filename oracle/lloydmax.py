@@ -24,7 +24,8 @@ centroid condition makes the cross terms vanish).
 Group quantizer (the reading used here; the paper gives no per-group
 normalisation for this quantizer, and TurboQuant scales by the vector
 norm): for one group x[0..31], with v = fp32(x) + 0 as in ``quant``,
-    s2    = sum_{i = 0..31, in this order} fp32(v_i * v_i), fp32 adds
+    s2    = fp32(S(0..15) + S(16..31)), S(i..j) = the fp32 sum of fp32(v_k * v_k)
+            for k = i..j in this order (two halves, added last)
     scale = fp16(fp32_sqrt(s2 / 32)),  zero = +0         (the group's RMS)
     L_c   = fp16(l_c)                                     (stored levels)
     T_i   = fp32(fp32((L_{i-1} + L_i) / 2) * sf),  i = 1..n-1
@@ -129,9 +130,13 @@ def quantize_groups(v: np.ndarray, b: int):
     with np.errstate(all="ignore"):
         finite = np.isfinite(v).all(axis=-1)
         vv = np.where(finite[..., None], v, np.float32(0.0))
-        s2 = np.zeros(vv.shape[:-1], dtype=np.float32)
-        for i in range(GROUP):                       # sequential fp32 sum of squares
-            s2 = (s2 + (vv[..., i] * vv[..., i]).astype(np.float32)).astype(np.float32)
+        halves = []
+        for h in range(2):                           # each half summed in order, in fp32
+            acc = np.zeros(vv.shape[:-1], dtype=np.float32)
+            for i in range(16 * h, 16 * h + 16):
+                acc = (acc + (vv[..., i] * vv[..., i]).astype(np.float32)).astype(np.float32)
+            halves.append(acc)
+        s2 = (halves[0] + halves[1]).astype(np.float32)
         rms = np.sqrt((s2 / np.float32(GROUP)).astype(np.float32)).astype(np.float32)
         scale = rms.astype(np.float16)
         bad = (~finite) | (~np.isfinite(scale))
