@@ -38,7 +38,7 @@ def _peaks():
         return FALLBACK_HBM_GBS, "fallback"
 
 
-QUANTIZERS = ["minmax", "absmax"]       # rq_quantizer values 0, 1
+QUANTIZERS = ["minmax", "absmax", "lloydmax"]       # rq_quantizer values 0, 1, 2
 
 
 def _workloads():
@@ -55,9 +55,9 @@ def _parse():
     ap.add_argument("--workload", default=None)
     ap.add_argument("--layers", type=int, default=None,
                     help="run only the first N layers (small cases for profiling)")
-    ap.add_argument("--k-quantizer", choices=["minmax", "absmax"], default=None,
+    ap.add_argument("--k-quantizer", choices=["minmax", "absmax", "lloydmax"], default=None,
                     help="override the workload's key quantizer (absmax = symmetric)")
-    ap.add_argument("--v-quantizer", choices=["minmax", "absmax"], default=None)
+    ap.add_argument("--v-quantizer", choices=["minmax", "absmax", "lloydmax"], default=None)
     ap.add_argument("--no-e2e", action="store_true")
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--cpu-leg", action="store_true", help=argparse.SUPPRESS)
@@ -465,7 +465,7 @@ def oracle_sample_run(wl, tokens: int, n_calib: int, heads: int = 1, budget_s: f
 
     t0 = time.perf_counter()
     groupings = [wl.k_grouping if i % 2 == 0 else wl.v_grouping for i in range(xs.shape[0])]
-    sym = [(wl.v_quantizer if i % 2 else wl.k_quantizer) == 1 for i in range(xs.shape[0])]
+    sym = [wl.v_quantizer if i % 2 else wl.k_quantizer for i in range(xs.shape[0])]
     mse = ocalib.distortion_sweep(xs, groupings, wl.hadamard, signs, symmetric=sym)
     mse_all = np.resize(mse, (n, 8))
     a, b, _ = ocalib.fit_distortion(mse_all, 2, 6, 0.96, np.arange(n) % 2)
@@ -489,7 +489,7 @@ def oracle_sample_run(wl, tokens: int, n_calib: int, heads: int = 1, budget_s: f
             t1 = time.perf_counter()
             ol = opipe.quantize_layer(ks[:, h:h + 1], vs[:, h:h + 1], bl, wl.k_grouping,
                                       wl.v_grouping, wl.hadamard, signs,
-                                      symmetric=(wl.k_quantizer == 1, wl.v_quantizer == 1))
+                                      symmetric=(wl.k_quantizer, wl.v_quantizer))
             opipe.attend_layer(qs[:, h * wl.g:(h + 1) * wl.g], ol)
             el += time.perf_counter() - t1
             packed = sum(nblk * 512 * (int(x) + 1) for x in bl.reshape(-1))

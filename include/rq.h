@@ -76,8 +76,16 @@ typedef enum { RQ_PER_TOKEN = 0, RQ_PER_CHANNEL = 1 } rq_grouping;
  *   the single level 0 (scale 0, zero 0, codes 0).
  * Codes are c = clamp(rint((x - zero) * (1/scale)), 0, c_max) in fp32 with
  * one rounding of the product, from the stored fp16 scale and zero, for
- * both; the decoder reads both the same way (x_hat = c * scale + zero). */
-typedef enum { RQ_MINMAX = 0, RQ_ABSMAX = 1 } rq_quantizer;
+ * both; the decoder reads both the same way (x_hat = c * scale + zero).
+ * RQ_LLOYDMAX: the 2^b-level Lloyd-Max codebook of a unit Gaussian (App. F
+ *   Table 8; TurboQuant's scalar quantizer, App. W) scaled by the group's
+ *   RMS: scale = fp16(sqrt(s2 / 32)) with s2 the fp32 sum of squares of
+ *   values 0..15 plus that of values 16..31 (each summed in order), zero = 0,
+ *   code = the number of thresholds fp32(fp32((L_{i-1} + L_i) / 2) * scale)
+ *   at or below the value (L = the fp16 levels of rq_lloydmax_levels),
+ *   x_hat = L_code * scale. Per-token groups only (RQ_ERR_INVALID_ARG with
+ *   per-channel groups), the grouping TurboQuant uses. */
+typedef enum { RQ_MINMAX = 0, RQ_ABSMAX = 1, RQ_LLOYDMAX = 2 } rq_quantizer;
 
 /* allocation flags */
 #define RQ_CAP_5X 1u /* w_i <- min(w_i, 5 * mean w) first (App. W "Mitigation") */
@@ -101,6 +109,13 @@ typedef struct {
 
 const char* rq_status_string(rq_status s);
 int32_t rq_abi_version(void);
+
+/* The fp16 levels (bit patterns, ascending, 2^b of them) of the RQ_LLOYDMAX
+ * codebook at b bits: the Lloyd-Max quantizer of N(0, 1), computed by the
+ * library on first use (Lloyd's iteration, then Newton's method on the same
+ * fixed point, in fp64) and rounded to nearest fp16. levels: host array of
+ * 2^b entries. Errors: RQ_ERR_INVALID_ARG (b outside 1..8, NULL). */
+rq_status rq_lloydmax_levels(int32_t b, uint16_t* levels);
 
 /* ---------------------------------------------------------------- host ---- */
 

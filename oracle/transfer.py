@@ -17,14 +17,15 @@ import numpy as np
 
 from .alloc import allocate
 from .calib import distortion_sweep, fit_distortion
-from .quant import PER_CHANNEL, PER_TOKEN
+from .quant import ABSMAX, LLOYDMAX, MINMAX, PER_CHANNEL, PER_TOKEN
 
-# name -> (key grouping, value grouping, hadamard, key symmetric, value symmetric)
+# name -> (key grouping, value grouping, hadamard, key form, value form)
 FAMILIES = {
-    "kivi": (PER_CHANNEL, PER_TOKEN, False, False, False),
-    "kivi_sym": (PER_CHANNEL, PER_TOKEN, False, True, False),
-    "rtn": (PER_TOKEN, PER_TOKEN, False, True, True),
-    "quarot": (PER_TOKEN, PER_TOKEN, True, True, True),
+    "kivi": (PER_CHANNEL, PER_TOKEN, False, MINMAX, MINMAX),
+    "kivi_sym": (PER_CHANNEL, PER_TOKEN, False, ABSMAX, MINMAX),
+    "rtn": (PER_TOKEN, PER_TOKEN, False, ABSMAX, ABSMAX),
+    "quarot": (PER_TOKEN, PER_TOKEN, True, ABSMAX, ABSMAX),
+    "turboquant": (PER_TOKEN, PER_TOKEN, True, LLOYDMAX, LLOYDMAX),
 }
 
 

@@ -76,6 +76,8 @@ struct DecodeArgs {
   float* partial;            // [B][H_q][splits][132]
   uint32_t* status;
   int layer, B, H, Hq, g, nblk, splits, bps, kg, vg, hadamard;
+  int kq, vq;                // rq_quantizer of keys / values
+  LMBook lm;                 // RQ_LLOYDMAX codebooks
 };
 
 __device__ __forceinline__ uint32_t h2u(__half2 h) { return *reinterpret_cast<uint32_t*>(&h); }
@@ -178,6 +180,15 @@ __device__ __forceinline__ uint32_t dequant(uint32_t sub, uint32_t m, uint32_t z
   return hfma2u(hsub2u(sub | kMagic, kMagic), m, z2);
 }
 
+// Lloyd-Max pair: the two codes of an extracted register (at bit E of each
+// half) looked up in the width's fp16 codebook (shared memory), scaled by m
+// and shifted by z2 (one fp16x2 FMA)
+template <int BW>
+__device__ __forceinline__ uint32_t lm_pair(uint32_t sub, int E, const uint16_t* tab) {
+  const uint32_t c0 = (sub >> E) & ((1u << BW) - 1u), c1 = (sub >> (16 + E)) & ((1u << BW) - 1u);
+  return static_cast<uint32_t>(tab[c0]) | (static_cast<uint32_t>(tab[c1]) << 16);
+}
+
 // ------------------------------------------------------------ block math ----
 // Lane (gid, tig) reads units u = 0..3 of its K words: unit u holds channels
 // 32 u + 8 tig + (0..7) of tokens gid + 8 (0..3); the k-steps 2u and 2u + 1
@@ -201,10 +212,10 @@ __device__ __forceinline__ uint32_t dequant(uint32_t sub, uint32_t m, uint32_t z
 // columns 4..7 (lanes gid >= 4 carry q of head gid - 4 and mneg = -1 there,
 // -0 elsewhere), and one shuffle adds the halves; otherwise hi and lo take
 // one MMA each.
-template <int BW, int KG, bool MERGED>
+template <int BW, int KG, bool MERGED, bool LM = false>
 __device__ __forceinline__ void qk_block(const uint8_t* img, int lane, const uint8_t* qtab,
                                          float qsc, float ms0, float ms1, uint32_t mneg,
-                                         float (&s)[2][4]) {
+                                         float (&s)[2][4], const uint16_t* lmtab = nullptr) {
   const int gid = lane >> 2, tig = lane & 3;
   uint32_t w[4 * BW];
   lane_words<BW>(img, lane, w);
@@ -284,19 +295,22 @@ __device__ __forceinline__ void qk_block(const uint8_t* img, int lane, const uin
 #pragma unroll
       for (int x = 0; x < 4; ++x) {
         const __half2 h = u2h(sz[x]);
-        m[x] = hmul2u(h2u(__low2half2(h)), pow2_neg_h2(fmt::exponent(BW, x)));
+        m[x] = LM ? h2u(__low2half2(h))          // codebook levels are real values
+                  : hmul2u(h2u(__low2half2(h)), pow2_neg_h2(fmt::exponent(BW, x)));
         z2[x] = h2u(__high2half2(h));
       }
+      auto deq = [&](int x, int y) -> uint32_t {
+        if constexpr (LM) return hfma2u(lm_pair<BW>(reg<BW>(w, u, x, y), fmt::exponent(BW, x), lmtab),
+                                        m[x], z2[x]);
+        else return dequant(reg<BW>(w, u, x, y), m[x], z2[x]);
+      };
 #pragma unroll
       for (int xs = 0; xs < 2; ++xs)
 #pragma unroll
         for (int mt = 0; mt < 2; ++mt) {
           // register (x = token 2mt + r, y = pair 2xs + h)
-          const uint32_t a[4] = {
-              dequant(reg<BW>(w, u, 2 * mt, 2 * xs), m[2 * mt], z2[2 * mt]),
-              dequant(reg<BW>(w, u, 2 * mt + 1, 2 * xs), m[2 * mt + 1], z2[2 * mt + 1]),
-              dequant(reg<BW>(w, u, 2 * mt, 2 * xs + 1), m[2 * mt], z2[2 * mt]),
-              dequant(reg<BW>(w, u, 2 * mt + 1, 2 * xs + 1), m[2 * mt + 1], z2[2 * mt + 1])};
+          const uint32_t a[4] = {deq(2 * mt, 2 * xs), deq(2 * mt + 1, 2 * xs),
+                                 deq(2 * mt, 2 * xs + 1), deq(2 * mt + 1, 2 * xs + 1)};
           mma16816(s[mt], a, qb[2 * xs], qb[2 * xs + 1]);
         }
     }
@@ -318,9 +332,10 @@ __device__ __forceinline__ void qk_block(const uint8_t* img, int lane, const uin
 // the scale is folded into P^T per group (one fp16x2 multiply per pair), the
 // zero-point term comes from MMAs whose A operand repeats z_tG in every row
 // of the group, and the codes' 2^(E - 24) is undone on the output rows.
-template <int BW, int VG>
+template <int BW, int VG, bool LM = false>
 __device__ __forceinline__ void pv_block(const uint8_t* img, int lane, const uint32_t (&pb)[2][2],
-                                         float (&o)[8][4], float (&bz)[2][4]) {
+                                         float (&o)[8][4], float (&bz)[2][4],
+                                         const uint16_t* lmtab = nullptr) {
   const int gid = lane >> 2, tig = lane & 3;
   uint32_t w[4 * BW];
   lane_words<BW>(img, lane, w);
@@ -356,9 +371,14 @@ __device__ __forceinline__ void pv_block(const uint8_t* img, int lane, const uin
         const uint32_t b1 = hmul2u(pb[ks][1], ms[2 * ks + 1][G]);
 #pragma unroll
         for (int mh = 0; mh < 2; ++mh) {
-          // register (x = row 2mh + r, y = token pair 2ks + h)
-          const uint32_t a[4] = {reg<BW>(w, G, 2 * mh, 2 * ks), reg<BW>(w, G, 2 * mh + 1, 2 * ks),
-                                 reg<BW>(w, G, 2 * mh, 2 * ks + 1), reg<BW>(w, G, 2 * mh + 1, 2 * ks + 1)};
+          // register (x = row 2mh + r, y = token pair 2ks + h); Lloyd-Max: the
+          // codebook levels (real values) instead of the subnormal codes
+          auto A = [&](int x, int y) -> uint32_t {
+            if constexpr (LM) return lm_pair<BW>(reg<BW>(w, G, x, y), fmt::exponent(BW, x), lmtab);
+            else return reg<BW>(w, G, x, y);
+          };
+          const uint32_t a[4] = {A(2 * mh, 2 * ks), A(2 * mh + 1, 2 * ks), A(2 * mh, 2 * ks + 1),
+                                 A(2 * mh + 1, 2 * ks + 1)};
           mma16816(o[2 * G + mh], a, b0, b1);
         }
       }
@@ -393,46 +413,49 @@ __device__ __forceinline__ void pv_block(const uint8_t* img, int lane, const uin
 template <int BW>
 __device__ __forceinline__ void qk_dispatch_g(int kg, const uint8_t* img, int lane,
                                               const uint8_t* qtab, float qsc, float ms0, float ms1,
-                                              float (&s)[2][4]) {
+                                              float (&s)[2][4], const uint16_t* lmtab) {
+  // mneg is unused off the merged path; lmtab is non-null for Lloyd-Max keys
   if (kg == RQ_PER_CHANNEL) qk_block<BW, RQ_PER_CHANNEL, false>(img, lane, qtab, qsc, ms0, ms1, 0u, s);
-  else qk_block<BW, RQ_PER_TOKEN, false>(img, lane, qtab, qsc, ms0, ms1, 0u, s);   // mneg unused
+  else if (lmtab) qk_block<BW, RQ_PER_TOKEN, false, true>(img, lane, qtab, qsc, ms0, ms1, 0u, s, lmtab);
+  else qk_block<BW, RQ_PER_TOKEN, false>(img, lane, qtab, qsc, ms0, ms1, 0u, s);
 }
 
 template <int BW>
 __device__ __forceinline__ void pv_dispatch_g(int vg, const uint8_t* img, int lane,
                                               const uint32_t (&pb)[2][2], float (&o)[8][4],
-                                              float (&bz)[2][4]) {
-  if (vg == RQ_PER_TOKEN) pv_block<BW, RQ_PER_TOKEN>(img, lane, pb, o, bz);
+                                              float (&bz)[2][4], const uint16_t* lmtab) {
+  if (vg == RQ_PER_TOKEN && lmtab) pv_block<BW, RQ_PER_TOKEN, true>(img, lane, pb, o, bz, lmtab);
+  else if (vg == RQ_PER_TOKEN) pv_block<BW, RQ_PER_TOKEN>(img, lane, pb, o, bz);
   else pv_block<BW, RQ_PER_CHANNEL>(img, lane, pb, o, bz);
 }
 
 __device__ __forceinline__ void qk_dispatch(int bw, int kg, const uint8_t* img, int lane,
                                             const uint8_t* qtab, float qsc, float ms0, float ms1,
-                                            float (&s)[2][4]) {
+                                            float (&s)[2][4], const uint16_t* lmtab) {
   switch (bw) {
-    case 1: qk_dispatch_g<1>(kg, img, lane, qtab, qsc, ms0, ms1, s); break;
-    case 2: qk_dispatch_g<2>(kg, img, lane, qtab, qsc, ms0, ms1, s); break;
-    case 3: qk_dispatch_g<3>(kg, img, lane, qtab, qsc, ms0, ms1, s); break;
-    case 4: qk_dispatch_g<4>(kg, img, lane, qtab, qsc, ms0, ms1, s); break;
-    case 5: qk_dispatch_g<5>(kg, img, lane, qtab, qsc, ms0, ms1, s); break;
-    case 6: qk_dispatch_g<6>(kg, img, lane, qtab, qsc, ms0, ms1, s); break;
-    case 7: qk_dispatch_g<7>(kg, img, lane, qtab, qsc, ms0, ms1, s); break;
-    default: qk_dispatch_g<8>(kg, img, lane, qtab, qsc, ms0, ms1, s); break;
+    case 1: qk_dispatch_g<1>(kg, img, lane, qtab, qsc, ms0, ms1, s, lmtab); break;
+    case 2: qk_dispatch_g<2>(kg, img, lane, qtab, qsc, ms0, ms1, s, lmtab); break;
+    case 3: qk_dispatch_g<3>(kg, img, lane, qtab, qsc, ms0, ms1, s, lmtab); break;
+    case 4: qk_dispatch_g<4>(kg, img, lane, qtab, qsc, ms0, ms1, s, lmtab); break;
+    case 5: qk_dispatch_g<5>(kg, img, lane, qtab, qsc, ms0, ms1, s, lmtab); break;
+    case 6: qk_dispatch_g<6>(kg, img, lane, qtab, qsc, ms0, ms1, s, lmtab); break;
+    case 7: qk_dispatch_g<7>(kg, img, lane, qtab, qsc, ms0, ms1, s, lmtab); break;
+    default: qk_dispatch_g<8>(kg, img, lane, qtab, qsc, ms0, ms1, s, lmtab); break;
   }
 }
 
 __device__ __forceinline__ void pv_dispatch(int bw, int vg, const uint8_t* img, int lane,
                                             const uint32_t (&pb)[2][2], float (&o)[8][4],
-                                            float (&bz)[2][4]) {
+                                            float (&bz)[2][4], const uint16_t* lmtab) {
   switch (bw) {
-    case 1: pv_dispatch_g<1>(vg, img, lane, pb, o, bz); break;
-    case 2: pv_dispatch_g<2>(vg, img, lane, pb, o, bz); break;
-    case 3: pv_dispatch_g<3>(vg, img, lane, pb, o, bz); break;
-    case 4: pv_dispatch_g<4>(vg, img, lane, pb, o, bz); break;
-    case 5: pv_dispatch_g<5>(vg, img, lane, pb, o, bz); break;
-    case 6: pv_dispatch_g<6>(vg, img, lane, pb, o, bz); break;
-    case 7: pv_dispatch_g<7>(vg, img, lane, pb, o, bz); break;
-    default: pv_dispatch_g<8>(vg, img, lane, pb, o, bz); break;
+    case 1: pv_dispatch_g<1>(vg, img, lane, pb, o, bz, lmtab); break;
+    case 2: pv_dispatch_g<2>(vg, img, lane, pb, o, bz, lmtab); break;
+    case 3: pv_dispatch_g<3>(vg, img, lane, pb, o, bz, lmtab); break;
+    case 4: pv_dispatch_g<4>(vg, img, lane, pb, o, bz, lmtab); break;
+    case 5: pv_dispatch_g<5>(vg, img, lane, pb, o, bz, lmtab); break;
+    case 6: pv_dispatch_g<6>(vg, img, lane, pb, o, bz, lmtab); break;
+    case 7: pv_dispatch_g<7>(vg, img, lane, pb, o, bz, lmtab); break;
+    default: pv_dispatch_g<8>(vg, img, lane, pb, o, bz, lmtab); break;
   }
 }
 
@@ -626,6 +649,8 @@ __device__ __forceinline__ void blocks_static(const WarpStream& ws, const uint8_
 // ---- streaming with runtime widths/groupings (every other combination)
 struct DynRing {
   int bK, bV, kg, vg, sK, sV, slot, ns;
+  const uint16_t* lmK;       // Lloyd-Max codebook of the key / value width (null: none)
+  const uint16_t* lmV;
 };
 
 __device__ __forceinline__ void issue_dyn(const WarpStream& ws, const DynRing& r, int e, int slot) {
@@ -649,7 +674,7 @@ __device__ __forceinline__ void blocks_dyn(const WarpStream& ws, const DynRing& 
     __syncwarp();
     float s[2][4];
     qk_dispatch(r.bK, r.kg, ws.ring_ptr + use * r.slot, ws.lane, qtab, qsc,
-                acc.m0 == -INFINITY ? 0.0f : acc.m0, acc.m1 == -INFINITY ? 0.0f : acc.m1, s);
+                acc.m0 == -INFINITY ? 0.0f : acc.m0, acc.m1 == -INFINITY ? 0.0f : acc.m1, s, r.lmK);
     __syncwarp();
     use = use + 1 == r.ns ? 0 : use + 1;
     uint32_t pb[2][2];
@@ -658,7 +683,7 @@ __device__ __forceinline__ void blocks_dyn(const WarpStream& ws, const DynRing& 
     iss = iss + 1 == r.ns ? 0 : iss + 1;
     cp_async_wait_dyn(r.ns - 1);
     __syncwarp();
-    pv_dispatch(r.bV, r.vg, ws.ring_ptr + use * r.slot, ws.lane, pb, acc.o, acc.bz);
+    pv_dispatch(r.bV, r.vg, ws.ring_ptr + use * r.slot, ws.lane, pb, acc.o, acc.bz, r.lmV);
     __syncwarp();
     use = use + 1 == r.ns ? 0 : use + 1;
   }
@@ -685,6 +710,7 @@ __global__ void __launch_bounds__(kThreads, RQ_DECODE_MIN_BLOCKS) decode_split_k
   uint8_t* rings = smem_raw + kQBytes;
   __shared__ float red_m[kWarps][kMaxHeads];
   __shared__ float red_l[kWarps][kMaxHeads];
+  __shared__ uint16_t lmtab[2][256];                // Lloyd-Max codebooks of this head's widths
   const int split = blockIdx.x, h = blockIdx.y, batch = blockIdx.z;
   const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
   const int gid = lane >> 2, tig = lane & 3;
@@ -702,6 +728,13 @@ __global__ void __launch_bounds__(kThreads, RQ_DECODE_MIN_BLOCKS) decode_split_k
   dr.bV = bV;
   dr.kg = a.kg;
   dr.vg = a.vg;
+  const bool lmk = valid && a.kq == RQ_LLOYDMAX, lmv = valid && a.vq == RQ_LLOYDMAX;
+  for (int i = threadIdx.x; i < 256; i += kThreads) {
+    if (lmk && i < (1 << bK)) lmtab[0][i] = a.lm.lv[lm_offset(bK) + i];
+    if (lmv && i < (1 << bV)) lmtab[1][i] = a.lm.lv[lm_offset(bV) + i];
+  }
+  dr.lmK = lmk ? lmtab[0] : nullptr;               // read after the barriers of the q prologue
+  dr.lmV = lmv ? lmtab[1] : nullptr;
   dr.sK = 512 * (bK + 1);
   dr.sV = 512 * (bV + 1);
   dr.slot = max(dr.sK, dr.sV);
@@ -716,7 +749,7 @@ __global__ void __launch_bounds__(kThreads, RQ_DECODE_MIN_BLOCKS) decode_split_k
   ws.ring = smem_u32(ws.ring_ptr);
   ws.kwarp = kbase + static_cast<size_t>(blk_first) * dr.sK;
   ws.vwarp = vbase + static_cast<size_t>(blk_first) * dr.sV;
-  const int key = valid ? fast_key(bK, bV, a.kg, a.vg) : -1;
+  const int key = valid && a.kq != RQ_LLOYDMAX && a.vq != RQ_LLOYDMAX ? fast_key(bK, bV, a.kg, a.vg) : -1;
   ws.merged = a.g <= kMaxHeads / 2 && key >= 0;   // the compile-time KIVI paths only
   ws.mneg = ws.merged && gid >= kMaxHeads / 2 ? 0xBC00BC00u : 0x80008000u;
 
@@ -811,7 +844,8 @@ __global__ void __launch_bounds__(kThreads, RQ_DECODE_MIN_BLOCKS) decode_split_k
     // of bz[G / 2] for even G, rows gid + 8 for odd G)
     float rf[4];
 #pragma unroll
-    for (int x = 0; x < 4; ++x) rf[x] = __int_as_float((127 + 24 - fmt::exponent(bV, x)) << 23);   // 2^(24 - E)
+    for (int x = 0; x < 4; ++x)       // 2^(24 - E); 1 for codebook levels
+      rf[x] = lmv ? 1.0f : __int_as_float((127 + 24 - fmt::exponent(bV, x)) << 23);
 #pragma unroll
     for (int mt = 0; mt < 8; ++mt) {
       const int G = mt >> 1;
@@ -1156,8 +1190,8 @@ rq_status check_desc(const rq_cache_desc* desc) {
   if (desc->dtype != RQ_F16 && desc->dtype != RQ_BF16) return RQ_ERR_INVALID_ARG;
   for (int g : {desc->k_grouping, desc->v_grouping})
     if (g != RQ_PER_TOKEN && g != RQ_PER_CHANNEL) return RQ_ERR_INVALID_ARG;
-  for (int qz : {desc->k_quantizer, desc->v_quantizer})
-    if (qz != RQ_MINMAX && qz != RQ_ABSMAX) return RQ_ERR_INVALID_ARG;
+  if (!quantizers_ok(desc->k_quantizer, desc->k_grouping, desc->v_quantizer, desc->v_grouping))
+    return RQ_ERR_INVALID_ARG;
   if (desc->d != kD || desc->group != kG || desc->S % kTile != 0 || desc->S == 0)
     return RQ_ERR_SHAPE;
   if (desc->H_q % desc->H_kv != 0 || desc->H_q / desc->H_kv > kMaxHeads) return RQ_ERR_SHAPE;
@@ -1190,6 +1224,9 @@ void fill_args(DecodeArgs& a, const rq_cache_desc* desc, int32_t layer, const vo
   a.kg = desc->k_grouping;
   a.vg = desc->v_grouping;
   a.hadamard = desc->hadamard ? 1 : 0;
+  a.kq = desc->k_quantizer;
+  a.vq = desc->v_quantizer;
+  if (a.kq == RQ_LLOYDMAX || a.vq == RQ_LLOYDMAX) fill_lm_book(a.lm);
 }
 
 template <typename T>

@@ -8,6 +8,7 @@
 //   Eq. 1               min sum w_i D_i(b_i), sum b_i = B, bounds
 //   Alg. 2, Prop. 3     greedy max-heap on marginal gain, optimal for convex D
 //   Thm. 1, App. B.1    continuous reverse waterfilling with iterative clipping
+#include <algorithm>
 #include <cmath>
 #include <cstdint>
 #include <cstring>
@@ -132,6 +133,118 @@ rq_status dp_alloc(int32_t n, const std::vector<double>& w, const double* alpha,
 
 }  // namespace
 
+// ------------------------------------------------------ Lloyd-Max codebook ----
+// The 2^b-level Lloyd-Max quantizer of a unit Gaussian (App. F Table 8;
+// TurboQuant's scalar quantizer): levels that are the centroids of their
+// nearest-level cells. Only the upper half is solved (the codebook is
+// symmetric): Lloyd's iteration, then Newton's method on the fixed point
+// (tridiagonal Jacobian: the centroid of cell i moves with its two edges,
+// dC/dt = phi(t) (C - t) / p at the lower edge and phi(t) (t - C) / p at the
+// upper one, each edge the midpoint of two levels).
+namespace {
+
+double gauss_pdf(double t) { return std::exp(-0.5 * t * t) * 0.3989422804014327; }
+// P(X > t) for t >= 0 without cancellation
+double gauss_tail(double t) { return 0.5 * std::erfc(t * 0.7071067811865476); }
+
+// positive levels y[0] < ... < y[m-1] of the 2m-level codebook; the cells are
+// [0, t_1), [t_1, t_2), ..., [t_{m-1}, inf) with t_k = (y[k-1] + y[k]) / 2
+void lm_centroids(const std::vector<double>& y, std::vector<double>& c, std::vector<double>& ga,
+                  std::vector<double>& gc) {
+  const size_t m = y.size();
+  for (size_t k = 0; k < m; ++k) {
+    const double a = k == 0 ? 0.0 : 0.5 * (y[k - 1] + y[k]);
+    const bool last = k + 1 == m;
+    const double hi = last ? 0.0 : 0.5 * (y[k] + y[k + 1]);
+    const double p = gauss_tail(a) - (last ? 0.0 : gauss_tail(hi));
+    const double cc = (gauss_pdf(a) - (last ? 0.0 : gauss_pdf(hi))) / p;
+    c[k] = cc;
+    ga[k] = k == 0 ? 0.0 : gauss_pdf(a) * (cc - a) / p;      // the cell at 0 has a fixed edge
+    gc[k] = last ? 0.0 : gauss_pdf(hi) * (hi - cc) / p;
+  }
+}
+
+std::vector<double> lloyd_max_positive(int b) {
+  const size_t m = static_cast<size_t>(1) << (b - 1);
+  std::vector<double> y(m), c(m), ga(m), gc(m);
+  // start: equally spaced over [0, 4]
+  for (size_t k = 0; k < m; ++k) y[k] = 4.0 * (k + 0.5) / m;
+  for (int it = 0; it < 400; ++it) {
+    lm_centroids(y, c, ga, gc);
+    y = c;
+  }
+  std::vector<double> lo(m), di(m), up(m), r(m), cp(m), dp(m), x(m);
+  for (int it = 0; it < 60; ++it) {
+    lm_centroids(y, c, ga, gc);
+    for (size_t k = 0; k < m; ++k) {
+      r[k] = c[k] - y[k];                        // Newton: (I - dC) step = C - y
+      di[k] = 1.0 - 0.5 * (ga[k] + gc[k]);
+      lo[k] = k ? -0.5 * ga[k] : 0.0;
+      up[k] = k + 1 < m ? -0.5 * gc[k] : 0.0;
+    }
+    // at the centre cell the lower edge is 0 for every level set (symmetry)
+    if (m > 0) di[0] = 1.0 - 0.5 * gc[0];
+    cp[0] = m > 1 ? up[0] / di[0] : 0.0;
+    dp[0] = r[0] / di[0];
+    for (size_t k = 1; k < m; ++k) {
+      const double den = di[k] - lo[k] * cp[k - 1];
+      cp[k] = k + 1 < m ? up[k] / den : 0.0;
+      dp[k] = (r[k] - lo[k] * dp[k - 1]) / den;
+    }
+    x[m - 1] = dp[m - 1];
+    for (size_t k = m - 1; k-- > 0;) x[k] = dp[k] - cp[k] * x[k + 1];
+    double big = 0.0;
+    for (size_t k = 0; k < m; ++k) {
+      y[k] += x[k];
+      big = std::max(big, std::fabs(x[k]));
+    }
+    if (big < 1e-15) break;
+  }
+  return y;
+}
+
+// round to nearest fp16, ties to even (|v| within the fp16 normal range)
+uint16_t to_half_bits(double v) {
+  const uint16_t sign = v < 0 ? 0x8000u : 0u;
+  const double a = std::fabs(v);
+  if (a == 0.0) return sign;
+  int e = 0;
+  std::frexp(a, &e);                              // a = f 2^e, f in [0.5, 1)
+  int E = e - 1;                                  // a = g 2^E, g in [1, 2)
+  if (E < -14) E = -14;                           // subnormal range: fixed step 2^-24
+  double mant = std::nearbyint(std::ldexp(a, 10 - E));     // rounds half to even
+  if (mant >= 2048.0) {
+    mant /= 2.0;
+    ++E;
+  }
+  if (mant < 1024.0) return static_cast<uint16_t>(sign | static_cast<uint16_t>(mant));
+  return static_cast<uint16_t>(sign | ((E + 15) << 10) | (static_cast<uint16_t>(mant) - 1024u));
+}
+
+struct LMCodebooks {
+  uint16_t lv[8][256];
+  LMCodebooks() {
+    for (int b = 1; b <= 8; ++b) {
+      const std::vector<double> y = lloyd_max_positive(b);
+      const int m = 1 << (b - 1);
+      for (int k = 0; k < m; ++k) {
+        lv[b - 1][m + k] = to_half_bits(y[k]);
+        lv[b - 1][m - 1 - k] = to_half_bits(-y[k]);
+      }
+    }
+  }
+};
+
+}  // namespace
+
+namespace rq {
+// fp16 bit patterns of the 2^b levels, ascending (computed once, on first use)
+const uint16_t* lloydmax_levels(int b) {
+  static const LMCodebooks books;
+  return books.lv[b - 1];
+}
+}  // namespace rq
+
 extern "C" {
 
 const char* rq_status_string(rq_status s) {
@@ -148,6 +261,12 @@ const char* rq_status_string(rq_status s) {
 }
 
 int32_t rq_abi_version(void) { return RQ_ABI_VERSION; }
+
+rq_status rq_lloydmax_levels(int32_t b, uint16_t* levels) {
+  if (b < 1 || b > 8 || !levels) return RQ_ERR_INVALID_ARG;
+  std::memcpy(levels, rq::lloydmax_levels(b), sizeof(uint16_t) << b);
+  return RQ_OK;
+}
 
 rq_status rq_fit_distortion(int32_t n, const double* mse, int32_t b_lo, int32_t b_hi,
                             double r2_min, const int32_t* classes, double* alpha, double* beta,

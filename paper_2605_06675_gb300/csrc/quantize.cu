@@ -24,7 +24,19 @@ struct CalibSmem {
   uint16_t x16[kTile * (kD + 8)];       // raw tile (column mode), rows 272 bytes apart
   int8_t signs[kD];
   double red[kThreads / 32][8];
+  float lm_lev[512];                    // Lloyd-Max levels of every width (at lm_offset(b))
+  float lm_mid[512];                    // and the midpoints between them
 };
+
+// Lloyd-Max code at a width known only at run time (the sweep's loop)
+__device__ __forceinline__ int lm_code_rt(float v, float sf, const float* mid, int b) {
+  int c = 0;
+  for (int k = b - 1; k >= 0; --k) {
+    const int cand = c + (1 << k);
+    c = v >= __fmul_rn(mid[cand - 1], sf) ? cand : c;
+  }
+  return sf != 0.0f ? c : 0;
+}
 constexpr int kX16Stride = kD + 8;
 
 template <typename T>
@@ -87,13 +99,23 @@ __global__ void __launch_bounds__(kThreads) calib_sweep_kernel(CalibArgs a) {
   long long tile = blockIdx.x;
   if (tile >= a.ntiles) return;
   if (threadIdx.x < kD) sm.signs[threadIdx.x] = a.signs ? a.signs[threadIdx.x] : int8_t(1);
+  if (a.kq == RQ_LLOYDMAX || a.vq == RQ_LLOYDMAX) {
+    for (int i = threadIdx.x; i < 510; i += kThreads) {
+      sm.lm_lev[i] = __half2float(__ushort_as_half(a.lm.lv[i]));
+    }
+    __syncthreads();
+    for (int b = 1; b <= 8; ++b)
+      for (int i = threadIdx.x; i < (1 << b) - 1; i += kThreads)
+        sm.lm_mid[lm_offset(b) + i] =
+            __fmul_rn(__fadd_rn(sm.lm_lev[lm_offset(b) + i], sm.lm_lev[lm_offset(b) + i + 1]), 0.5f);
+  }
   __syncthreads();
   const bool had = a.hadamard != 0;
   const T* xbase = static_cast<const T*>(a.x);
   const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
 
   int grouping = (static_cast<int>(tile / a.ntile) & 1) ? a.vg : a.kg;
-  bool sym = ((static_cast<int>(tile / a.ntile) & 1) ? a.vq : a.kq) == RQ_ABSMAX;
+  int form = (static_cast<int>(tile / a.ntile) & 1) ? a.vq : a.kq;
   bool row_mode = grouping == RQ_PER_TOKEN || had;
   uint4 ld[4];
   calib_load<T>(xbase + tile * kTile * kD, row_mode, ld);
@@ -101,9 +123,9 @@ __global__ void __launch_bounds__(kThreads) calib_sweep_kernel(CalibArgs a) {
     float v[kG];
     calib_group_values<T>(ld, row_mode, grouping, had, sm, x32, v);
     const long long next = tile + stride;
-    const bool sym_now = sym;
+    const int form_now = form;
     if (next < a.ntiles) {
-      sym = ((static_cast<int>(next / a.ntile) & 1) ? a.vq : a.kq) == RQ_ABSMAX;
+      form = (static_cast<int>(next / a.ntile) & 1) ? a.vq : a.kq;
       grouping = (static_cast<int>(next / a.ntile) & 1) ? a.vg : a.kg;
       row_mode = grouping == RQ_PER_TOKEN || had;
       calib_load<T>(xbase + next * kTile * kD, row_mode, ld);
@@ -114,9 +136,35 @@ __global__ void __launch_bounds__(kThreads) calib_sweep_kernel(CalibArgs a) {
     mn = __fadd_rn(mn, 0.0f);
     mx = __fadd_rn(mx, 0.0f);
     double acc[8];
+    if (form_now == RQ_LLOYDMAX) {
+      // the group's RMS scale (as the quantizer computes it), then every width
+      const float s2s = __fadd_rn(sumsq16(v), sumsq16(v + 16));
+      float sf = __half2float(__float2half_rn(__fsqrt_rn(__fmul_rn(s2s, 0.03125f))));
+      if (!finite || !isfinite(sf)) {
+        set_status(a.status, RQ_STATUS_NUMERIC);
+        sf = 0.0f;
+      }
+      float vz[kG];
+#pragma unroll
+      for (int i = 0; i < kG; ++i) vz[i] = __fadd_rn(v[i], 0.0f);
+#pragma unroll 1
+      for (int b = 1; b <= 8; ++b) {
+        const float* mid = sm.lm_mid + lm_offset(b);
+        const float* lev = sm.lm_lev + lm_offset(b);
+        float2 s2 = make_float2(0.0f, 0.0f);
+#pragma unroll
+        for (int i = 0; i < kG; i += 2) {
+          const float x0 = __fmul_rn(lev[lm_code_rt(vz[i], sf, mid, b)], sf);
+          const float x1 = __fmul_rn(lev[lm_code_rt(vz[i + 1], sf, mid, b)], sf);
+          const float2 e = __fadd2_rn(make_float2(v[i], v[i + 1]), make_float2(-x0, -x1));
+          s2 = __ffma2_rn(e, e, s2);
+        }
+        acc[b - 1] = static_cast<double>(s2.x) + static_cast<double>(s2.y);
+      }
+    } else {
 #pragma unroll
     for (int b = 1; b <= 8; ++b) {
-      const GroupParams g = group_params(mn, mx, finite, b, sym_now);
+      const GroupParams g = group_params(mn, mx, finite, b, form_now == RQ_ABSMAX);
       if (b == 1 && g.bad) set_status(a.status, RQ_STATUS_NUMERIC);
       const float2 sf = make_float2(g.sf, g.sf), zf = make_float2(g.zf, g.zf);
       float2 s2 = make_float2(0.0f, 0.0f);
@@ -130,6 +178,7 @@ __global__ void __launch_bounds__(kThreads) calib_sweep_kernel(CalibArgs a) {
         s2 = __ffma2_rn(e, e, s2);
       }
       acc[b - 1] = static_cast<double>(s2.x) + static_cast<double>(s2.y);
+    }
     }
 #pragma unroll
     for (int k = 0; k < 8; ++k) {
@@ -179,8 +228,8 @@ extern "C" rq_status rq_quantize_pack(const rq_cache_desc* desc, int32_t layer, 
   if (desc->dtype != RQ_F16 && desc->dtype != RQ_BF16) return RQ_ERR_INVALID_ARG;
   for (int g : {desc->k_grouping, desc->v_grouping})
     if (g != RQ_PER_TOKEN && g != RQ_PER_CHANNEL) return RQ_ERR_INVALID_ARG;
-  for (int qz : {desc->k_quantizer, desc->v_quantizer})
-    if (qz != RQ_MINMAX && qz != RQ_ABSMAX) return RQ_ERR_INVALID_ARG;
+  if (!quantizers_ok(desc->k_quantizer, desc->k_grouping, desc->v_quantizer, desc->v_grouping))
+    return RQ_ERR_INVALID_ARG;
   if (desc->d != kD || desc->group != kG || desc->S % kTile != 0) return RQ_ERR_SHAPE;
   if (!aligned16(k) || !aligned16(v) || !aligned16(packed)) return RQ_ERR_ALIGNMENT;
   QuantArgs a;
@@ -200,6 +249,7 @@ extern "C" rq_status rq_quantize_pack(const rq_cache_desc* desc, int32_t layer, 
   a.vg = desc->v_grouping;
   a.kq = desc->k_quantizer;
   a.vq = desc->v_quantizer;
+  if (a.kq == RQ_LLOYDMAX || a.vq == RQ_LLOYDMAX) fill_lm_book(a.lm);
   a.hadamard = desc->hadamard ? 1 : 0;
   a.j_dst0 = 0;
   a.ntiles = static_cast<long long>(desc->B) * desc->H_kv * 2 * a.nblk;
@@ -227,8 +277,7 @@ extern "C" rq_status rq_calibrate_distortion(const void* x, int32_t dtype, int32
   if (dtype != RQ_F16 && dtype != RQ_BF16) return RQ_ERR_INVALID_ARG;
   for (int g : {k_grouping, v_grouping})
     if (g != RQ_PER_TOKEN && g != RQ_PER_CHANNEL) return RQ_ERR_INVALID_ARG;
-  for (int qz : {k_quantizer, v_quantizer})
-    if (qz != RQ_MINMAX && qz != RQ_ABSMAX) return RQ_ERR_INVALID_ARG;
+  if (!quantizers_ok(k_quantizer, k_grouping, v_quantizer, v_grouping)) return RQ_ERR_INVALID_ARG;
   if (T % kTile != 0) return RQ_ERR_SHAPE;
   if (!aligned16(x) || !aligned16(ws) || (reinterpret_cast<uintptr_t>(mse_dev) & 7u))
     return RQ_ERR_ALIGNMENT;
@@ -245,6 +294,7 @@ extern "C" rq_status rq_calibrate_distortion(const void* x, int32_t dtype, int32
   a.vg = v_grouping;
   a.kq = k_quantizer;
   a.vq = v_quantizer;
+  if (a.kq == RQ_LLOYDMAX || a.vq == RQ_LLOYDMAX) fill_lm_book(a.lm);
   a.hadamard = hadamard ? 1 : 0;
   a.ntiles = static_cast<long long>(n) * a.ntile;
   cudaStream_t st = static_cast<cudaStream_t>(stream);
@@ -300,8 +350,8 @@ extern "C" rq_status rq_append(const rq_cache_desc* desc, int32_t layer, int32_t
   if (desc->dtype != RQ_F16 && desc->dtype != RQ_BF16) return RQ_ERR_INVALID_ARG;
   for (int g : {desc->k_grouping, desc->v_grouping})
     if (g != RQ_PER_TOKEN && g != RQ_PER_CHANNEL) return RQ_ERR_INVALID_ARG;
-  for (int qz : {desc->k_quantizer, desc->v_quantizer})
-    if (qz != RQ_MINMAX && qz != RQ_ABSMAX) return RQ_ERR_INVALID_ARG;
+  if (!quantizers_ok(desc->k_quantizer, desc->k_grouping, desc->v_quantizer, desc->v_grouping))
+    return RQ_ERR_INVALID_ARG;
   if (desc->d != kD || desc->group != kG || desc->S % kTile != 0) return RQ_ERR_SHAPE;
   if (!aligned16(k_new) || !aligned16(v_new) || !aligned16(residual) || !aligned16(packed))
     return RQ_ERR_ALIGNMENT;
@@ -335,6 +385,7 @@ extern "C" rq_status rq_append(const rq_cache_desc* desc, int32_t layer, int32_t
   a.vg = desc->v_grouping;
   a.kq = desc->k_quantizer;
   a.vq = desc->v_quantizer;
+  if (a.kq == RQ_LLOYDMAX || a.vq == RQ_LLOYDMAX) fill_lm_book(a.lm);
   a.hadamard = desc->hadamard ? 1 : 0;
   a.j_dst0 = pos / kTile;
   a.ntiles = static_cast<long long>(desc->B) * desc->H_kv * 2;

@@ -46,6 +46,7 @@ struct QuantArgs {
   int kq, vq;                // rq_quantizer of keys / values
   int j_dst0;                // packed block index of each stream's first tile
   long long ntiles;
+  LMBook lm;                 // RQ_LLOYDMAX codebooks
 };
 
 struct CalibArgs {
@@ -56,6 +57,7 @@ struct CalibArgs {
   int n, T, ntile, kg, vg, hadamard;
   int kq, vq;                // rq_quantizer of keys / values
   long long ntiles;
+  LMBook lm;                 // RQ_LLOYDMAX codebooks
 };
 
 // one launcher per quantize_pack_kernel instance (quantize_k_*.cu)
@@ -77,7 +79,9 @@ constexpr int kRowBytes = 320;
 constexpr int kTileBytes = kTile * kRowBytes;
 constexpr int kX32S = kD + 4;           // rotated fp32 row (floats)
 
-enum { kModeKC = 0, kModeKT = 1, kModeVT = 2, kModeVC = 3 };
+// layouts: keys per channel / per token, values per token / per channel, and
+// the Lloyd-Max codebook quantizer on per-token keys / values
+enum { kModeKC = 0, kModeKT = 1, kModeVT = 2, kModeVC = 3, kModeKTL = 4, kModeVTL = 5 };
 
 // 16-byte multiple: the rotated fp32 tile follows it (float4 accesses)
 struct alignas(16) QSmem {
@@ -86,6 +90,7 @@ struct alignas(16) QSmem {
   float inv[kD];                // 1 / scale (0 for a group without codes)
   uint2 xchg[kThreads];         // per-channel min/max of half the tokens (rotated tiles)
   float top;                    // magic + the largest code of the tile's quantizer
+  float lm_mid[256];            // Lloyd-Max: midpoints of the tile width's levels
   int8_t signs[kD];
 };
 
@@ -185,6 +190,9 @@ __device__ __forceinline__ void issue_tile(uint8_t* buf, const void* src) {
 }
 
 // ------------------------------------------------------------- phase 1 ----
+// phase 1's grouping argument: RQ_PER_TOKEN, RQ_PER_CHANNEL, or per-token
+// Lloyd-Max groups
+constexpr int kGroupingLM = 2;
 
 struct GroupOut {
   bool slow, bad;
@@ -241,6 +249,71 @@ __device__ __forceinline__ GroupOut finish_group(int kind, int grouping, int t, 
   const float uM = __fmaf_rn(__fsub_rn(mx, g.zf), g.inv, kRoundMagic);
   o.slow = um < kRoundMagic || uM > kRoundMagic + g.cmax;
   return o;
+}
+
+// Lloyd-Max group (per-token groups only): scale = fp16(sqrt(s2 / 32)) of the
+// fp32 sum of squares s2 = (v0^2 + ... + v15^2) + (v16^2 + ... + v31^2), each
+// half summed in order; zero = +0. The table gets sf (codes come from the
+// thresholds mid * sf). No clamping variant is needed.
+__device__ __forceinline__ float sumsq16(const float* v) {
+  float s = 0.0f;
+#pragma unroll
+  for (int i = 0; i < 16; ++i) s = __fadd_rn(s, __fmul_rn(v[i], v[i]));
+  return s;
+}
+
+__device__ __forceinline__ GroupOut finish_group_lm(int kind, int t, int G, const float (&v)[kG],
+                                                    bool finite, uint8_t* meta, QSmem& sm) {
+  const float s2 = __fadd_rn(sumsq16(v), sumsq16(v + 16));
+  const float rms = __fsqrt_rn(__fmul_rn(s2, 0.03125f));
+  __half scale = __float2half_rn(rms);
+  float sf = __half2float(scale);
+  GroupOut o;
+  o.bad = !finite || !isfinite(sf);
+  o.slow = false;
+  if (o.bad) {
+    scale = __float2half_rn(0.0f);
+    sf = 0.0f;
+  }
+  const uint32_t sb = __half_as_ushort(scale);
+  uint16_t* m16 = reinterpret_cast<uint16_t*>(meta);
+  uint32_t* m32 = reinterpret_cast<uint32_t*>(meta);
+  if (kind == 0) {
+    m32[16 * (t & 7) + 4 * G + (t >> 3)] = sb;            // (scale, zero = +0)
+  } else {
+    const int Q = t >> 1;
+    const int zw = 64 + 32 * (Q >> 3) + 8 * (Q & 3) + 4 * (G >> 1) + 2 * ((Q >> 2) & 1) + (G & 1);
+    m16[2 * (4 * Q + G) + (t & 1)] = static_cast<uint16_t>(sb);
+    m16[2 * zw + (t & 1)] = 0;
+  }
+  sm.nz[32 * G + t] = sf;
+  return o;
+}
+
+// per-token Lloyd-Max groups on the raw tile: thread 4 t + G, values in order
+template <typename T>
+__device__ __forceinline__ GroupOut phase1_rows_lm(const uint8_t* tile, int kind, uint8_t* meta,
+                                                   QSmem& sm) {
+  const int tau = threadIdx.x, t = tau >> 2, G = tau & 3;
+  const uint8_t* row = tile + t * kRowBytes + 64 * G;
+  float v[kG];
+#pragma unroll
+  for (int i = 0; i < 4; ++i) {
+    const uint4 u = *reinterpret_cast<const uint4*>(row + 16 * i);
+    const uint32_t w[4] = {u.x, u.y, u.z, u.w};
+#pragma unroll
+    for (int e = 0; e < 4; ++e) {
+      v[8 * i + 2 * e] = lo_f32<T>(w[e]);
+      v[8 * i + 2 * e + 1] = hi_f32<T>(w[e]);
+    }
+  }
+  bool finite = true;
+#pragma unroll
+  for (int i = 0; i < kG; ++i) {
+    finite = finite && isfinite(v[i]);
+    v[i] = __fadd_rn(v[i], 0.0f);
+  }
+  return finish_group_lm(kind, t, G, v, finite, meta, sm);
 }
 
 // Per-channel groups on the raw tile: thread 2p + hv (channel pair p, token
@@ -389,6 +462,15 @@ __device__ __forceinline__ GroupOut phase1_rotated(const uint8_t* tile, float* x
     return finish_group(kind, RQ_PER_TOKEN, t, G, 0, __fadd_rn(mn, 0.0f), __fadd_rn(mx, 0.0f),
                         finite, q, meta, sm);
   }
+  if (grouping == kGroupingLM) {            // Lloyd-Max, per token, on the rotated values
+    bool finite = true;
+#pragma unroll
+    for (int i = 0; i < kG; ++i) {
+      finite = finite && isfinite(v[i]);
+      v[i] = __fadd_rn(v[i], 0.0f);
+    }
+    return finish_group_lm(kind, t, G, v, finite, meta, sm);
+  }
   __syncthreads();
   const int p = tau & 63, hv = tau >> 6;
   const float* col = x32 + 16 * hv * kX32S + 2 * p;
@@ -412,10 +494,11 @@ __device__ __forceinline__ GroupOut phase1_rotated(const uint8_t* tile, float* x
 }
 
 template <typename T, bool HAD, bool SYM>
-__device__ __noinline__ GroupOut phase1(const uint8_t* tile, float* x32, int kind, int grouping,
-                                           int b, uint8_t* meta, QSmem& sm) {
+__device__ __forceinline__ GroupOut phase1(const uint8_t* tile, float* x32, int kind, int grouping,
+                                              int b, uint8_t* meta, QSmem& sm) {
   const TileQ<SYM> q{b};
   if constexpr (HAD) return phase1_rotated<T>(tile, x32, kind, grouping, q, meta, sm);
+  else if (grouping == kGroupingLM) return phase1_rows_lm<T>(tile, kind, meta, sm);
   else if (grouping == RQ_PER_CHANNEL) return phase1_cols<T>(tile, kind, q, meta, sm);
   else return phase1_rows<T>(tile, kind, q, meta, sm);
 }
@@ -475,6 +558,26 @@ __device__ __forceinline__ void emit(uint32_t (&uw)[B], int x, int y, float2 v, 
   fmt::place<B>(uw, x, y, __byte_perm(__float_as_uint(q.x), __float_as_uint(q.y), 0x5410u));
 }
 
+// Lloyd-Max code: the number of thresholds fp32(mid_i * sf), i = 0..2^B - 2,
+// at or below v (binary search over the ascending thresholds); 0 for a group
+// without a scale
+template <int B>
+__device__ __forceinline__ uint32_t lm_code(float v, float sf, const float* mid) {
+  int c = 0;
+#pragma unroll
+  for (int k = B - 1; k >= 0; --k) {
+    const int cand = c + (1 << k);
+    c = v >= __fmul_rn(mid[cand - 1], sf) ? cand : c;
+  }
+  return sf != 0.0f ? static_cast<uint32_t>(c) : 0u;
+}
+
+template <int B>
+__device__ __forceinline__ void emit_lm(uint32_t (&uw)[B], int x, int y, float2 v, float2 sf,
+                                        const float* mid) {
+  fmt::place<B>(uw, x, y, lm_code<B>(v.x, sf.x, mid) | (lm_code<B>(v.y, sf.y, mid) << 16));
+}
+
 // Thread -> (lane gid/tig of the packed format, unit u). K: warp = unit,
 // lane = format lane. V: a half warp is (gid 0..7) x (two units), so the
 // 8-byte reads of one token row hit 16 distinct bank pairs.
@@ -483,7 +586,7 @@ __device__ __forceinline__ void phase2(const uint8_t* tile, const float* x32, co
                                        uint32_t* blk) {
   const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
   int gid, tig, u;
-  if (MODE == kModeKC || MODE == kModeKT) {
+  if (MODE == kModeKC || MODE == kModeKT || MODE == kModeKTL) {
     gid = lane >> 2;
     tig = lane & 3;
     u = warp;
@@ -514,6 +617,18 @@ __device__ __forceinline__ void phase2(const uint8_t* tile, const float* x32, co
 #pragma unroll
       for (int x = 0; x < 4; ++x) emit<B, CLAMP>(uw, x, y, v[x], nz[x], iv[x]);
     }
+  } else if constexpr (MODE == kModeKTL) {
+    // as kModeKT, codes from the Lloyd-Max thresholds (the table holds sf)
+    const int c = 32 * u + 8 * tig;
+#pragma unroll
+    for (int x = 0; x < 4; ++x) {
+      const int t = 8 * x + gid;
+      const float sf = sm.nz[32 * u + t];
+      float2 v[4];
+      load_pairs<T, F32>(tile, x32, t, c, v);
+#pragma unroll
+      for (int y = 0; y < 4; ++y) emit_lm<B>(uw, x, y, v[y], make_float2(sf, sf), sm.lm_mid);
+    }
   } else if constexpr (MODE == kModeKT) {
     // token 8x + gid, channels 32u + 8tig + 2y + h; group = (token, G = u)
     const int c = 32 * u + 8 * tig;
@@ -540,7 +655,11 @@ __device__ __forceinline__ void phase2(const uint8_t* tile, const float* x32, co
       float a[4], b[4];
       load_quad<T, F32>(tile, x32, t, c, a);
       load_quad<T, F32>(tile, x32, t + 1, c, b);
-      if constexpr (MODE == kModeVT) {
+      if constexpr (MODE == kModeVTL) {
+        const float2 sf = *reinterpret_cast<const float2*>(sm.nz + 32 * u + t);
+#pragma unroll
+        for (int x = 0; x < 4; ++x) emit_lm<B>(uw, x, y, make_float2(a[x], b[x]), sf, sm.lm_mid);
+      } else if constexpr (MODE == kModeVT) {
         const float2 nz = *reinterpret_cast<const float2*>(sm.nz + 32 * u + t);
         const float2 iv = *reinterpret_cast<const float2*>(sm.inv + 32 * u + t);
 #pragma unroll
@@ -606,9 +725,10 @@ struct Segment {
   int n;
 };
 
-__host__ __device__ constexpr int mode_of(int kind, int grouping) {
-  return kind == 0 ? (grouping == RQ_PER_CHANNEL ? kModeKC : kModeKT)
-                   : (grouping == RQ_PER_TOKEN ? kModeVT : kModeVC);
+__host__ __device__ constexpr int mode_of(int kind, int grouping, bool lloydmax) {
+  return lloydmax ? (kind == 0 ? kModeKTL : kModeVTL)
+                  : kind == 0 ? (grouping == RQ_PER_CHANNEL ? kModeKC : kModeKT)
+                              : (grouping == RQ_PER_TOKEN ? kModeVT : kModeVC);
 }
 
 // One stream's tiles with the layout (MODE) and width (B) fixed at compile
@@ -620,8 +740,10 @@ __device__ __forceinline__ int run_segment(const QuantArgs& a, QSmem& sm, float*
                                            const Segment& seg, int it) {
   constexpr int kTileSrcBytes = kTile * kD * static_cast<int>(sizeof(T));
   constexpr int kBlkBytes = 512 * (B + 1);
-  constexpr int kind = (MODE == kModeKC || MODE == kModeKT) ? 0 : 1;
-  constexpr int grouping = (MODE == kModeKC || MODE == kModeVC) ? RQ_PER_CHANNEL : RQ_PER_TOKEN;
+  constexpr int kind = (MODE == kModeKC || MODE == kModeKT || MODE == kModeKTL) ? 0 : 1;
+  constexpr bool LM = MODE == kModeKTL || MODE == kModeVTL;
+  constexpr int grouping = LM ? kGroupingLM
+                              : (MODE == kModeKC || MODE == kModeVC) ? RQ_PER_CHANNEL : RQ_PER_TOKEN;
   const bool sym = (kind ? a.vq : a.kq) == RQ_ABSMAX;      // kernel parameters, no register
   for (int k = 0; k < seg.n; ++k, ++it) {
     const uint8_t* buf = sm.tile[it & 1];
@@ -634,6 +756,13 @@ __device__ __forceinline__ int run_segment(const QuantArgs& a, QSmem& sm, float*
     uint8_t* meta = blk + 512 * B;
     if (threadIdx.x == 0)        // read by phase 2, after the barrier below
       sm.top = kRoundMagic + static_cast<float>(sym ? (1 << B) - 2 : (1 << B) - 1);
+    if constexpr (LM) {          // the thresholds' midpoints, exact in fp32
+      for (int i = threadIdx.x; i < (1 << B) - 1; i += kThreads) {
+        const float l0 = __half2float(__ushort_as_half(a.lm.lv[lm_offset(B) + i]));
+        const float l1 = __half2float(__ushort_as_half(a.lm.lv[lm_offset(B) + i + 1]));
+        sm.lm_mid[i] = __fmul_rn(__fadd_rn(l0, l1), 0.5f);
+      }
+    }
     GroupOut g;
     if (sym) g = phase1<T, HAD, true>(buf, x32, kind, grouping, B, meta, sm);
     else g = phase1<T, HAD, false>(buf, x32, kind, grouping, B, meta, sm);
@@ -709,10 +838,13 @@ __global__ void __launch_bounds__(kThreads, RQ_QUANT_MIN_BLOCKS) quantize_pack_k
     if (b < 1 || b > 8) {
       it = skip_segment(a, sm, seg, it, kTileSrcBytes);
     } else {
-      switch (mode_of(cur.kind, cur.grouping)) {
+      const bool lm = (cur.kind ? a.vq : a.kq) == RQ_LLOYDMAX;
+      switch (mode_of(cur.kind, cur.grouping, lm)) {
         case kModeKC: it = run_segment_b<T, HAD, kModeKC>(a, sm, x32, seg, it, b); break;
         case kModeKT: it = run_segment_b<T, HAD, kModeKT>(a, sm, x32, seg, it, b); break;
         case kModeVT: it = run_segment_b<T, HAD, kModeVT>(a, sm, x32, seg, it, b); break;
+        case kModeKTL: it = run_segment_b<T, HAD, kModeKTL>(a, sm, x32, seg, it, b); break;
+        case kModeVTL: it = run_segment_b<T, HAD, kModeVTL>(a, sm, x32, seg, it, b); break;
         default: it = run_segment_b<T, HAD, kModeVC>(a, sm, x32, seg, it, b); break;
       }
     }

@@ -28,6 +28,31 @@ inline rq_status launch_status() {
   return cudaGetLastError() == cudaSuccess ? RQ_OK : RQ_ERR_CUDA;
 }
 
+// The Lloyd-Max codebooks (RQ_LLOYDMAX) of every width, passed to the kernels
+// by value: fp16 bit patterns, ascending, width b at lv[2^b - 2 ..].
+struct LMBook {
+  uint16_t lv[510];
+};
+__host__ __device__ constexpr int lm_offset(int b) { return (1 << b) - 2; }
+// the library's codebook (host.cpp), and one filled LMBook
+const uint16_t* lloydmax_levels(int b);
+// a quantizer choice of keys and values is supported: min-max and absmax with
+// either grouping, Lloyd-Max with per-token groups
+inline bool quantizers_ok(int kq, int kg, int vq, int vg) {
+  for (int i = 0; i < 2; ++i) {
+    const int q = i ? vq : kq, g = i ? vg : kg;
+    if (q != RQ_MINMAX && q != RQ_ABSMAX && q != RQ_LLOYDMAX) return false;
+    if (q == RQ_LLOYDMAX && g != RQ_PER_TOKEN) return false;
+  }
+  return true;
+}
+inline void fill_lm_book(LMBook& book) {
+  for (int b = 1; b <= 8; ++b) {
+    const uint16_t* lv = lloydmax_levels(b);
+    for (int i = 0; i < (1 << b); ++i) book.lv[lm_offset(b) + i] = lv[i];
+  }
+}
+
 // ---------------------------------------------------------- device side ----
 
 template <typename T>

@@ -18,7 +18,7 @@ LIB_PATH = os.path.join(_HERE, "librq.so")
 RQ_OK = 0
 RQ_F16, RQ_BF16 = 0, 1
 RQ_PER_TOKEN, RQ_PER_CHANNEL = 0, 1
-RQ_MINMAX, RQ_ABSMAX = 0, 1
+RQ_MINMAX, RQ_ABSMAX, RQ_LLOYDMAX = 0, 1, 2
 RQ_CAP_5X = 1
 RQ_STATUS_NUMERIC = 1
 RQ_STATUS_BAD_BITS = 2
@@ -30,7 +30,7 @@ STATUS_NAMES = {0: "RQ_OK", 1: "RQ_ERR_INVALID_ARG", 2: "RQ_ERR_INFEASIBLE", 3: 
                 4: "RQ_ERR_ALIGNMENT", 5: "RQ_ERR_WORKSPACE", 6: "RQ_ERR_CUDA"}
 
 # every symbol include/rq.h declares
-EXPORTS = ["rq_status_string", "rq_abi_version", "rq_fit_distortion", "rq_alloc",
+EXPORTS = ["rq_status_string", "rq_abi_version", "rq_lloydmax_levels", "rq_fit_distortion", "rq_alloc",
            "rq_alloc_continuous", "rq_packed_layout", "rq_calibrate_workspace_bytes",
            "rq_calibrate_distortion", "rq_quantize_pack", "rq_decode_workspace_bytes",
            "rq_decode_attention", "rq_decode_attention_static", "rq_residual_bytes",
@@ -66,6 +66,7 @@ def lib() -> ctypes.CDLL:
         sig = {
             "rq_status_string": ([_I], ctypes.c_char_p),
             "rq_abi_version": ([], _I),
+            "rq_lloydmax_levels": ([_I, _P], _I),
             "rq_fit_distortion": ([_I, _P, _I, _I, _D, _P, _P, _P, _P], _I),
             "rq_alloc": ([_I, _P, _P, _P, _D, _U, _U, _P, _P], _I),
             "rq_alloc_continuous": ([_I, _P, _P, _P, _D, _D, _D, _P], _I),
@@ -147,6 +148,13 @@ def rq_status_string(status: int) -> str:
 
 def rq_abi_version() -> int:
     return lib().rq_abi_version()
+
+
+def rq_lloydmax_levels(b: int) -> np.ndarray:
+    """The library's fp16 Lloyd-Max codebook at b bits (2^b levels, ascending)."""
+    out = np.zeros(2 ** b, dtype=np.uint16)
+    _check("rq_lloydmax_levels", lib().rq_lloydmax_levels(b, _hp(out)))
+    return out.view(np.float16)
 
 
 def rq_fit_distortion(mse, b_lo=2, b_hi=6, r2_min=0.96, classes=None):

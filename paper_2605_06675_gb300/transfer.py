@@ -19,6 +19,8 @@ Sec. 3.4 "K/V separation"):
             values per token min-max
   rtn       keys and values per token absmax (Table 16)
   quarot    Hadamard rotation, then per token absmax (Sec. 4.1)
+  turboquant Hadamard rotation, then the per-token Lloyd-Max codebook
+            quantizer (App. F Table 8, App. W)
 The "uniform" column gives every key ceil(avg_bits) and every value
 floor(avg_bits) bits (one width per kind; the same width when avg_bits is
 an integer).
@@ -43,6 +45,8 @@ FAMILIES = {
                 k_quantizer=rq.RQ_ABSMAX, v_quantizer=rq.RQ_ABSMAX),
     "quarot": dict(k_grouping=PER_TOKEN, v_grouping=PER_TOKEN, hadamard=True,
                    k_quantizer=rq.RQ_ABSMAX, v_quantizer=rq.RQ_ABSMAX),
+    "turboquant": dict(k_grouping=PER_TOKEN, v_grouping=PER_TOKEN, hadamard=True,
+                       k_quantizer=rq.RQ_LLOYDMAX, v_quantizer=rq.RQ_LLOYDMAX),
 }
 
 
@@ -99,19 +103,19 @@ def format_matrix(res: dict) -> str:
     """The matrix as text: rows = allocation's family, columns = quantizer,
     entries J / J(matched)."""
     names = res["names"]
-    head = "alloc \\ quant".ljust(14) + "".join(n.rjust(10) for n in names)
+    head = "alloc \\ quant".ljust(14) + "".join(n.rjust(11) for n in names)
     lines = [head]
     for a in names:
         lines.append(a.ljust(14) + "".join(
-            f"{res['J'][a][b] / res['J'][b][b]:10.3f}" for b in names))
+            f"{res['J'][a][b] / res['J'][b][b]:11.3f}" for b in names))
     lines.append("uniform".ljust(14) + "".join(
-        f"{res['uniform'][b] / res['J'][b][b]:10.3f}" for b in names))
+        f"{res['uniform'][b] / res['J'][b][b]:11.3f}" for b in names))
     lines.append("mean beta K".ljust(14) + "".join(
-        f"{float(np.mean(res['beta'][b][0::2])):10.2f}" for b in names))
+        f"{float(np.mean(res['beta'][b][0::2])):11.2f}" for b in names))
     lines.append("mean beta V".ljust(14) + "".join(
-        f"{float(np.mean(res['beta'][b][1::2])):10.2f}" for b in names))
+        f"{float(np.mean(res['beta'][b][1::2])):11.2f}" for b in names))
     lines.append("mean bits K/V".ljust(14) + "".join(
-        f"{float(np.mean(res['bits'][b][0::2])):5.2f}/{float(np.mean(res['bits'][b][1::2])):4.2f}"
+        f"{float(np.mean(res['bits'][b][0::2])):6.2f}/{float(np.mean(res['bits'][b][1::2])):4.2f}"
         for b in names))
     return "\n".join(lines)
 

@@ -176,3 +176,15 @@ def test_scale_division_method_is_exact(tmp_path):
     subprocess.run([cc, "-O2", "-ffp-contract=off", "-o", str(exe), str(src), "-lm"], check=True)
     out = subprocess.run([str(exe)], capture_output=True, text=True, check=True).stdout
     assert out.strip() == "0"
+
+
+def test_lloydmax_codebook_matches_the_oracle(rq):
+    # the library solves the codebook on its own (C++, upper half, Newton);
+    # its fp16 levels must equal the oracle's at every width
+    from oracle import lloydmax
+    for b in range(1, 9):
+        got = rq.rq_lloydmax_levels(b)
+        want = lloydmax.levels_f16(b)
+        assert np.array_equal(got.view(np.uint16), want.view(np.uint16)), b
+    with pytest.raises(rq.RQError):
+        rq.rq_lloydmax_levels(9)
