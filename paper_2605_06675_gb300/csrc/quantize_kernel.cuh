@@ -493,11 +493,26 @@ __device__ __forceinline__ GroupOut phase1_rotated(const uint8_t* tile, float* x
                       __fadd_rn(mx, 0.0f), finite, q, meta, sm);
 }
 
+// The rotated phase 1 is large (the FWHT unrolled over 32 values) and runs
+// once per tile: one out-of-line copy per (dtype, quantizer form), shared by
+// every layout and width, keeps the kernel's code within the instruction
+// cache. Shared memory is re-derived from the dynamic-shared symbol so its
+// accesses stay shared-memory instructions.
+template <typename T, bool SYM>
+__device__ __noinline__ GroupOut phase1_rot_call(int buf, int kind, int grouping, int b,
+                                                 uint8_t* meta) {
+  extern __shared__ __align__(16) unsigned char smem_raw[];
+  QSmem& sm = *reinterpret_cast<QSmem*>(smem_raw);
+  float* x32 = reinterpret_cast<float*>(smem_raw + sizeof(QSmem));
+  const TileQ<SYM> q{b};
+  return phase1_rotated<T>(sm.tile[buf], x32, kind, grouping, q, meta, sm);
+}
+
 template <typename T, bool HAD, bool SYM>
 __device__ __forceinline__ GroupOut phase1(const uint8_t* tile, float* x32, int kind, int grouping,
-                                              int b, uint8_t* meta, QSmem& sm) {
+                                              int b, uint8_t* meta, QSmem& sm, int buf) {
   const TileQ<SYM> q{b};
-  if constexpr (HAD) return phase1_rotated<T>(tile, x32, kind, grouping, q, meta, sm);
+  if constexpr (HAD) return phase1_rot_call<T, SYM>(buf, kind, grouping, b, meta);
   else if (grouping == kGroupingLM) return phase1_rows_lm<T>(tile, kind, meta, sm);
   else if (grouping == RQ_PER_CHANNEL) return phase1_cols<T>(tile, kind, q, meta, sm);
   else return phase1_rows<T>(tile, kind, q, meta, sm);
@@ -693,6 +708,17 @@ __device__ __forceinline__ void phase2(const uint8_t* tile, const float* x32, co
   }
 }
 
+// The clamping variant of phase 2 (rare: degenerate groups, codes that could
+// leave their range): out of line, so each layout and width carries one
+// inlined phase 2 only.
+template <int MODE, typename T, int B, bool F32>
+__device__ __noinline__ void phase2_clamp_call(int buf, uint32_t* blk) {
+  extern __shared__ __align__(16) unsigned char smem_raw[];
+  const QSmem& sm = *reinterpret_cast<const QSmem*>(smem_raw);
+  const float* x32 = F32 ? reinterpret_cast<const float*>(smem_raw + sizeof(QSmem)) : nullptr;
+  phase2<MODE, T, B, true, F32>(sm.tile[buf], x32, sm, blk);
+}
+
 // Per-stream constants (recomputed when the walk crosses into a stream).
 struct StreamState {
   const uint8_t* src;     // first tile of the stream (raw values)
@@ -764,12 +790,12 @@ __device__ __forceinline__ int run_segment(const QuantArgs& a, QSmem& sm, float*
       }
     }
     GroupOut g;
-    if (sym) g = phase1<T, HAD, true>(buf, x32, kind, grouping, B, meta, sm);
-    else g = phase1<T, HAD, false>(buf, x32, kind, grouping, B, meta, sm);
+    if (sym) g = phase1<T, HAD, true>(buf, x32, kind, grouping, B, meta, sm, it & 1);
+    else g = phase1<T, HAD, false>(buf, x32, kind, grouping, B, meta, sm, it & 1);
     if (g.bad) set_status(a.status, RQ_STATUS_NUMERIC);
     const bool slow = __syncthreads_or(g.slow) != 0;
     uint32_t* blk32 = reinterpret_cast<uint32_t*>(blk);
-    if (slow) phase2<MODE, T, B, true, HAD>(buf, x32, sm, blk32);
+    if (slow) phase2_clamp_call<MODE, T, B, HAD>(it & 1, blk32);
     else phase2<MODE, T, B, false, HAD>(buf, x32, sm, blk32);
   }
   return it;
