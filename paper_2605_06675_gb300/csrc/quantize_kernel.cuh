@@ -77,7 +77,12 @@ constexpr int kThreads = 128;
 // 16 banks apart (conflict-free 16-byte reads of neighbouring tokens)
 constexpr int kRowBytes = 320;
 constexpr int kTileBytes = kTile * kRowBytes;
-constexpr int kX32S = kD + 4;           // rotated fp32 row (floats)
+// Rotated fp32 tile: channel c of token t at x32_at(t, c) = 164 t + c + 8 (c / 32).
+// The 8-float gap per 32-channel group puts the four group quarters of a
+// token written together in phase 1 on distinct banks, and the row stride
+// (4 mod 32 banks) keeps phase 2's reads of neighbouring tokens apart.
+constexpr int kX32S = 164;
+__device__ __forceinline__ int x32_at(int t, int c) { return t * kX32S + c + 8 * (c >> 5); }
 
 // layouts: keys per channel / per token, values per token / per channel, and
 // the Lloyd-Max codebook quantizer on per-token keys / values
@@ -451,7 +456,7 @@ __device__ __forceinline__ GroupOut phase1_rotated(const uint8_t* tile, float* x
     }
   }
   rotate_group(v, G, sm.signs);
-  float* xr = x32 + t * kX32S + 32 * G;
+  float* xr = x32 + x32_at(t, 32 * G);
 #pragma unroll
   for (int i = 0; i < kG; i += 4)
     *reinterpret_cast<float4*>(xr + i) = make_float4(v[i], v[i + 1], v[i + 2], v[i + 3]);
@@ -473,7 +478,7 @@ __device__ __forceinline__ GroupOut phase1_rotated(const uint8_t* tile, float* x
   }
   __syncthreads();
   const int p = tau & 63, hv = tau >> 6;
-  const float* col = x32 + 16 * hv * kX32S + 2 * p;
+  const float* col = x32 + x32_at(16 * hv, 2 * p);
   float2 lo = *reinterpret_cast<const float2*>(col), hi = lo;
 #pragma unroll
   for (int i = 1; i < 16; ++i) {
@@ -525,8 +530,8 @@ template <typename T, bool F32>
 __device__ __forceinline__ void load_pairs(const uint8_t* tile, const float* x32, int t, int c,
                                            float2 (&v)[4]) {
   if constexpr (F32) {
-    const float4 a = *reinterpret_cast<const float4*>(x32 + t * kX32S + c);
-    const float4 b = *reinterpret_cast<const float4*>(x32 + t * kX32S + c + 4);
+    const float4 a = *reinterpret_cast<const float4*>(x32 + x32_at(t, c));
+    const float4 b = *reinterpret_cast<const float4*>(x32 + x32_at(t, c) + 4);
     v[0] = make_float2(a.x, a.y);
     v[1] = make_float2(a.z, a.w);
     v[2] = make_float2(b.x, b.y);
@@ -545,7 +550,7 @@ template <typename T, bool F32>
 __device__ __forceinline__ void load_quad(const uint8_t* tile, const float* x32, int t, int c,
                                           float (&v)[4]) {
   if constexpr (F32) {
-    const float4 a = *reinterpret_cast<const float4*>(x32 + t * kX32S + c);
+    const float4 a = *reinterpret_cast<const float4*>(x32 + x32_at(t, c));
     v[0] = a.x;
     v[1] = a.y;
     v[2] = a.z;
