@@ -96,7 +96,7 @@ struct alignas(16) QSmem {
   uint2 xchg[kThreads];         // per-channel min/max of half the tokens (rotated tiles)
   float top;                    // magic + the largest code of the tile's quantizer
   float lm_mid[256];            // Lloyd-Max: midpoints of the tile width's levels
-  int8_t signs[kD];
+  uint32_t negmask[4];          // rotation signs: bit i of word G = channel 32 G + i negated
 };
 
 static_assert(sizeof(QSmem) % 16 == 0, "the rotated tile after QSmem must stay 16-byte aligned");
@@ -405,14 +405,8 @@ __device__ __forceinline__ void minmax32(const float (&v)[kG], float& mn, float&
   mx = hi[0];
 }
 
-// y = FWHT(x * sigma) / sqrt(128) of token t's channels 32 G .. 32 G + 31
-// held by thread 4 t + G: butterflies of stride 1..16 in registers, strides
-// 32 and 64 with the lanes holding G ^ 1, G ^ 2 (the lower channel of a
-// pair takes a + b, the upper a - b), in that order.
-__device__ __forceinline__ void rotate_group(float (&v)[kG], int G, const int8_t* signs) {
-#pragma unroll
-  for (int i = 0; i < kG; ++i)
-    if (signs[32 * G + i] < 0) v[i] = -v[i];
+// the butterflies of rotate_group on values whose signs are already applied
+__device__ __forceinline__ void rotate_group_signed(float (&v)[kG], int G) {
 #pragma unroll
   for (int h = 1; h < kG; h <<= 1) {
 #pragma unroll
@@ -436,6 +430,25 @@ __device__ __forceinline__ void rotate_group(float (&v)[kG], int G, const int8_t
   for (int i = 0; i < kG; ++i) v[i] = __fmul_rn(v[i], kInvSqrt128);
 }
 
+// sign flips of a thread's 32 channels from a bit mask (bit i: channel
+// 32 G + i is negated), on the sign bit: no shared-memory reads per value
+__device__ __forceinline__ void apply_sign_mask(float (&v)[kG], uint32_t neg) {
+#pragma unroll
+  for (int i = 0; i < kG; ++i)
+    v[i] = __uint_as_float(__float_as_uint(v[i]) ^ ((neg << (31 - i)) & 0x80000000u));
+}
+
+// y = FWHT(x * sigma) / sqrt(128) of token t's channels 32 G .. 32 G + 31
+// held by thread 4 t + G: butterflies of stride 1..16 in registers, strides
+// 32 and 64 with the lanes holding G ^ 1, G ^ 2 (the lower channel of a
+// pair takes a + b, the upper a - b), in that order.
+__device__ __forceinline__ void rotate_group(float (&v)[kG], int G, const int8_t* signs) {
+#pragma unroll
+  for (int i = 0; i < kG; ++i)
+    if (signs[32 * G + i] < 0) v[i] = -v[i];
+  rotate_group_signed(v, G);
+}
+
 // Rotated tiles: every thread rotates one 32-channel quarter of a token and
 // writes it to the fp32 tile x32; groups are then formed on x32.
 template <typename T, bool SYM>
@@ -455,7 +468,8 @@ __device__ __forceinline__ GroupOut phase1_rotated(const uint8_t* tile, float* x
       v[8 * i + 2 * e + 1] = hi_f32<T>(w[e]);
     }
   }
-  rotate_group(v, G, sm.signs);
+  apply_sign_mask(v, sm.negmask[G]);
+  rotate_group_signed(v, G);
   float* xr = x32 + x32_at(t, 32 * G);
 #pragma unroll
   for (int i = 0; i < kG; i += 4)
@@ -847,7 +861,11 @@ __global__ void __launch_bounds__(kThreads, RQ_QUANT_MIN_BLOCKS) quantize_pack_k
   const long long t0 = a.ntiles * blockIdx.x / gridDim.x;
   const long long t1 = a.ntiles * (blockIdx.x + 1) / gridDim.x;
   if (t0 >= t1) return;
-  if (HAD && threadIdx.x < kD) sm.signs[threadIdx.x] = a.signs ? a.signs[threadIdx.x] : int8_t(1);
+  if (HAD) {                     // warp w's ballot is the sign mask of channels 32 w .. 32 w + 31
+    const bool neg = a.signs && a.signs[threadIdx.x] < 0;
+    const uint32_t m = __ballot_sync(0xffffffffu, neg);
+    if ((threadIdx.x & 31) == 0) sm.negmask[threadIdx.x >> 5] = m;
+  }
 
   const int nblk = a.nblk;
   constexpr int kTileSrcBytes = kTile * kD * static_cast<int>(sizeof(T));
