@@ -213,7 +213,8 @@ rq_status rq_decode_workspace_bytes(const rq_cache_desc* desc, size_t* bytes);
 /* Decode attention of one query per (batch, query head) over all S cached
  * tokens of one layer, reading the packed mixed-bit cache directly
  * (App. W "Kernel fusion"): out[b][j] = sum_t softmax_t(q_j . k_hat_t / sqrt(128)) v_hat_t
- * with k_hat, v_hat the dequantized cache of kv head j / (H_q / H_kv); with
+ * with k_hat, v_hat the dequantized cache of kv head j / (H_q / H_kv)
+ * (x_hat = c * scale + zero, or L_c * scale for RQ_LLOYDMAX groups); with
  * desc->hadamard the rotated cache is used as Q(XR)R^T (App. W "QuaRot kernel").
  * Split-K over the sequence, then a log-sum-exp merge kernel launched as a
  * programmatic dependent of the split kernel (it overlaps the split grid's
