@@ -31,6 +31,7 @@ CHECKPOINTS = (1, 17, 31, 32, 33, 64, 95, 96, 100, 128, 159, 160)
     ("float16", PER_TOKEN, PER_CHANNEL, False, (1, 2, 4), 0, 0),
     ("bfloat16", PER_CHANNEL, PER_TOKEN, False, (2, 3, 4, 6), 1, 0),     # KIVI symmetric keys
     ("bfloat16", PER_TOKEN, PER_TOKEN, True, (2, 4, 5, 8), 1, 1),        # QuaRot symmetric
+    ("float16", PER_TOKEN, PER_TOKEN, True, (1, 3, 4, 6), 2, 2),         # Lloyd-Max codebook
 ])
 def test_append_then_decode_matches_oracle(dtype, kg, vg, hadamard, allowed, kq, vq):
     ensure_built()
@@ -57,7 +58,7 @@ def test_append_then_decode_matches_oracle(dtype, kg, vg, hadamard, allowed, kq,
         ol = {}
         if s_pk:
             ol = oracle_layer(k[:, :, :s_pk], v[:, :, :s_pk], bits[layer], kg, vg, hadamard, signs,
-                              symmetric=(kq == 1, vq == 1))
+                              symmetric=(kq, vq))
             for (bb, h, kind), r in ol.items():   # the packed prefix, bit for bit
                 words = r["words"].view(np.uint8)
                 got = path.stream_bytes(layer, bb, h, kind)[:words.size].cpu().numpy()

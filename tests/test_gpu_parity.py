@@ -31,7 +31,8 @@ def small_wl(L=2, B=2, H=4, g=4, S=96, dtype="float16", kg=PER_CHANNEL, vg=PER_T
 
 
 def symmetric_of(wl):
-    return (wl.k_quantizer == 1, wl.v_quantizer == 1)
+    """The oracle's quantizer forms (0 min-max, 1 absmax, 2 Lloyd-Max) of K and V."""
+    return (int(wl.k_quantizer), int(wl.v_quantizer))
 
 
 def run_layers(rq, wl, bits, layers=None, q_seed=0, kv_scale=1.0):

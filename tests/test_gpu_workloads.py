@@ -62,8 +62,11 @@ def test_tiny_workload_end_to_end(rq, kg):
     assert int(path.status.item()) == 0
 
 
-@pytest.mark.parametrize("wl", [LLAMA3_8B_32K, QWEN3_8B_8K, LONG_70B_128K],
-                         ids=lambda w: w.name)
+@pytest.mark.parametrize("wl", [
+    LLAMA3_8B_32K, QWEN3_8B_8K, LONG_70B_128K,
+    LLAMA3_8B_32K.scaled(name="llama3_absmax_keys", k_quantizer=1),            # KIVI symmetric keys
+    QWEN3_8B_8K.scaled(name="qwen3_lloydmax", k_quantizer=2, v_quantizer=2),   # TurboQuant-style
+], ids=lambda w: w.name)
 def test_full_size_layer_sampled(rq, wl):
     bits = bits_cycle(wl.L, wl.H_kv, wl.allowed)
     layer = wl.L - 1                      # last layer: largest stream offsets
