@@ -78,7 +78,10 @@ rq_status greedy_alloc(int32_t n, const std::vector<double>& w, const double* al
 }
 
 // Exact optimum for any allowed set: suffix table g[i][r] = least cost of
-// components i..n-1 spending r bits above the smallest allowed width.
+// components i..n-1 spending r bits above the smallest allowed width. Only two
+// rows of g are kept; choice[i][r] records the width that attains g[i][r]
+// (the largest one on a tie, as the reconstruction has always taken it), and
+// the bits are read off the choices from (0, R).
 rq_status dp_alloc(int32_t n, const std::vector<double>& w, const double* alpha,
                    const double* beta, int64_t B, uint32_t mask, uint8_t* bits) {
   std::vector<int> widths;
@@ -90,45 +93,37 @@ rq_status dp_alloc(int32_t n, const std::vector<double>& w, const double* alpha,
   if (static_cast<double>(n + 1) * static_cast<double>(R + 1) > 4.0e8) return RQ_ERR_INVALID_ARG;
   const double inf = std::numeric_limits<double>::infinity();
   const size_t W = static_cast<size_t>(R + 1);
-  std::vector<double> g(static_cast<size_t>(n + 1) * W, inf);
-  g[static_cast<size_t>(n) * W + 0] = 0.0;
+  std::vector<double> cur(W, inf), next(W, inf);
+  std::vector<uint8_t> choice(static_cast<size_t>(n) * W, 0);
+  next[0] = 0.0;                                  // g[n][r]: nothing left to spend
   const size_t nw = widths.size();
-  std::vector<double> cost(static_cast<size_t>(n) * nw);
-  for (int32_t i = 0; i < n; ++i)
-    for (size_t k = 0; k < nw; ++k) cost[i * nw + k] = component_cost(w[i], alpha[i], beta[i], widths[k]);
   for (int32_t i = n - 1; i >= 0; --i) {
-    double* gi = &g[static_cast<size_t>(i) * W];
-    const double* gn = &g[static_cast<size_t>(i + 1) * W];
-    for (int64_t r = 0; r <= R; ++r) {
-      double best = inf;
-      for (size_t k = 0; k < nw; ++k) {
-        const int64_t dlt = widths[k] - lo;
-        if (dlt > r || gn[r - dlt] == inf) continue;
-        const double v = cost[i * nw + k] + gn[r - dlt];
-        if (v < best) best = v;
+    // g[i][r] = min over widths k of cost_k + g[i+1][r - (w_k - lo)]: one
+    // branch-free pass per width over the shifted row; visiting the widths in
+    // ascending order with <= keeps the largest width on a tie
+    uint8_t* ch = &choice[static_cast<size_t>(i) * W];
+    std::fill(cur.begin(), cur.end(), inf);
+    for (size_t k = 0; k < nw; ++k) {
+      const int64_t dlt = widths[k] - lo;
+      const double c = component_cost(w[i], alpha[i], beta[i], widths[k]);
+      const uint8_t kk = static_cast<uint8_t>(k);
+      for (int64_t r = dlt; r <= R; ++r) {
+        const double v = c + next[r - dlt];
+        const bool take = v <= cur[r] && v != inf;
+        cur[r] = take ? v : cur[r];
+        ch[r] = take ? kk : ch[r];
       }
-      gi[r] = best;
     }
+    cur.swap(next);
   }
-  if (g[R] == inf) return RQ_ERR_INFEASIBLE;
+  if (next[R] == inf) return RQ_ERR_INFEASIBLE;
   int64_t r = R;
   for (int32_t i = 0; i < n; ++i) {
-    const double* gi = &g[static_cast<size_t>(i) * W];
-    const double* gn = &g[static_cast<size_t>(i + 1) * W];
-    bool placed = false;
-    for (int k = static_cast<int>(nw) - 1; k >= 0; --k) {
-      const int64_t dlt = widths[k] - lo;
-      if (dlt > r || gn[r - dlt] == inf) continue;
-      if (cost[i * nw + k] + gn[r - dlt] == gi[r]) {
-        bits[i] = static_cast<uint8_t>(widths[k]);
-        r -= dlt;
-        placed = true;
-        break;
-      }
-    }
-    if (!placed) return RQ_ERR_INFEASIBLE;  // unreachable when g[R] is finite
+    const int k = choice[static_cast<size_t>(i) * W + r];
+    bits[i] = static_cast<uint8_t>(widths[k]);
+    r -= widths[k] - lo;
   }
-  return RQ_OK;
+  return r == 0 ? RQ_OK : RQ_ERR_INFEASIBLE;
 }
 
 }  // namespace

@@ -10,9 +10,11 @@
 // rotation (QuaRot, App. W "QuaRot kernel"); the sweep measures the MSE at
 // every b for the fit of D(b) = alpha beta^-b (Alg. 1 stage 2, Sec. 3.4).
 //
-// quantize_pack_kernel: persistent CTAs of 128 threads; a CTA owns one
-// 32-token x 128-channel tile (one packed block) at a time, staged raw in
-// shared memory by cp.async one tile ahead. Per tile:
+// quantize_pack_kernel: persistent CTAs of 128 threads; a CTA walks a
+// contiguous range of 32-token x 128-channel tiles (one packed block each)
+// one stream at a time, each stream with a loop compiled for its layout and
+// width; a tile is staged raw in shared memory by cp.async one tile ahead.
+// Per tile:
 //   phase 1, one group per thread: min / max with NaN-propagating fp16x2 or
 //     bf16x2 compares on the raw values, the group's fp16 scale and zero
 //     (its meta words go straight to global memory) and (-zero, 1/scale)
@@ -24,6 +26,8 @@
 //     with vector stores. Codes never pass through shared memory.
 // Phase 1 flags a tile whose codes could leave [0, largest code], or that holds a
 // degenerate group; such a tile takes the clamping variant of phase 2.
+// Lloyd-Max groups (per token): phase 1 computes the group's RMS scale, phase 2
+// finds each code by a binary search over the scaled level midpoints.
 #pragma once
 
 #include <algorithm>
