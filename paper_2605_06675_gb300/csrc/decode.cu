@@ -283,7 +283,57 @@ __device__ __forceinline__ void qk_block(const uint8_t* img, int lane, const uin
       s[mt][2] = __fmaf_rn(s[mt][2], f, c0);
       s[mt][3] = __fmaf_rn(s[mt][3], f, c1);
     }
-  } else {                    // per-token keys: dequantize in registers
+  } else if constexpr (!LM) {
+    // Per-token keys: k_hat[t][c] = code s_tG + z_tG, so for group G = unit u
+    //   scores[t][j] += s_tG sum_{c in G} code[t][c] q_jc + z_tG sum_{c in G} q_jc:
+    // the codes enter the MMA undequantized (two k-steps per group into a
+    // group accumulator), and the group's scale (with the codes' 2^(24 - E)
+    // of the token row) and zero term are applied to that accumulator in fp32.
+    // qsum (the QF area of the table) holds sum_{c in G} q_jc for [G][head].
+    const float* qsum = reinterpret_cast<const float*>(qtab + 2048);
+#pragma unroll
+    for (int u = 0; u < 4; ++u) {
+      // (scale, zero) of tokens 8x + gid, group u: words 16 gid + 4u + x
+      const uint4 SZ = lds128(meta + 4 * (16 * gid + 4 * u));
+      const uint4 QB = lds128(qtab + 16 * (32 * u + lane));
+      const float2 qs = *reinterpret_cast<const float2*>(qsum + 8 * u + 2 * tig);
+      const uint32_t qb[4] = {QB.x, QB.y, QB.z, QB.w};
+      const uint32_t sz[4] = {SZ.x, SZ.y, SZ.z, SZ.w};
+      float acc[2][4];
+#pragma unroll
+      for (int mt = 0; mt < 2; ++mt)
+#pragma unroll
+        for (int r = 0; r < 4; ++r) acc[mt][r] = 0.0f;
+#pragma unroll
+      for (int xs = 0; xs < 2; ++xs)
+#pragma unroll
+        for (int mt = 0; mt < 2; ++mt) {
+          // register (x = token 2mt + r, y = pair 2xs + h)
+          const uint32_t a[4] = {reg<BW>(w, u, 2 * mt, 2 * xs), reg<BW>(w, u, 2 * mt + 1, 2 * xs),
+                                 reg<BW>(w, u, 2 * mt, 2 * xs + 1), reg<BW>(w, u, 2 * mt + 1, 2 * xs + 1)};
+          mma16816(acc[mt], a, qb[2 * xs], qb[2 * xs + 1]);
+        }
+#pragma unroll
+      for (int mt = 0; mt < 2; ++mt) {
+        // rows gid / gid + 8: tokens of class x = 2mt / 2mt + 1
+        const __half2 h0 = u2h(sz[2 * mt]), h1 = u2h(sz[2 * mt + 1]);
+        const float s0 = __fmul_rn(__low2float(h0), __int_as_float((127 + 24 - fmt::exponent(BW, 2 * mt)) << 23));
+        const float s1 = __fmul_rn(__low2float(h1), __int_as_float((127 + 24 - fmt::exponent(BW, 2 * mt + 1)) << 23));
+        const float z0 = __high2float(h0), z1 = __high2float(h1);
+        s[mt][0] = __fmaf_rn(acc[mt][0], s0, __fmaf_rn(z0, qs.x, s[mt][0]));
+        s[mt][1] = __fmaf_rn(acc[mt][1], s0, __fmaf_rn(z0, qs.y, s[mt][1]));
+        s[mt][2] = __fmaf_rn(acc[mt][2], s1, __fmaf_rn(z1, qs.x, s[mt][2]));
+        s[mt][3] = __fmaf_rn(acc[mt][3], s1, __fmaf_rn(z1, qs.y, s[mt][3]));
+      }
+    }
+#pragma unroll
+    for (int mt = 0; mt < 2; ++mt) {
+      s[mt][0] = __fmaf_rn(s[mt][0], qsc, -ms0);
+      s[mt][1] = __fmaf_rn(s[mt][1], qsc, -ms1);
+      s[mt][2] = __fmaf_rn(s[mt][2], qsc, -ms0);
+      s[mt][3] = __fmaf_rn(s[mt][3], qsc, -ms1);
+    }
+  } else {                    // Lloyd-Max per-token keys: codebook levels in registers
 #pragma unroll
     for (int u = 0; u < 4; ++u) {
       // (scale, zero) of tokens 8x + gid, group u: words 16 gid + 4u + x
@@ -802,15 +852,24 @@ __global__ void __launch_bounds__(kThreads, RQ_DECODE_MIN_BLOCKS) decode_split_k
         qf[u][x] = hmul2u(qb[u][x], ef[x]);
       }
   }
+  // per-token keys: sum over each 32-channel group of the q operand the MMA
+  // sees (fp16 q scaled by qpow), [group G = lane / 8][head n = lane % 8]
+  float qgsum = 0.0f;
+  if (warp == 0 && a.kg == RQ_PER_TOKEN) {
+    const float* qr = qs + (lane & 7) * kD + 32 * (lane >> 3);
+    for (int c = 0; c < 32; ++c) qgsum += __half2float(__float2half_rn(qr[c] * qpow));
+  }
   __syncthreads();                  // qs is read; its space becomes the q operand table
   uint8_t* qtab = smem_raw;
   if (warp == 0) {
 #pragma unroll
     for (int u = 0; u < 4; ++u) {
       *reinterpret_cast<uint4*>(qtab + 16 * (32 * u + lane)) = make_uint4(qb[u][0], qb[u][1], qb[u][2], qb[u][3]);
-      *reinterpret_cast<uint4*>(qtab + 2048 + 16 * (32 * u + lane)) =
-          make_uint4(qf[u][0], qf[u][1], qf[u][2], qf[u][3]);
+      if (a.kg == RQ_PER_CHANNEL)
+        *reinterpret_cast<uint4*>(qtab + 2048 + 16 * (32 * u + lane)) =
+            make_uint4(qf[u][0], qf[u][1], qf[u][2], qf[u][3]);
     }
+    if (a.kg == RQ_PER_TOKEN) reinterpret_cast<float*>(qtab + 2048)[lane] = qgsum;   // [G][n]
   }
   __syncthreads();
 
