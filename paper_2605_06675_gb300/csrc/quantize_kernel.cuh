@@ -31,6 +31,7 @@
 #pragma once
 
 #include <algorithm>
+#include <cstddef>
 
 #include "format.cuh"
 #include "rq_internal.cuh"
@@ -82,12 +83,13 @@ constexpr int kThreads = 128;
 // 16 banks apart (conflict-free 16-byte reads of neighbouring tokens)
 constexpr int kRowBytes = 320;
 constexpr int kTileBytes = kTile * kRowBytes;
-// Rotated fp32 tile: channel c of token t at x32_at(t, c) = 164 t + c + 8 (c / 32).
-// The 8-float gap per 32-channel group puts the four group quarters of a
-// token written together in phase 1 on distinct banks, and the row stride
-// (4 mod 32 banks) keeps phase 2's reads of neighbouring tokens apart.
+// Rotated fp32 tile: channel c of token t at x32_at(t, c) = 164 t + c. The
+// row stride (4 mod 32 banks) keeps reads of neighbouring tokens apart; the
+// four quarters of a token are written in the chunk order i ^ G of
+// phase1_rotated, which puts each quarter-warp's 16-byte stores on distinct
+// banks.
 constexpr int kX32S = 164;
-__device__ __forceinline__ int x32_at(int t, int c) { return t * kX32S + c + 8 * (c >> 5); }
+__device__ __forceinline__ int x32_at(int t, int c) { return t * kX32S + c; }
 
 // layouts: keys per channel / per token, values per token / per channel, and
 // the Lloyd-Max codebook quantizer on per-token keys / values
@@ -101,10 +103,13 @@ struct alignas(16) QSmem {
   uint2 xchg[kThreads];         // per-channel min/max of half the tokens (rotated tiles)
   float top;                    // magic + the largest code of the tile's quantizer
   float lm_mid[256];            // Lloyd-Max: midpoints of the tile width's levels
-  uint32_t negmask[4];          // rotation signs: bit i of word G = channel 32 G + i negated
+  alignas(16) uint32_t negw[4][16];   // rotation signs (read as uint4): word k of row G flips the sign bits (15, 31)
+                                //   of the raw pair of channels 32 G + 2k, 32 G + 2k + 1
 };
 
 static_assert(sizeof(QSmem) % 16 == 0, "the rotated tile after QSmem must stay 16-byte aligned");
+static_assert(offsetof(QSmem, tile) % 16 == 0 && offsetof(QSmem, negw) % 16 == 0 &&
+              offsetof(QSmem, xchg) % 16 == 0, "16-byte shared-memory accesses");
 
 // sm.top, read where it is used (a volatile load from a fixed shared address,
 // so the clamping variant keeps no register for it)
@@ -125,6 +130,16 @@ __device__ __forceinline__ float fmin_nan(float a, float b) {
 __device__ __forceinline__ float fmax_nan(float a, float b) {
   float r;
   asm("max.NaN.f32 %0, %1, %2;" : "=f"(r) : "f"(a), "f"(b));
+  return r;
+}
+__device__ __forceinline__ float fmin3_nan(float a, float b, float c) {
+  float r;
+  asm("min.NaN.f32 %0, %1, %2, %3;" : "=f"(r) : "f"(a), "f"(b), "f"(c));
+  return r;
+}
+__device__ __forceinline__ float fmax3_nan(float a, float b, float c) {
+  float r;
+  asm("max.NaN.f32 %0, %1, %2, %3;" : "=f"(r) : "f"(a), "f"(b), "f"(c));
   return r;
 }
 
@@ -364,7 +379,7 @@ __device__ __forceinline__ GroupOut phase1_rows(const uint8_t* tile, int kind, T
   uint32_t w[16];
 #pragma unroll
   for (int i = 0; i < 4; ++i) {
-    const uint4 u = *reinterpret_cast<const uint4*>(row + 16 * ((i + (t >> 1)) & 3));
+    const uint4 u = *reinterpret_cast<const uint4*>(row + 16 * (i ^ G));
     w[4 * i] = u.x;
     w[4 * i + 1] = u.y;
     w[4 * i + 2] = u.z;
@@ -391,56 +406,70 @@ __device__ __forceinline__ GroupOut phase1_rows(const uint8_t* tile, int kind, T
   return finish_group(kind, RQ_PER_TOKEN, t, G, 0, mn, mx, finite, q, meta, sm);
 }
 
-// min / max of 32 fp32 values; NaN propagates
+// min / max of 32 fp32 values; NaN propagates. Three-input min / max
+// (exact and order-free): 32 -> 12 -> 4 -> 2 -> 1 values, 16 each.
 __device__ __forceinline__ void minmax32(const float (&v)[kG], float& mn, float& mx) {
-  float lo[16], hi[16];
+  float lo[12], hi[12];
 #pragma unroll
-  for (int i = 0; i < 16; ++i) {
-    lo[i] = fmin_nan(v[2 * i], v[2 * i + 1]);
-    hi[i] = fmax_nan(v[2 * i], v[2 * i + 1]);
+  for (int i = 0; i < 10; ++i) {
+    lo[i] = fmin3_nan(v[3 * i], v[3 * i + 1], v[3 * i + 2]);
+    hi[i] = fmax3_nan(v[3 * i], v[3 * i + 1], v[3 * i + 2]);
   }
+  lo[10] = hi[10] = v[30];
+  lo[11] = hi[11] = v[31];
 #pragma unroll
-  for (int w = 8; w >= 1; w >>= 1)
-#pragma unroll
-    for (int i = 0; i < w; ++i) {
-      lo[i] = fmin_nan(lo[i], lo[i + w]);
-      hi[i] = fmax_nan(hi[i], hi[i + w]);
-    }
-  mn = lo[0];
-  mx = hi[0];
+  for (int i = 0; i < 4; ++i) {
+    lo[i] = fmin3_nan(lo[3 * i], lo[3 * i + 1], lo[3 * i + 2]);
+    hi[i] = fmax3_nan(hi[3 * i], hi[3 * i + 1], hi[3 * i + 2]);
+  }
+  mn = fmin_nan(fmin3_nan(lo[0], lo[1], lo[2]), lo[3]);
+  mx = fmax_nan(fmax3_nan(hi[0], hi[1], hi[2]), hi[3]);
 }
 
-// the butterflies of rotate_group on values whose signs are already applied
+// RN(a - b) per component: the product b * -1 is exact and the fused add
+// rounds once (no fp32x2 subtract instruction)
+__device__ __forceinline__ float2 fsub2_rn(float2 a, float2 b) {
+  return __ffma2_rn(b, make_float2(-1.0f, -1.0f), a);
+}
+
+// the butterflies of rotate_group on values whose signs are already applied.
+// Stride 1 pairs the two halves of a register pair, so it runs on scalars;
+// strides 2..16 and the two lane stages run on pairs (v[2k], v[2k + 1]) with
+// fp32x2 instructions, each component rounded exactly as the scalar form.
 __device__ __forceinline__ void rotate_group_signed(float (&v)[kG], int G) {
+  float2 p[kG / 2];
 #pragma unroll
-  for (int h = 1; h < kG; h <<= 1) {
+  for (int k = 0; k < kG / 2; ++k)
+    p[k] = make_float2(__fadd_rn(v[2 * k], v[2 * k + 1]), __fsub_rn(v[2 * k], v[2 * k + 1]));
 #pragma unroll
-    for (int i = 0; i < kG; ++i) {
-      if (i & h) continue;
-      const float a = v[i], b = v[i + h];
-      v[i] = __fadd_rn(a, b);
-      v[i + h] = __fsub_rn(a, b);
+  for (int h = 1; h < kG / 2; h <<= 1) {
+#pragma unroll
+    for (int k = 0; k < kG / 2; ++k) {
+      if (k & h) continue;
+      const float2 a = p[k], b = p[k + h];
+      p[k] = __fadd2_rn(a, b);
+      p[k + h] = fsub2_rn(a, b);
     }
   }
 #pragma unroll
   for (int s = 1; s <= 2; s <<= 1) {
-    const bool upper = (G & s) != 0;
+    // lower channel of a pair: v + o; upper: o - v; both as fma(v, +-1, o)
+    const float sg = (G & s) ? -1.0f : 1.0f;
+    const float2 sg2 = make_float2(sg, sg);
 #pragma unroll
-    for (int i = 0; i < kG; ++i) {
-      const float o = __shfl_xor_sync(0xffffffffu, v[i], s);
-      v[i] = upper ? __fsub_rn(o, v[i]) : __fadd_rn(v[i], o);
+    for (int k = 0; k < kG / 2; ++k) {
+      const float2 o = make_float2(__shfl_xor_sync(0xffffffffu, p[k].x, s),
+                                   __shfl_xor_sync(0xffffffffu, p[k].y, s));
+      p[k] = __ffma2_rn(p[k], sg2, o);
     }
   }
+  const float2 r = make_float2(kInvSqrt128, kInvSqrt128);
 #pragma unroll
-  for (int i = 0; i < kG; ++i) v[i] = __fmul_rn(v[i], kInvSqrt128);
-}
-
-// sign flips of a thread's 32 channels from a bit mask (bit i: channel
-// 32 G + i is negated), on the sign bit: no shared-memory reads per value
-__device__ __forceinline__ void apply_sign_mask(float (&v)[kG], uint32_t neg) {
-#pragma unroll
-  for (int i = 0; i < kG; ++i)
-    v[i] = __uint_as_float(__float_as_uint(v[i]) ^ ((neg << (31 - i)) & 0x80000000u));
+  for (int k = 0; k < kG / 2; ++k) {
+    const float2 y = __fmul2_rn(p[k], r);
+    v[2 * k] = y.x;
+    v[2 * k + 1] = y.y;
+  }
 }
 
 // y = FWHT(x * sigma) / sqrt(128) of token t's channels 32 G .. 32 G + 31
@@ -454,8 +483,69 @@ __device__ __forceinline__ void rotate_group(float (&v)[kG], int G, const int8_t
   rotate_group_signed(v, G);
 }
 
+// rotate_group_signed for a thread whose 8-value chunks are permuted: slot
+// 8 i + j holds channel 32 G + 8 (i ^ G) + j. Strides 1, 2, 4 are as there.
+// At strides 8 and 16 the lower channel of a slot pair sits in the upper
+// slot when bit 0 / bit 1 of G is set, so each output is fma(own, +-1,
+// other) with the lane's signs (the same single rounding as a + b, a - b).
+// The lane stages take, from the partner, the slot that holds the same
+// channel there (slot ^ 8 for G ^ 1, slot ^ 16 for G ^ 2).
+__device__ __forceinline__ void rotate_group_perm(float (&v)[kG], int G) {
+  float2 p[kG / 2];
+#pragma unroll
+  for (int k = 0; k < kG / 2; ++k)
+    p[k] = make_float2(__fadd_rn(v[2 * k], v[2 * k + 1]), __fsub_rn(v[2 * k], v[2 * k + 1]));
+#pragma unroll
+  for (int h = 1; h <= 2; h <<= 1) {          // strides 2, 4
+#pragma unroll
+    for (int k = 0; k < kG / 2; ++k) {
+      if (k & h) continue;
+      const float2 a = p[k], b = p[k + h];
+      p[k] = __fadd2_rn(a, b);
+      p[k + h] = fsub2_rn(a, b);
+    }
+  }
+#pragma unroll
+  for (int h = 4; h <= 8; h <<= 1) {          // strides 8, 16
+    const float sg = (G & (h >> 2)) ? -1.0f : 1.0f;
+    const float2 s2 = make_float2(sg, sg), n2 = make_float2(-sg, -sg);
+#pragma unroll
+    for (int k = 0; k < kG / 2; ++k) {
+      if (k & h) continue;
+      const float2 a = p[k], b = p[k + h];
+      p[k] = __ffma2_rn(a, s2, b);
+      p[k + h] = __ffma2_rn(b, n2, a);
+    }
+  }
+#pragma unroll
+  for (int s = 1; s <= 2; s <<= 1) {          // strides 32, 64: lanes G ^ 1, G ^ 2
+    const int d = 4 * s;                      // pair offset of slot ^ 8 / slot ^ 16
+    const float sg = (G & s) ? -1.0f : 1.0f;
+    const float2 sg2 = make_float2(sg, sg);
+#pragma unroll
+    for (int k = 0; k < kG / 2; ++k) {
+      if (k & d) continue;
+      const float2 ok = make_float2(__shfl_xor_sync(0xffffffffu, p[k + d].x, s),
+                                    __shfl_xor_sync(0xffffffffu, p[k + d].y, s));
+      const float2 od = make_float2(__shfl_xor_sync(0xffffffffu, p[k].x, s),
+                                    __shfl_xor_sync(0xffffffffu, p[k].y, s));
+      p[k] = __ffma2_rn(p[k], sg2, ok);
+      p[k + d] = __ffma2_rn(p[k + d], sg2, od);
+    }
+  }
+  const float2 r = make_float2(kInvSqrt128, kInvSqrt128);
+#pragma unroll
+  for (int k = 0; k < kG / 2; ++k) {
+    const float2 y = __fmul2_rn(p[k], r);
+    v[2 * k] = y.x;
+    v[2 * k + 1] = y.y;
+  }
+}
+
 // Rotated tiles: every thread rotates one 32-channel quarter of a token and
-// writes it to the fp32 tile x32; groups are then formed on x32.
+// writes it to the fp32 tile x32; groups are then formed on x32. The thread
+// takes its quarter's 16-byte chunks in the order i ^ G, which puts the
+// reads and writes of each quarter-warp on distinct banks.
 template <typename T, bool SYM>
 __device__ __forceinline__ GroupOut phase1_rotated(const uint8_t* tile, float* x32, int kind,
                                                    int grouping, TileQ<SYM> q, uint8_t* meta,
@@ -465,21 +555,27 @@ __device__ __forceinline__ GroupOut phase1_rotated(const uint8_t* tile, float* x
   const uint8_t* row = tile + t * kRowBytes + 64 * G;
 #pragma unroll
   for (int i = 0; i < 4; ++i) {
-    const uint4 u = *reinterpret_cast<const uint4*>(row + 16 * i);
-    const uint32_t w[4] = {u.x, u.y, u.z, u.w};
+    // sign flips on the raw pairs (bits 15 and 31 are the two signs)
+    const int c = i ^ G;
+    const uint4 u = *reinterpret_cast<const uint4*>(row + 16 * c);
+    const uint4 n = *reinterpret_cast<const uint4*>(&sm.negw[G][4 * c]);
+    const uint32_t w[4] = {u.x ^ n.x, u.y ^ n.y, u.z ^ n.z, u.w ^ n.w};
 #pragma unroll
     for (int e = 0; e < 4; ++e) {
       v[8 * i + 2 * e] = lo_f32<T>(w[e]);
       v[8 * i + 2 * e + 1] = hi_f32<T>(w[e]);
     }
   }
-  apply_sign_mask(v, sm.negmask[G]);
-  rotate_group_signed(v, G);
+  rotate_group_perm(v, G);
   float* xr = x32 + x32_at(t, 32 * G);
 #pragma unroll
-  for (int i = 0; i < kG; i += 4)
-    *reinterpret_cast<float4*>(xr + i) = make_float4(v[i], v[i + 1], v[i + 2], v[i + 3]);
-  if (grouping == RQ_PER_TOKEN) {
+  for (int i = 0; i < 4; ++i) {
+    float* xc = xr + 8 * (i ^ G);
+    *reinterpret_cast<float4*>(xc) = make_float4(v[8 * i], v[8 * i + 1], v[8 * i + 2], v[8 * i + 3]);
+    *reinterpret_cast<float4*>(xc + 4) =
+        make_float4(v[8 * i + 4], v[8 * i + 5], v[8 * i + 6], v[8 * i + 7]);
+  }
+  if (grouping == RQ_PER_TOKEN) {             // min / max: any order
     float mn, mx;
     minmax32(v, mn, mx);
     const bool finite = isfinite(mn) && isfinite(mx);
@@ -487,6 +583,15 @@ __device__ __forceinline__ GroupOut phase1_rotated(const uint8_t* tile, float* x
                         finite, q, meta, sm);
   }
   if (grouping == kGroupingLM) {            // Lloyd-Max, per token, on the rotated values
+    // the sum of squares is ordered: the quarter back from x32 in channel order
+#pragma unroll
+    for (int i = 0; i < kG; i += 4) {
+      const float4 y = *reinterpret_cast<const float4*>(xr + i);
+      v[i] = y.x;
+      v[i + 1] = y.y;
+      v[i + 2] = y.z;
+      v[i + 3] = y.w;
+    }
     bool finite = true;
 #pragma unroll
     for (int i = 0; i < kG; ++i) {
@@ -869,7 +974,9 @@ __global__ void __launch_bounds__(kThreads, RQ_QUANT_MIN_BLOCKS) quantize_pack_k
   if (HAD) {                     // warp w's ballot is the sign mask of channels 32 w .. 32 w + 31
     const bool neg = a.signs && a.signs[threadIdx.x] < 0;
     const uint32_t m = __ballot_sync(0xffffffffu, neg);
-    if ((threadIdx.x & 31) == 0) sm.negmask[threadIdx.x >> 5] = m;
+    const int k = threadIdx.x & 31;
+    if (k < 16)
+      sm.negw[threadIdx.x >> 5][k] = ((m >> (2 * k)) & 1u) << 15 | ((m >> (2 * k + 1)) & 1u) << 31;
   }
 
   const int nblk = a.nblk;
