@@ -225,14 +225,7 @@ __device__ __forceinline__ void qk_block(const uint8_t* img, int lane, const uin
 #pragma unroll
     for (int r = 0; r < 4; ++r) s[mt][r] = 0.0f;
   if constexpr (KG == RQ_PER_CHANNEL) {
-    // two accumulators per m-tile (pair halves xs = 0, 1): chains of four
-    // dependent MMAs instead of eight
-    float zb[2][4] = {{0.0f, 0.0f, 0.0f, 0.0f}, {0.0f, 0.0f, 0.0f, 0.0f}};
-    float s2[2][4];
-#pragma unroll
-    for (int mt = 0; mt < 2; ++mt)
-#pragma unroll
-      for (int r = 0; r < 4; ++r) s2[mt][r] = 0.0f;
+    float zb[4] = {0.0f, 0.0f, 0.0f, 0.0f};
 #pragma unroll
     for (int u = 0; u < 4; ++u) {
       // channel pairs P = 16u + 4tig + x: zeros at word 2P, scales at 2P + 1,
@@ -249,8 +242,7 @@ __device__ __forceinline__ void qk_block(const uint8_t* img, int lane, const uin
         const uint32_t h0 = hmul2u(qf[2 * xs], MZ.y);
         const uint32_t h1 = hmul2u(qf[2 * xs + 1], MZ.w);
         const uint32_t az[4] = {MZ.x, MZ.y, MZ.z, MZ.w};
-        mma16816(zb[xs], az, qb[2 * xs], qb[2 * xs + 1]);
-        float (&sa)[2][4] = xs ? s2 : s;
+        mma16816(zb, az, qb[2 * xs], qb[2 * xs + 1]);
         if constexpr (MERGED) {
           // hi lanes: fma(q, s, hi * -0) = hi; lo lanes: fma(q, s, -hi) = lo
           // (fp16 multiplies, not bitwise ops: they run on the FMA pipe,
@@ -261,7 +253,7 @@ __device__ __forceinline__ void qk_block(const uint8_t* img, int lane, const uin
           for (int mt = 0; mt < 2; ++mt) {
             const uint32_t a[4] = {reg<BW>(w, u, 2 * xs, 2 * mt), reg<BW>(w, u, 2 * xs, 2 * mt + 1),
                                    reg<BW>(w, u, 2 * xs + 1, 2 * mt), reg<BW>(w, u, 2 * xs + 1, 2 * mt + 1)};
-            mma16816(sa[mt], a, b0, b1);
+            mma16816(s[mt], a, b0, b1);
           }
         } else {
           const uint32_t l0 = hfma2u(qf[2 * xs], MZ.y, h0 ^ 0x80008000u);
@@ -270,23 +262,19 @@ __device__ __forceinline__ void qk_block(const uint8_t* img, int lane, const uin
           for (int mt = 0; mt < 2; ++mt) {
             const uint32_t a[4] = {reg<BW>(w, u, 2 * xs, 2 * mt), reg<BW>(w, u, 2 * xs, 2 * mt + 1),
                                    reg<BW>(w, u, 2 * xs + 1, 2 * mt), reg<BW>(w, u, 2 * xs + 1, 2 * mt + 1)};
-            mma16816(sa[mt], a, h0, h1);
-            mma16816(sa[mt], a, l0, l1);
+            mma16816(s[mt], a, h0, h1);
+            mma16816(s[mt], a, l0, l1);
           }
         }
       }
     }
-#pragma unroll
-    for (int mt = 0; mt < 2; ++mt)
-#pragma unroll
-      for (int r = 0; r < 4; ++r) s[mt][r] += s2[mt][r];
     if constexpr (MERGED) {   // columns j and j + 4 of the accumulator: hi + lo
 #pragma unroll
       for (int mt = 0; mt < 2; ++mt)
 #pragma unroll
         for (int r = 0; r < 4; ++r) s[mt][r] += __shfl_xor_sync(0xffffffffu, s[mt][r], 2);
     }
-    const float c0 = __fmaf_rn(zb[0][0] + zb[1][0], qsc, -ms0), c1 = __fmaf_rn(zb[0][1] + zb[1][1], qsc, -ms1);
+    const float c0 = __fmaf_rn(zb[0], qsc, -ms0), c1 = __fmaf_rn(zb[1], qsc, -ms1);
     const float f = kTwo24 * qsc;
 #pragma unroll
     for (int mt = 0; mt < 2; ++mt) {
