@@ -740,18 +740,30 @@ __device__ __forceinline__ void blocks_dyn(const WarpStream& ws, const DynRing& 
   cp_async_wait<0>();
 }
 
-// KIVI layout (per-channel K, per-token V) at widths {2, 3, 4, 8}: key for
-// the compile-time path, or -1
+// Key of the compile-time path, or -1: keys 0..15 for the KIVI layout
+// (per-channel K, per-token V) at widths {2, 3, 4, 8}; keys 16..24 for
+// per-token K and V (the rotated caches) at widths {3, 4, 5}, the widths an
+// allocation at about 4 bits per code mostly gives.
 __device__ __forceinline__ int fast_key(int bK, int bV, int kg, int vg) {
-  auto idx = [](int b) { return b == 2 ? 0 : b == 3 ? 1 : b == 4 ? 2 : b == 8 ? 3 : -1; };
-  if (kg != RQ_PER_CHANNEL || vg != RQ_PER_TOKEN) return -1;
-  const int ik = idx(bK), iv = idx(bV);
-  return (ik < 0 || iv < 0) ? -1 : 4 * ik + iv;
+  if (kg == RQ_PER_CHANNEL && vg == RQ_PER_TOKEN) {
+    auto idx = [](int b) { return b == 2 ? 0 : b == 3 ? 1 : b == 4 ? 2 : b == 8 ? 3 : -1; };
+    const int ik = idx(bK), iv = idx(bV);
+    return (ik < 0 || iv < 0) ? -1 : 4 * ik + iv;
+  }
+  if (kg == RQ_PER_TOKEN && vg == RQ_PER_TOKEN) {
+    auto idx = [](int b) { return b >= 3 && b <= 5 ? b - 3 : -1; };
+    const int ik = idx(bK), iv = idx(bV);
+    return (ik < 0 || iv < 0) ? -1 : 16 + 3 * ik + iv;
+  }
+  return -1;
 }
 
 #define RQ_FAST_CASES(X) \
   X(0, 2, 2) X(1, 2, 3) X(2, 2, 4) X(3, 2, 8) X(4, 3, 2) X(5, 3, 3) X(6, 3, 4) X(7, 3, 8) \
   X(8, 4, 2) X(9, 4, 3) X(10, 4, 4) X(11, 4, 8) X(12, 8, 2) X(13, 8, 3) X(14, 8, 4) X(15, 8, 8)
+#define RQ_TOKEN_CASES(X) \
+  X(16, 3, 3) X(17, 3, 4) X(18, 3, 5) X(19, 4, 3) X(20, 4, 4) X(21, 4, 5) X(22, 5, 3) X(23, 5, 4) \
+  X(24, 5, 5)
 
 template <typename T>
 __global__ void __launch_bounds__(kThreads, RQ_DECODE_MIN_BLOCKS) decode_split_kernel(DecodeArgs a) {
@@ -800,13 +812,14 @@ __global__ void __launch_bounds__(kThreads, RQ_DECODE_MIN_BLOCKS) decode_split_k
   ws.kwarp = kbase + static_cast<size_t>(blk_first) * dr.sK;
   ws.vwarp = vbase + static_cast<size_t>(blk_first) * dr.sV;
   const int key = valid && a.kq != RQ_LLOYDMAX && a.vq != RQ_LLOYDMAX ? fast_key(bK, bV, a.kg, a.vg) : -1;
-  ws.merged = a.g <= kMaxHeads / 2 && key >= 0;   // the compile-time KIVI paths only
+  ws.merged = a.g <= kMaxHeads / 2 && key >= 0 && key < 16;   // the compile-time KIVI paths only
   ws.mneg = ws.merged && gid >= kMaxHeads / 2 ? 0xBC00BC00u : 0x80008000u;
 
   // start streaming the first entries before the q prologue
   switch (key) {
 #define RQ_PRO(k, BK, BV) case k: prologue_static<BK, BV>(ws); break;
     RQ_FAST_CASES(RQ_PRO)
+    RQ_TOKEN_CASES(RQ_PRO)
 #undef RQ_PRO
     default: prologue_dyn(ws, dr); break;
   }
@@ -893,6 +906,10 @@ __global__ void __launch_bounds__(kThreads, RQ_DECODE_MIN_BLOCKS) decode_split_k
     break;
     RQ_FAST_CASES(RQ_BLK)
 #undef RQ_BLK
+#define RQ_TBLK(k, BK, BV)                                                                  \
+  case k: blocks_static<BK, RQ_PER_TOKEN, BV, RQ_PER_TOKEN, false>(ws, qtab, qscale, acc); break;
+    RQ_TOKEN_CASES(RQ_TBLK)
+#undef RQ_TBLK
     default: blocks_dyn(ws, dr, qtab, qscale, acc); break;
   }
   // the merge kernel may be scheduled now; it waits for this grid to finish
