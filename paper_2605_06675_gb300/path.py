@@ -60,8 +60,16 @@ class PackedKVPath:
         offsets, total = rq.rq_packed_layout(self.desc, bits)
         self.bits_host = np.asarray(bits, dtype=np.uint8).reshape(self.wl.L, self.wl.H_kv, 2)
         self.offsets_host = offsets
-        self.bits = torch.from_numpy(self.bits_host.copy()).to(self.device)
-        self.offsets = torch.from_numpy(offsets.view(np.int64).copy()).to(self.device)
+        # update the device tables in place when their shapes allow, so that
+        # work captured in a CUDA graph reads the new widths and offsets
+        bits_t = torch.from_numpy(self.bits_host.copy())
+        offs_t = torch.from_numpy(offsets.view(np.int64).copy())
+        if getattr(self, "bits", None) is not None and self.bits.shape == bits_t.shape:
+            self.bits.copy_(bits_t)
+            self.offsets.copy_(offs_t)
+        else:
+            self.bits = bits_t.to(self.device)
+            self.offsets = offs_t.to(self.device)
         self.total_bytes = total
         cap = max(total, capacity or 0)
         if self.packed is None or self.packed.numel() < cap:
