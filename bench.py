@@ -174,17 +174,43 @@ class ClockSampler:
 # were taken on)
 # --------------------------------------------------------------------------
 
+def strip_comments(src: str) -> str:
+    """C/C++/CUDA source without its comments, whitespace runs collapsed to
+    one blank (string and character literals kept as written)."""
+    out, i, n = [], 0, len(src)
+    while i < n:
+        c = src[i]
+        if c == "/" and i + 1 < n and src[i + 1] == "/":
+            j = src.find("\n", i)
+            i = n if j < 0 else j
+        elif c == "/" and i + 1 < n and src[i + 1] == "*":
+            j = src.find("*/", i + 2)
+            i = n if j < 0 else j + 2
+            out.append(" ")
+        elif c in "\"'":
+            j = i + 1
+            while j < n and src[j] != c:
+                j += 2 if src[j] == "\\" else 1
+            out.append(src[i:j + 1])
+            i = j + 1
+        else:
+            out.append(c)
+            i += 1
+    return " ".join("".join(out).split())
+
+
 def kernel_source_hash(name: str) -> str:
     """sha256[:16] of a kernel's translation unit together with the library's
-    headers (every .cuh and rq.h), so a record goes stale when any of them
-    changes."""
+    headers (every .cuh and rq.h), comments stripped: a record goes stale when
+    the code of any of them changes, not when a comment does."""
     import hashlib
     csrc = os.path.join(ROOT, "paper_2605_06675_gb300", "csrc")
     h = hashlib.sha256()
     headers = sorted(f for f in os.listdir(csrc) if f.endswith(".cuh"))
     for path in ([os.path.join(csrc, name)] + [os.path.join(csrc, f) for f in headers] +
                  [os.path.join(ROOT, "include", "rq.h")]):
-        h.update(open(path, "rb").read())
+        h.update(strip_comments(open(path, encoding="utf-8").read()).encode())
+        h.update(b"\0")
     return h.hexdigest()[:16]
 
 

@@ -369,8 +369,10 @@ __device__ __forceinline__ GroupOut phase1_cols(const uint8_t* tile, int kind, T
 }
 
 // Per-token groups on the raw tile: thread 4 t + G takes token t, channels
-// 32 G .. 32 G + 31 (four 16-byte reads, started at a rotating chunk so the
-// eight threads of a read phase hit distinct banks).
+// 32 G .. 32 G + 31 as four 16-byte reads in the chunk order i ^ G, which
+// puts the eight threads of a quarter-warp (two tokens x four quarters, rows
+// 320 bytes apart) on eight distinct 16-byte bank groups; min / max do not
+// depend on the order.
 template <typename T, bool SYM>
 __device__ __forceinline__ GroupOut phase1_rows(const uint8_t* tile, int kind, TileQ<SYM> q,
                                                 uint8_t* meta, QSmem& sm) {
