@@ -231,9 +231,8 @@ rq_status rq_decode_attention(const rq_cache_desc* desc, int32_t layer, const vo
 
 /* Allocation-free variant of rq_decode_attention (the paper has no counterpart;
  * this is a library convenience). Some callers cannot allocate device memory
- * at the point where they decode: code running inside a captured or
- * replayed CUDA graph, embedding runtimes whose allocator is owned by
- * someone else, or plugins that are handed only the tensors they read and
+ * where they decode: embedding runtimes whose device allocator belongs to
+ * someone else, and plugins that are handed only the tensors they read and
  * write. This entry point takes the same arguments minus the workspace: the
  * split-K partials live in a fixed device array inside librq of
  * RQ_STATIC_SCRATCH_BYTES bytes, reserved on every GPU that loads the
@@ -243,7 +242,9 @@ rq_status rq_decode_attention(const rq_cache_desc* desc, int32_t layer, const vo
  *    anything is launched.
  *  - The first call on a device looks up the array's device address
  *    (cudaGetSymbolAddress) with that device current; make that first call
- *    before any stream capture.
+ *    before any stream capture. The address is cached for the life of the
+ *    process: a device reset (cudaDeviceReset) invalidates it and is not
+ *    supported.
  *  - Every call on a device shares the one array, which keeps the previous
  *    call's contents (each call overwrites every record it reads, so nothing
  *    needs clearing). Calls that can overlap on the GPU (different streams

@@ -1,34 +1,11 @@
-// Split-K GQA decode attention that reads the packed mixed-bit cache
-// directly, plus the log-sum-exp combine of the split partials.
-//
-// RateQuant (arXiv 2605.06675): the allocation table is a static lookup
-// indexed at run time (App. M, App. U) and the quantizers are fused with the
-// consumer so the full-precision cache is never materialised (App. W "Kernel
-// fusion"). Attention itself is standard decode attention (Sec. 1) with GQA
-// (Sec. 4.1 "Models"); the QuaRot cache is used as Q(XR)R^T (App. W).
-//
-// Design (sm_103a): one CTA = (split of the sequence, kv head, batch), four
-// warps, each warp walking its own 32-token blocks. Per block a warp runs
-//   scores^T[32 tok x 8 heads] = K_hat[32 x 128] . q^T      (mma m16n8k16)
-//   online softmax in fp32 (log2 domain), P^T via movmatrix.trans
-//   o^T[128 x 8 heads]       += V_hat^T[128 x 32] . P^T    (mma m16n8k16)
-// The GQA group (g <= 8 query heads) is the MMA n dimension, so it is never
-// padded to 16. Each warp streams its K and V block images through its own
-// ring of shared-memory slots with cp.async, several entries ahead of use.
-// Codes are stored in the MMA-fragment order of format.cuh: one AND of a
-// word yields a register's two codes as exact fp16 subnormals c * 2^(E - 24)
-// that enter the tensor cores undequantized. For the KIVI layouts
-// (per-channel keys, per-token values) the group scales and 2^-E are folded
-// into the small operand (q or P) or the output rows, and the zero-points are
-// added by extra MMAs whose A operand is the meta image as read; the other
-// layouts dequantize in registers (fp16 1024 exponent, one fp16x2 FMA).
-// Split records are merged by decode_merge_kernel, a programmatic dependent
-// launch of the split kernel.
+// Host side of decode attention: the split plan of a call, workspace
+// layout, argument checks and the C entry points. The kernels are in
+// decode_kernel.cuh (one instance per input dtype: decode_f16.cu,
+// decode_bf16.cu).
 #include <algorithm>
 #include <atomic>
 
-#include "format.cuh"
-#include "rq_internal.cuh"
+#include "decode_kernel.cuh"
 
 namespace rq {
 
@@ -50,1161 +27,11 @@ rq_status current_sm_count(int* sms) {
   *sms = v;
   return RQ_OK;
 }
-
 namespace {
 
-// CTAs per SM the decoder's register budget is sized for
-#ifndef RQ_DECODE_MIN_BLOCKS
-#define RQ_DECODE_MIN_BLOCKS 4
-#endif
-constexpr int kWarps = 4;
-constexpr int kThreads = 32 * kWarps;
-constexpr int kPart = kD + 4;        // partial record: o[128], m (log2 domain), l, 2 pad (16-byte rows)
-constexpr int kMaxHeads = 8;         // MMA n
-constexpr int kRingBytes = 11264;    // per-warp ring of shared-memory slots
-constexpr int kMaxSlots = 8;
-constexpr int kQBytes = kMaxHeads * kD * 4;
-constexpr int kSmemBytes = kQBytes + kWarps * kRingBytes;   // 49152: 4 CTAs per SM
-static_assert(kWarps * kMaxHeads * kD * 4 <= kWarps * kRingBytes, "merge buffer aliases rings");
-
-struct DecodeArgs {
-  const void* q;
-  const uint8_t* packed;
-  const uint8_t* bits;
-  const uint64_t* offsets;
-  const int8_t* signs;
-  float* partial;            // [B][H_q][splits][132]
-  uint32_t* status;
-  int layer, B, H, Hq, g, nblk, splits, bps, kg, vg, hadamard;
-  int kq, vq;                // rq_quantizer of keys / values
-  LMBook lm;                 // RQ_LLOYDMAX codebooks
-};
-
-__device__ __forceinline__ uint32_t h2u(__half2 h) { return *reinterpret_cast<uint32_t*>(&h); }
-__device__ __forceinline__ __half2 u2h(uint32_t u) { return *reinterpret_cast<__half2*>(&u); }
-__device__ __forceinline__ uint32_t pack_f16x2(float lo, float hi) {
-  return h2u(__floats2half2_rn(lo, hi));
-}
-
-__device__ __forceinline__ void mma16816(float (&d)[4], const uint32_t (&a)[4], uint32_t b0,
-                                         uint32_t b1) {
-  asm("mma.sync.aligned.m16n8k16.row.col.f32.f16.f16.f32 {%0,%1,%2,%3}, {%4,%5,%6,%7}, "
-      "{%8,%9}, {%0,%1,%2,%3};\n"
-      : "+f"(d[0]), "+f"(d[1]), "+f"(d[2]), "+f"(d[3])
-      : "r"(a[0]), "r"(a[1]), "r"(a[2]), "r"(a[3]), "r"(b0), "r"(b1));
-}
-
-__device__ __forceinline__ uint32_t movmatrix_trans(uint32_t x) {
-  uint32_t y;
-  asm volatile("movmatrix.sync.aligned.m8n8.trans.b16 %0, %1;\n" : "=r"(y) : "r"(x));
-  return y;
-}
-
-__device__ __forceinline__ uint32_t smem_u32(const void* p) {
-  return static_cast<uint32_t>(__cvta_generic_to_shared(p));
-}
-
-__device__ __forceinline__ void cp_async16(uint32_t dst, const void* src) {
-  asm volatile("cp.async.cg.shared.global [%0], [%1], 16;\n" ::"r"(dst), "l"(src));
-}
-__device__ __forceinline__ void cp_async_commit() { asm volatile("cp.async.commit_group;\n" ::); }
-template <int N>
-__device__ __forceinline__ void cp_async_wait() { asm volatile("cp.async.wait_group %0;\n" ::"n"(N)); }
-__device__ __forceinline__ void cp_async_wait_dyn(int n) {
-  switch (n) {
-    case 0: cp_async_wait<0>(); break;
-    case 1: cp_async_wait<1>(); break;
-    case 2: cp_async_wait<2>(); break;
-    case 3: cp_async_wait<3>(); break;
-    case 4: cp_async_wait<4>(); break;
-    case 5: cp_async_wait<5>(); break;
-    case 6: cp_async_wait<6>(); break;
-    default: cp_async_wait<7>(); break;
-  }
-}
-
-// 2^x with the MUFU approximation (x <= 0 or small; -inf gives 0)
-__device__ __forceinline__ float fast_exp2(float x) {
-  float y;
-  asm("ex2.approx.ftz.f32 %0, %1;" : "=f"(y) : "f"(x));
-  return y;
-}
-
-__device__ __forceinline__ uint4 lds128(const uint8_t* p) {
-  return *reinterpret_cast<const uint4*>(p);
-}
-
-// ------------------------------------------------------- code extraction ----
-// The lane's 4*BW code words of one block image (16-byte piece i of lane L at
-// byte 16*(32 i + L)); unit u's words are w[BW u .. BW u + BW - 1].
-template <int BW>
-__device__ __forceinline__ void lane_words(const uint8_t* img, int lane, uint32_t (&w)[4 * BW]) {
-#pragma unroll
-  for (int i = 0; i < BW; ++i) {
-    const uint4 u = lds128(img + 16 * (32 * i + lane));
-    w[4 * i + 0] = u.x;
-    w[4 * i + 1] = u.y;
-    w[4 * i + 2] = u.z;
-    w[4 * i + 3] = u.w;
-  }
-}
-
-constexpr uint32_t kMagic = 0x64006400u;      // fp16 1024.0 in both halves
-constexpr float kTwo24 = 16777216.0f;         // codes enter the MMA as c * 2^(E - 24)
-
-__device__ __forceinline__ uint32_t hfma2u(uint32_t x, uint32_t m, uint32_t a) {
-  return h2u(__hfma2(u2h(x), u2h(m), u2h(a)));
-}
-__device__ __forceinline__ uint32_t hsub2u(uint32_t x, uint32_t y) {
-  return h2u(__hsub2(u2h(x), u2h(y)));
-}
-__device__ __forceinline__ uint32_t hmul2u(uint32_t x, uint32_t y) {
-  return h2u(__hmul2(u2h(x), u2h(y)));
-}
-
-// 2^-E in both fp16 halves (E <= 14)
-__host__ __device__ constexpr uint32_t pow2_neg_h2(int E) {
-  return (static_cast<uint32_t>(15 - E) << 10) * 0x00010001u;
-}
-
-// register (x, y) of unit u of the lane's words: c * 2^(E - 24) per half
-template <int BW>
-__device__ __forceinline__ uint32_t reg(const uint32_t (&w)[4 * BW], int u, int x, int y) {
-  return fmt::extract<BW>(w + BW * u, x, y);
-}
-
-// dequantized pair s * c + z from an extracted register (layouts whose scale
-// cannot be folded): the subnormal c * 2^E under the 1024 exponent, minus
-// 1024 (exact), times m = s * 2^-E plus z (one rounding)
-__device__ __forceinline__ uint32_t dequant(uint32_t sub, uint32_t m, uint32_t z2) {
-  return hfma2u(hsub2u(sub | kMagic, kMagic), m, z2);
-}
-
-// Lloyd-Max pair: the two codes of an extracted register (at bit E of each
-// half) looked up in the width's fp16 codebook (shared memory), scaled by m
-// and shifted by z2 (one fp16x2 FMA)
-template <int BW>
-__device__ __forceinline__ uint32_t lm_pair(uint32_t sub, int E, const uint16_t* tab) {
-  const uint32_t c0 = (sub >> E) & ((1u << BW) - 1u), c1 = (sub >> (16 + E)) & ((1u << BW) - 1u);
-  return static_cast<uint32_t>(tab[c0]) | (static_cast<uint32_t>(tab[c1]) << 16);
-}
-
-// ------------------------------------------------------------ block math ----
-// Lane (gid, tig) reads units u = 0..3 of its K words: unit u holds channels
-// 32 u + 8 tig + (0..7) of tokens gid + 8 (0..3); the k-steps 2u and 2u + 1
-// of the scores MMA are its channel pairs x = 0, 1 and 2, 3 (format.cuh).
-//
-// scores^T[mt] (tokens 16 mt + gid (+8), heads 2 tig (+1)) of one K block image.
-// Per-channel keys: k_hat[t][c] = code s_c + z_c, so
-//   scores[t][j] = sum_c code[t][c] (q_jc s_c) + sum_c z_c q_jc:
-// the scale (and the code's 2^-E) is folded into q, one fp16x2 multiply per
-// q pair; the zero-point term, the same for every token, comes from MMAs
-// whose A operand carries z in rows gid. Codes enter the tensor cores as
-// exact fp16 subnormals c 2^(E - 24); the accumulator is scaled by 2^24.
-// q operands of lane L for unit u: qtab + 16 (32 u + L) holds q pairs x = 0..3
-// (channels 32u + 8tig + 2x), qtab + 2048 + the same with 2^-E(x) folded in.
-// s is returned in log2 units (q . k times qsc = log2(e) / sqrt(128), applied
-// here in fp32 so q enters the MMAs unscaled) relative to the running max
-// (ms0, ms1: the max of heads 2tig, 2tig + 1, 0 while unset).
-// q s 2^-E enters as an fp16 sum hi + lo (lo = the exact remainder, one fp16
-// FMA), so the products keep ~22 bits. With g <= 4 query heads (MERGED)
-// the MMA's 8 columns hold hi for heads 0..3 and lo for the same heads in
-// columns 4..7 (lanes gid >= 4 carry q of head gid - 4 and mneg = -1 there,
-// -0 elsewhere), and one shuffle adds the halves; otherwise hi and lo take
-// one MMA each.
-template <int BW, int KG, bool MERGED, bool LM = false>
-__device__ __forceinline__ void qk_block(const uint8_t* img, int lane, const uint8_t* qtab,
-                                         float qsc, float ms0, float ms1, uint32_t mneg,
-                                         float (&s)[2][4], const uint16_t* lmtab = nullptr) {
-  const int gid = lane >> 2, tig = lane & 3;
-  uint32_t w[4 * BW];
-  lane_words<BW>(img, lane, w);
-  const uint8_t* meta = img + 512 * BW;
-#pragma unroll
-  for (int mt = 0; mt < 2; ++mt)
-#pragma unroll
-    for (int r = 0; r < 4; ++r) s[mt][r] = 0.0f;
-  if constexpr (KG == RQ_PER_CHANNEL) {
-    float zb[4] = {0.0f, 0.0f, 0.0f, 0.0f};
-#pragma unroll
-    for (int u = 0; u < 4; ++u) {
-      // channel pairs P = 16u + 4tig + x: zeros at word 2P, scales at 2P + 1,
-      // so each 16-byte read {z(x), s(x), z(x+1), s(x+1)} is the A operand of
-      // a zero-point MMA (rows gid take z; rows gid + 8 take s and are unused)
-      const uint4 MZ0 = lds128(meta + 4 * (32 * u + 8 * tig));
-      const uint4 MZ1 = lds128(meta + 4 * (32 * u + 8 * tig + 4));
-      const uint4 QB = lds128(qtab + 16 * (32 * u + lane));
-      const uint4 QF = lds128(qtab + 2048 + 16 * (32 * u + lane));
-      const uint32_t qb[4] = {QB.x, QB.y, QB.z, QB.w}, qf[4] = {QF.x, QF.y, QF.z, QF.w};
-#pragma unroll
-      for (int xs = 0; xs < 2; ++xs) {
-        const uint4 MZ = xs ? MZ1 : MZ0;
-        const uint32_t h0 = hmul2u(qf[2 * xs], MZ.y);
-        const uint32_t h1 = hmul2u(qf[2 * xs + 1], MZ.w);
-        const uint32_t az[4] = {MZ.x, MZ.y, MZ.z, MZ.w};
-        mma16816(zb, az, qb[2 * xs], qb[2 * xs + 1]);
-        if constexpr (MERGED) {
-          // hi lanes: fma(q, s, hi * -0) = hi; lo lanes: fma(q, s, -hi) = lo
-          // (fp16 multiplies, not bitwise ops: they run on the FMA pipe,
-          // which the code extraction leaves idle)
-          const uint32_t b0 = hfma2u(qf[2 * xs], MZ.y, hmul2u(h0, mneg));
-          const uint32_t b1 = hfma2u(qf[2 * xs + 1], MZ.w, hmul2u(h1, mneg));
-#pragma unroll
-          for (int mt = 0; mt < 2; ++mt) {
-            const uint32_t a[4] = {reg<BW>(w, u, 2 * xs, 2 * mt), reg<BW>(w, u, 2 * xs, 2 * mt + 1),
-                                   reg<BW>(w, u, 2 * xs + 1, 2 * mt), reg<BW>(w, u, 2 * xs + 1, 2 * mt + 1)};
-            mma16816(s[mt], a, b0, b1);
-          }
-        } else {
-          const uint32_t l0 = hfma2u(qf[2 * xs], MZ.y, h0 ^ 0x80008000u);
-          const uint32_t l1 = hfma2u(qf[2 * xs + 1], MZ.w, h1 ^ 0x80008000u);
-#pragma unroll
-          for (int mt = 0; mt < 2; ++mt) {
-            const uint32_t a[4] = {reg<BW>(w, u, 2 * xs, 2 * mt), reg<BW>(w, u, 2 * xs, 2 * mt + 1),
-                                   reg<BW>(w, u, 2 * xs + 1, 2 * mt), reg<BW>(w, u, 2 * xs + 1, 2 * mt + 1)};
-            mma16816(s[mt], a, h0, h1);
-            mma16816(s[mt], a, l0, l1);
-          }
-        }
-      }
-    }
-    if constexpr (MERGED) {   // columns j and j + 4 of the accumulator: hi + lo
-#pragma unroll
-      for (int mt = 0; mt < 2; ++mt)
-#pragma unroll
-        for (int r = 0; r < 4; ++r) s[mt][r] += __shfl_xor_sync(0xffffffffu, s[mt][r], 2);
-    }
-    const float c0 = __fmaf_rn(zb[0], qsc, -ms0), c1 = __fmaf_rn(zb[1], qsc, -ms1);
-    const float f = kTwo24 * qsc;
-#pragma unroll
-    for (int mt = 0; mt < 2; ++mt) {
-      s[mt][0] = __fmaf_rn(s[mt][0], f, c0);
-      s[mt][1] = __fmaf_rn(s[mt][1], f, c1);
-      s[mt][2] = __fmaf_rn(s[mt][2], f, c0);
-      s[mt][3] = __fmaf_rn(s[mt][3], f, c1);
-    }
-  } else if constexpr (!LM) {
-    // Per-token keys: k_hat[t][c] = code s_tG + z_tG, so for group G = unit u
-    //   scores[t][j] += s_tG sum_{c in G} code[t][c] q_jc + z_tG sum_{c in G} q_jc:
-    // the codes enter the MMA undequantized (two k-steps per group into a
-    // group accumulator), and the group's scale (with the codes' 2^(24 - E)
-    // of the token row) and zero term are applied to that accumulator in fp32.
-    // qsum (the QF area of the table) holds sum_{c in G} q_jc for [G][head].
-    const float* qsum = reinterpret_cast<const float*>(qtab + 2048);
-#pragma unroll
-    for (int u = 0; u < 4; ++u) {
-      // (scale, zero) of tokens 8x + gid, group u: words 16 gid + 4u + x
-      const uint4 SZ = lds128(meta + 4 * (16 * gid + 4 * u));
-      const uint4 QB = lds128(qtab + 16 * (32 * u + lane));
-      const float2 qs = *reinterpret_cast<const float2*>(qsum + 8 * u + 2 * tig);
-      const uint32_t qb[4] = {QB.x, QB.y, QB.z, QB.w};
-      const uint32_t sz[4] = {SZ.x, SZ.y, SZ.z, SZ.w};
-      float acc[2][4];
-#pragma unroll
-      for (int mt = 0; mt < 2; ++mt)
-#pragma unroll
-        for (int r = 0; r < 4; ++r) acc[mt][r] = 0.0f;
-#pragma unroll
-      for (int xs = 0; xs < 2; ++xs)
-#pragma unroll
-        for (int mt = 0; mt < 2; ++mt) {
-          // register (x = token 2mt + r, y = pair 2xs + h)
-          const uint32_t a[4] = {reg<BW>(w, u, 2 * mt, 2 * xs), reg<BW>(w, u, 2 * mt + 1, 2 * xs),
-                                 reg<BW>(w, u, 2 * mt, 2 * xs + 1), reg<BW>(w, u, 2 * mt + 1, 2 * xs + 1)};
-          mma16816(acc[mt], a, qb[2 * xs], qb[2 * xs + 1]);
-        }
-#pragma unroll
-      for (int mt = 0; mt < 2; ++mt) {
-        // rows gid / gid + 8: tokens of class x = 2mt / 2mt + 1
-        const __half2 h0 = u2h(sz[2 * mt]), h1 = u2h(sz[2 * mt + 1]);
-        const float s0 = __fmul_rn(__low2float(h0), __int_as_float((127 + 24 - fmt::exponent(BW, 2 * mt)) << 23));
-        const float s1 = __fmul_rn(__low2float(h1), __int_as_float((127 + 24 - fmt::exponent(BW, 2 * mt + 1)) << 23));
-        const float z0 = __high2float(h0), z1 = __high2float(h1);
-        s[mt][0] = __fmaf_rn(acc[mt][0], s0, __fmaf_rn(z0, qs.x, s[mt][0]));
-        s[mt][1] = __fmaf_rn(acc[mt][1], s0, __fmaf_rn(z0, qs.y, s[mt][1]));
-        s[mt][2] = __fmaf_rn(acc[mt][2], s1, __fmaf_rn(z1, qs.x, s[mt][2]));
-        s[mt][3] = __fmaf_rn(acc[mt][3], s1, __fmaf_rn(z1, qs.y, s[mt][3]));
-      }
-    }
-#pragma unroll
-    for (int mt = 0; mt < 2; ++mt) {
-      s[mt][0] = __fmaf_rn(s[mt][0], qsc, -ms0);
-      s[mt][1] = __fmaf_rn(s[mt][1], qsc, -ms1);
-      s[mt][2] = __fmaf_rn(s[mt][2], qsc, -ms0);
-      s[mt][3] = __fmaf_rn(s[mt][3], qsc, -ms1);
-    }
-  } else {                    // Lloyd-Max per-token keys: codebook levels in registers
-#pragma unroll
-    for (int u = 0; u < 4; ++u) {
-      // (scale, zero) of tokens 8x + gid, group u: words 16 gid + 4u + x
-      const uint4 SZ = lds128(meta + 4 * (16 * gid + 4 * u));
-      const uint4 QB = lds128(qtab + 16 * (32 * u + lane));
-      const uint32_t qb[4] = {QB.x, QB.y, QB.z, QB.w};
-      const uint32_t sz[4] = {SZ.x, SZ.y, SZ.z, SZ.w};
-      uint32_t m[4], z2[4];
-#pragma unroll
-      for (int x = 0; x < 4; ++x) {
-        const __half2 h = u2h(sz[x]);
-        m[x] = LM ? h2u(__low2half2(h))          // codebook levels are real values
-                  : hmul2u(h2u(__low2half2(h)), pow2_neg_h2(fmt::exponent(BW, x)));
-        z2[x] = h2u(__high2half2(h));
-      }
-      auto deq = [&](int x, int y) -> uint32_t {
-        if constexpr (LM) return hfma2u(lm_pair<BW>(reg<BW>(w, u, x, y), fmt::exponent(BW, x), lmtab),
-                                        m[x], z2[x]);
-        else return dequant(reg<BW>(w, u, x, y), m[x], z2[x]);
-      };
-#pragma unroll
-      for (int xs = 0; xs < 2; ++xs)
-#pragma unroll
-        for (int mt = 0; mt < 2; ++mt) {
-          // register (x = token 2mt + r, y = pair 2xs + h)
-          const uint32_t a[4] = {deq(2 * mt, 2 * xs), deq(2 * mt + 1, 2 * xs),
-                                 deq(2 * mt, 2 * xs + 1), deq(2 * mt + 1, 2 * xs + 1)};
-          mma16816(s[mt], a, qb[2 * xs], qb[2 * xs + 1]);
-        }
-    }
-#pragma unroll
-    for (int mt = 0; mt < 2; ++mt) {
-      s[mt][0] = __fmaf_rn(s[mt][0], qsc, -ms0);
-      s[mt][1] = __fmaf_rn(s[mt][1], qsc, -ms1);
-      s[mt][2] = __fmaf_rn(s[mt][2], qsc, -ms0);
-      s[mt][3] = __fmaf_rn(s[mt][3], qsc, -ms1);
-    }
-  }
-}
-
-// o^T[mt] (channel rows 16 mt + gid (+8), heads 2 tig (+1)) += V_hat^T . P^T of
-// one V block image. Unit u = channel group G holds channels 32u + 4gid + x
-// (rows of m-tiles 2u, 2u + 1) of tokens 8y + 2tig + (0, 1).
-// Per-token values: v_hat[t][c] = code s_tG + z_tG, so
-//   o[c][j] += sum_t code[t][c] (p_tj s_tG) + sum_t z_tG p_tj:
-// the scale is folded into P^T per group (one fp16x2 multiply per pair), the
-// zero-point term comes from MMAs whose A operand repeats z_tG in every row
-// of the group, and the codes' 2^(E - 24) is undone on the output rows.
-template <int BW, int VG, bool LM = false>
-__device__ __forceinline__ void pv_block(const uint8_t* img, int lane, const uint32_t (&pb)[2][2],
-                                         float (&o)[8][4], float (&bz)[2][4],
-                                         const uint16_t* lmtab = nullptr) {
-  const int gid = lane >> 2, tig = lane & 3;
-  uint32_t w[4 * BW];
-  lane_words<BW>(img, lane, w);
-  const uint8_t* meta = img + 512 * BW;
-  if constexpr (VG == RQ_PER_TOKEN) {
-    // zero-points: rows gid of the A operand carry group 2gp, rows gid + 8
-    // group 2gp + 1; columns are token pairs 2ks (k 2tig..) and 2ks + 1.
-    // Zero pairs are stored so that each 16-byte read is an A operand:
-    // words 64 + 32ks + 8tig + 4gp + {0..3} = z of (token pair 2ks, group
-    // 2gp), (2ks, 2gp+1), (2ks+1, 2gp), (2ks+1, 2gp+1).
-#pragma unroll
-    for (int ks = 0; ks < 2; ++ks)
-#pragma unroll
-      for (int gp = 0; gp < 2; ++gp) {
-        const uint4 Z = lds128(meta + 4 * (64 + 32 * ks + 8 * tig + 4 * gp));
-        const uint32_t az[4] = {Z.x, Z.y, Z.z, Z.w};
-        mma16816(bz[gp], az, pb[ks][0], pb[ks][1]);
-      }
-    uint32_t ms[4][4];        // scale pairs [token pair y][group G]: words 16y + 4tig + G
-#pragma unroll
-    for (int y = 0; y < 4; ++y) {
-      const uint4 S = lds128(meta + 4 * (16 * y + 4 * tig));
-      ms[y][0] = S.x;
-      ms[y][1] = S.y;
-      ms[y][2] = S.z;
-      ms[y][3] = S.w;
-    }
-#pragma unroll
-    for (int ks = 0; ks < 2; ++ks)
-#pragma unroll
-      for (int G = 0; G < 4; ++G) {
-        const uint32_t b0 = hmul2u(pb[ks][0], ms[2 * ks][G]);
-        const uint32_t b1 = hmul2u(pb[ks][1], ms[2 * ks + 1][G]);
-#pragma unroll
-        for (int mh = 0; mh < 2; ++mh) {
-          // register (x = row 2mh + r, y = token pair 2ks + h); Lloyd-Max: the
-          // codebook levels (real values) instead of the subnormal codes
-          auto A = [&](int x, int y) -> uint32_t {
-            if constexpr (LM) return lm_pair<BW>(reg<BW>(w, G, x, y), fmt::exponent(BW, x), lmtab);
-            else return reg<BW>(w, G, x, y);
-          };
-          const uint32_t a[4] = {A(2 * mh, 2 * ks), A(2 * mh + 1, 2 * ks), A(2 * mh, 2 * ks + 1),
-                                 A(2 * mh + 1, 2 * ks + 1)};
-          mma16816(o[2 * G + mh], a, b0, b1);
-        }
-      }
-  } else {                    // per-channel values: dequantize in registers
-#pragma unroll
-    for (int u = 0; u < 4; ++u) {
-      // (scale, zero) of channels 32u + 4gid + x: words 32u + 4gid + x
-      const uint4 SZ = lds128(meta + 4 * (32 * u + 4 * gid));
-      const uint32_t sz[4] = {SZ.x, SZ.y, SZ.z, SZ.w};
-      uint32_t m[4], z2[4];
-#pragma unroll
-      for (int x = 0; x < 4; ++x) {
-        const __half2 h = u2h(sz[x]);
-        m[x] = hmul2u(h2u(__low2half2(h)), pow2_neg_h2(fmt::exponent(BW, x)));
-        z2[x] = h2u(__high2half2(h));
-      }
-#pragma unroll
-      for (int ks = 0; ks < 2; ++ks)
-#pragma unroll
-        for (int mh = 0; mh < 2; ++mh) {
-          const uint32_t a[4] = {
-              dequant(reg<BW>(w, u, 2 * mh, 2 * ks), m[2 * mh], z2[2 * mh]),
-              dequant(reg<BW>(w, u, 2 * mh + 1, 2 * ks), m[2 * mh + 1], z2[2 * mh + 1]),
-              dequant(reg<BW>(w, u, 2 * mh, 2 * ks + 1), m[2 * mh], z2[2 * mh]),
-              dequant(reg<BW>(w, u, 2 * mh + 1, 2 * ks + 1), m[2 * mh + 1], z2[2 * mh + 1])};
-          mma16816(o[2 * u + mh], a, pb[ks][0], pb[ks][1]);
-        }
-    }
-  }
-}
-
-template <int BW>
-__device__ __forceinline__ void qk_dispatch_g(int kg, const uint8_t* img, int lane,
-                                              const uint8_t* qtab, float qsc, float ms0, float ms1,
-                                              float (&s)[2][4], const uint16_t* lmtab) {
-  // mneg is unused off the merged path; lmtab is non-null for Lloyd-Max keys
-  if (kg == RQ_PER_CHANNEL) qk_block<BW, RQ_PER_CHANNEL, false>(img, lane, qtab, qsc, ms0, ms1, 0u, s);
-  else if (lmtab) qk_block<BW, RQ_PER_TOKEN, false, true>(img, lane, qtab, qsc, ms0, ms1, 0u, s, lmtab);
-  else qk_block<BW, RQ_PER_TOKEN, false>(img, lane, qtab, qsc, ms0, ms1, 0u, s);
-}
-
-template <int BW>
-__device__ __forceinline__ void pv_dispatch_g(int vg, const uint8_t* img, int lane,
-                                              const uint32_t (&pb)[2][2], float (&o)[8][4],
-                                              float (&bz)[2][4], const uint16_t* lmtab) {
-  if (vg == RQ_PER_TOKEN && lmtab) pv_block<BW, RQ_PER_TOKEN, true>(img, lane, pb, o, bz, lmtab);
-  else if (vg == RQ_PER_TOKEN) pv_block<BW, RQ_PER_TOKEN>(img, lane, pb, o, bz);
-  else pv_block<BW, RQ_PER_CHANNEL>(img, lane, pb, o, bz);
-}
-
-__device__ __forceinline__ void qk_dispatch(int bw, int kg, const uint8_t* img, int lane,
-                                            const uint8_t* qtab, float qsc, float ms0, float ms1,
-                                            float (&s)[2][4], const uint16_t* lmtab) {
-  switch (bw) {
-    case 1: qk_dispatch_g<1>(kg, img, lane, qtab, qsc, ms0, ms1, s, lmtab); break;
-    case 2: qk_dispatch_g<2>(kg, img, lane, qtab, qsc, ms0, ms1, s, lmtab); break;
-    case 3: qk_dispatch_g<3>(kg, img, lane, qtab, qsc, ms0, ms1, s, lmtab); break;
-    case 4: qk_dispatch_g<4>(kg, img, lane, qtab, qsc, ms0, ms1, s, lmtab); break;
-    case 5: qk_dispatch_g<5>(kg, img, lane, qtab, qsc, ms0, ms1, s, lmtab); break;
-    case 6: qk_dispatch_g<6>(kg, img, lane, qtab, qsc, ms0, ms1, s, lmtab); break;
-    case 7: qk_dispatch_g<7>(kg, img, lane, qtab, qsc, ms0, ms1, s, lmtab); break;
-    default: qk_dispatch_g<8>(kg, img, lane, qtab, qsc, ms0, ms1, s, lmtab); break;
-  }
-}
-
-__device__ __forceinline__ void pv_dispatch(int bw, int vg, const uint8_t* img, int lane,
-                                            const uint32_t (&pb)[2][2], float (&o)[8][4],
-                                            float (&bz)[2][4], const uint16_t* lmtab) {
-  switch (bw) {
-    case 1: pv_dispatch_g<1>(vg, img, lane, pb, o, bz, lmtab); break;
-    case 2: pv_dispatch_g<2>(vg, img, lane, pb, o, bz, lmtab); break;
-    case 3: pv_dispatch_g<3>(vg, img, lane, pb, o, bz, lmtab); break;
-    case 4: pv_dispatch_g<4>(vg, img, lane, pb, o, bz, lmtab); break;
-    case 5: pv_dispatch_g<5>(vg, img, lane, pb, o, bz, lmtab); break;
-    case 6: pv_dispatch_g<6>(vg, img, lane, pb, o, bz, lmtab); break;
-    case 7: pv_dispatch_g<7>(vg, img, lane, pb, o, bz, lmtab); break;
-    default: pv_dispatch_g<8>(vg, img, lane, pb, o, bz, lmtab); break;
-  }
-}
-
-// 128-point FWHT of each of `rows` rows of x (row stride 128), strides 1..64
-__device__ void fwht_smem(float* x, int rows) {
-  for (int lh = 0; lh < 7; ++lh) {
-    const int h = 1 << lh;
-    for (int p = threadIdx.x; p < rows * 64; p += blockDim.x) {
-      const int row = p >> 6, pi = p & 63;
-      const int i = ((pi >> lh) << (lh + 1)) | (pi & (h - 1));
-      float* r = x + row * kD;
-      const float a = r[i], b = r[i + h];
-      r[i] = a + b;
-      r[i + h] = a - b;
-    }
-    __syncthreads();
-  }
-}
-
-// Issue the cp.async copies of one ring entry (the K or V image of one
-// block, `bytes` long, at `src`) into the slot at shared address `dst`; one
-// commit group per entry (empty when there is nothing left, so the group
-// count stays uniform).
-__device__ __forceinline__ void issue_entry(bool live, int lane, uint32_t dst, const uint8_t* src,
-                                            int bytes) {
-  if (live) {
-    const int chunks = bytes >> 4;
-    for (int ch = lane; ch < chunks; ch += 32) cp_async16(dst + 16 * ch, src + 16 * ch);
-  }
-  cp_async_commit();
-}
-
-// Per-warp streaming state: the warp's blocks are blk_first, blk_first + 4,
-// ... of one (batch, kv head) K and V stream; ring entry e is the K image
-// (e even) or V image (e odd) of the warp's block e / 2.
-struct WarpStream {
-  const uint8_t* kwarp;   // K image of the warp's first block
-  const uint8_t* vwarp;
-  uint8_t* ring_ptr;      // this warp's ring of slots
-  uint32_t ring;          // its shared-memory address
-  int lane, nb;
-  bool merged;            // g <= 4: hi and lo q operands share one MMA
-  uint32_t mneg;          // merged: fp16x2 -1 on the lanes that carry lo (gid >= 4), else -0
-};
-
-// online-softmax state of one warp: o^T accumulators and per-column max/sum
-struct SoftmaxAcc {
-  float o[8][4];
-  float bz[2][4];   // per-token V zero-point sums: rows gid -> groups 0/2, rows gid+8 -> 1/3
-  float m0, m1, l0, l1;
-};
-
-// softmax of one block's scores (log2 units) into the accumulator; returns
-// the B fragments of P^T. The running max only moves when a block max
-// exceeds it by more than 8, so p <= 2^8 and rescaling is rare.
-__device__ __forceinline__ void softmax_block(float (&s)[2][4], SoftmaxAcc& acc,
-                                              uint32_t (&pb)[2][2]) {
-  // s holds score - running max (log2 units). Each lane checks its own
-  // values; only when one exceeds the bound is the column max reduced across
-  // the lanes and the running max moved (rare), so p <= 2^8 always.
-  float bm0 = fmaxf(fmaxf(s[0][0], s[0][2]), fmaxf(s[1][0], s[1][2]));
-  float bm1 = fmaxf(fmaxf(s[0][1], s[0][3]), fmaxf(s[1][1], s[1][3]));
-  const bool first = acc.m0 == -INFINITY;      // the warp's first block: set the max
-  if (__any_sync(0xffffffffu, first || bm0 > 8.0f || bm1 > 8.0f)) {
-#pragma unroll
-    for (int off = 4; off <= 16; off <<= 1) {
-      bm0 = fmaxf(bm0, __shfl_xor_sync(0xffffffffu, bm0, off));
-      bm1 = fmaxf(bm1, __shfl_xor_sync(0xffffffffu, bm1, off));
-    }
-    // first block: max = block max (s holds raw scores); later: the max moves
-    // up by d = max(block max - m, 0) and the state is scaled by 2^-d
-    float d0, d1, al0, al1;
-    if (first) {
-      d0 = bm0;
-      d1 = bm1;
-      al0 = al1 = 0.0f;
-      acc.m0 = bm0;
-      acc.m1 = bm1;
-    } else {
-      d0 = fmaxf(bm0, 0.0f);
-      d1 = fmaxf(bm1, 0.0f);
-      al0 = fast_exp2(-d0);
-      al1 = fast_exp2(-d1);
-      acc.m0 += d0;
-      acc.m1 += d1;
-    }
-#pragma unroll
-    for (int mt = 0; mt < 2; ++mt) {
-      s[mt][0] -= d0;
-      s[mt][1] -= d1;
-      s[mt][2] -= d0;
-      s[mt][3] -= d1;
-    }
-    acc.l0 *= al0;
-    acc.l1 *= al1;
-#pragma unroll
-    for (int mt = 0; mt < 8; ++mt) {
-      acc.o[mt][0] *= al0;
-      acc.o[mt][1] *= al1;
-      acc.o[mt][2] *= al0;
-      acc.o[mt][3] *= al1;
-    }
-#pragma unroll
-    for (int gp = 0; gp < 2; ++gp) {
-      acc.bz[gp][0] *= al0;
-      acc.bz[gp][1] *= al1;
-      acc.bz[gp][2] *= al0;
-      acc.bz[gp][3] *= al1;
-    }
-  }
-  float p[2][4];
-#pragma unroll
-  for (int mt = 0; mt < 2; ++mt)
-#pragma unroll
-    for (int r = 0; r < 4; ++r) p[mt][r] = fast_exp2(s[mt][r]);
-  acc.l0 += (p[0][0] + p[0][2]) + (p[1][0] + p[1][2]);
-  acc.l1 += (p[0][1] + p[0][3]) + (p[1][1] + p[1][3]);
-#pragma unroll
-  for (int ks = 0; ks < 2; ++ks) {
-    pb[ks][0] = movmatrix_trans(pack_f16x2(p[ks][0], p[ks][1]));
-    pb[ks][1] = movmatrix_trans(pack_f16x2(p[ks][2], p[ks][3]));
-  }
-}
-
-// ---- streaming with widths and groupings fixed at compile time: slot sizes,
-// slot counts, copy counts and the wait depth are constants, and the fp16
-// constants of the code extraction stay in registers across the loop.
-template <int BK, int BV>
-struct Ring {
-  static constexpr int kSK = 512 * (BK + 1), kSV = 512 * (BV + 1);
-  static constexpr int kSlot = kSK > kSV ? kSK : kSV;
-  static constexpr int kRaw = kRingBytes / kSlot;
-  static constexpr int kSlots = kRaw > kMaxSlots ? kMaxSlots : kRaw;
-};
-
-template <int BK, int BV>
-__device__ __forceinline__ void issue_static(const WarpStream& ws, int e, int slot) {
-  using R = Ring<BK, BV>;
-  if (e < 2 * ws.nb) {
-    const int i = e >> 1;
-    const uint32_t dst = ws.ring + slot * R::kSlot;
-    if ((e & 1) == 0) {
-      const uint8_t* src = ws.kwarp + i * (kWarps * R::kSK);
-#pragma unroll
-      for (int c = 0; c < R::kSK / 512; ++c) cp_async16(dst + 16 * (ws.lane + 32 * c), src + 16 * (ws.lane + 32 * c));
-    } else {
-      const uint8_t* src = ws.vwarp + i * (kWarps * R::kSV);
-#pragma unroll
-      for (int c = 0; c < R::kSV / 512; ++c) cp_async16(dst + 16 * (ws.lane + 32 * c), src + 16 * (ws.lane + 32 * c));
-    }
-  }
-  cp_async_commit();
-}
-
-template <int BK, int BV>
-__device__ __forceinline__ void prologue_static(const WarpStream& ws) {
-#pragma unroll
-  for (int e = 0; e < Ring<BK, BV>::kSlots - 1; ++e) issue_static<BK, BV>(ws, e, e);
-}
-
-template <int BK, int KG, int BV, int VG, bool MERGED>
-__device__ __forceinline__ void blocks_static(const WarpStream& ws, const uint8_t* qtab, float qsc,
-                                              SoftmaxAcc& acc) {
-  using R = Ring<BK, BV>;
-  constexpr int NS = R::kSlots;
-  int use = 0, iss = NS - 1;          // slot of the next entry to use / to issue
-  for (int i = 0; i < ws.nb; ++i) {
-    issue_static<BK, BV>(ws, 2 * i + NS - 1, iss);
-    iss = iss + 1 == NS ? 0 : iss + 1;
-    cp_async_wait<NS - 1>();
-    __syncwarp();
-    float s[2][4];
-    qk_block<BK, KG, MERGED>(ws.ring_ptr + use * R::kSlot, ws.lane, qtab, qsc,
-                     acc.m0 == -INFINITY ? 0.0f : acc.m0, acc.m1 == -INFINITY ? 0.0f : acc.m1,
-                     ws.mneg, s);
-    __syncwarp();
-    use = use + 1 == NS ? 0 : use + 1;
-    uint32_t pb[2][2];
-    softmax_block(s, acc, pb);
-    issue_static<BK, BV>(ws, 2 * i + NS, iss);
-    iss = iss + 1 == NS ? 0 : iss + 1;
-    cp_async_wait<NS - 1>();
-    __syncwarp();
-    pv_block<BV, VG>(ws.ring_ptr + use * R::kSlot, ws.lane, pb, acc.o, acc.bz);
-    __syncwarp();
-    use = use + 1 == NS ? 0 : use + 1;
-  }
-  cp_async_wait<0>();
-}
-
-// ---- streaming with runtime widths/groupings (every other combination)
-struct DynRing {
-  int bK, bV, kg, vg, sK, sV, slot, ns;
-  const uint16_t* lmK;       // Lloyd-Max codebook of the key / value width (null: none)
-  const uint16_t* lmV;
-};
-
-__device__ __forceinline__ void issue_dyn(const WarpStream& ws, const DynRing& r, int e, int slot) {
-  const int i = e >> 1;
-  const bool isK = (e & 1) == 0;
-  issue_entry(e < 2 * ws.nb, ws.lane, ws.ring + slot * r.slot,
-              isK ? ws.kwarp + i * (kWarps * r.sK) : ws.vwarp + i * (kWarps * r.sV), isK ? r.sK : r.sV);
-}
-
-__device__ __forceinline__ void prologue_dyn(const WarpStream& ws, const DynRing& r) {
-  for (int e = 0; e < r.ns - 1; ++e) issue_dyn(ws, r, e, e);
-}
-
-__device__ __forceinline__ void blocks_dyn(const WarpStream& ws, const DynRing& r,
-                                           const uint8_t* qtab, float qsc, SoftmaxAcc& acc) {
-  int use = 0, iss = r.ns - 1;
-  for (int i = 0; i < ws.nb; ++i) {
-    issue_dyn(ws, r, 2 * i + r.ns - 1, iss);
-    iss = iss + 1 == r.ns ? 0 : iss + 1;
-    cp_async_wait_dyn(r.ns - 1);
-    __syncwarp();
-    float s[2][4];
-    qk_dispatch(r.bK, r.kg, ws.ring_ptr + use * r.slot, ws.lane, qtab, qsc,
-                acc.m0 == -INFINITY ? 0.0f : acc.m0, acc.m1 == -INFINITY ? 0.0f : acc.m1, s, r.lmK);
-    __syncwarp();
-    use = use + 1 == r.ns ? 0 : use + 1;
-    uint32_t pb[2][2];
-    softmax_block(s, acc, pb);
-    issue_dyn(ws, r, 2 * i + r.ns, iss);
-    iss = iss + 1 == r.ns ? 0 : iss + 1;
-    cp_async_wait_dyn(r.ns - 1);
-    __syncwarp();
-    pv_dispatch(r.bV, r.vg, ws.ring_ptr + use * r.slot, ws.lane, pb, acc.o, acc.bz, r.lmV);
-    __syncwarp();
-    use = use + 1 == r.ns ? 0 : use + 1;
-  }
-  cp_async_wait<0>();
-}
-
-// Key of the compile-time path, or -1: keys 0..15 for the KIVI layout
-// (per-channel K, per-token V) at widths {2, 3, 4, 8}; keys 16..24 for
-// per-token K and V (the rotated caches) at widths {3, 4, 5}, the widths an
-// allocation at about 4 bits per code mostly gives.
-__device__ __forceinline__ int fast_key(int bK, int bV, int kg, int vg) {
-  if (kg == RQ_PER_CHANNEL && vg == RQ_PER_TOKEN) {
-    auto idx = [](int b) { return b == 2 ? 0 : b == 3 ? 1 : b == 4 ? 2 : b == 8 ? 3 : -1; };
-    const int ik = idx(bK), iv = idx(bV);
-    return (ik < 0 || iv < 0) ? -1 : 4 * ik + iv;
-  }
-  if (kg == RQ_PER_TOKEN && vg == RQ_PER_TOKEN) {
-    auto idx = [](int b) { return b >= 3 && b <= 5 ? b - 3 : -1; };
-    const int ik = idx(bK), iv = idx(bV);
-    return (ik < 0 || iv < 0) ? -1 : 16 + 3 * ik + iv;
-  }
-  return -1;
-}
-
-#define RQ_FAST_CASES(X) \
-  X(0, 2, 2) X(1, 2, 3) X(2, 2, 4) X(3, 2, 8) X(4, 3, 2) X(5, 3, 3) X(6, 3, 4) X(7, 3, 8) \
-  X(8, 4, 2) X(9, 4, 3) X(10, 4, 4) X(11, 4, 8) X(12, 8, 2) X(13, 8, 3) X(14, 8, 4) X(15, 8, 8)
-#define RQ_TOKEN_CASES(X) \
-  X(16, 3, 3) X(17, 3, 4) X(18, 3, 5) X(19, 4, 3) X(20, 4, 4) X(21, 4, 5) X(22, 5, 3) X(23, 5, 4) \
-  X(24, 5, 5)
-
-template <typename T>
-__global__ void __launch_bounds__(kThreads, RQ_DECODE_MIN_BLOCKS) decode_split_kernel(DecodeArgs a) {
-  extern __shared__ __align__(16) unsigned char smem_raw[];
-  float* qs = reinterpret_cast<float*>(smem_raw);                  // [8][128]
-  uint8_t* rings = smem_raw + kQBytes;
-  __shared__ float red_m[kWarps][kMaxHeads];
-  __shared__ float red_l[kWarps][kMaxHeads];
-  __shared__ uint16_t lmtab[2][256];                // Lloyd-Max codebooks of this head's widths
-  const int split = blockIdx.x, h = blockIdx.y, batch = blockIdx.z;
-  const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
-  const int gid = lane >> 2, tig = lane & 3;
-
-  const int bK = a.bits[(a.layer * a.H + h) * 2 + 0];
-  const int bV = a.bits[(a.layer * a.H + h) * 2 + 1];
-  const bool valid = bK >= 1 && bK <= 8 && bV >= 1 && bV <= 8;
-  if (!valid && threadIdx.x == 0) set_status(a.status, RQ_STATUS_BAD_BITS);
-  const uint64_t* offp =
-      a.offsets + ((static_cast<long long>(a.layer) * a.B + batch) * a.H + h) * 2;
-  const uint8_t* kbase = a.packed + (valid ? offp[0] : 0);
-  const uint8_t* vbase = a.packed + (valid ? offp[1] : 0);
-  DynRing dr;
-  dr.bK = bK;
-  dr.bV = bV;
-  dr.kg = a.kg;
-  dr.vg = a.vg;
-  const bool lmk = valid && a.kq == RQ_LLOYDMAX, lmv = valid && a.vq == RQ_LLOYDMAX;
-  for (int i = threadIdx.x; i < 256; i += kThreads) {
-    if (lmk && i < (1 << bK)) lmtab[0][i] = a.lm.lv[lm_offset(bK) + i];
-    if (lmv && i < (1 << bV)) lmtab[1][i] = a.lm.lv[lm_offset(bV) + i];
-  }
-  dr.lmK = lmk ? lmtab[0] : nullptr;               // read after the barriers of the q prologue
-  dr.lmV = lmv ? lmtab[1] : nullptr;
-  dr.sK = 512 * (bK + 1);
-  dr.sV = 512 * (bV + 1);
-  dr.slot = max(dr.sK, dr.sV);
-  dr.ns = valid ? min(kMaxSlots, kRingBytes / dr.slot) : 2;
-  const int blk0 = split * a.bps;
-  const int blk1 = min(a.nblk, blk0 + a.bps);
-  const int blk_first = blk0 + warp;
-  WarpStream ws;
-  ws.lane = lane;
-  ws.nb = valid && blk_first < blk1 ? (blk1 - blk_first + kWarps - 1) / kWarps : 0;
-  ws.ring_ptr = rings + warp * kRingBytes;
-  ws.ring = smem_u32(ws.ring_ptr);
-  ws.kwarp = kbase + static_cast<size_t>(blk_first) * dr.sK;
-  ws.vwarp = vbase + static_cast<size_t>(blk_first) * dr.sV;
-  const int key = valid && a.kq != RQ_LLOYDMAX && a.vq != RQ_LLOYDMAX ? fast_key(bK, bV, a.kg, a.vg) : -1;
-  ws.merged = a.g <= kMaxHeads / 2 && key >= 0 && key < 16;   // the compile-time KIVI paths only
-  ws.mneg = ws.merged && gid >= kMaxHeads / 2 ? 0xBC00BC00u : 0x80008000u;
-
-  // start streaming the first entries before the q prologue
-  switch (key) {
-#define RQ_PRO(k, BK, BV) case k: prologue_static<BK, BV>(ws); break;
-    RQ_FAST_CASES(RQ_PRO)
-    RQ_TOKEN_CASES(RQ_PRO)
-#undef RQ_PRO
-    default: prologue_dyn(ws, dr); break;
-  }
-
-  // q of the g query heads of this kv head (rows >= g are zero), rotated
-  // into the cache's domain when the cache is Hadamard-rotated
-  const T* qp = static_cast<const T*>(a.q) + (static_cast<long long>(batch) * a.Hq +
-                                              static_cast<long long>(h) * a.g) * kD;
-  for (int idx = threadIdx.x; idx < kMaxHeads * kD; idx += kThreads) {
-    const int n = idx >> 7, d = idx & 127;
-    float x = 0.0f;
-    if (n < a.g) {
-      x = to_f32<T>(qp[n * kD + d]);
-      if (a.hadamard && a.signs && a.signs[d] < 0) x = -x;
-    }
-    qs[idx] = x;
-  }
-  __syncthreads();
-  if (a.hadamard) fwht_smem(qs, kMaxHeads);
-  // q enters the MMAs scaled by a power of two only (no rounding beyond its
-  // fp16 conversion); the rest of the softmax scale 1/sqrt(128) * log2(e) is
-  // applied to the fp32 scores (log2 units).
-  // K unit u, pair x of lane (gid, tig) is channels 32u + 8tig + 2x (+1);
-  // qf carries the per-channel-key codes' 2^-E(x) as well.
-  // q is scaled by a power of two only (exact: headroom for q . scale in
-  // fp16), the rest of the softmax scale is applied in fp32
-  const float qpow = a.hadamard ? 0.015625f : 0.125f;
-  const float qscale = kLog2e * kInvSqrt128 * (a.hadamard ? kInvSqrt128 : 1.0f) / qpow;
-  uint32_t qb[4][4], qf[4][4];
-  uint32_t ef[4];
-#pragma unroll
-  for (int x = 0; x < 4; ++x) ef[x] = pow2_neg_h2(a.kg == RQ_PER_CHANNEL && valid ? fmt::exponent(bK, x) : 0);
-  if (warp == 0) {
-    // merged (g <= 4): columns 4..7 repeat heads 0..3 (they carry lo in the
-    // scores MMA; elsewhere they give duplicate results that are not stored)
-    const int qrow = ws.merged ? (gid & 3) : gid;
-#pragma unroll
-    for (int u = 0; u < 4; ++u)
-#pragma unroll
-      for (int x = 0; x < 4; ++x) {
-        const float* qr = qs + qrow * kD + 32 * u + 8 * tig + 2 * x;
-        qb[u][x] = pack_f16x2(qr[0] * qpow, qr[1] * qpow);
-        qf[u][x] = hmul2u(qb[u][x], ef[x]);
-      }
-  }
-  // per-token keys: sum over each 32-channel group of the q operand the MMA
-  // sees (fp16 q scaled by qpow), [group G = lane / 8][head n = lane % 8]
-  float qgsum = 0.0f;
-  if (warp == 0 && a.kg == RQ_PER_TOKEN) {
-    const float* qr = qs + (lane & 7) * kD + 32 * (lane >> 3);
-    for (int c = 0; c < 32; ++c) qgsum += __half2float(__float2half_rn(qr[c] * qpow));
-  }
-  __syncthreads();                  // qs is read; its space becomes the q operand table
-  uint8_t* qtab = smem_raw;
-  if (warp == 0) {
-#pragma unroll
-    for (int u = 0; u < 4; ++u) {
-      *reinterpret_cast<uint4*>(qtab + 16 * (32 * u + lane)) = make_uint4(qb[u][0], qb[u][1], qb[u][2], qb[u][3]);
-      if (a.kg == RQ_PER_CHANNEL)
-        *reinterpret_cast<uint4*>(qtab + 2048 + 16 * (32 * u + lane)) =
-            make_uint4(qf[u][0], qf[u][1], qf[u][2], qf[u][3]);
-    }
-    if (a.kg == RQ_PER_TOKEN) reinterpret_cast<float*>(qtab + 2048)[lane] = qgsum;   // [G][n]
-  }
-  __syncthreads();
-
-  SoftmaxAcc acc;
-#pragma unroll
-  for (int mt = 0; mt < 8; ++mt)
-#pragma unroll
-    for (int r = 0; r < 4; ++r) acc.o[mt][r] = 0.0f;
-#pragma unroll
-  for (int gp = 0; gp < 2; ++gp)
-#pragma unroll
-    for (int r = 0; r < 4; ++r) acc.bz[gp][r] = 0.0f;
-  acc.m0 = acc.m1 = -INFINITY;
-  acc.l0 = acc.l1 = 0.0f;
-
-  switch (key) {
-#define RQ_BLK(k, BK, BV)                                                                        \
-  case k:                                                                                        \
-    if (ws.merged) blocks_static<BK, RQ_PER_CHANNEL, BV, RQ_PER_TOKEN, true>(ws, qtab, qscale, acc); \
-    else blocks_static<BK, RQ_PER_CHANNEL, BV, RQ_PER_TOKEN, false>(ws, qtab, qscale, acc);        \
-    break;
-    RQ_FAST_CASES(RQ_BLK)
-#undef RQ_BLK
-#define RQ_TBLK(k, BK, BV)                                                                  \
-  case k: blocks_static<BK, RQ_PER_TOKEN, BV, RQ_PER_TOKEN, false>(ws, qtab, qscale, acc); break;
-    RQ_TOKEN_CASES(RQ_TBLK)
-#undef RQ_TBLK
-    default: blocks_dyn(ws, dr, qtab, qscale, acc); break;
-  }
-  // the merge kernel may be scheduled now; it waits for this grid to finish
-  asm volatile("griddepcontrol.launch_dependents;\n" ::: "memory");
-  if (a.vg == RQ_PER_TOKEN && valid) {
-    // rows of m-tile mt are classes x = 2 (mt & 1) + r of unit mt / 2: undo
-    // their codes' 2^(E(x) - 24), then add group G's zero-point sum (rows gid
-    // of bz[G / 2] for even G, rows gid + 8 for odd G)
-    float rf[4];
-#pragma unroll
-    for (int x = 0; x < 4; ++x)       // 2^(24 - E); 1 for codebook levels
-      rf[x] = lmv ? 1.0f : __int_as_float((127 + 24 - fmt::exponent(bV, x)) << 23);
-#pragma unroll
-    for (int mt = 0; mt < 8; ++mt) {
-      const int G = mt >> 1;
-      const float z0 = (G & 1) ? acc.bz[G >> 1][2] : acc.bz[G >> 1][0];
-      const float z1 = (G & 1) ? acc.bz[G >> 1][3] : acc.bz[G >> 1][1];
-      const float f0 = rf[2 * (mt & 1)], f1 = rf[2 * (mt & 1) + 1];
-      acc.o[mt][0] = __fmaf_rn(acc.o[mt][0], f0, z0);
-      acc.o[mt][1] = __fmaf_rn(acc.o[mt][1], f0, z1);
-      acc.o[mt][2] = __fmaf_rn(acc.o[mt][2], f1, z0);
-      acc.o[mt][3] = __fmaf_rn(acc.o[mt][3], f1, z1);
-    }
-  }
-  float m0 = acc.m0, m1 = acc.m1, l0 = acc.l0, l1 = acc.l1;
-#pragma unroll
-  for (int off = 4; off <= 16; off <<= 1) {
-    l0 += __shfl_xor_sync(0xffffffffu, l0, off);
-    l1 += __shfl_xor_sync(0xffffffffu, l1, off);
-  }
-  // merge the four warps (log-sum-exp), one partial record per query head;
-  // the merge buffer reuses the rings
-  __syncthreads();
-  float* red_o = reinterpret_cast<float*>(rings);   // [warp][head][channel]
-#pragma unroll
-  for (int mt = 0; mt < 8; ++mt) {
-    // row r of m-tile mt is channel 32 (mt / 2) + 4 gid + 2 (mt & 1) + r
-    float* r0 = red_o + (warp * kMaxHeads + 2 * tig) * kD;
-    float* r1 = r0 + kD;
-    const int ch = 32 * (mt >> 1) + 4 * gid + 2 * (mt & 1);
-    r0[ch] = acc.o[mt][0];
-    r1[ch] = acc.o[mt][1];
-    r0[ch + 1] = acc.o[mt][2];
-    r1[ch + 1] = acc.o[mt][3];
-  }
-  if (gid == 0) {
-    red_m[warp][2 * tig] = m0;
-    red_m[warp][2 * tig + 1] = m1;
-    red_l[warp][2 * tig] = l0;
-    red_l[warp][2 * tig + 1] = l1;
-  }
-  __syncthreads();
-  const int d = threadIdx.x;
-  for (int n = 0; n < a.g; ++n) {
-    float M = -INFINITY;
-#pragma unroll
-    for (int w = 0; w < kWarps; ++w) M = fmaxf(M, red_m[w][n]);
-    float osum = 0.0f, lsum = 0.0f;
-#pragma unroll
-    for (int w = 0; w < kWarps; ++w) {
-      const float mw = red_m[w][n];
-      const float sc = (mw == -INFINITY) ? 0.0f : exp2f(mw - M);
-      osum += sc * red_o[(w * kMaxHeads + n) * kD + d];
-      lsum += sc * red_l[w][n];
-    }
-    float* dst = a.partial + ((static_cast<long long>(batch) * a.Hq + h * a.g + n) * a.splits + split) * kPart;
-    dst[d] = osum;
-    if (d == 0) {
-      dst[kD] = M;
-      dst[kD + 1] = lsum;
-    }
-  }
-}
-
-// ------------------------------------------------------------ split merge ----
-// out_n = sum_s 2^(m_ns - M_n) o_ns / sum_s 2^(m_ns - M_n) l_ns for the g
-// query rows n of one (batch, kv head), rotated back (o R^T =
-// FWHT(o) / sqrt(128) * signs) for a Hadamard cache. A CTA owns one (batch,
-// kv head) and 128 / CQ channels of its rows (the whole row when CQ = 1, as
-// the rotation needs). It is launched as a programmatic dependent of the
-// split kernel and waits for it on entry. Records are pulled into shared
-// memory with cp.async, a chunk of splits at a time (one round trip per
-// chunk), and merged there with a running max per row.
-constexpr int kMergeSmem = 64 * 1024;
-
-// The unquantized residual tokens (decode-time append) of one (batch, kv
-// head): their exact fp32 attention record (m, l, o) for the g query rows
-// starts the running merge. Scores use the unrotated q and keys (a rotation
-// leaves dot products unchanged); the value sum is rotated into the cache's
-// domain when the cache is rotated. Whole CTA; sm: 64 KB of shared memory.
-template <int CQ, typename T>
-__device__ __forceinline__ void residual_record(const T* q, const T* res, int R, int g,
-                                                const int8_t* signs, int hadamard, int part,
-                                                float* sm, float* y, float* run_m, float* run_l,
-                                                float (&acc)[kMaxHeads * (kD / CQ) / kThreads]) {
-  constexpr int CW = kD / CQ;
-  constexpr int PAIRS = kMaxHeads * CW / kThreads;
-  const int tid = threadIdx.x;
-  float* qf = sm;                                  // [g][128], scaled to log2 units
-  float* kr = qf + kMaxHeads * kD;                 // [32][129]
-  float* vr = kr + kTile * (kD + 1);               // [32][128]
-  float* sc = vr + kTile * kD;                     // [g][32]
-  const float qscale = kLog2e * kInvSqrt128;
-  for (int n = 0; n < g; ++n) qf[n * kD + tid] = to_f32<T>(q[n * kD + tid]) * qscale;
-  for (int t = 0; t < R; ++t) {
-    kr[t * (kD + 1) + tid] = to_f32<T>(res[t * kD + tid]);
-    vr[t * kD + tid] = to_f32<T>(res[(kTile + t) * kD + tid]);
-  }
-  __syncthreads();
-  for (int idx = tid; idx < g * R; idx += kThreads) {
-    const int n = idx / R, t = idx % R;
-    float sdot = 0.0f;
-    for (int c = 0; c < kD; ++c) sdot = __fmaf_rn(qf[n * kD + c], kr[t * (kD + 1) + c], sdot);
-    sc[n * kTile + t] = sdot;
-  }
-  __syncthreads();
-#pragma unroll
-  for (int k = 0; k < PAIRS; ++k) {
-    const int pi = tid + kThreads * k, n = pi / CW, c = pi % CW;
-    if (n < g) {
-      float m = -INFINITY;
-      for (int t = 0; t < R; ++t) m = fmaxf(m, sc[n * kTile + t]);
-      float l = 0.0f, o = 0.0f;
-      for (int t = 0; t < R; ++t) {
-        const float p = exp2f(sc[n * kTile + t] - m);
-        l += p;
-        o = __fmaf_rn(p, vr[t * kD + part * CW + c], o);
-      }
-      acc[k] = o;
-      if (c == 0) {
-        run_m[n] = m;
-        run_l[n] = l;
-      }
-    }
-  }
-  if (CQ == 1 && hadamard) {                       // o R = FWHT(o * signs) / sqrt(128)
-#pragma unroll
-    for (int k = 0; k < PAIRS; ++k) {
-      const int pi = tid + kThreads * k, c = pi % CW;
-      if (pi / CW < g) y[pi] = (signs && signs[c] < 0) ? -acc[k] : acc[k];
-    }
-    __syncthreads();
-    fwht_smem(y, g);
-#pragma unroll
-    for (int k = 0; k < PAIRS; ++k) {
-      const int pi = tid + kThreads * k;
-      if (pi / CW < g) acc[k] = y[pi] * kInvSqrt128;
-    }
-  }
-  __syncthreads();
-}
-
-template <int CQ, typename T>
-__global__ void __launch_bounds__(kThreads) decode_merge_kernel(const float* partial, float* out,
-                                                                const int8_t* signs,
-                                                                uint32_t* status, int Hq, int H,
-                                                                int g, int splits, int hadamard,
-                                                                const T* q, const T* residual,
-                                                                int R) {
-  asm volatile("griddepcontrol.wait;\n" ::: "memory");
-  constexpr int CW = kD / CQ;          // channels of this CTA
-  constexpr int CH = CW / 4;           // 16-byte pieces of a record's o slice
-  constexpr int SLOT = CH + 1;         // pieces per (row, split): o slice, then (m, l, pad)
-  constexpr int PAIRS = kMaxHeads * CW / kThreads;   // (row, channel) pairs per thread, at most
-  extern __shared__ float4 msm[];
-  __shared__ float wgt[kMaxHeads][64];
-  __shared__ float run_m[kMaxHeads], run_l[kMaxHeads], run_scale[kMaxHeads];
-  __shared__ float y[kMaxHeads * kD];
-  const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
-  const int batch = blockIdx.x / H, h = blockIdx.x % H, part = blockIdx.y;
-  const long long row0 = static_cast<long long>(batch) * Hq + h * g;
-  const long long rstride = static_cast<long long>(splits) * kPart;
-  const float* p = partial + row0 * rstride + part * CW;     // o slice of row 0, split 0
-  const float* pml = partial + row0 * rstride + kD;           // (m, l) of row 0, split 0
-  // splits per chunk: shared budget, and at most 64 (one weight per lane pair)
-  const int cs_max = min(64, kMergeSmem / (g * SLOT * 16));
-  if (tid < kMaxHeads) {
-    run_m[tid] = -INFINITY;
-    run_l[tid] = 0.0f;
-  }
-  float acc[PAIRS];
-#pragma unroll
-  for (int k = 0; k < PAIRS; ++k) acc[k] = 0.0f;
-  __syncthreads();
-  if (R > 0)
-    residual_record<CQ, T>(q + row0 * kD, residual + (static_cast<long long>(batch) * H + h) * 2 * kTile * kD,
-                           R, g, signs, hadamard, part, reinterpret_cast<float*>(msm), y, run_m, run_l,
-                           acc);
-  const uint32_t sbase = static_cast<uint32_t>(__cvta_generic_to_shared(msm));
-
-  for (int c0 = 0; c0 < splits; c0 += cs_max) {
-    const int cs = min(cs_max, splits - c0);
-    // piece (n, s, i): i < CH the o slice, i == CH (m, l, pad, pad)
-    const int npieces = g * cs * SLOT;
-    for (int x = tid; x < npieces; x += kThreads) {
-      const int i = x % SLOT, ns = x / SLOT, n = ns / cs, sl = ns % cs;
-      const float* src = (i < CH ? p + 4 * i : pml) + n * rstride + static_cast<long long>(c0 + sl) * kPart;
-      asm volatile("cp.async.cg.shared.global [%0], [%1], 16;\n" ::"r"(sbase + 16 * x), "l"(src));
-    }
-    asm volatile("cp.async.commit_group;\n" ::);
-    asm volatile("cp.async.wait_group 0;\n" ::);
-    __syncthreads();
-    // warp w: rows w, w + 4; lanes over the chunk's splits (two per lane)
-#pragma unroll
-    for (int k = 0; k < 2; ++k) {
-      const int n = warp + kWarps * k;
-      if (n < g) {
-        float mv[2], lv[2], mx = -INFINITY;
-#pragma unroll
-        for (int r = 0; r < 2; ++r) {
-          const int sl = lane + 32 * r;
-          mv[r] = -INFINITY;
-          lv[r] = 0.0f;
-          if (sl < cs) {
-            const float4 ml = msm[(n * cs + sl) * SLOT + CH];
-            mv[r] = ml.x;
-            lv[r] = ml.y;
-          }
-          mx = fmaxf(mx, mv[r]);
-        }
-#pragma unroll
-        for (int off = 16; off >= 1; off >>= 1) mx = fmaxf(mx, __shfl_xor_sync(0xffffffffu, mx, off));
-        const float mold = run_m[n];
-        const float mnew = fmaxf(mold, mx);
-        float l = 0.0f;
-#pragma unroll
-        for (int r = 0; r < 2; ++r) {
-          const int sl = lane + 32 * r;
-          const float wv = (mv[r] == -INFINITY) ? 0.0f : exp2f(mv[r] - mnew);
-          if (sl < cs) wgt[n][sl] = wv;
-          l += wv * lv[r];
-        }
-#pragma unroll
-        for (int off = 16; off >= 1; off >>= 1) l += __shfl_xor_sync(0xffffffffu, l, off);
-        __syncwarp();
-        if (lane == 0) {
-          const float sc = (mold == -INFINITY) ? 0.0f : exp2f(mold - mnew);
-          run_scale[n] = sc;
-          run_l[n] = run_l[n] * sc + l;
-          run_m[n] = mnew;
-        }
-      }
-    }
-    __syncthreads();
-#pragma unroll
-    for (int k = 0; k < PAIRS; ++k) {
-      const int pi = tid + kThreads * k, n = pi / CW, c = pi % CW;
-      if (n < g) {
-        float a = acc[k] * run_scale[n];
-        const float* o = reinterpret_cast<const float*>(msm + n * cs * SLOT) + c;
-        const float* wn = wgt[n];
-#pragma unroll 4
-        for (int sl = 0; sl < cs; ++sl) a += wn[sl] * o[sl * SLOT * 4];
-        acc[k] = a;
-      }
-    }
-    __syncthreads();
-  }
-#pragma unroll
-  for (int k = 0; k < PAIRS; ++k) {
-    const int n = (tid + kThreads * k) / CW;
-    if (n < g) {
-      const float L = run_l[n];
-      float v = L > 0.0f ? acc[k] / L : 0.0f;
-      if (!(L > 0.0f) || !isfinite(v)) {
-        set_status(status, RQ_STATUS_NUMERIC);
-        if (!isfinite(v)) v = 0.0f;
-      }
-      acc[k] = v;
-    }
-  }
-  if (CQ == 1 && hadamard) {
-#pragma unroll
-    for (int k = 0; k < PAIRS; ++k) {
-      const int pi = tid + kThreads * k;
-      if (pi / CW < g) y[pi] = acc[k];
-    }
-    __syncthreads();
-    fwht_smem(y, g);
-#pragma unroll
-    for (int k = 0; k < PAIRS; ++k) {
-      const int pi = tid + kThreads * k, c = pi % CW;
-      if (pi / CW < g) {
-        float v = y[pi] * kInvSqrt128;
-        if (signs && signs[c] < 0) v = -v;
-        acc[k] = v;
-      }
-    }
-  }
-#pragma unroll
-  for (int k = 0; k < PAIRS; ++k) {
-    const int pi = tid + kThreads * k, n = pi / CW, c = pi % CW;
-    if (n < g) out[(row0 + n) * kD + part * CW + c] = acc[k];
-  }
-}
+using dk::DecodeArgs;
+using dk::kMaxHeads;
+using dk::kPart;
 
 // Resident split-kernel CTAs per SM on the current device (cached per device).
 rq_status split_ctas_per_sm(int* per_sm) {
@@ -1218,15 +45,8 @@ rq_status split_ctas_per_sm(int* per_sm) {
       return RQ_OK;
     }
   }
-  auto kern = decode_split_kernel<__nv_bfloat16>;
-  if (cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, kSmemBytes) != cudaSuccess ||
-      cudaFuncSetAttribute(kern, cudaFuncAttributePreferredSharedMemoryCarveout,
-                           cudaSharedmemCarveoutMaxShared) != cudaSuccess)
-    return RQ_ERR_CUDA;
   int v = 0;
-  if (cudaOccupancyMaxActiveBlocksPerMultiprocessor(&v, kern, kThreads, kSmemBytes) != cudaSuccess)
-    return RQ_ERR_CUDA;
-  v = std::max(v, 1);
+  if (decode_split_ctas_per_sm(&v) != RQ_OK) return RQ_ERR_CUDA;
   if (dev >= 0 && dev < 64) cache[dev].store(v, std::memory_order_relaxed);
   *per_sm = v;
   return RQ_OK;
@@ -1305,54 +125,11 @@ void fill_args(DecodeArgs& a, const rq_cache_desc* desc, int32_t layer, const vo
   if (a.kq == RQ_LLOYDMAX || a.vq == RQ_LLOYDMAX) fill_lm_book(a.lm);
 }
 
-template <typename T>
-rq_status launch_split(const DecodeArgs& a, const dim3& grid, cudaStream_t s) {
-  auto kern = decode_split_kernel<T>;
-  if (cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, kSmemBytes) != cudaSuccess ||
-      cudaFuncSetAttribute(kern, cudaFuncAttributePreferredSharedMemoryCarveout,
-                           cudaSharedmemCarveoutMaxShared) != cudaSuccess)
-    return RQ_ERR_CUDA;
-  kern<<<grid, kThreads, kSmemBytes, s>>>(a);
-  return launch_status();
-}
-
-// split kernel, then the merge kernel as its programmatic dependent
-template <typename T>
-rq_status launch_merge(const DecodeArgs& a, const rq_cache_desc* desc, float* out,
-                       const void* res_layer, int R, cudaStream_t s) {
-  // a whole row per CTA for a rotated cache (the rotation mixes channels),
-  // a quarter of the channels otherwise (four times the CTAs)
-  const int cq = a.hadamard ? 1 : 4;
-  cudaLaunchConfig_t cfg = {};
-  cfg.gridDim = dim3(static_cast<unsigned>(desc->B * desc->H_kv), static_cast<unsigned>(cq));
-  cfg.blockDim = dim3(kThreads);
-  cfg.dynamicSmemBytes = kMergeSmem;
-  cfg.stream = s;
-  cudaLaunchAttribute attr[1];
-  attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
-  attr[0].val.programmaticStreamSerializationAllowed = 1;
-  cfg.attrs = attr;
-  cfg.numAttrs = 1;
-  auto kern = a.hadamard ? decode_merge_kernel<1, T> : decode_merge_kernel<4, T>;
-  if (cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, kMergeSmem) != cudaSuccess)
-    return RQ_ERR_CUDA;
-  if (cudaLaunchKernelEx(&cfg, kern, static_cast<const float*>(a.partial), out, a.signs, a.status,
-                         a.Hq, a.H, a.g, a.splits, a.hadamard, static_cast<const T*>(a.q),
-                         static_cast<const T*>(res_layer), R) != cudaSuccess)
-    return RQ_ERR_CUDA;
-  return launch_status();
-}
-
 // split kernel, then the merge kernel as its programmatic dependent
 rq_status launch_decode(const DecodeArgs& a, const rq_cache_desc* desc, float* out, cudaStream_t s,
                         const void* res_layer = nullptr, int R = 0) {
-  const dim3 grid(static_cast<unsigned>(a.splits), static_cast<unsigned>(desc->H_kv),
-                  static_cast<unsigned>(desc->B));
-  const bool f16 = desc->dtype == RQ_F16;
-  const rq_status st = f16 ? launch_split<__half>(a, grid, s) : launch_split<__nv_bfloat16>(a, grid, s);
-  if (st != RQ_OK) return st;
-  return f16 ? launch_merge<__half>(a, desc, out, res_layer, R, s)
-             : launch_merge<__nv_bfloat16>(a, desc, out, res_layer, R, s);
+  return desc->dtype == RQ_F16 ? launch_decode_f16(a, out, res_layer, R, s)
+                               : launch_decode_bf16(a, out, res_layer, R, s);
 }
 
 }  // namespace
@@ -1396,8 +173,9 @@ extern "C" rq_status rq_decode_attention(const rq_cache_desc* desc, int32_t laye
 // ---------------------------------------------------------------------------
 // Allocation-free decode: the split-K partials live in a fixed device array
 // of this library instead of a caller-supplied workspace, for callers that
-// cannot allocate (graph replays, foreign allocators, plugins handed only
-// their inputs and outputs). The array is shared by every call on a device.
+// cannot allocate (runtimes whose allocator belongs to someone else, plugins
+// handed only their inputs and outputs). The array is shared by every call
+// on a device.
 namespace rq {
 namespace {
 
@@ -1489,3 +267,4 @@ extern "C" rq_status rq_decode_attention_len(const rq_cache_desc* desc, int32_t 
             : nullptr;
   return launch_decode(a, desc, out, static_cast<cudaStream_t>(stream), res_layer, R);
 }
+

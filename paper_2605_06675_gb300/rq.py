@@ -245,9 +245,10 @@ def rq_decode_attention(desc, layer, q, packed, bits_dev, offsets_dev, signs, ou
 def rq_decode_attention_static(desc, layer, q, packed, bits_dev, offsets_dev, signs, out,
                                status=None, stream=None):
     """rq_decode_attention without a workspace argument: for callers that
-    cannot allocate device memory (graph replays, foreign allocators,
-    plugins). Uses librq's fixed RQ_STATIC_SCRATCH_BYTES device array, shared
-    by every call on the device, so concurrent calls on unordered streams race."""
+    cannot allocate device memory where they decode (runtimes whose allocator
+    belongs to someone else, plugins handed only their inputs and outputs).
+    Uses librq's fixed RQ_STATIC_SCRATCH_BYTES device array, shared by every
+    call on the device, so concurrent calls on unordered streams race."""
     _check("rq_decode_attention_static", lib().rq_decode_attention_static(
         ctypes.byref(desc), layer, _dp(q), _dp(packed), _dp(bits_dev), _dp(offsets_dev),
         _dp(signs), _dp(out), _dp(status), _stream(stream)))

@@ -321,3 +321,4 @@ def test_quantizer_argument_errors(rq):
         rq.rq_calibrate_distortion(x, 1, 0, False, None, mse, ws, k_quantizer=3)
     assert e.value.status == 1
 
+

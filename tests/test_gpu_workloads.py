@@ -85,3 +85,47 @@ def test_full_size_layer_sampled(rq, wl):
     assert torch.isfinite(out).all()
     del k, v
     torch.cuda.empty_cache()
+
+
+def test_llama3_bench_path_allocator_widths(rq):
+    """The bench's configuration as bench.py runs it, on one full-size layer:
+    calibrate on the workload's calibration sample, fit + allocate with the
+    library (bit-exact against the oracle's fit and allocation on the same
+    MSE), lay out every layer at the allocator's widths in a buffer of the
+    bench's capacity, quantize + decode the last layer, and compare every
+    (batch 0, kv head) stream and one kv head of every other batch with the
+    oracle: packed bytes bit-exact, attention within the tolerance."""
+    wl = LLAMA3_8B_32K
+    path = PackedKVPath(wl, DEV)
+    X = synth.calibration_sample(wl, device=DEV)
+    mse = path.calibrate(X).cpu().numpy()
+    n = X.shape[0]
+    w = synth.importances(n, wl.sigma_lnw, wl.seed)
+    bits, (_, _, _, J) = path.allocate(mse, w)
+    oa, ob, _ = ocalib.fit_distortion(mse, 2, 6, 0.96, np.arange(n) % 2)
+    obits, oJ = oalloc.allocate(w, oa, ob, wl.avg_bits, wl.allowed_mask)
+    assert list(bits.reshape(-1)) == obits and J == oJ
+    assert int(bits.sum()) == oalloc.budget(wl.avg_bits, n)
+    # the sweep on every 37th component against the oracle's
+    idx = np.arange(0, n, 37)
+    xs = to_np(X[torch.as_tensor(idx, device=X.device)])
+    ref_mse = ocalib.distortion_sweep(xs, [wl.k_grouping if i % 2 == 0 else wl.v_grouping
+                                           for i in idx])
+    assert (np.abs(mse[idx] - ref_mse) / ref_mse).max() < MSE_RTOL
+    del X
+    # capacity as bench.py sizes it: every stream at the widest allowed width
+    cap = wl.L * wl.B * wl.H_kv * 2 * (wl.S // 32) * 512 * (max(wl.allowed) + 1)
+    path.set_bits(bits, capacity=cap)
+    layer = wl.L - 1
+    k, v = synth.kv_layer(wl.B, wl.H_kv, wl.S, wl.dtype, wl.seed, layer, wl.value_dist, DEV)
+    q = synth.queries(wl.B, wl.H_q, wl.dtype, wl.seed, layer, DEV)
+    out = torch.empty((wl.B, wl.H_q, 128), dtype=torch.float32, device=DEV)
+    path.quantize(layer, k, v)
+    path.decode(layer, q, out)
+    torch.cuda.synchronize()
+    streams = [(0, h) for h in range(wl.H_kv)] + [(bb, bb % wl.H_kv) for bb in range(1, wl.B)]
+    check_layer(path, wl, layer, k, v, q, out, None, streams)
+    assert int(path.status.item()) == 0
+    assert torch.isfinite(out).all()
+    del k, v
+    torch.cuda.empty_cache()
