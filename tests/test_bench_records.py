@@ -51,3 +51,19 @@ def test_records_parse_and_go_stale(tmp_path, monkeypatch):
     assert bench.recorded_traffic("kern", "missing") is None
     (csrc / "k.cu").write_text("__global__ void g() { }\n__global__ void h() {}\n")
     assert bench.recorded_traffic("kern", "wl") is None
+
+
+def test_only_included_headers_enter_the_hash(tmp_path, monkeypatch):
+    csrc = tmp_path / "paper_2605_06675_gb300" / "csrc"
+    csrc.mkdir(parents=True)
+    (tmp_path / "include").mkdir()
+    (tmp_path / "include" / "rq.h").write_text("int rq_x(void);\n")
+    (csrc / "a.cuh").write_text('#include "rq.h"\n__device__ int f(int x) { return x; }\n')
+    (csrc / "b.cuh").write_text("__device__ int g(int x) { return -x; }\n")
+    (csrc / "k.cu").write_text('#include "a.cuh"\n__global__ void k(int* p) { *p = f(*p); }\n')
+    monkeypatch.setattr(bench, "ROOT", str(tmp_path))
+    h0 = bench.kernel_source_hash("k.cu")
+    (csrc / "b.cuh").write_text("__device__ int g(int x) { return x * 3; }\n")   # not included
+    assert bench.kernel_source_hash("k.cu") == h0
+    (tmp_path / "include" / "rq.h").write_text("int rq_x(void); int rq_y(void);\n")  # included via a.cuh
+    assert bench.kernel_source_hash("k.cu") != h0
