@@ -14,7 +14,7 @@ import numpy as np
 
 from . import pack
 from .attention import decode_attention, unrotate
-from .quant import quantize_stream
+from .quant import quantize_stream, storage_grouping
 
 
 def quantize_layer(k, v, bits, k_grouping, v_grouping, hadamard=False, signs=None,
@@ -40,7 +40,8 @@ def quantize_layer(k, v, bits, k_grouping, v_grouping, hadamard=False, signs=Non
         for kind, x, grouping in ((pack.KIND_K, k, k_grouping), (pack.KIND_V, v, v_grouping)):
             b = int(bits[h, kind])
             r = quantize_stream(x[bb, h], grouping, b, signs, hadamard, int(sym[kind]))
-            words = pack.pack_stream(r["codes"], r["scale"], r["zero"], kind, grouping, b)
+            words = pack.pack_stream(r["codes"], r["scale"], r["zero"], kind,
+                                     storage_grouping(grouping), b)
             xhat = r["xhat"].astype(np.float64)
             if hadamard:
                 xhat = unrotate(xhat, signs)

@@ -51,6 +51,15 @@ decoder serves both), in the same precision steps as above:
 so level c sits at fp16(c sf + zf) ~ (c - M) sf, off the exact symmetric grid
 only by the fp16 rounding of zero (at most 2^-12 |zero|).
 
+TurboQuant group sizes (App. W "TurboQuant kernel": absmax per-group
+symmetric, groups of 128 elements for keys and 64 for values). Reading: the
+groups run along the head dimension of one token (PER_TOKEN_128: a key's
+whole 128-channel row; PER_TOKEN_64: each half of a value's row); a, M, the
+stored scale and zero and the codes follow the absmax steps above over the
+group's 128 or 64 values (min-max works the same way over them). In the
+packed format every group of 32 channels of the token stores its wide
+group's (scale, zero), so the 32-token block format is unchanged.
+
 Rotation (QuaRot reading of "Hadamard" / "random orthogonal R"):
   y = FWHT(x * sigma) * fp32_rn(1/sqrt(128)), in fp32, butterfly stages with
   stride 1, 2, 4, ..., 64 in that order; each stage maps the pair (i, i+h),
@@ -65,6 +74,18 @@ GROUP = 32
 HEAD_DIM = 128
 PER_TOKEN = 0
 PER_CHANNEL = 1
+PER_TOKEN_64 = 2       # groups of 64 consecutive channels of one token
+PER_TOKEN_128 = 3      # the whole 128-channel row of one token
+# elements per group of each grouping
+GROUP_LEN = {PER_TOKEN: 32, PER_CHANNEL: 32, PER_TOKEN_64: 64, PER_TOKEN_128: 128}
+
+
+def storage_grouping(grouping: int) -> int:
+    """The packed format's grouping of a stream: the wide per-token groups are
+    stored as per-token groups of 32 whose (scale, zero) repeat their wide
+    group's (reading: TurboQuant's 128 / 64-element groups in the 32-token
+    block format)."""
+    return PER_CHANNEL if grouping == PER_CHANNEL else PER_TOKEN
 
 # fp32 round-to-nearest of 1/sqrt(128) = 2^-3.5
 INV_SQRT_128_F32 = np.float32(0.08838834764831845)
@@ -93,7 +114,7 @@ def hadamard_rotate(x: np.ndarray, signs: np.ndarray | None) -> np.ndarray:
 
 
 def quantize_groups(v: np.ndarray, b: int, symmetric: bool = False):
-    """Quantize groups along the last axis (length 32) at b bits.
+    """Quantize groups along the last axis (length 32, 64 or 128) at b bits.
 
     Returns (codes uint8, scale float16, zero float16, bad bool), the last
     three with the group shape (last axis removed). ``symmetric``: the absmax
@@ -101,7 +122,7 @@ def quantize_groups(v: np.ndarray, b: int, symmetric: bool = False):
     """
     assert 1 <= b <= 8
     v = canonical(v)
-    assert v.shape[-1] == GROUP
+    assert v.shape[-1] in (32, 64, 128)
     with np.errstate(all="ignore"):
         finite = np.isfinite(v).all(axis=-1)
         vv = np.where(finite[..., None], v, np.float32(0.0))
@@ -143,22 +164,25 @@ def dequantize_groups(codes: np.ndarray, scale: np.ndarray, zero: np.ndarray) ->
 
 
 def to_groups(x: np.ndarray, grouping: int) -> np.ndarray:
-    """View one stream x[S, 128] as groups of 32.
+    """View one stream x[S, 128] as its groups.
 
-    PER_TOKEN:   groups[t, G, :]   = x[t, 32G : 32G+32]
-    PER_CHANNEL: groups[blk, c, :] = x[32 blk : 32 blk + 32, c]   (S % 32 == 0)
+    PER_TOKEN:     groups[t, G, :]   = x[t, 32G : 32G+32]
+    PER_TOKEN_64:  groups[t, G, :]   = x[t, 64G : 64G+64]
+    PER_TOKEN_128: groups[t, 0, :]   = x[t, :]
+    PER_CHANNEL:   groups[blk, c, :] = x[32 blk : 32 blk + 32, c]   (S % 32 == 0)
     """
     S, d = x.shape
     assert d == HEAD_DIM
-    if grouping == PER_TOKEN:
-        return x.reshape(S, HEAD_DIM // GROUP, GROUP)
+    if grouping != PER_CHANNEL:
+        n = GROUP_LEN[grouping]
+        return x.reshape(S, HEAD_DIM // n, n)
     assert S % GROUP == 0, "per-channel groups need S % 32 == 0"
     return x.reshape(S // GROUP, GROUP, HEAD_DIM).transpose(0, 2, 1)
 
 
 def from_groups(g: np.ndarray, grouping: int) -> np.ndarray:
     """Inverse of ``to_groups``: back to [S, 128]."""
-    if grouping == PER_TOKEN:
+    if grouping != PER_CHANNEL:
         S = g.shape[0]
         return g.reshape(S, HEAD_DIM)
     nblk = g.shape[0]
@@ -175,8 +199,11 @@ def quantize_stream(x: np.ndarray, grouping: int, b: int, signs: np.ndarray | No
     ``symmetric`` selects the group quantizer: False / MINMAX, True / ABSMAX,
     or LLOYDMAX (the codebook quantizer of ``lloydmax``).
     Returns dict with the quantizer-domain values ``y`` [S,128] (rotated when
-    ``hadamard``), ``codes`` [S,128] uint8 (element order), group-shaped
-    ``scale``/``zero``/``bad``, and ``xhat`` [S,128] fp32 in the quantizer domain.
+    ``hadamard``), ``codes`` [S,128] uint8 (element order), ``scale``/``zero``/
+    ``bad`` in the shape of the stored groups of 32 (for the wide per-token
+    groupings each wide group's values repeated over its groups of 32;
+    ``group_scale``/``group_zero`` hold one per wide group), and ``xhat``
+    [S,128] fp32 in the quantizer domain.
     """
     x = np.asarray(x, dtype=np.float32)
     y = hadamard_rotate(x, signs) if hadamard else x.astype(np.float32)
@@ -184,17 +211,21 @@ def quantize_stream(x: np.ndarray, grouping: int, b: int, signs: np.ndarray | No
     g = to_groups(y, grouping)
     form = int(symmetric)
     if form == LLOYDMAX:
+        assert grouping == PER_TOKEN, "Lloyd-Max groups are per-token groups of 32"
         from . import lloydmax
         codes, scale, zero, bad = lloydmax.quantize_groups(g, b)
         xhat = lloydmax.dequantize_groups(codes, scale, b)
     else:
         codes, scale, zero, bad = quantize_groups(g, b, form == ABSMAX)
         xhat = dequantize_groups(codes, scale, zero)
+    rep = GROUP_LEN[grouping] // GROUP if grouping != PER_CHANNEL else 1
     return {
         "y": y,
         "codes": from_groups(codes, grouping),
-        "scale": scale,
-        "zero": zero,
-        "bad": bad,
+        "scale": np.repeat(scale, rep, axis=-1),
+        "zero": np.repeat(zero, rep, axis=-1),
+        "bad": np.repeat(bad, rep, axis=-1),
+        "group_scale": scale,
+        "group_zero": zero,
         "xhat": from_groups(xhat, grouping),
     }

@@ -17,7 +17,7 @@ import numpy as np
 
 from .alloc import allocate
 from .calib import distortion_sweep, fit_distortion
-from .quant import ABSMAX, LLOYDMAX, MINMAX, PER_CHANNEL, PER_TOKEN
+from .quant import ABSMAX, LLOYDMAX, MINMAX, PER_CHANNEL, PER_TOKEN, PER_TOKEN_64, PER_TOKEN_128
 
 # name -> (key grouping, value grouping, hadamard, key form, value form)
 FAMILIES = {
@@ -26,6 +26,7 @@ FAMILIES = {
     "rtn": (PER_TOKEN, PER_TOKEN, False, ABSMAX, ABSMAX),
     "quarot": (PER_TOKEN, PER_TOKEN, True, ABSMAX, ABSMAX),
     "turboquant": (PER_TOKEN, PER_TOKEN, True, LLOYDMAX, LLOYDMAX),
+    "turboquant_absmax": (PER_TOKEN_128, PER_TOKEN_64, False, ABSMAX, ABSMAX),
 }
 
 

@@ -236,3 +236,26 @@ def test_stream_offsets_order():
     expect = np.cumsum([0] + sizes * 2)[:-1].reshape(1, 2, 2, 2)
     assert np.array_equal(off.astype(np.int64), expect)
     assert total == 2 * sum(sizes)
+
+
+def test_hand_meta_words_wide_groups():
+    # the wide per-token groups are stored as per-token groups of 32: a key
+    # row (group of 128) with scale 2.0 (0x4000) and zero -14.0 (0xCB00)
+    # gives word 16 (t mod 8) + 4 G + t / 8 = 0xCB004000 for all four G
+    from oracle import pipeline, quant
+    x = np.zeros((1, 1, 32, 128), dtype=np.float32)
+    x[..., 3] = 14.0
+    ol = pipeline.quantize_layer(x, x, np.array([[4, 4]]), quant.PER_TOKEN_128, quant.PER_TOKEN_64,
+                                 symmetric=(quant.ABSMAX, quant.ABSMAX))
+    words = ol[(0, 0, 0)]["words"]
+    meta = words[128 * 4:]
+    for t in range(32):
+        for G in range(4):
+            assert meta[16 * (t % 8) + 4 * G + t // 8] == 0xCB004000
+    # values: halves of 64; the row's second half is all zero: scale 0, zero +0
+    vm = ol[(0, 0, 1)]["words"][128 * 4:]
+    s, z = pack.unpack_meta_block(vm, pack.KIND_V, PER_TOKEN)
+    s = s.reshape(32, 4)
+    z = z.reshape(32, 4)
+    assert (s[:, :2] == 2.0).all() and (z[:, :2] == -14.0).all()
+    assert (s[:, 2:] == 0.0).all() and (z[:, 2:].view(np.uint16) == 0).all()

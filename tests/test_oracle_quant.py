@@ -344,3 +344,72 @@ def test_symmetric_costs_one_level():
             c, s, z, _ = quant.quantize_groups(x, b, symmetric=sym)
             ms.append(((quant.dequantize_groups(c, s, z) - x) ** 2).mean())
         assert ms[1] > ms[0]
+
+
+# ---- TurboQuant group sizes (App. W "TurboQuant kernel": absmax per group,
+# 128 elements for keys, 64 for values, along one token's head dimension)
+
+def test_wide_groups_match_printed_absmax_formula():
+    # round(x M / a) a / M with a = max |x| over each group of 128 (one key
+    # row) or 64 (half a value row), when a / M is a power of two and no value
+    # sits on a tie
+    rng = np.random.default_rng(31)
+    for grouping, n in ((quant.PER_TOKEN_128, 128), (quant.PER_TOKEN_64, 64)):
+        for b in (2, 3, 4, 8):
+            M = 2 ** (b - 1) - 1
+            e = rng.integers(-4, 4, size=(48, 128 // n))          # a / M = 2^e per group
+            a = M * 2.0 ** e
+            x = rng.uniform(-1, 1, size=(48, 128 // n, n)) * a[..., None]
+            x[:, :, 7] = a                                       # the group's absmax
+            x = x.astype(np.float16).astype(np.float32).reshape(48, 128)
+            u = (x.reshape(48, 128 // n, n).astype(np.float64) * M / a[..., None]).reshape(48, 128)
+            keep = np.abs(u - np.floor(u) - 0.5) > 1e-9
+            r = quant.quantize_stream(x, grouping, b, symmetric=quant.ABSMAX)
+            assert (r["group_scale"] == 2.0 ** e).all() and not r["bad"].any()
+            want = np.round(u) * np.repeat(a / M, n, axis=1)
+            got = r["xhat"].astype(np.float64)
+            assert np.array_equal(got[keep], want[keep]), (n, b)
+            assert np.array_equal((r["codes"].astype(np.int64) - M)[keep], np.round(u).astype(np.int64)[keep])
+
+
+def test_wide_groups_store_their_parameters_on_every_group_of_32():
+    # a key row of 128 with absmax 14 at 4 bits: scale 2, zero -14 on all four
+    # stored groups of 32; a value row whose halves have absmax 14 and 7:
+    # scales 2, 2, 1, 1 and zeros -14, -14, -7, -7
+    x = np.zeros((32, 128), dtype=np.float32)
+    x[:, 3] = 14.0
+    x[:, 100] = -6.0
+    r = quant.quantize_stream(x, quant.PER_TOKEN_128, 4, symmetric=quant.ABSMAX)
+    assert r["scale"].shape == (32, 4) and (r["scale"] == 2.0).all() and (r["zero"] == -14.0).all()
+    assert (r["group_scale"].shape == (32, 1))
+    assert (r["codes"][:, 3] == 14).all() and (r["codes"][:, 100] == 4).all() and (r["codes"][:, 0] == 7).all()
+    y = np.zeros((32, 128), dtype=np.float32)
+    y[:, 10] = -14.0
+    y[:, 64 + 20] = 7.0
+    r = quant.quantize_stream(y, quant.PER_TOKEN_64, 4, symmetric=quant.ABSMAX)
+    assert (r["scale"] == np.float16([2, 2, 1, 1])).all() and (r["zero"] == np.float16([-14, -14, -7, -7])).all()
+    assert (r["codes"][:, 10] == 0).all() and (r["codes"][:, 84] == 14).all()
+
+
+def test_wide_groups_equal_groups_of_32_when_their_quarters_agree():
+    # every group of 32 of a row holding the same absmax: the wide group's
+    # parameters are the same as each quarter's, so the codes agree
+    rng = np.random.default_rng(33)
+    x = rng.standard_normal((64, 128)).astype(np.float16).astype(np.float32)
+    x[:, [0, 32, 64, 96]] = 5.0
+    r32 = quant.quantize_stream(x, quant.PER_TOKEN, 3, symmetric=quant.ABSMAX)
+    for g in (quant.PER_TOKEN_64, quant.PER_TOKEN_128):
+        r = quant.quantize_stream(x, g, 3, symmetric=quant.ABSMAX)
+        assert np.array_equal(r["codes"], r32["codes"]) and np.array_equal(r["scale"], r32["scale"])
+
+
+def test_wider_groups_cost_distortion():
+    # on Gaussian rows a larger group has a larger absmax, so a coarser step:
+    # MSE(128) > MSE(64) > MSE(32) at every width (statistical, 4096 tokens)
+    x = np.random.default_rng(34).standard_normal((4096, 128)).astype(np.float32)
+    for b in (2, 3, 4, 6):
+        mse = []
+        for g in (quant.PER_TOKEN, quant.PER_TOKEN_64, quant.PER_TOKEN_128):
+            r = quant.quantize_stream(x, g, b, symmetric=quant.ABSMAX)
+            mse.append(float(np.mean((r["y"].astype(np.float64) - r["xhat"]) ** 2)))
+        assert mse[0] < mse[1] < mse[2], (b, mse)
