@@ -62,8 +62,18 @@ typedef enum { RQ_F16 = 0, RQ_BF16 = 1 } rq_dtype;
 
 /* RQ_PER_TOKEN: a group is 32 consecutive channels of one token (KIVI values,
  * QuaRot); RQ_PER_CHANNEL: 32 consecutive tokens of one channel (KIVI keys).
- * Sec. 2 "KV cache quantization", App. W "KIVI kernel". */
-typedef enum { RQ_PER_TOKEN = 0, RQ_PER_CHANNEL = 1 } rq_grouping;
+ * Sec. 2 "KV cache quantization", App. W "KIVI kernel".
+ * RQ_PER_TOKEN_64 / RQ_PER_TOKEN_128: 64 consecutive channels of one token /
+ * a token's whole 128-channel row, the value / key group sizes of App. W
+ * "TurboQuant kernel" (min-max or absmax, not Lloyd-Max). They are stored
+ * like RQ_PER_TOKEN: every group of 32 channels carries its wide group's
+ * fp16 (scale, zero), so the block format and its size are unchanged. */
+typedef enum {
+  RQ_PER_TOKEN = 0,
+  RQ_PER_CHANNEL = 1,
+  RQ_PER_TOKEN_64 = 2,
+  RQ_PER_TOKEN_128 = 3
+} rq_grouping;
 
 /* Per-group quantizer of a kind (keys or values), groups of 32 either way.
  * RQ_MINMAX: asymmetric min-max, scale = fp16(fp32(max - min) / (2^b - 1)),
@@ -77,6 +87,8 @@ typedef enum { RQ_PER_TOKEN = 0, RQ_PER_CHANNEL = 1 } rq_grouping;
  * Codes are c = clamp(rint((x - zero) * (1/scale)), 0, c_max) in fp32 with
  * one rounding of the product, from the stored fp16 scale and zero, for
  * both; the decoder reads both the same way (x_hat = c * scale + zero).
+ * For the wide per-token groupings the group's min, max or max |x| is taken
+ * over its 64 or 128 values, and the codes from its stored scale and zero.
  * RQ_LLOYDMAX: the 2^b-level Lloyd-Max codebook of a unit Gaussian (App. F
  *   Table 8; TurboQuant's scalar quantizer, App. W) scaled by the group's
  *   RMS: scale = fp16(sqrt(s2 / 32)) with s2 the fp32 sum of squares of

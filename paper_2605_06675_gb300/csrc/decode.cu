@@ -85,7 +85,7 @@ rq_status check_desc(const rq_cache_desc* desc) {
     return RQ_ERR_INVALID_ARG;
   if (desc->dtype != RQ_F16 && desc->dtype != RQ_BF16) return RQ_ERR_INVALID_ARG;
   for (int g : {desc->k_grouping, desc->v_grouping})
-    if (g != RQ_PER_TOKEN && g != RQ_PER_CHANNEL) return RQ_ERR_INVALID_ARG;
+    if (!grouping_ok(g)) return RQ_ERR_INVALID_ARG;
   if (!quantizers_ok(desc->k_quantizer, desc->k_grouping, desc->v_quantizer, desc->v_grouping))
     return RQ_ERR_INVALID_ARG;
   if (desc->d != kD || desc->group != kG || desc->S % kTile != 0 || desc->S == 0)
@@ -117,8 +117,8 @@ void fill_args(DecodeArgs& a, const rq_cache_desc* desc, int32_t layer, const vo
   a.nblk = desc->S / kTile;
   a.splits = splits;
   a.bps = bps;
-  a.kg = desc->k_grouping;
-  a.vg = desc->v_grouping;
+  a.kg = stored_grouping(desc->k_grouping);   // wide per-token groups are stored as groups of 32
+  a.vg = stored_grouping(desc->v_grouping);
   a.hadamard = desc->hadamard ? 1 : 0;
   a.kq = desc->k_quantizer;
   a.vq = desc->v_quantizer;

@@ -123,7 +123,8 @@ __global__ void __launch_bounds__(kThreads) calib_sweep_kernel(CalibArgs a) {
     float v[kG];
     calib_group_values<T>(ld, row_mode, grouping, had, sm, x32, v);
     const long long next = tile + stride;
-    const int form_now = form;
+    const int form_now = form, grouping_now = grouping;
+    const int span_now = (static_cast<int>(tile / a.ntile) & 1) ? a.vspan : a.kspan;
     if (next < a.ntiles) {
       form = (static_cast<int>(next / a.ntile) & 1) ? a.vq : a.kq;
       grouping = (static_cast<int>(next / a.ntile) & 1) ? a.vg : a.kg;
@@ -132,6 +133,7 @@ __global__ void __launch_bounds__(kThreads) calib_sweep_kernel(CalibArgs a) {
     }
     float mn, mx;
     minmax32(v, mn, mx);
+    if (grouping_now == RQ_PER_TOKEN) join_quarters(mn, mx, span_now);   // wide per-token groups
     const bool finite = isfinite(mn) && isfinite(mx);
     mn = __fadd_rn(mn, 0.0f);
     mx = __fadd_rn(mx, 0.0f);
@@ -227,7 +229,7 @@ extern "C" rq_status rq_quantize_pack(const rq_cache_desc* desc, int32_t layer, 
   if (layer < 0 || layer >= desc->L) return RQ_ERR_INVALID_ARG;
   if (desc->dtype != RQ_F16 && desc->dtype != RQ_BF16) return RQ_ERR_INVALID_ARG;
   for (int g : {desc->k_grouping, desc->v_grouping})
-    if (g != RQ_PER_TOKEN && g != RQ_PER_CHANNEL) return RQ_ERR_INVALID_ARG;
+    if (!grouping_ok(g)) return RQ_ERR_INVALID_ARG;
   if (!quantizers_ok(desc->k_quantizer, desc->k_grouping, desc->v_quantizer, desc->v_grouping))
     return RQ_ERR_INVALID_ARG;
   if (desc->d != kD || desc->group != kG || desc->S % kTile != 0) return RQ_ERR_SHAPE;
@@ -245,8 +247,10 @@ extern "C" rq_status rq_quantize_pack(const rq_cache_desc* desc, int32_t layer, 
   a.H = desc->H_kv;
   a.S = desc->S;
   a.nblk = desc->S / kTile;
-  a.kg = desc->k_grouping;
-  a.vg = desc->v_grouping;
+  a.kg = stored_grouping(desc->k_grouping);
+  a.vg = stored_grouping(desc->v_grouping);
+  a.kspan = token_span(desc->k_grouping);
+  a.vspan = token_span(desc->v_grouping);
   a.kq = desc->k_quantizer;
   a.vq = desc->v_quantizer;
   if (a.kq == RQ_LLOYDMAX || a.vq == RQ_LLOYDMAX) fill_lm_book(a.lm);
@@ -276,7 +280,7 @@ extern "C" rq_status rq_calibrate_distortion(const void* x, int32_t dtype, int32
   if (!x || !mse_dev || !ws || n <= 0 || T <= 0) return RQ_ERR_INVALID_ARG;
   if (dtype != RQ_F16 && dtype != RQ_BF16) return RQ_ERR_INVALID_ARG;
   for (int g : {k_grouping, v_grouping})
-    if (g != RQ_PER_TOKEN && g != RQ_PER_CHANNEL) return RQ_ERR_INVALID_ARG;
+    if (!grouping_ok(g)) return RQ_ERR_INVALID_ARG;
   if (!quantizers_ok(k_quantizer, k_grouping, v_quantizer, v_grouping)) return RQ_ERR_INVALID_ARG;
   if (T % kTile != 0) return RQ_ERR_SHAPE;
   if (!aligned16(x) || !aligned16(ws) || (reinterpret_cast<uintptr_t>(mse_dev) & 7u))
@@ -290,8 +294,10 @@ extern "C" rq_status rq_calibrate_distortion(const void* x, int32_t dtype, int32
   a.n = n;
   a.T = T;
   a.ntile = T / kTile;
-  a.kg = k_grouping;
-  a.vg = v_grouping;
+  a.kg = stored_grouping(k_grouping);
+  a.vg = stored_grouping(v_grouping);
+  a.kspan = token_span(k_grouping);
+  a.vspan = token_span(v_grouping);
   a.kq = k_quantizer;
   a.vq = v_quantizer;
   if (a.kq == RQ_LLOYDMAX || a.vq == RQ_LLOYDMAX) fill_lm_book(a.lm);
@@ -349,7 +355,7 @@ extern "C" rq_status rq_append(const rq_cache_desc* desc, int32_t layer, int32_t
   if (layer < 0 || layer >= desc->L || pos < 0 || pos >= desc->S) return RQ_ERR_INVALID_ARG;
   if (desc->dtype != RQ_F16 && desc->dtype != RQ_BF16) return RQ_ERR_INVALID_ARG;
   for (int g : {desc->k_grouping, desc->v_grouping})
-    if (g != RQ_PER_TOKEN && g != RQ_PER_CHANNEL) return RQ_ERR_INVALID_ARG;
+    if (!grouping_ok(g)) return RQ_ERR_INVALID_ARG;
   if (!quantizers_ok(desc->k_quantizer, desc->k_grouping, desc->v_quantizer, desc->v_grouping))
     return RQ_ERR_INVALID_ARG;
   if (desc->d != kD || desc->group != kG || desc->S % kTile != 0) return RQ_ERR_SHAPE;
@@ -381,8 +387,10 @@ extern "C" rq_status rq_append(const rq_cache_desc* desc, int32_t layer, int32_t
   a.H = desc->H_kv;
   a.S = 2 * kTile;
   a.nblk = 1;
-  a.kg = desc->k_grouping;
-  a.vg = desc->v_grouping;
+  a.kg = stored_grouping(desc->k_grouping);
+  a.vg = stored_grouping(desc->v_grouping);
+  a.kspan = token_span(desc->k_grouping);
+  a.vspan = token_span(desc->v_grouping);
   a.kq = desc->k_quantizer;
   a.vq = desc->v_quantizer;
   if (a.kq == RQ_LLOYDMAX || a.vq == RQ_LLOYDMAX) fill_lm_book(a.lm);

@@ -47,7 +47,8 @@ struct QuantArgs {
   const uint64_t* offsets;   // [L][B][H][2]
   uint8_t* packed;
   uint32_t* status;
-  int layer, B, H, S, nblk, kg, vg, hadamard;
+  int layer, B, H, S, nblk, kg, vg, hadamard;   // kg, vg: the stored grouping
+  int kspan, vspan;          // groups of 32 channels per per-token group (1, 2 or 4)
   int kq, vq;                // rq_quantizer of keys / values
   int j_dst0;                // packed block index of each stream's first tile
   long long ntiles;
@@ -59,7 +60,8 @@ struct CalibArgs {
   const int8_t* signs;
   double* partial;           // [n][T/32][8]
   uint32_t* status;
-  int n, T, ntile, kg, vg, hadamard;
+  int n, T, ntile, kg, vg, hadamard;   // kg, vg: the stored grouping
+  int kspan, vspan;          // groups of 32 channels per per-token group (1, 2 or 4)
   int kq, vq;                // rq_quantizer of keys / values
   long long ntiles;
   LMBook lm;                 // RQ_LLOYDMAX codebooks
@@ -141,6 +143,21 @@ __device__ __forceinline__ float fmax3_nan(float a, float b, float c) {
   float r;
   asm("max.NaN.f32 %0, %1, %2, %3;" : "=f"(r) : "f"(a), "f"(b), "f"(c));
   return r;
+}
+
+// min / max of a wide per-token group (64 or 128 channels of one token) from
+// its quarters: thread 4 t + G holds quarter G (channels 32 G .. 32 G + 31) of
+// token t; span 2 joins quarters (0, 1) and (2, 3), span 4 all four (NaN
+// propagates). Every lane of the warp takes part.
+__device__ __forceinline__ void join_quarters(float& mn, float& mx, int span) {
+  if (span >= 2) {
+    mn = fmin_nan(mn, __shfl_xor_sync(0xffffffffu, mn, 1));
+    mx = fmax_nan(mx, __shfl_xor_sync(0xffffffffu, mx, 1));
+  }
+  if (span >= 4) {
+    mn = fmin_nan(mn, __shfl_xor_sync(0xffffffffu, mn, 2));
+    mx = fmax_nan(mx, __shfl_xor_sync(0xffffffffu, mx, 2));
+  }
 }
 
 // NaN-propagating min / max of two packed 16-bit pairs
@@ -375,7 +392,7 @@ __device__ __forceinline__ GroupOut phase1_cols(const uint8_t* tile, int kind, T
 // depend on the order.
 template <typename T, bool SYM>
 __device__ __forceinline__ GroupOut phase1_rows(const uint8_t* tile, int kind, TileQ<SYM> q,
-                                                uint8_t* meta, QSmem& sm) {
+                                                uint8_t* meta, QSmem& sm, int span) {
   const int tau = threadIdx.x, t = tau >> 2, G = tau & 3;
   const uint8_t* row = tile + t * kRowBytes + 64 * G;
   uint32_t w[16];
@@ -402,6 +419,7 @@ __device__ __forceinline__ GroupOut phase1_rows(const uint8_t* tile, int kind, T
     }
   float mn = fmin_nan(lo_f32<T>(lo[0]), hi_f32<T>(lo[0]));
   float mx = fmax_nan(lo_f32<T>(hi[0]), hi_f32<T>(hi[0]));
+  join_quarters(mn, mx, span);
   const bool finite = isfinite(mn) && isfinite(mx);
   mn = __fadd_rn(mn, 0.0f);
   mx = __fadd_rn(mx, 0.0f);
@@ -551,7 +569,7 @@ __device__ __forceinline__ void rotate_group_perm(float (&v)[kG], int G) {
 template <typename T, bool SYM>
 __device__ __forceinline__ GroupOut phase1_rotated(const uint8_t* tile, float* x32, int kind,
                                                    int grouping, TileQ<SYM> q, uint8_t* meta,
-                                                   QSmem& sm) {
+                                                   QSmem& sm, int span) {
   const int tau = threadIdx.x, t = tau >> 2, G = tau & 3;
   float v[kG];
   const uint8_t* row = tile + t * kRowBytes + 64 * G;
@@ -580,6 +598,7 @@ __device__ __forceinline__ GroupOut phase1_rotated(const uint8_t* tile, float* x
   if (grouping == RQ_PER_TOKEN) {             // min / max: any order
     float mn, mx;
     minmax32(v, mn, mx);
+    join_quarters(mn, mx, span);
     const bool finite = isfinite(mn) && isfinite(mx);
     return finish_group(kind, RQ_PER_TOKEN, t, G, 0, __fadd_rn(mn, 0.0f), __fadd_rn(mx, 0.0f),
                         finite, q, meta, sm);
@@ -631,22 +650,22 @@ __device__ __forceinline__ GroupOut phase1_rotated(const uint8_t* tile, float* x
 // accesses stay shared-memory instructions.
 template <typename T, bool SYM>
 __device__ __noinline__ GroupOut phase1_rot_call(int buf, int kind, int grouping, int b,
-                                                 uint8_t* meta) {
+                                                 uint8_t* meta, int span) {
   extern __shared__ __align__(16) unsigned char smem_raw[];
   QSmem& sm = *reinterpret_cast<QSmem*>(smem_raw);
   float* x32 = reinterpret_cast<float*>(smem_raw + sizeof(QSmem));
   const TileQ<SYM> q{b};
-  return phase1_rotated<T>(sm.tile[buf], x32, kind, grouping, q, meta, sm);
+  return phase1_rotated<T>(sm.tile[buf], x32, kind, grouping, q, meta, sm, span);
 }
 
 template <typename T, bool HAD, bool SYM>
 __device__ __forceinline__ GroupOut phase1(const uint8_t* tile, float* x32, int kind, int grouping,
-                                              int b, uint8_t* meta, QSmem& sm, int buf) {
+                                              int b, uint8_t* meta, QSmem& sm, int buf, int span) {
   const TileQ<SYM> q{b};
-  if constexpr (HAD) return phase1_rot_call<T, SYM>(buf, kind, grouping, b, meta);
+  if constexpr (HAD) return phase1_rot_call<T, SYM>(buf, kind, grouping, b, meta, span);
   else if (grouping == kGroupingLM) return phase1_rows_lm<T>(tile, kind, meta, sm);
   else if (grouping == RQ_PER_CHANNEL) return phase1_cols<T>(tile, kind, q, meta, sm);
-  else return phase1_rows<T>(tile, kind, q, meta, sm);
+  else return phase1_rows<T>(tile, kind, q, meta, sm, span);
 }
 
 // ------------------------------------------------------------- phase 2 ----
@@ -921,8 +940,9 @@ __device__ __forceinline__ int run_segment(const QuantArgs& a, QSmem& sm, float*
       }
     }
     GroupOut g;
-    if (sym) g = phase1<T, HAD, true>(buf, x32, kind, grouping, B, meta, sm, it & 1);
-    else g = phase1<T, HAD, false>(buf, x32, kind, grouping, B, meta, sm, it & 1);
+    const int span = kind ? a.vspan : a.kspan;             // kernel parameters, no register
+    if (sym) g = phase1<T, HAD, true>(buf, x32, kind, grouping, B, meta, sm, it & 1, span);
+    else g = phase1<T, HAD, false>(buf, x32, kind, grouping, B, meta, sm, it & 1, span);
     if (g.bad) set_status(a.status, RQ_STATUS_NUMERIC);
     const bool slow = __syncthreads_or(g.slow) != 0;
     uint32_t* blk32 = reinterpret_cast<uint32_t*>(blk);

@@ -36,11 +36,26 @@ struct LMBook {
 __host__ __device__ constexpr int lm_offset(int b) { return (1 << b) - 2; }
 // the library's codebook (host.cpp), and one filled LMBook
 const uint16_t* lloydmax_levels(int b);
+// rq_grouping values; the wide per-token groupings (64 or 128 channels of
+// one token) are stored as per-token groups of 32 that repeat their wide
+// group's scale and zero
+inline bool grouping_ok(int g) {
+  return g == RQ_PER_TOKEN || g == RQ_PER_CHANNEL || g == RQ_PER_TOKEN_64 || g == RQ_PER_TOKEN_128;
+}
+// the grouping of the packed format (RQ_PER_TOKEN or RQ_PER_CHANNEL)
+__host__ __device__ constexpr int stored_grouping(int g) {
+  return g == RQ_PER_CHANNEL ? RQ_PER_CHANNEL : RQ_PER_TOKEN;
+}
+// groups of 32 channels in one group of a per-token grouping (1, 2 or 4)
+__host__ __device__ constexpr int token_span(int g) {
+  return g == RQ_PER_TOKEN_128 ? 4 : g == RQ_PER_TOKEN_64 ? 2 : 1;
+}
 // a quantizer choice of keys and values is supported: min-max and absmax with
-// either grouping, Lloyd-Max with per-token groups
+// any grouping, Lloyd-Max with per-token groups of 32
 inline bool quantizers_ok(int kq, int kg, int vq, int vg) {
   for (int i = 0; i < 2; ++i) {
     const int q = i ? vq : kq, g = i ? vg : kg;
+    if (!grouping_ok(g)) return false;
     if (q != RQ_MINMAX && q != RQ_ABSMAX && q != RQ_LLOYDMAX) return false;
     if (q == RQ_LLOYDMAX && g != RQ_PER_TOKEN) return false;
   }

@@ -17,7 +17,7 @@ LIB_PATH = os.path.join(_HERE, "librq.so")
 
 RQ_OK = 0
 RQ_F16, RQ_BF16 = 0, 1
-RQ_PER_TOKEN, RQ_PER_CHANNEL = 0, 1
+RQ_PER_TOKEN, RQ_PER_CHANNEL, RQ_PER_TOKEN_64, RQ_PER_TOKEN_128 = 0, 1, 2, 3
 RQ_MINMAX, RQ_ABSMAX, RQ_LLOYDMAX = 0, 1, 2
 RQ_CAP_5X = 1
 RQ_STATUS_NUMERIC = 1

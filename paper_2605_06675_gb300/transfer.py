@@ -21,6 +21,9 @@ Sec. 3.4 "K/V separation"):
   quarot    Hadamard rotation, then per token absmax (Sec. 4.1)
   turboquant Hadamard rotation, then the per-token Lloyd-Max codebook
             quantizer (App. F Table 8, App. W)
+  turboquant_absmax  absmax per group with TurboQuant's group sizes
+            (App. W "TurboQuant kernel"): 128 channels for keys (a whole
+            row), 64 for values
 The "uniform" column gives every key ceil(avg_bits) and every value
 floor(avg_bits) bits (one width per kind; the same width when avg_bits is
 an integer).
@@ -34,7 +37,7 @@ import torch
 
 from . import rq, synth
 from .path import PackedKVPath
-from .workloads import PER_CHANNEL, PER_TOKEN, Workload
+from .workloads import PER_CHANNEL, PER_TOKEN, PER_TOKEN_64, PER_TOKEN_128, Workload
 
 FAMILIES = {
     "kivi": dict(k_grouping=PER_CHANNEL, v_grouping=PER_TOKEN, hadamard=False,
@@ -47,6 +50,8 @@ FAMILIES = {
                    k_quantizer=rq.RQ_ABSMAX, v_quantizer=rq.RQ_ABSMAX),
     "turboquant": dict(k_grouping=PER_TOKEN, v_grouping=PER_TOKEN, hadamard=True,
                        k_quantizer=rq.RQ_LLOYDMAX, v_quantizer=rq.RQ_LLOYDMAX),
+    "turboquant_absmax": dict(k_grouping=PER_TOKEN_128, v_grouping=PER_TOKEN_64, hadamard=False,
+                              k_quantizer=rq.RQ_ABSMAX, v_quantizer=rq.RQ_ABSMAX),
 }
 
 

@@ -11,6 +11,7 @@ from __future__ import annotations
 from dataclasses import dataclass
 
 PER_TOKEN, PER_CHANNEL = 0, 1
+PER_TOKEN_64, PER_TOKEN_128 = 2, 3     # TurboQuant's value / key groups (64 / 128 channels)
 
 
 def mask_of(bits) -> int:

@@ -8,7 +8,8 @@ import torch
 from oracle import calib as ocalib
 from paper_2605_06675_gb300 import synth
 from paper_2605_06675_gb300.path import PackedKVPath
-from paper_2605_06675_gb300.workloads import PER_CHANNEL, PER_TOKEN, Workload
+from paper_2605_06675_gb300.workloads import (PER_CHANNEL, PER_TOKEN, PER_TOKEN_64, PER_TOKEN_128,
+                                              Workload)
 
 from .gpu_helpers import (TOL, attn_err, bits_cycle, ensure_built, oracle_attention,
                           oracle_layer, to_np)
@@ -270,6 +271,65 @@ def test_symmetric_all_widths_bit_exact_and_attention(rq, name, dtype, kg, vg, h
     for l, (k, v, q, out) in res.items():
         check_layer(path, wl, l, k, v, q, out, signs)
     assert int(path.status.item()) == 0
+
+
+# ---- TurboQuant's group sizes (App. W "TurboQuant kernel"): absmax over a
+# key's whole 128-channel row and over each 64-channel half of a value row;
+# also min-max over the wide groups, rotated caches and per-channel partners
+WIDE_CASES = [
+    ("turboquant_absmax", "bfloat16", PER_TOKEN_128, PER_TOKEN_64, False, 1, 1),
+    ("turboquant_absmax", "float16", PER_TOKEN_128, PER_TOKEN_64, False, 1, 1),
+    ("minmax_wide", "bfloat16", PER_TOKEN_64, PER_TOKEN_128, False, 0, 0),
+    ("rotated_wide", "bfloat16", PER_TOKEN_128, PER_TOKEN_64, True, 1, 1),
+    ("kivi_keys_wide_values", "float16", PER_CHANNEL, PER_TOKEN_128, False, 0, 1),
+]
+
+
+@pytest.mark.parametrize("name,dtype,kg,vg,hadamard,kq,vq", WIDE_CASES)
+def test_wide_groups_all_widths_bit_exact_and_attention(rq, name, dtype, kg, vg, hadamard, kq, vq):
+    wl = small_wl(dtype=dtype, kg=kg, vg=vg, hadamard=hadamard, S=96, seed=65, kq=kq, vq=vq)
+    bits = bits_cycle(wl.L, wl.H_kv, range(1, 9), offset=3)
+    path, res, signs = run_layers(rq, wl, bits)
+    for l, (k, v, q, out) in res.items():
+        check_layer(path, wl, l, k, v, q, out, signs)
+    assert int(path.status.item()) == 0
+
+
+@pytest.mark.parametrize("name,dtype,kg,vg,hadamard,kq,vq", WIDE_CASES[:1] + WIDE_CASES[2:4])
+def test_wide_groups_calibration_matches_oracle(rq, name, dtype, kg, vg, hadamard, kq, vq):
+    wl = small_wl(L=2, H=4, S=96, dtype=dtype, hadamard=hadamard, seed=66, kg=kg, vg=vg, kq=kq, vq=vq)
+    x = synth.calibration_sample(wl, T=96, device=DEV)
+    signs = synth.hadamard_signs(wl.seed) if hadamard else None
+    path = PackedKVPath(wl, DEV, signs)
+    mse = path.calibrate(x).cpu().numpy()
+    torch.cuda.synchronize()
+    n = x.shape[0]
+    groupings = [wl.k_grouping if i % 2 == 0 else wl.v_grouping for i in range(n)]
+    sym = [symmetric_of(wl)[i % 2] for i in range(n)]
+    ref = ocalib.distortion_sweep(to_np(x), groupings, hadamard,
+                                  None if signs is None else signs.numpy(), symmetric=sym)
+    rel = np.abs(mse - ref) / np.abs(ref)
+    assert rel.max() < MSE_RTOL, rel.max()
+    assert np.all(np.diff(mse[:, 1:], axis=1) < 0)
+
+
+def test_wide_groups_flag_a_non_finite_quarter(rq):
+    # one NaN in a 128-channel key row makes the whole row's group bad (codes,
+    # scale and zero 0, status NUMERIC), not just its quarter
+    wl = small_wl(L=1, B=1, H=2, g=4, S=64, dtype="bfloat16", kg=PER_TOKEN_128, vg=PER_TOKEN_64,
+                  seed=67, kq=1, vq=1)
+    path = PackedKVPath(wl, DEV)
+    path.set_bits(np.full((1, 2, 2), 4, dtype=np.uint8))
+    k, v = synth.kv_layer(1, 2, 64, "bfloat16", 67, 0, device=DEV)
+    k[0, 0, 5, 100] = float("nan")
+    path.quantize(0, k, v)
+    torch.cuda.synchronize()
+    assert int(path.status.item()) & 1
+    ol = oracle_layer(k, v, path.bits_host[0], wl.k_grouping, wl.v_grouping, False, None,
+                      [(0, 0)], symmetric_of(wl))
+    got = path.stream_bytes(0, 0, 0, 0).cpu().numpy()
+    assert np.array_equal(got, ol[(0, 0, 0)]["words"].view(np.uint8))
+    assert ol[(0, 0, 0)]["bad"][5].all()
 
 
 @pytest.mark.parametrize("kq,vq", [(1, 1), (0, 1)])
