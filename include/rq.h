@@ -57,6 +57,8 @@ typedef enum {
 /* bits OR-ed into *status_dev by the kernels */
 #define RQ_STATUS_NUMERIC 1u  /* a group held NaN/inf or its fp16 scale/zero overflowed */
 #define RQ_STATUS_BAD_BITS 2u /* a device bit-table entry was outside 1..8; stream skipped */
+#define RQ_STATUS_BAD_POSITION 4u /* a per-row position or token count (rq_append_rows,
+                                     rq_decode_attention_rows) was out of range; row skipped */
 
 typedef enum { RQ_F16 = 0, RQ_BF16 = 1 } rq_dtype;
 
@@ -310,6 +312,35 @@ rq_status rq_decode_attention_len(const rq_cache_desc* desc, int32_t layer, int3
                                   const uint64_t* offsets_dev, const int8_t* signs_dev,
                                   const void* residual, float* out, void* ws, size_t ws_bytes,
                                   uint32_t* status_dev, void* stream);
+
+/* Decode-time append for a batch whose rows are at different lengths (a
+ * ragged decode batch): as rq_append, with one position per batch row in
+ * pos_dev (device int32 [B], 4-byte aligned). Row b's new token goes to slot
+ * pos_dev[b] % 32 of its windows; when that is slot 31 the row's windows are
+ * quantized and packed as block pos_dev[b] / 32 of its streams. A negative
+ * position appends nothing for that row (a row that is not decoding this
+ * step); a position at or past desc->S sets RQ_STATUS_BAD_POSITION and skips
+ * the row. Always launches (the positions are read on the device).
+ * Errors: as rq_append. */
+rq_status rq_append_rows(const rq_cache_desc* desc, int32_t layer, const int32_t* pos_dev,
+                         const void* k_new, const void* v_new, void* residual,
+                         const int8_t* signs_dev, const uint8_t* bits_dev,
+                         const uint64_t* offsets_dev, void* packed, uint32_t* status_dev,
+                         void* stream);
+
+/* Decode attention with one token count per batch row: row b attends its
+ * first n_dev[b] tokens (device int32 [B], 4-byte aligned; 1 <= n <= desc->S):
+ * the packed blocks below 32 * (n / 32) and the last n % 32 from its residual
+ * windows, as rq_decode_attention_len does for one n. residual is required.
+ * The split plan is that of the capacity desc->S; each row's split CTAs stop
+ * at its own packed length. A count outside 1..desc->S sets
+ * RQ_STATUS_BAD_POSITION and that row's output is 0. Workspace and other
+ * arguments as rq_decode_attention_len. */
+rq_status rq_decode_attention_rows(const rq_cache_desc* desc, int32_t layer, const int32_t* n_dev,
+                                   const void* q, const void* packed, const uint8_t* bits_dev,
+                                   const uint64_t* offsets_dev, const int8_t* signs_dev,
+                                   const void* residual, float* out, void* ws, size_t ws_bytes,
+                                   uint32_t* status_dev, void* stream);
 
 #ifdef __cplusplus
 }

@@ -108,6 +108,7 @@ void fill_args(DecodeArgs& a, const rq_cache_desc* desc, int32_t layer, const vo
   a.offsets = offsets_dev;
   a.signs = signs_dev;
   a.partial = static_cast<float*>(ws);
+  a.n_rows = nullptr;
   a.status = status_dev;
   a.layer = layer;
   a.B = desc->B;
@@ -268,3 +269,36 @@ extern "C" rq_status rq_decode_attention_len(const rq_cache_desc* desc, int32_t 
   return launch_decode(a, desc, out, static_cast<cudaStream_t>(stream), res_layer, R);
 }
 
+
+// --------------------------------------- decode with a token count per row ----
+extern "C" rq_status rq_decode_attention_rows(const rq_cache_desc* desc, int32_t layer,
+                                              const int32_t* n_dev, const void* q,
+                                              const void* packed, const uint8_t* bits_dev,
+                                              const uint64_t* offsets_dev, const int8_t* signs_dev,
+                                              const void* residual, float* out, void* ws,
+                                              size_t ws_bytes, uint32_t* status_dev, void* stream) {
+  using namespace rq;
+  const rq_status st = check_desc(desc);
+  if (st != RQ_OK) return st;
+  if (!n_dev || !q || !packed || !bits_dev || !offsets_dev || !residual || !out || !ws)
+    return RQ_ERR_INVALID_ARG;
+  if (layer < 0 || layer >= desc->L) return RQ_ERR_INVALID_ARG;
+  if (!aligned16(packed) || !aligned16(ws) || !aligned16(residual) ||
+      (reinterpret_cast<uintptr_t>(n_dev) & 3u) || (reinterpret_cast<uintptr_t>(q) & 1u) ||
+      (reinterpret_cast<uintptr_t>(out) & 3u))
+    return RQ_ERR_ALIGNMENT;
+  if (desc->B == 0) return RQ_OK;
+  int slots = 0;
+  if (decode_slots(&slots) != RQ_OK) return RQ_ERR_CUDA;
+  // the split plan of the capacity; each row's CTAs stop at its own length
+  int splits = 1, bps = 1;
+  const int nblk = desc->S / kTile;
+  decode_plan(desc, nblk, slots, &splits, &bps);
+  if (ws_bytes < workspace_bytes(desc, splits)) return RQ_ERR_WORKSPACE;
+  DecodeArgs a;
+  fill_args(a, desc, layer, q, packed, bits_dev, offsets_dev, signs_dev, ws, status_dev, splits, bps);
+  a.n_rows = n_dev;
+  const void* res_layer = static_cast<const uint8_t*>(residual) +
+                          static_cast<size_t>(layer) * desc->B * desc->H_kv * 2 * kTile * kD * 2;
+  return launch_decode(a, desc, out, static_cast<cudaStream_t>(stream), res_layer, 0);
+}

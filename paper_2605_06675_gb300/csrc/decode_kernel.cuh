@@ -56,6 +56,7 @@ struct DecodeArgs {
   const uint64_t* offsets;
   const int8_t* signs;
   float* partial;            // [B][H_q][splits][132]
+  const int32_t* n_rows;     // tokens attended per batch row (rq_decode_attention_rows) or null
   uint32_t* status;
   int layer, B, H, Hq, g, nblk, splits, bps, kg, vg, hadamard;
   int kq, vq;                // rq_quantizer of keys / values
@@ -787,8 +788,15 @@ __global__ void __launch_bounds__(kThreads, RQ_DECODE_MIN_BLOCKS) decode_split_k
   dr.sV = 512 * (bV + 1);
   dr.slot = max(dr.sK, dr.sV);
   dr.ns = valid ? min(kMaxSlots, kRingBytes / dr.slot) : 2;
+  // the packed blocks of this batch row: all nblk, or those below 32 * floor(n / 32)
+  // of its own token count n (1 <= n <= 32 * nblk; another n attends nothing)
+  int nblk_row = a.nblk;
+  if (a.n_rows) {
+    const int n = a.n_rows[batch];
+    nblk_row = (n >= 1 && n <= a.nblk * kTile) ? n / kTile : 0;
+  }
   const int blk0 = split * a.bps;
-  const int blk1 = min(a.nblk, blk0 + a.bps);
+  const int blk1 = min(nblk_row, blk0 + a.bps);
   const int blk_first = blk0 + warp;
   WarpStream ws;
   ws.lane = lane;
@@ -1054,8 +1062,17 @@ __global__ void __launch_bounds__(kThreads) decode_merge_kernel(const float* par
                                                                 uint32_t* status, int Hq, int H,
                                                                 int g, int splits, int hadamard,
                                                                 const T* q, const T* residual,
-                                                                int R) {
+                                                                int R, const int32_t* n_rows,
+                                                                int cap) {
   asm volatile("griddepcontrol.wait;\n" ::: "memory");
+  bool row_ok = true;
+  if (n_rows) {                  // a token count per batch row: its own residual tokens
+    const int n = n_rows[blockIdx.x / H];
+    row_ok = n >= 1 && n <= cap;
+    R = row_ok ? n % kTile : 0;
+    if (!row_ok && threadIdx.x == 0 && blockIdx.x % H == 0 && blockIdx.y == 0)
+      set_status(status, RQ_STATUS_BAD_POSITION);
+  }
   constexpr int CW = kD / CQ;          // channels of this CTA
   constexpr int CH = CW / 4;           // 16-byte pieces of a record's o slice
   constexpr int SLOT = CH + 1;         // pieces per (row, split): o slice, then (m, l, pad)
@@ -1160,10 +1177,11 @@ __global__ void __launch_bounds__(kThreads) decode_merge_kernel(const float* par
     if (n < g) {
       const float L = run_l[n];
       float v = L > 0.0f ? acc[k] / L : 0.0f;
-      if (!(L > 0.0f) || !isfinite(v)) {
+      if (row_ok && (!(L > 0.0f) || !isfinite(v))) {
         set_status(status, RQ_STATUS_NUMERIC);
         if (!isfinite(v)) v = 0.0f;
       }
+      if (!row_ok) v = 0.0f;
       acc[k] = v;
     }
   }
@@ -1198,6 +1216,7 @@ __global__ void __launch_bounds__(kThreads) decode_merge_kernel(const float* par
 template <typename T>
 inline rq_status launch_decode_t(const DecodeArgs& a, float* out, const void* res_layer, int R,
                                  cudaStream_t s) {
+  // a token count per batch row: every row may hold residual tokens
   auto kern = decode_split_kernel<T>;
   if (cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, kSmemBytes) != cudaSuccess ||
       cudaFuncSetAttribute(kern, cudaFuncAttributePreferredSharedMemoryCarveout,
@@ -1224,7 +1243,7 @@ inline rq_status launch_decode_t(const DecodeArgs& a, float* out, const void* re
     return RQ_ERR_CUDA;
   if (cudaLaunchKernelEx(&cfg, mk, static_cast<const float*>(a.partial), out, a.signs, a.status,
                          a.Hq, a.H, a.g, a.splits, a.hadamard, static_cast<const T*>(a.q),
-                         static_cast<const T*>(res_layer), R) != cudaSuccess)
+                         static_cast<const T*>(res_layer), R, a.n_rows, a.nblk * kTile) != cudaSuccess)
     return RQ_ERR_CUDA;
   return launch_status();
 }

@@ -256,6 +256,8 @@ extern "C" rq_status rq_quantize_pack(const rq_cache_desc* desc, int32_t layer, 
   if (a.kq == RQ_LLOYDMAX || a.vq == RQ_LLOYDMAX) fill_lm_book(a.lm);
   a.hadamard = desc->hadamard ? 1 : 0;
   a.j_dst0 = 0;
+  a.row_pos = nullptr;
+  a.cap = desc->S;
   a.ntiles = static_cast<long long>(desc->B) * desc->H_kv * 2 * a.nblk;
   if (a.ntiles == 0) return RQ_OK;
   cudaStream_t st = static_cast<cudaStream_t>(stream);
@@ -329,6 +331,22 @@ __global__ void append_token_kernel(const uint4* k_new, const uint4* v_new, uint
   residual_layer[(bh * 2 + kind) * 32 * 16 + slot * 16 + ch] = *src;
 }
 
+// As append_token_kernel with a position per batch row: a negative position
+// appends nothing for that row, one at or past the capacity is reported.
+__global__ void append_token_rows_kernel(const uint4* k_new, const uint4* v_new,
+                                         uint4* residual_layer, const int32_t* pos, int H,
+                                         int cap, uint32_t* status) {
+  const int bh = blockIdx.x, t = threadIdx.x, kind = t >> 4, ch = t & 15;
+  const int p = pos[bh / H];
+  if (p < 0) return;
+  if (p >= cap) {
+    if (t == 0 && bh % H == 0) set_status(status, RQ_STATUS_BAD_POSITION);
+    return;
+  }
+  const uint4* src = (kind ? v_new : k_new) + bh * 16 + ch;
+  residual_layer[(bh * 2 + kind) * 32 * 16 + (p % kTile) * 16 + ch] = *src;
+}
+
 size_t residual_layer_elems(const rq_cache_desc* desc) {
   return static_cast<size_t>(desc->B) * desc->H_kv * 2 * kTile * kD;
 }
@@ -396,6 +414,68 @@ extern "C" rq_status rq_append(const rq_cache_desc* desc, int32_t layer, int32_t
   if (a.kq == RQ_LLOYDMAX || a.vq == RQ_LLOYDMAX) fill_lm_book(a.lm);
   a.hadamard = desc->hadamard ? 1 : 0;
   a.j_dst0 = pos / kTile;
+  a.row_pos = nullptr;
+  a.cap = desc->S;
+  a.ntiles = static_cast<long long>(desc->B) * desc->H_kv * 2;
+  if (desc->dtype == RQ_F16)
+    return a.hadamard ? launch_quantize_f16_rot(a, st) : launch_quantize_f16(a, st);
+  return a.hadamard ? launch_quantize_bf16_rot(a, st) : launch_quantize_bf16(a, st);
+}
+
+// ---- decode-time append with a position per batch row ----------------------
+extern "C" rq_status rq_append_rows(const rq_cache_desc* desc, int32_t layer,
+                                    const int32_t* pos_dev, const void* k_new, const void* v_new,
+                                    void* residual, const int8_t* signs_dev,
+                                    const uint8_t* bits_dev, const uint64_t* offsets_dev,
+                                    void* packed, uint32_t* status_dev, void* stream) {
+  using namespace rq;
+  if (!desc || !pos_dev || !k_new || !v_new || !residual || !bits_dev || !offsets_dev || !packed)
+    return RQ_ERR_INVALID_ARG;
+  if (desc->L <= 0 || desc->B < 0 || desc->H_kv <= 0 || desc->S < 0) return RQ_ERR_INVALID_ARG;
+  if (layer < 0 || layer >= desc->L) return RQ_ERR_INVALID_ARG;
+  if (desc->dtype != RQ_F16 && desc->dtype != RQ_BF16) return RQ_ERR_INVALID_ARG;
+  for (int g : {desc->k_grouping, desc->v_grouping})
+    if (!grouping_ok(g)) return RQ_ERR_INVALID_ARG;
+  if (!quantizers_ok(desc->k_quantizer, desc->k_grouping, desc->v_quantizer, desc->v_grouping))
+    return RQ_ERR_INVALID_ARG;
+  if (desc->d != kD || desc->group != kG || desc->S % kTile != 0) return RQ_ERR_SHAPE;
+  if (!aligned16(k_new) || !aligned16(v_new) || !aligned16(residual) || !aligned16(packed) ||
+      (reinterpret_cast<uintptr_t>(pos_dev) & 3u))
+    return RQ_ERR_ALIGNMENT;
+  if (desc->B == 0) return RQ_OK;
+  cudaStream_t st = static_cast<cudaStream_t>(stream);
+  const size_t layer_bytes = residual_layer_elems(desc) * 2;
+  uint8_t* res_layer = static_cast<uint8_t*>(residual) + static_cast<size_t>(layer) * layer_bytes;
+  append_token_rows_kernel<<<static_cast<unsigned>(desc->B * desc->H_kv), 32, 0, st>>>(
+      static_cast<const uint4*>(k_new), static_cast<const uint4*>(v_new),
+      reinterpret_cast<uint4*>(res_layer), pos_dev, desc->H_kv, desc->S, status_dev);
+  if (launch_status() != RQ_OK) return RQ_ERR_CUDA;
+  // every row whose window is now full (its position is 31 mod 32) packs it
+  // as block position / 32; the kernel reads the positions and skips the rest
+  QuantArgs a;
+  a.k = res_layer;
+  a.v = res_layer + static_cast<size_t>(kTile) * kD * 2;
+  a.signs = signs_dev;
+  a.bits = bits_dev;
+  a.offsets = offsets_dev;
+  a.packed = static_cast<uint8_t*>(packed);
+  a.status = status_dev;
+  a.layer = layer;
+  a.B = desc->B;
+  a.H = desc->H_kv;
+  a.S = 2 * kTile;
+  a.nblk = 1;
+  a.kg = stored_grouping(desc->k_grouping);
+  a.vg = stored_grouping(desc->v_grouping);
+  a.kspan = token_span(desc->k_grouping);
+  a.vspan = token_span(desc->v_grouping);
+  a.kq = desc->k_quantizer;
+  a.vq = desc->v_quantizer;
+  if (a.kq == RQ_LLOYDMAX || a.vq == RQ_LLOYDMAX) fill_lm_book(a.lm);
+  a.hadamard = desc->hadamard ? 1 : 0;
+  a.j_dst0 = 0;
+  a.row_pos = pos_dev;
+  a.cap = desc->S;
   a.ntiles = static_cast<long long>(desc->B) * desc->H_kv * 2;
   if (desc->dtype == RQ_F16)
     return a.hadamard ? launch_quantize_f16_rot(a, st) : launch_quantize_f16(a, st);

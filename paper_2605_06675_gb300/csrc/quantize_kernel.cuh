@@ -51,6 +51,10 @@ struct QuantArgs {
   int kspan, vspan;          // groups of 32 channels per per-token group (1, 2 or 4)
   int kq, vq;                // rq_quantizer of keys / values
   int j_dst0;                // packed block index of each stream's first tile
+  const int32_t* row_pos;    // decode-time append per batch row (or null): the window of row
+                             // b is packed as block row_pos[b] / 32 when row_pos[b] % 32 == 31
+                             // and 0 <= row_pos[b] < cap, and skipped otherwise
+  int cap;                   // the cache's capacity in tokens (row_pos only)
   long long ntiles;
   LMBook lm;                 // RQ_LLOYDMAX codebooks
 };
@@ -874,6 +878,7 @@ struct StreamState {
   const uint8_t* src;     // first tile of the stream (raw values)
   uint8_t* dst;           // first packed block of the stream
   int b, kind, grouping;
+  bool skip;              // row_pos: this row's window is not full (nothing to write)
 };
 
 template <typename T>
@@ -885,9 +890,16 @@ __device__ __forceinline__ StreamState stream_state(const QuantArgs& a, int sk) 
   st.grouping = st.kind ? a.vg : a.kg;
   st.src = reinterpret_cast<const uint8_t*>(static_cast<const T*>(st.kind ? a.v : a.k) +
                                             static_cast<long long>(sk >> 1) * a.S * kD);
+  int j = a.j_dst0;
+  st.skip = false;
+  if (a.row_pos) {
+    const int p = a.row_pos[(sk >> 1) / a.H];
+    st.skip = !(p >= 0 && p < a.cap && p % kTile == kTile - 1);
+    j = st.skip ? 0 : p / kTile;
+  }
   // offsets[layer][batch][h][kind] = offsets[layer * B * H * 2 + sk]
   st.dst = a.packed + a.offsets[static_cast<long long>(a.layer) * a.B * a.H * 2 + sk] +
-           static_cast<long long>(a.j_dst0) * (512 * (st.b + 1));
+           static_cast<long long>(j) * (512 * (st.b + 1));
   return st;
 }
 
@@ -952,10 +964,10 @@ __device__ __forceinline__ int run_segment(const QuantArgs& a, QSmem& sm, float*
   return it;
 }
 
-// a stream whose device bit-width is outside 1..8: keep the tile pipeline
-// going, write nothing, report it
+// a stream whose device bit-width is outside 1..8 (reported), or a window
+// with nothing to pack: keep the tile pipeline going, write nothing
 __device__ __forceinline__ int skip_segment(const QuantArgs& a, QSmem& sm, const Segment& seg,
-                                            int it, int tile_bytes) {
+                                            int it, int tile_bytes, bool report) {
   for (int k = 0; k < seg.n; ++k, ++it) {
     cp_async_wait_all();
     __syncthreads();
@@ -963,7 +975,7 @@ __device__ __forceinline__ int skip_segment(const QuantArgs& a, QSmem& sm, const
     else if (seg.next) issue_tile(sm.tile[(it + 1) & 1], seg.next);
     cp_async_commit();
   }
-  if (threadIdx.x == 0) set_status(a.status, RQ_STATUS_BAD_BITS);
+  if (report && threadIdx.x == 0) set_status(a.status, RQ_STATUS_BAD_BITS);
   return it;
 }
 
@@ -1018,8 +1030,8 @@ __global__ void __launch_bounds__(kThreads, RQ_QUANT_MIN_BLOCKS) quantize_pack_k
     seg.next = more ? nxt.src : nullptr;
     seg.n = static_cast<int>(end - t);
     const int b = cur.b;
-    if (b < 1 || b > 8) {
-      it = skip_segment(a, sm, seg, it, kTileSrcBytes);
+    if (cur.skip || b < 1 || b > 8) {
+      it = skip_segment(a, sm, seg, it, kTileSrcBytes, !cur.skip);
     } else {
       const bool lm = (cur.kind ? a.vq : a.kq) == RQ_LLOYDMAX;
       switch (mode_of(cur.kind, cur.grouping, lm)) {

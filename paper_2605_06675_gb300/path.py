@@ -112,6 +112,21 @@ class PackedKVPath:
                                    self.offsets, self.signs, self.residual(), out, ws,
                                    self.status, stream)
 
+    def append_rows(self, layer: int, pos: torch.Tensor, k_new: torch.Tensor, v_new: torch.Tensor,
+                    stream=None):
+        """Append one token per batch row at positions ``pos`` (CUDA int32 [B];
+        negative: the row appends nothing)."""
+        rq.rq_append_rows(self.desc, layer, pos, k_new, v_new, self.residual(), self.signs,
+                          self.bits, self.offsets, self.packed, self.status, stream)
+
+    def decode_rows(self, layer: int, n_tokens: torch.Tensor, q: torch.Tensor, out: torch.Tensor,
+                    stream=None):
+        """Decode attention, batch row b over its first n_tokens[b] tokens."""
+        ws = self.decode_workspace()
+        rq.rq_decode_attention_rows(self.desc, layer, n_tokens, q, self.packed, self.bits,
+                                    self.offsets, self.signs, self.residual(), out, ws,
+                                    self.status, stream)
+
     def stream_bytes(self, layer: int, batch: int, head: int, kind: int) -> torch.Tensor:
         """The packed bytes of one stream (a view into the packed buffer)."""
         off = int(self.offsets_host[layer, batch, head, kind])

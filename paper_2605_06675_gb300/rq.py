@@ -22,6 +22,7 @@ RQ_MINMAX, RQ_ABSMAX, RQ_LLOYDMAX = 0, 1, 2
 RQ_CAP_5X = 1
 RQ_STATUS_NUMERIC = 1
 RQ_STATUS_BAD_BITS = 2
+RQ_STATUS_BAD_POSITION = 4
 RQ_STATIC_SCRATCH_BYTES = 8 << 20
 HEAD_DIM = 128
 GROUP = 32
@@ -34,7 +35,7 @@ EXPORTS = ["rq_status_string", "rq_abi_version", "rq_lloydmax_levels", "rq_fit_d
            "rq_alloc_continuous", "rq_packed_layout", "rq_calibrate_workspace_bytes",
            "rq_calibrate_distortion", "rq_quantize_pack", "rq_decode_workspace_bytes",
            "rq_decode_attention", "rq_decode_attention_static", "rq_residual_bytes",
-           "rq_append", "rq_decode_attention_len"]
+           "rq_append", "rq_decode_attention_len", "rq_append_rows", "rq_decode_attention_rows"]
 
 
 class RQError(RuntimeError):
@@ -82,6 +83,9 @@ def lib() -> ctypes.CDLL:
             "rq_append": ([_P, _I, _I, _P, _P, _P, _P, _P, _P, _P, _P, _P], _I),
             "rq_decode_attention_len": ([_P, _I, _I, _P, _P, _P, _P, _P, _P, _P, _P, _SZ, _P, _P],
                                         _I),
+            "rq_append_rows": ([_P, _I, _P, _P, _P, _P, _P, _P, _P, _P, _P, _P], _I),
+            "rq_decode_attention_rows": ([_P, _I, _P, _P, _P, _P, _P, _P, _P, _P, _P, _SZ, _P, _P],
+                                         _I),
         }
         for name, (args, res) in sig.items():
             f = getattr(L, name)
@@ -273,5 +277,24 @@ def rq_decode_attention_len(desc, layer, n_tokens, q, packed, bits_dev, offsets_
     the residual window's last n_tokens % 32 tokens."""
     _check("rq_decode_attention_len", lib().rq_decode_attention_len(
         ctypes.byref(desc), layer, n_tokens, _dp(q), _dp(packed), _dp(bits_dev),
+        _dp(offsets_dev), _dp(signs), _dp(residual), _dp(out), _dp(ws),
+        ws.numel() * ws.element_size(), _dp(status), _stream(stream)))
+
+
+def rq_append_rows(desc, layer, pos, k_new, v_new, residual, signs, bits_dev, offsets_dev, packed,
+                   status=None, stream=None):
+    """Append one token per batch row at the rows' own positions (``pos``:
+    CUDA int32 [B]; a negative entry appends nothing for that row)."""
+    _check("rq_append_rows", lib().rq_append_rows(
+        ctypes.byref(desc), layer, _dp(pos), _dp(k_new), _dp(v_new), _dp(residual), _dp(signs),
+        _dp(bits_dev), _dp(offsets_dev), _dp(packed), _dp(status), _stream(stream)))
+
+
+def rq_decode_attention_rows(desc, layer, n_tokens, q, packed, bits_dev, offsets_dev, signs,
+                             residual, out, ws, status=None, stream=None):
+    """Decode attention with a token count per batch row (``n_tokens``: CUDA
+    int32 [B])."""
+    _check("rq_decode_attention_rows", lib().rq_decode_attention_rows(
+        ctypes.byref(desc), layer, _dp(n_tokens), _dp(q), _dp(packed), _dp(bits_dev),
         _dp(offsets_dev), _dp(signs), _dp(residual), _dp(out), _dp(ws),
         ws.numel() * ws.element_size(), _dp(status), _stream(stream)))

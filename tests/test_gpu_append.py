@@ -117,3 +117,76 @@ def test_decode_len_argument_errors():
         rq.rq_append(path.desc, 0, 64, kn, kn, path.residual(), None, path.bits, path.offsets,
                      path.packed)
     assert e.value.status == 1
+
+
+# ---- a ragged decode batch: every row at its own position ---------------------
+@pytest.mark.gpu
+@pytest.mark.parametrize("dtype,kg,vg,hadamard,allowed,kq,vq", [
+    ("bfloat16", PER_CHANNEL, PER_TOKEN, False, (2, 3, 4), 0, 0),
+    ("float16", PER_TOKEN, PER_TOKEN, True, (3, 4, 5), 1, 1),
+])
+def test_ragged_rows_append_and_decode_match_oracle(dtype, kg, vg, hadamard, allowed, kq, vq):
+    """Three rows appended one token per step until each reaches its own
+    length (160, 97 and 33 tokens; a row that has stopped passes position -1),
+    decoded with a token count per row: each row's packed prefix bit for bit
+    and its attention against the oracle's, over its own prefix and
+    residual tokens."""
+    ensure_built()
+    lengths = (160, 97, 33)
+    wl = Workload("ragged", L=2, B=3, H_kv=2, H_q=8, S=160, dtype=dtype, k_grouping=kg,
+                  v_grouping=vg, hadamard=hadamard, allowed=allowed, avg_bits=3.0, sigma_lnw=0.5,
+                  value_dist="gaussian", seed=57, k_quantizer=kq, v_quantizer=vq)
+    layer = 0
+    signs = synth.hadamard_signs(wl.seed).to(DEV) if hadamard else None
+    path = PackedKVPath(wl, DEV, signs)
+    bits = bits_cycle(wl.L, wl.H_kv, allowed, offset=2)
+    path.set_bits(bits)
+    k, v = synth.kv_layer(wl.B, wl.H_kv, wl.S, wl.dtype, wl.seed, layer, device=DEV)
+    out = torch.empty((wl.B, wl.H_q, 128), dtype=torch.float32, device=DEV)
+    checkpoints = {1, 31, 32, 33, 50, 96, 97, 98, 130, 160}
+    for step in range(wl.S):
+        pos = torch.tensor([step if step < n else -1 for n in lengths], dtype=torch.int32,
+                           device=DEV)
+        path.append_rows(layer, pos, k[:, :, step].contiguous(), v[:, :, step].contiguous())
+        if step + 1 not in checkpoints:
+            continue
+        n_rows = [min(step + 1, n) for n in lengths]
+        q = synth.queries(wl.B, wl.H_q, wl.dtype, wl.seed + step, layer, DEV)
+        path.decode_rows(layer, torch.tensor(n_rows, dtype=torch.int32, device=DEV), q, out)
+        torch.cuda.synchronize()
+        for bb, n in enumerate(n_rows):
+            s_pk = 32 * (n // 32)
+            ol = {}
+            if s_pk:
+                ol = oracle_layer(k[bb:bb + 1, :, :s_pk], v[bb:bb + 1, :, :s_pk], bits[layer], kg, vg,
+                                  hadamard, signs, symmetric=(kq, vq))
+                for (_, h, kind), r in ol.items():
+                    words = r["words"].view(np.uint8)
+                    got = path.stream_bytes(layer, bb, h, kind)[:words.size].cpu().numpy()
+                    assert np.array_equal(got, words), (step, bb, h, kind)
+            ref = opipe.attend_with_residual(to_np(q[bb:bb + 1]), ol, to_np(k[bb:bb + 1, :, s_pk:n]),
+                                             to_np(v[bb:bb + 1, :, s_pk:n]))
+            err = attn_err(to_np(out[bb:bb + 1]), ref)
+            assert err <= TOL, (step, bb, n, err)
+    assert int(path.status.item()) == 0
+
+
+@pytest.mark.gpu
+def test_ragged_rows_out_of_range_are_reported():
+    ensure_built()
+    wl = Workload("ragged_err", L=1, B=2, H_kv=2, H_q=4, S=64, dtype="bfloat16",
+                  k_grouping=PER_CHANNEL, v_grouping=PER_TOKEN, hadamard=False,
+                  allowed=(2, 3, 4), avg_bits=3.0, sigma_lnw=0.5, value_dist="gaussian", seed=58)
+    path = PackedKVPath(wl, DEV)
+    path.set_bits(bits_cycle(1, 2, wl.allowed))
+    kn = torch.zeros((2, 2, 128), dtype=torch.bfloat16, device=DEV)
+    path.append_rows(0, torch.tensor([0, 64], dtype=torch.int32, device=DEV), kn, kn)   # 64 = S
+    torch.cuda.synchronize()
+    assert int(path.status.item()) & 4
+    path.status.zero_()
+    q = torch.zeros((2, 4, 128), dtype=torch.bfloat16, device=DEV)
+    out = torch.full((2, 4, 128), 7.0, dtype=torch.float32, device=DEV)
+    path.decode_rows(0, torch.tensor([1, 0], dtype=torch.int32, device=DEV), q, out)      # 0 < 1
+    torch.cuda.synchronize()
+    assert int(path.status.item()) & 4
+    assert torch.isfinite(out).all() and (out[1] == 0).all()
