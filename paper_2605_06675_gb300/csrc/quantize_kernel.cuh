@@ -507,14 +507,14 @@ __device__ __forceinline__ void rotate_group(float (&v)[kG], int G, const int8_t
   rotate_group_signed(v, G);
 }
 
-// rotate_group_signed for a thread whose 8-value chunks are permuted: slot
-// 8 i + j holds channel 32 G + 8 (i ^ G) + j. Strides 1, 2, 4 are as there.
-// At strides 8 and 16 the lower channel of a slot pair sits in the upper
-// slot when bit 0 / bit 1 of G is set, so each output is fma(own, +-1,
-// other) with the lane's signs (the same single rounding as a + b, a - b).
-// The lane stages take, from the partner, the slot that holds the same
-// channel there (slot ^ 8 for G ^ 1, slot ^ 16 for G ^ 2).
-__device__ __forceinline__ void rotate_group_perm(float (&v)[kG], int G) {
+// Strides 1 .. 16 of the FWHT of a thread's quarter whose 8-value chunks are
+// permuted: slot 8 i + j holds channel 32 G + 8 (i ^ G) + j. Strides 1, 2, 4
+// are as in rotate_group_signed. At strides 8 and 16 the lower channel of a
+// slot pair sits in the upper slot when bit 0 / bit 1 of G is set, so each
+// output is fma(own, +-1, other) with the lane's signs (the same single
+// rounding as a + b, a - b). The values stay unscaled; strides 32 and 64
+// follow in rotate_lanes_x32.
+__device__ __forceinline__ void rotate_quarter_perm(float (&v)[kG], int G) {
   float2 p[kG / 2];
 #pragma unroll
   for (int k = 0; k < kG / 2; ++k)
@@ -542,27 +542,55 @@ __device__ __forceinline__ void rotate_group_perm(float (&v)[kG], int G) {
     }
   }
 #pragma unroll
-  for (int s = 1; s <= 2; s <<= 1) {          // strides 32, 64: lanes G ^ 1, G ^ 2
-    const int d = 4 * s;                      // pair offset of slot ^ 8 / slot ^ 16
-    const float sg = (G & s) ? -1.0f : 1.0f;
-    const float2 sg2 = make_float2(sg, sg);
+  for (int k = 0; k < kG / 2; ++k) {
+    v[2 * k] = p[k].x;
+    v[2 * k + 1] = p[k].y;
+  }
+}
+
+// Strides 32 and 64 of token t's FWHT through the fp32 tile, in place: the
+// four quarters (after strides 1 .. 16) are in x32; thread 4 t + G takes
+// channel offsets 8 G .. 8 G + 7 of all four quarters, runs stride 32 on the
+// quarter pairs (0, 1), (2, 3) and stride 64 on (0, 2), (1, 3) (the
+// oracle's butterfly order, each output one fp32 rounding), scales by
+// fp32(1/sqrt(128)) and writes the results back to the same places. The four
+// threads of a token are consecutive lanes, so a warp barrier orders the
+// exchange; the 16-byte accesses of a quarter-warp fall on distinct bank
+// groups (rows 164 words apart). Returns each quarter's min / max over the
+// thread's eight values.
+__device__ __forceinline__ void rotate_lanes_x32(float* x32, int t, int G, float (&mnq)[4],
+                                                 float (&mxq)[4]) {
+  __syncwarp();
+  float2 y[4][4];                            // [quarter][pair of offsets]
 #pragma unroll
-    for (int k = 0; k < kG / 2; ++k) {
-      if (k & d) continue;
-      const float2 ok = make_float2(__shfl_xor_sync(0xffffffffu, p[k + d].x, s),
-                                    __shfl_xor_sync(0xffffffffu, p[k + d].y, s));
-      const float2 od = make_float2(__shfl_xor_sync(0xffffffffu, p[k].x, s),
-                                    __shfl_xor_sync(0xffffffffu, p[k].y, s));
-      p[k] = __ffma2_rn(p[k], sg2, ok);
-      p[k + d] = __ffma2_rn(p[k + d], sg2, od);
-    }
+  for (int Q = 0; Q < 4; ++Q) {
+    const float* src = x32 + x32_at(t, 32 * Q + 8 * G);
+    const float4 a = *reinterpret_cast<const float4*>(src);
+    const float4 b = *reinterpret_cast<const float4*>(src + 4);
+    y[Q][0] = make_float2(a.x, a.y);
+    y[Q][1] = make_float2(a.z, a.w);
+    y[Q][2] = make_float2(b.x, b.y);
+    y[Q][3] = make_float2(b.z, b.w);
   }
   const float2 r = make_float2(kInvSqrt128, kInvSqrt128);
 #pragma unroll
-  for (int k = 0; k < kG / 2; ++k) {
-    const float2 y = __fmul2_rn(p[k], r);
-    v[2 * k] = y.x;
-    v[2 * k + 1] = y.y;
+  for (int k = 0; k < 4; ++k) {
+    const float2 s01 = __fadd2_rn(y[0][k], y[1][k]), d01 = fsub2_rn(y[0][k], y[1][k]);
+    const float2 s23 = __fadd2_rn(y[2][k], y[3][k]), d23 = fsub2_rn(y[2][k], y[3][k]);
+    y[0][k] = __fmul2_rn(__fadd2_rn(s01, s23), r);
+    y[2][k] = __fmul2_rn(fsub2_rn(s01, s23), r);
+    y[1][k] = __fmul2_rn(__fadd2_rn(d01, d23), r);
+    y[3][k] = __fmul2_rn(fsub2_rn(d01, d23), r);
+  }
+#pragma unroll
+  for (int Q = 0; Q < 4; ++Q) {
+    float* dst = x32 + x32_at(t, 32 * Q + 8 * G);
+    *reinterpret_cast<float4*>(dst) = make_float4(y[Q][0].x, y[Q][0].y, y[Q][1].x, y[Q][1].y);
+    *reinterpret_cast<float4*>(dst + 4) = make_float4(y[Q][2].x, y[Q][2].y, y[Q][3].x, y[Q][3].y);
+    mnq[Q] = fmin_nan(fmin3_nan(fmin3_nan(y[Q][0].x, y[Q][0].y, y[Q][1].x), y[Q][1].y, y[Q][2].x),
+                      fmin3_nan(y[Q][2].y, y[Q][3].x, y[Q][3].y));
+    mxq[Q] = fmax_nan(fmax3_nan(fmax3_nan(y[Q][0].x, y[Q][0].y, y[Q][1].x), y[Q][1].y, y[Q][2].x),
+                      fmax3_nan(y[Q][2].y, y[Q][3].x, y[Q][3].y));
   }
 }
 
@@ -590,7 +618,7 @@ __device__ __forceinline__ GroupOut phase1_rotated(const uint8_t* tile, float* x
       v[8 * i + 2 * e + 1] = hi_f32<T>(w[e]);
     }
   }
-  rotate_group_perm(v, G);
+  rotate_quarter_perm(v, G);
   float* xr = x32 + x32_at(t, 32 * G);
 #pragma unroll
   for (int i = 0; i < 4; ++i) {
@@ -599,9 +627,25 @@ __device__ __forceinline__ GroupOut phase1_rotated(const uint8_t* tile, float* x
     *reinterpret_cast<float4*>(xc + 4) =
         make_float4(v[8 * i + 4], v[8 * i + 5], v[8 * i + 6], v[8 * i + 7]);
   }
+  float mnq[4], mxq[4];
+  rotate_lanes_x32(x32, t, G, mnq, mxq);
   if (grouping == RQ_PER_TOKEN) {             // min / max: any order
+    // reduce-scatter over the token's four threads: thread G ends with
+    // quarter G's min / max (lane G ^ 2 first takes the other half of the
+    // quarters, lane G ^ 1 then the other quarter of the pair); wide
+    // groups then join quarters as in the plain layout
     float mn, mx;
-    minmax32(v, mn, mx);
+    {
+      const bool h = G & 2, l = G & 1;
+      float a0 = h ? mnq[2] : mnq[0], a1 = h ? mnq[3] : mnq[1];
+      float b0 = h ? mxq[2] : mxq[0], b1 = h ? mxq[3] : mxq[1];
+      a0 = fmin_nan(a0, __shfl_xor_sync(0xffffffffu, h ? mnq[0] : mnq[2], 2));
+      a1 = fmin_nan(a1, __shfl_xor_sync(0xffffffffu, h ? mnq[1] : mnq[3], 2));
+      b0 = fmax_nan(b0, __shfl_xor_sync(0xffffffffu, h ? mxq[0] : mxq[2], 2));
+      b1 = fmax_nan(b1, __shfl_xor_sync(0xffffffffu, h ? mxq[1] : mxq[3], 2));
+      mn = fmin_nan(l ? a1 : a0, __shfl_xor_sync(0xffffffffu, l ? a0 : a1, 1));
+      mx = fmax_nan(l ? b1 : b0, __shfl_xor_sync(0xffffffffu, l ? b0 : b1, 1));
+    }
     join_quarters(mn, mx, span);
     const bool finite = isfinite(mn) && isfinite(mx);
     return finish_group(kind, RQ_PER_TOKEN, t, G, 0, __fadd_rn(mn, 0.0f), __fadd_rn(mx, 0.0f),
@@ -609,6 +653,8 @@ __device__ __forceinline__ GroupOut phase1_rotated(const uint8_t* tile, float* x
   }
   if (grouping == kGroupingLM) {            // Lloyd-Max, per token, on the rotated values
     // the sum of squares is ordered: the quarter back from x32 in channel order
+    // (written by the token's four threads)
+    __syncwarp();
 #pragma unroll
     for (int i = 0; i < kG; i += 4) {
       const float4 y = *reinterpret_cast<const float4*>(xr + i);
