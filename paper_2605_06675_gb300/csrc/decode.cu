@@ -52,24 +52,58 @@ rq_status split_ctas_per_sm(int* per_sm) {
   return RQ_OK;
 }
 
-// Splits of the sequence per (batch, kv head): as many as fit in one wave of
-// resident CTAs (slots = SMs x CTAs per SM), so every CTA streams a long run
-// of blocks and none waits for a second wave; at least one.
+struct SplitPlan {
+  int splits, bps;      // units [u_lo, B * H_kv): CTAs and blocks per CTA
+  int s_lo, bps_lo;     // units [0, u_lo)
+  int u_lo;
+};
+
+// Splits of the sequence per (batch, kv head) unit: as many CTAs as fit in one
+// wave of resident CTAs (slots = SMs x CTAs per SM), so every CTA streams a
+// long run of blocks and none waits for a second wave; at least one per unit.
+// When the units do not divide the slots, the wave is filled with two split
+// counts: units [0, u_lo) take s_lo = slots / units splits and the rest
+// s_lo + 1, so that every SM holds the same number of CTAs (a grid of
+// units x s_lo CTAs would leave some SMs one CTA short and the others, with
+// their full complement, setting the time). The s_lo-split units' CTAs (the
+// larger ones) come first in the grid, so the round-robin dispatch spreads
+// them over the SMs.
 // nblk: the packed blocks attended (<= the capacity's); splits <= the
 // capacity's split bound (max_splits), which sizes the workspace.
 int max_splits(const rq_cache_desc* desc, int slots) {
   const long long units = static_cast<long long>(desc->B) * desc->H_kv;
-  const long long sp = units > 0 ? slots / units : 1;
+  long long sp = units > 0 ? slots / units : 1;
+  if (units > 0 && units <= slots && slots % units != 0) ++sp;
   return static_cast<int>(std::max<long long>(1, std::min<long long>(sp, desc->S / kTile)));
 }
 
-void decode_plan(const rq_cache_desc* desc, int nblk, int slots, int* splits, int* bps) {
-  const long long units = static_cast<long long>(desc->B) * desc->H_kv;
-  long long sp = units > 0 ? slots / units : 1;
+namespace {
+// blocks per CTA and the resulting split count for sp requested splits
+void split_even(int nblk, long long sp, int* splits, int* bps) {
   sp = std::max<long long>(1, std::min<long long>(sp, nblk));
-  const int b = static_cast<int>((nblk + sp - 1) / sp);
-  *bps = std::max(b, 1);
+  *bps = std::max(1, static_cast<int>((nblk + sp - 1) / sp));
   *splits = std::max(1, (nblk + *bps - 1) / *bps);
+}
+}  // namespace
+
+SplitPlan decode_plan(const rq_cache_desc* desc, int nblk, int slots) {
+  SplitPlan p;
+  const long long units = static_cast<long long>(desc->B) * desc->H_kv;
+  const long long sp = units > 0 ? slots / units : 1;
+  split_even(nblk, sp, &p.splits, &p.bps);
+  p.s_lo = p.splits;
+  p.bps_lo = p.bps;
+  p.u_lo = static_cast<int>(units);
+  if (units > 0 && units <= slots && slots % units != 0 && sp < nblk) {
+    int s_hi = 1, bps_hi = 1;
+    split_even(nblk, sp + 1, &s_hi, &bps_hi);
+    if (s_hi > p.s_lo) {
+      p.splits = s_hi;
+      p.bps = bps_hi;
+      p.u_lo = static_cast<int>(units - (slots - units * sp));
+    }
+  }
+  return p;
 }
 
 rq_status decode_slots(int* slots) {
@@ -101,7 +135,7 @@ size_t workspace_bytes(const rq_cache_desc* desc, int splits) {
 
 void fill_args(DecodeArgs& a, const rq_cache_desc* desc, int32_t layer, const void* q,
                const void* packed, const uint8_t* bits_dev, const uint64_t* offsets_dev,
-               const int8_t* signs_dev, void* ws, uint32_t* status_dev, int splits, int bps) {
+               const int8_t* signs_dev, void* ws, uint32_t* status_dev, const SplitPlan& plan) {
   a.q = q;
   a.packed = static_cast<const uint8_t*>(packed);
   a.bits = bits_dev;
@@ -116,8 +150,11 @@ void fill_args(DecodeArgs& a, const rq_cache_desc* desc, int32_t layer, const vo
   a.Hq = desc->H_q;
   a.g = desc->H_q / desc->H_kv;
   a.nblk = desc->S / kTile;
-  a.splits = splits;
-  a.bps = bps;
+  a.splits = plan.splits;
+  a.bps = plan.bps;
+  a.s_lo = plan.s_lo;
+  a.bps_lo = plan.bps_lo;
+  a.u_lo = plan.u_lo;
   a.kg = stored_grouping(desc->k_grouping);   // wide per-token groups are stored as groups of 32
   a.vg = stored_grouping(desc->v_grouping);
   a.hadamard = desc->hadamard ? 1 : 0;
@@ -163,11 +200,10 @@ extern "C" rq_status rq_decode_attention(const rq_cache_desc* desc, int32_t laye
   if (desc->B == 0) return RQ_OK;
   int slots = 0;
   if (decode_slots(&slots) != RQ_OK) return RQ_ERR_CUDA;
-  int splits = 1, bps = 1;
-  decode_plan(desc, desc->S / kTile, slots, &splits, &bps);
-  if (ws_bytes < workspace_bytes(desc, splits)) return RQ_ERR_WORKSPACE;
+  const SplitPlan plan = decode_plan(desc, desc->S / kTile, slots);
+  if (ws_bytes < workspace_bytes(desc, plan.splits)) return RQ_ERR_WORKSPACE;
   DecodeArgs a;
-  fill_args(a, desc, layer, q, packed, bits_dev, offsets_dev, signs_dev, ws, status_dev, splits, bps);
+  fill_args(a, desc, layer, q, packed, bits_dev, offsets_dev, signs_dev, ws, status_dev, plan);
   return launch_decode(a, desc, out, static_cast<cudaStream_t>(stream));
 }
 
@@ -223,14 +259,12 @@ extern "C" rq_status rq_decode_attention_static(const rq_cache_desc* desc, int32
   if (desc->B == 0) return RQ_OK;
   int slots = 0;
   if (decode_slots(&slots) != RQ_OK) return RQ_ERR_CUDA;
-  int splits = 1, bps = 1;
-  decode_plan(desc, desc->S / kTile, slots, &splits, &bps);
-  if (workspace_bytes(desc, splits) > RQ_STATIC_SCRATCH_BYTES) return RQ_ERR_WORKSPACE;
+  const SplitPlan plan = decode_plan(desc, desc->S / kTile, slots);
+  if (workspace_bytes(desc, plan.splits) > RQ_STATIC_SCRATCH_BYTES) return RQ_ERR_WORKSPACE;
   float* scratch = nullptr;
   if (static_scratch_ptr(&scratch) != RQ_OK) return RQ_ERR_CUDA;
   DecodeArgs a;
-  fill_args(a, desc, layer, q, packed, bits_dev, offsets_dev, signs_dev, scratch, status_dev, splits,
-            bps);
+  fill_args(a, desc, layer, q, packed, bits_dev, offsets_dev, signs_dev, scratch, status_dev, plan);
   return launch_decode(a, desc, out, static_cast<cudaStream_t>(stream));
 }
 
@@ -254,12 +288,11 @@ extern "C" rq_status rq_decode_attention_len(const rq_cache_desc* desc, int32_t 
   if (desc->B == 0) return RQ_OK;
   int slots = 0;
   if (decode_slots(&slots) != RQ_OK) return RQ_ERR_CUDA;
-  int splits = 1, bps = 1;
   const int nblk = n_tokens / kTile;
-  decode_plan(desc, nblk, slots, &splits, &bps);
-  if (ws_bytes < workspace_bytes(desc, splits)) return RQ_ERR_WORKSPACE;
+  const SplitPlan plan = decode_plan(desc, nblk, slots);
+  if (ws_bytes < workspace_bytes(desc, plan.splits)) return RQ_ERR_WORKSPACE;
   DecodeArgs a;
-  fill_args(a, desc, layer, q, packed, bits_dev, offsets_dev, signs_dev, ws, status_dev, splits, bps);
+  fill_args(a, desc, layer, q, packed, bits_dev, offsets_dev, signs_dev, ws, status_dev, plan);
   a.nblk = nblk;
   // this layer's residual windows: [B][H][2][32][128] values of the cache dtype
   const void* res_layer =
@@ -291,12 +324,11 @@ extern "C" rq_status rq_decode_attention_rows(const rq_cache_desc* desc, int32_t
   int slots = 0;
   if (decode_slots(&slots) != RQ_OK) return RQ_ERR_CUDA;
   // the split plan of the capacity; each row's CTAs stop at its own length
-  int splits = 1, bps = 1;
   const int nblk = desc->S / kTile;
-  decode_plan(desc, nblk, slots, &splits, &bps);
-  if (ws_bytes < workspace_bytes(desc, splits)) return RQ_ERR_WORKSPACE;
+  const SplitPlan plan = decode_plan(desc, nblk, slots);
+  if (ws_bytes < workspace_bytes(desc, plan.splits)) return RQ_ERR_WORKSPACE;
   DecodeArgs a;
-  fill_args(a, desc, layer, q, packed, bits_dev, offsets_dev, signs_dev, ws, status_dev, splits, bps);
+  fill_args(a, desc, layer, q, packed, bits_dev, offsets_dev, signs_dev, ws, status_dev, plan);
   a.n_rows = n_dev;
   const void* res_layer = static_cast<const uint8_t*>(residual) +
                           static_cast<size_t>(layer) * desc->B * desc->H_kv * 2 * kTile * kD * 2;

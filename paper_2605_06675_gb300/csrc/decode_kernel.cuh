@@ -58,7 +58,11 @@ struct DecodeArgs {
   float* partial;            // [B][H_q][splits][132]
   const int32_t* n_rows;     // tokens attended per batch row (rq_decode_attention_rows) or null
   uint32_t* status;
-  int layer, B, H, Hq, g, nblk, splits, bps, kg, vg, hadamard;
+  // split plan: (batch, kv head) units [0, u_lo) take s_lo CTAs of bps_lo
+  // blocks, the others `splits` CTAs of bps blocks (splits = s_lo or s_lo + 1;
+  // it is also the record stride per query row); the grid is 1-D, the
+  // s_lo-split units' (larger) CTAs first
+  int layer, B, H, Hq, g, nblk, splits, bps, s_lo, bps_lo, u_lo, kg, vg, hadamard;
   int kq, vq;                // rq_quantizer of keys / values
   LMBook lm;                 // RQ_LLOYDMAX codebooks
 };
@@ -760,7 +764,21 @@ __global__ void __launch_bounds__(kThreads, RQ_DECODE_MIN_BLOCKS) decode_split_k
   __shared__ float red_m[kWarps][kMaxHeads];
   __shared__ float red_l[kWarps][kMaxHeads];
   __shared__ uint16_t lmtab[2][256];                // Lloyd-Max codebooks of this head's widths
-  const int split = blockIdx.x, h = blockIdx.y, batch = blockIdx.z;
+  int unit, split, bps;
+  {
+    const int c = blockIdx.x, nlo = a.u_lo * a.s_lo;
+    if (c < nlo) {
+      unit = c / a.s_lo;
+      split = c - unit * a.s_lo;
+      bps = a.bps_lo;
+    } else {
+      const int c2 = c - nlo, u2 = c2 / a.splits;
+      unit = a.u_lo + u2;
+      split = c2 - u2 * a.splits;
+      bps = a.bps;
+    }
+  }
+  const int batch = unit / a.H, h = unit - batch * a.H;
   const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
   const int gid = lane >> 2, tig = lane & 3;
 
@@ -795,8 +813,8 @@ __global__ void __launch_bounds__(kThreads, RQ_DECODE_MIN_BLOCKS) decode_split_k
     const int n = a.n_rows[batch];
     nblk_row = (n >= 1 && n <= a.nblk * kTile) ? n / kTile : 0;
   }
-  const int blk0 = split * a.bps;
-  const int blk1 = min(nblk_row, blk0 + a.bps);
+  const int blk0 = split * bps;
+  const int blk1 = min(nblk_row, blk0 + bps);
   const int blk_first = blk0 + warp;
   WarpStream ws;
   ws.lane = lane;
@@ -1060,7 +1078,8 @@ template <int CQ, typename T>
 __global__ void __launch_bounds__(kThreads) decode_merge_kernel(const float* partial, float* out,
                                                                 const int8_t* signs,
                                                                 uint32_t* status, int Hq, int H,
-                                                                int g, int splits, int hadamard,
+                                                                int g, int splits, int s_lo,
+                                                                int u_lo, int hadamard,
                                                                 const T* q, const T* residual,
                                                                 int R, const int32_t* n_rows,
                                                                 int cap) {
@@ -1085,6 +1104,7 @@ __global__ void __launch_bounds__(kThreads) decode_merge_kernel(const float* par
   const int batch = blockIdx.x / H, h = blockIdx.x % H, part = blockIdx.y;
   const long long row0 = static_cast<long long>(batch) * Hq + h * g;
   const long long rstride = static_cast<long long>(splits) * kPart;
+  const int ns = static_cast<int>(blockIdx.x) < u_lo ? s_lo : splits;   // this unit's records
   const float* p = partial + row0 * rstride + part * CW;     // o slice of row 0, split 0
   const float* pml = partial + row0 * rstride + kD;           // (m, l) of row 0, split 0
   // splits per chunk: shared budget, and at most 64 (one weight per lane pair)
@@ -1103,8 +1123,8 @@ __global__ void __launch_bounds__(kThreads) decode_merge_kernel(const float* par
                            acc);
   const uint32_t sbase = static_cast<uint32_t>(__cvta_generic_to_shared(msm));
 
-  for (int c0 = 0; c0 < splits; c0 += cs_max) {
-    const int cs = min(cs_max, splits - c0);
+  for (int c0 = 0; c0 < ns; c0 += cs_max) {
+    const int cs = min(cs_max, ns - c0);
     // piece (n, s, i): i < CH the o slice, i == CH (m, l, pad, pad)
     const int npieces = g * cs * SLOT;
     for (int x = tid; x < npieces; x += kThreads) {
@@ -1222,8 +1242,9 @@ inline rq_status launch_decode_t(const DecodeArgs& a, float* out, const void* re
       cudaFuncSetAttribute(kern, cudaFuncAttributePreferredSharedMemoryCarveout,
                            cudaSharedmemCarveoutMaxShared) != cudaSuccess)
     return RQ_ERR_CUDA;
-  const dim3 grid(static_cast<unsigned>(a.splits), static_cast<unsigned>(a.H), static_cast<unsigned>(a.B));
-  kern<<<grid, kThreads, kSmemBytes, s>>>(a);
+  const long long nlo = static_cast<long long>(a.u_lo) * a.s_lo;
+  const long long ncta = nlo + (static_cast<long long>(a.B) * a.H - a.u_lo) * a.splits;
+  kern<<<static_cast<unsigned>(ncta), kThreads, kSmemBytes, s>>>(a);
   if (cudaGetLastError() != cudaSuccess) return RQ_ERR_CUDA;
   // a whole row per CTA for a rotated cache (the rotation mixes channels),
   // a quarter of the channels otherwise (four times the CTAs)
@@ -1242,7 +1263,7 @@ inline rq_status launch_decode_t(const DecodeArgs& a, float* out, const void* re
   if (cudaFuncSetAttribute(mk, cudaFuncAttributeMaxDynamicSharedMemorySize, kMergeSmem) != cudaSuccess)
     return RQ_ERR_CUDA;
   if (cudaLaunchKernelEx(&cfg, mk, static_cast<const float*>(a.partial), out, a.signs, a.status,
-                         a.Hq, a.H, a.g, a.splits, a.hadamard, static_cast<const T*>(a.q),
+                         a.Hq, a.H, a.g, a.splits, a.s_lo, a.u_lo, a.hadamard, static_cast<const T*>(a.q),
                          static_cast<const T*>(res_layer), R, a.n_rows, a.nblk * kTile) != cudaSuccess)
     return RQ_ERR_CUDA;
   return launch_status();
