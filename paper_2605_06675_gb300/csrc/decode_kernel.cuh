@@ -1083,7 +1083,8 @@ __global__ void __launch_bounds__(kThreads) decode_merge_kernel(const float* par
                                                                 const T* q, const T* residual,
                                                                 int R, const int32_t* n_rows,
                                                                 int cap) {
-  asm volatile("griddepcontrol.wait;\n" ::: "memory");
+  // everything up to the wait reads only this call's inputs, so it overlaps
+  // the split grid's tail
   bool row_ok = true;
   if (n_rows) {                  // a token count per batch row: its own residual tokens
     const int n = n_rows[blockIdx.x / H];
@@ -1096,6 +1097,7 @@ __global__ void __launch_bounds__(kThreads) decode_merge_kernel(const float* par
   constexpr int CH = CW / 4;           // 16-byte pieces of a record's o slice
   constexpr int SLOT = CH + 1;         // pieces per (row, split): o slice, then (m, l, pad)
   constexpr int PAIRS = kMaxHeads * CW / kThreads;   // (row, channel) pairs per thread, at most
+  static_assert(PAIRS >= 1, "every thread owns a (row, channel) pair");
   extern __shared__ float4 msm[];
   __shared__ float wgt[kMaxHeads][64];
   __shared__ float run_m[kMaxHeads], run_l[kMaxHeads], run_scale[kMaxHeads];
@@ -1103,10 +1105,16 @@ __global__ void __launch_bounds__(kThreads) decode_merge_kernel(const float* par
   const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
   const int batch = blockIdx.x / H, h = blockIdx.x % H, part = blockIdx.y;
   const long long row0 = static_cast<long long>(batch) * Hq + h * g;
-  const long long rstride = static_cast<long long>(splits) * kPart;
+  const int rs = splits * kPart;                               // floats between query rows
   const int ns = static_cast<int>(blockIdx.x) < u_lo ? s_lo : splits;   // this unit's records
-  const float* p = partial + row0 * rstride + part * CW;     // o slice of row 0, split 0
-  const float* pml = partial + row0 * rstride + kD;           // (m, l) of row 0, split 0
+  const float* base = partial + row0 * rs;                     // row 0, split 0
+  // sign flips of the thread's channels for the rotation back (bit k: pair k)
+  uint32_t negmask = 0;
+  if (CQ == 1 && hadamard && signs) {
+#pragma unroll
+    for (int k = 0; k < PAIRS; ++k)
+      if (signs[(tid + kThreads * k) % CW] < 0) negmask |= 1u << k;
+  }
   // splits per chunk: shared budget, and at most 64 (one weight per lane pair)
   const int cs_max = min(64, kMergeSmem / (g * SLOT * 16));
   if (tid < kMaxHeads) {
@@ -1122,15 +1130,32 @@ __global__ void __launch_bounds__(kThreads) decode_merge_kernel(const float* par
                            R, g, signs, hadamard, part, reinterpret_cast<float*>(msm), y, run_m, run_l,
                            acc);
   const uint32_t sbase = static_cast<uint32_t>(__cvta_generic_to_shared(msm));
+  asm volatile("griddepcontrol.wait;\n" ::: "memory");
 
   for (int c0 = 0; c0 < ns; c0 += cs_max) {
     const int cs = min(cs_max, ns - c0);
-    // piece (n, s, i): i < CH the o slice, i == CH (m, l, pad, pad)
+    // piece x = (n cs + sl) SLOT + i: i < CH the o slice, i == CH (m, l, pad,
+    // pad); the thread steps x by kThreads with a mixed-radix carry instead
+    // of dividing per piece
     const int npieces = g * cs * SLOT;
-    for (int x = tid; x < npieces; x += kThreads) {
-      const int i = x % SLOT, ns = x / SLOT, n = ns / cs, sl = ns % cs;
-      const float* src = (i < CH ? p + 4 * i : pml) + n * rstride + static_cast<long long>(c0 + sl) * kPart;
-      asm volatile("cp.async.cg.shared.global [%0], [%1], 16;\n" ::"r"(sbase + 16 * x), "l"(src));
+    {
+      constexpr int DI = kThreads % SLOT, DR = kThreads / SLOT;
+      int i = tid % SLOT, sl = tid / SLOT, n = sl / cs;
+      sl -= n * cs;
+      for (int x = tid; x < npieces; x += kThreads) {
+        const int off = n * rs + (c0 + sl) * kPart + (i < CH ? part * CW + 4 * i : kD);
+        asm volatile("cp.async.cg.shared.global [%0], [%1], 16;\n" ::"r"(sbase + 16 * x), "l"(base + off));
+        i += DI;
+        sl += DR;
+        if (i >= SLOT) {
+          i -= SLOT;
+          ++sl;
+        }
+        while (sl >= cs) {
+          sl -= cs;
+          ++n;
+        }
+      }
     }
     asm volatile("cp.async.commit_group;\n" ::);
     asm volatile("cp.async.wait_group 0;\n" ::);
@@ -1215,11 +1240,10 @@ __global__ void __launch_bounds__(kThreads) decode_merge_kernel(const float* par
     fwht_smem(y, g);
 #pragma unroll
     for (int k = 0; k < PAIRS; ++k) {
-      const int pi = tid + kThreads * k, c = pi % CW;
+      const int pi = tid + kThreads * k;
       if (pi / CW < g) {
-        float v = y[pi] * kInvSqrt128;
-        if (signs && signs[c] < 0) v = -v;
-        acc[k] = v;
+        const float v = y[pi] * kInvSqrt128;
+        acc[k] = (negmask >> k) & 1u ? -v : v;
       }
     }
   }
@@ -1247,8 +1271,10 @@ inline rq_status launch_decode_t(const DecodeArgs& a, float* out, const void* re
   kern<<<static_cast<unsigned>(ncta), kThreads, kSmemBytes, s>>>(a);
   if (cudaGetLastError() != cudaSuccess) return RQ_ERR_CUDA;
   // a whole row per CTA for a rotated cache (the rotation mixes channels),
-  // a quarter of the channels otherwise (four times the CTAs)
-  const int cq = a.hadamard ? 1 : 4;
+  // a quarter of the channels otherwise (four times the CTAs), an eighth when
+  // there are few (batch, kv head) units (the records of a unit are then
+  // many, and more CTAs pull them in parallel)
+  const int cq = a.hadamard ? 1 : (static_cast<long long>(a.B) * a.H <= 32 ? 8 : 4);
   cudaLaunchConfig_t cfg = {};
   cfg.gridDim = dim3(static_cast<unsigned>(a.B * a.H), static_cast<unsigned>(cq));
   cfg.blockDim = dim3(kThreads);
@@ -1259,7 +1285,7 @@ inline rq_status launch_decode_t(const DecodeArgs& a, float* out, const void* re
   attr[0].val.programmaticStreamSerializationAllowed = 1;
   cfg.attrs = attr;
   cfg.numAttrs = 1;
-  auto mk = a.hadamard ? decode_merge_kernel<1, T> : decode_merge_kernel<4, T>;
+  auto mk = cq == 1 ? decode_merge_kernel<1, T> : cq == 8 ? decode_merge_kernel<8, T> : decode_merge_kernel<4, T>;
   if (cudaFuncSetAttribute(mk, cudaFuncAttributeMaxDynamicSharedMemorySize, kMergeSmem) != cudaSuccess)
     return RQ_ERR_CUDA;
   if (cudaLaunchKernelEx(&cfg, mk, static_cast<const float*>(a.partial), out, a.signs, a.status,
