@@ -1006,6 +1006,7 @@ __global__ void __launch_bounds__(kThreads, RQ_DECODE_MIN_BLOCKS) decode_split_k
 // memory with cp.async, a chunk of splits at a time (one round trip per
 // chunk), and merged there with a running max per row.
 constexpr int kMergeSmem = 64 * 1024;
+constexpr int kMergeChunk = 128;     // split records merged per round trip, at most
 
 // The unquantized residual tokens (decode-time append) of one (batch, kv
 // head): their exact fp32 attention record (m, l, o) for the g query rows
@@ -1099,7 +1100,7 @@ __global__ void __launch_bounds__(kThreads) decode_merge_kernel(const float* par
   constexpr int PAIRS = kMaxHeads * CW / kThreads;   // (row, channel) pairs per thread, at most
   static_assert(PAIRS >= 1, "every thread owns a (row, channel) pair");
   extern __shared__ float4 msm[];
-  __shared__ float wgt[kMaxHeads][64];
+  __shared__ float wgt[kMaxHeads][kMergeChunk];
   __shared__ float run_m[kMaxHeads], run_l[kMaxHeads], run_scale[kMaxHeads];
   __shared__ float y[kMaxHeads * kD];
   const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
@@ -1115,8 +1116,8 @@ __global__ void __launch_bounds__(kThreads) decode_merge_kernel(const float* par
     for (int k = 0; k < PAIRS; ++k)
       if (signs[(tid + kThreads * k) % CW] < 0) negmask |= 1u << k;
   }
-  // splits per chunk: shared budget, and at most 64 (one weight per lane pair)
-  const int cs_max = min(64, kMergeSmem / (g * SLOT * 16));
+  // splits per chunk: shared budget, and at most kMergeChunk (four weights per lane)
+  const int cs_max = min(kMergeChunk, kMergeSmem / (g * SLOT * 16));
   if (tid < kMaxHeads) {
     run_m[tid] = -INFINITY;
     run_l[tid] = 0.0f;
@@ -1160,14 +1161,14 @@ __global__ void __launch_bounds__(kThreads) decode_merge_kernel(const float* par
     asm volatile("cp.async.commit_group;\n" ::);
     asm volatile("cp.async.wait_group 0;\n" ::);
     __syncthreads();
-    // warp w: rows w, w + 4; lanes over the chunk's splits (two per lane)
+    // warp w: rows w, w + 4; lanes over the chunk's splits (four per lane)
 #pragma unroll
     for (int k = 0; k < 2; ++k) {
       const int n = warp + kWarps * k;
       if (n < g) {
-        float mv[2], lv[2], mx = -INFINITY;
+        float mv[kMergeChunk / 32], lv[kMergeChunk / 32], mx = -INFINITY;
 #pragma unroll
-        for (int r = 0; r < 2; ++r) {
+        for (int r = 0; r < kMergeChunk / 32; ++r) {
           const int sl = lane + 32 * r;
           mv[r] = -INFINITY;
           lv[r] = 0.0f;
@@ -1184,7 +1185,7 @@ __global__ void __launch_bounds__(kThreads) decode_merge_kernel(const float* par
         const float mnew = fmaxf(mold, mx);
         float l = 0.0f;
 #pragma unroll
-        for (int r = 0; r < 2; ++r) {
+        for (int r = 0; r < kMergeChunk / 32; ++r) {
           const int sl = lane + 32 * r;
           const float wv = (mv[r] == -INFINITY) ? 0.0f : exp2f(mv[r] - mnew);
           if (sl < cs) wgt[n][sl] = wv;
@@ -1231,20 +1232,39 @@ __global__ void __launch_bounds__(kThreads) decode_merge_kernel(const float* par
     }
   }
   if (CQ == 1 && hadamard) {
+    // FWHT of each row: thread c holds channel c of every row (acc[k] is row
+    // k); strides 1 .. 16 are lane exchanges, strides 32 and 64 go through
+    // shared memory. Every output is one fp32 a + b or a - b, as in the
+    // butterfly order of the in-place transform.
 #pragma unroll
-    for (int k = 0; k < PAIRS; ++k) {
-      const int pi = tid + kThreads * k;
-      if (pi / CW < g) y[pi] = acc[k];
-    }
-    __syncthreads();
-    fwht_smem(y, g);
+    for (int st = 1; st <= 16; st <<= 1) {
+      const bool up = lane & st;
 #pragma unroll
-    for (int k = 0; k < PAIRS; ++k) {
-      const int pi = tid + kThreads * k;
-      if (pi / CW < g) {
-        const float v = y[pi] * kInvSqrt128;
-        acc[k] = (negmask >> k) & 1u ? -v : v;
+      for (int k = 0; k < PAIRS; ++k) {
+        const float o = __shfl_xor_sync(0xffffffffu, acc[k], st);
+        acc[k] = up ? o - acc[k] : acc[k] + o;
       }
+    }
+#pragma unroll
+    for (int st = 32; st <= 64; st <<= 1) {
+      const bool up = tid & st;
+#pragma unroll
+      for (int k = 0; k < PAIRS; ++k)
+        if (k < g) y[k * kD + tid] = acc[k];
+      __syncthreads();
+#pragma unroll
+      for (int k = 0; k < PAIRS; ++k) {
+        if (k < g) {
+          const float o = y[k * kD + (tid ^ st)];
+          acc[k] = up ? o - acc[k] : acc[k] + o;
+        }
+      }
+      __syncthreads();
+    }
+#pragma unroll
+    for (int k = 0; k < PAIRS; ++k) {
+      const float v = acc[k] * kInvSqrt128;
+      acc[k] = (negmask >> k) & 1u ? -v : v;
     }
   }
 #pragma unroll
