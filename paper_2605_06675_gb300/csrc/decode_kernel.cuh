@@ -782,6 +782,18 @@ __global__ void __launch_bounds__(kThreads, RQ_DECODE_MIN_BLOCKS) decode_split_k
   const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
   const int gid = lane >> 2, tig = lane & 3;
 
+  // q of the g query heads of this kv head (rows >= g are zero), sign-flipped
+  // for a Hadamard-rotated cache. Its loads go out first: issued after the
+  // ring's first copies (every CTA's at once) they would queue behind them,
+  // and the q prologue, which the block loop waits for, with them.
+  static_assert(kD == kThreads, "thread d loads channel d of every row");
+  const T* qp = static_cast<const T*>(a.q) + (static_cast<long long>(batch) * a.Hq +
+                                              static_cast<long long>(h) * a.g) * kD;
+  float qreg[kMaxHeads];
+#pragma unroll
+  for (int n = 0; n < kMaxHeads; ++n) qreg[n] = n < a.g ? to_f32<T>(qp[n * kD + threadIdx.x]) : 0.0f;
+  const bool qneg = a.hadamard && a.signs && a.signs[threadIdx.x] < 0;
+
   const int bK = a.bits[(a.layer * a.H + h) * 2 + 0];
   const int bV = a.bits[(a.layer * a.H + h) * 2 + 1];
   const bool valid = bK >= 1 && bK <= 8 && bV >= 1 && bV <= 8;
@@ -836,21 +848,12 @@ __global__ void __launch_bounds__(kThreads, RQ_DECODE_MIN_BLOCKS) decode_split_k
     default: prologue_dyn(ws, dr); break;
   }
 
-  // q of the g query heads of this kv head (rows >= g are zero), rotated
-  // into the cache's domain when the cache is Hadamard-rotated
-  const T* qp = static_cast<const T*>(a.q) + (static_cast<long long>(batch) * a.Hq +
-                                              static_cast<long long>(h) * a.g) * kD;
-  for (int idx = threadIdx.x; idx < kMaxHeads * kD; idx += kThreads) {
-    const int n = idx >> 7, d = idx & 127;
-    float x = 0.0f;
-    if (n < a.g) {
-      x = to_f32<T>(qp[n * kD + d]);
-      if (a.hadamard && a.signs && a.signs[d] < 0) x = -x;
-    }
-    qs[idx] = x;
-  }
+  // q into shared memory, rotated into the cache's domain when the cache is
+  // Hadamard-rotated (rows >= g stay zero)
+#pragma unroll
+  for (int n = 0; n < kMaxHeads; ++n) qs[n * kD + threadIdx.x] = qneg ? -qreg[n] : qreg[n];
   __syncthreads();
-  if (a.hadamard) fwht_smem(qs, kMaxHeads);
+  if (a.hadamard) fwht_smem(qs, a.g);
   // q enters the MMAs scaled by a power of two only (no rounding beyond its
   // fp16 conversion); the rest of the softmax scale 1/sqrt(128) * log2(e) is
   // applied to the fp32 scores (log2 units).
