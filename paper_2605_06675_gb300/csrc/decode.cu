@@ -33,7 +33,8 @@ using dk::DecodeArgs;
 using dk::kMaxHeads;
 using dk::kPart;
 
-// Resident split-kernel CTAs per SM on the current device (cached per device).
+// Resident splits per SM on the current device (cached per device): resident
+// split-kernel CTAs x the split groups of a CTA.
 rq_status split_ctas_per_sm(int* per_sm) {
   static std::atomic<int> cache[64];
   int dev = 0;
@@ -53,21 +54,21 @@ rq_status split_ctas_per_sm(int* per_sm) {
 }
 
 struct SplitPlan {
-  int splits, bps;      // units [u_lo, B * H_kv): CTAs and blocks per CTA
+  int splits, bps;      // units [u_lo, B * H_kv): splits and blocks per split
   int s_lo, bps_lo;     // units [0, u_lo)
   int u_lo;
 };
 
-// Splits of the sequence per (batch, kv head) unit: as many CTAs as fit in one
-// wave of resident CTAs (slots = SMs x CTAs per SM), so every CTA streams a
-// long run of blocks and none waits for a second wave; at least one per unit.
-// When the units do not divide the slots, the wave is filled with two split
-// counts: units [0, u_lo) take s_lo = slots / units splits and the rest
-// s_lo + 1, so that every SM holds the same number of CTAs (a grid of
-// units x s_lo CTAs would leave some SMs one CTA short and the others, with
-// their full complement, setting the time). The s_lo-split units' CTAs (the
-// larger ones) come first in the grid, so the round-robin dispatch spreads
-// them over the SMs.
+// Splits of the sequence per (batch, kv head) unit: as many as fit in one
+// wave of resident splits (slots = SMs x splits per SM), so every split
+// streams a long run of blocks and none waits for a second wave; at least one
+// per unit. When the units do not divide the slots, the wave is filled with
+// two split counts: units [0, u_lo) take s_lo = slots / units splits and the
+// rest s_lo + 1, so that every SM holds the same number of splits (units x
+// s_lo splits would leave some SMs one split short and the others, with
+// their full complement, setting the time). The s_lo-split units' splits
+// (the larger ones) come first in the plan; the kernel deals the plan's
+// quarters to the four groups of its CTAs, so every SM gets a like mix.
 // nblk: the packed blocks attended (<= the capacity's); splits <= the
 // capacity's split bound (max_splits), which sizes the workspace.
 int max_splits(const rq_cache_desc* desc, int slots) {

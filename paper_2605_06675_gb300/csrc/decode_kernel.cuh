@@ -35,18 +35,20 @@
 namespace rq {
 namespace dk {
 
-// CTAs per SM the decoder's register budget is sized for
-#ifndef RQ_DECODE_MIN_BLOCKS
-#define RQ_DECODE_MIN_BLOCKS 4
-#endif
-constexpr int kWarps = 4;
+constexpr int kWarps = 4;                 // warps per split (a group; the merge kernel's CTA)
 constexpr int kThreads = 32 * kWarps;
+constexpr int kGroups = 4;                // split groups per decode CTA
 constexpr int kPart = kD + 4;        // partial record: o[128], m (log2 domain), l, 2 pad (16-byte rows)
 constexpr int kMaxHeads = 8;         // MMA n
 constexpr int kRingBytes = 11264;    // per-warp ring of shared-memory slots
 constexpr int kMaxSlots = 8;
 constexpr int kQBytes = kMaxHeads * kD * 4;
-constexpr int kSmemBytes = kQBytes + kWarps * kRingBytes;   // 49152: 4 CTAs per SM
+constexpr int kSmemBytes = kQBytes + kWarps * kRingBytes;   // 49152: q table and rings of a split group
+// a split group's shared memory: q table, rings, the warps' (m, l) and two
+// Lloyd-Max codebooks (50432 bytes, a multiple of 128)
+constexpr int kGroupBytes = kSmemBytes + 2 * kWarps * kMaxHeads * 4 + 2 * 256 * 2;
+constexpr int kSplitSmem = kGroups * kGroupBytes;            // per four-group CTA
+static_assert(kGroupBytes % 128 == 0, "group areas start on 128-byte boundaries");
 static_assert(kWarps * kMaxHeads * kD * 4 <= kWarps * kRingBytes, "merge buffer aliases rings");
 
 struct DecodeArgs {
@@ -497,6 +499,35 @@ __device__ __forceinline__ void pv_dispatch(int bw, int vg, const uint8_t* img, 
 }
 
 // 128-point FWHT of each of `rows` rows of x (row stride 128), strides 1..64
+// named barrier of split group grp (kThreads threads; barrier 0 is the
+// CTA's). Immediate barrier ids: a register id would reserve all 16 of the
+// CTA's barriers.
+__device__ __forceinline__ void group_sync(int grp) {
+  switch (grp) {
+    case 0: asm volatile("bar.sync 1, %0;\n" ::"n"(kThreads) : "memory"); break;
+    case 1: asm volatile("bar.sync 2, %0;\n" ::"n"(kThreads) : "memory"); break;
+    case 2: asm volatile("bar.sync 3, %0;\n" ::"n"(kThreads) : "memory"); break;
+    default: asm volatile("bar.sync 4, %0;\n" ::"n"(kThreads) : "memory"); break;
+  }
+}
+static_assert(kGroups == 4, "group_sync names four barriers");
+
+// fwht_smem for one split group: thread tl of group grp
+__device__ inline void fwht_smem_group(float* x, int rows, int tl, int grp) {
+  for (int lh = 0; lh < 7; ++lh) {
+    const int h = 1 << lh;
+    for (int p = tl; p < rows * 64; p += kThreads) {
+      const int row = p >> 6, pi = p & 63;
+      const int i = ((pi >> lh) << (lh + 1)) | (pi & (h - 1));
+      float* r = x + row * kD;
+      const float a = r[i], b = r[i + h];
+      r[i] = a + b;
+      r[i + h] = a - b;
+    }
+    group_sync(grp);
+  }
+}
+
 __device__ inline void fwht_smem(float* x, int rows) {
   for (int lh = 0; lh < 7; ++lh) {
     const int h = 1 << lh;
@@ -753,20 +784,36 @@ __device__ __forceinline__ int fast_key(int bK, int bV, int kg, int vg) {
   X(24, 5, 5)
 
 template <typename T>
-__global__ void __launch_bounds__(kThreads, RQ_DECODE_MIN_BLOCKS) decode_split_kernel(DecodeArgs a) {
-  // The dynamic area starts on a 128-byte boundary (the static arrays below
-  // are 1280 bytes): the cp.async rings in it then take whole 128-byte lines
-  // per 8 lanes; a ring off that boundary doubles the L2 sectors every copy
-  // moves.
-  extern __shared__ __align__(128) unsigned char smem_raw[];
+__global__ void __launch_bounds__(kThreads * kGroups, 1) decode_split_kernel(DecodeArgs a) {
+  // A CTA is G = blockDim.x / kThreads (1 or kGroups) independent groups of
+  // kWarps warps, one split each (split c = group * CTAs + CTA index, so that
+  // with four groups every CTA takes splits from each quarter of the plan: as
+  // many of the larger ones as the others); a group synchronises on its own
+  // named barrier. The warp schedulers serve the warps of one CTA evenly but
+  // favour the CTAs that reached an SM first: four one-group CTAs per SM
+  // finish far apart (the last ones alone on their SMs), one four-group CTA
+  // per SM finishes together but streams a little slower per SM. The launch
+  // picks the layout per query-group size.
+  // No static shared memory: every group's area starts on a 128-byte
+  // boundary, so its cp.async rings take whole 128-byte lines per 8 lanes (a
+  // ring off that boundary doubles the L2 sectors every copy moves).
+  extern __shared__ __align__(128) unsigned char smem_dyn[];
+  const int grp = threadIdx.x / kThreads, tl = threadIdx.x % kThreads;   // G = blockDim.x / kThreads
+  const long long c = static_cast<long long>(grp) * gridDim.x + blockIdx.x;
+  {
+    const long long units = static_cast<long long>(a.B) * a.H;
+    if (c >= units * a.s_lo + (units - a.u_lo) * (a.splits - a.s_lo)) return;   // no split
+  }
+  unsigned char* smem_raw = smem_dyn + grp * kGroupBytes;
   float* qs = reinterpret_cast<float*>(smem_raw);                  // [8][128]
   uint8_t* rings = smem_raw + kQBytes;
-  __shared__ float red_m[kWarps][kMaxHeads];
-  __shared__ float red_l[kWarps][kMaxHeads];
-  __shared__ uint16_t lmtab[2][256];                // Lloyd-Max codebooks of this head's widths
+  float (*red_m)[kMaxHeads] = reinterpret_cast<float (*)[kMaxHeads]>(smem_raw + kSmemBytes);
+  float (*red_l)[kMaxHeads] = red_m + kWarps;
+  // Lloyd-Max codebooks of the group's widths
+  uint16_t (*lmtab)[256] = reinterpret_cast<uint16_t (*)[256]>(red_l + kWarps);
   int unit, split, bps;
   {
-    const int c = blockIdx.x, nlo = a.u_lo * a.s_lo;
+    const int nlo = a.u_lo * a.s_lo;
     if (c < nlo) {
       unit = c / a.s_lo;
       split = c - unit * a.s_lo;
@@ -779,7 +826,7 @@ __global__ void __launch_bounds__(kThreads, RQ_DECODE_MIN_BLOCKS) decode_split_k
     }
   }
   const int batch = unit / a.H, h = unit - batch * a.H;
-  const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+  const int lane = tl & 31, warp = tl >> 5;
   const int gid = lane >> 2, tig = lane & 3;
 
   // q of the g query heads of this kv head (rows >= g are zero), sign-flipped
@@ -791,13 +838,13 @@ __global__ void __launch_bounds__(kThreads, RQ_DECODE_MIN_BLOCKS) decode_split_k
                                               static_cast<long long>(h) * a.g) * kD;
   float qreg[kMaxHeads];
 #pragma unroll
-  for (int n = 0; n < kMaxHeads; ++n) qreg[n] = n < a.g ? to_f32<T>(qp[n * kD + threadIdx.x]) : 0.0f;
-  const bool qneg = a.hadamard && a.signs && a.signs[threadIdx.x] < 0;
+  for (int n = 0; n < kMaxHeads; ++n) qreg[n] = n < a.g ? to_f32<T>(qp[n * kD + tl]) : 0.0f;
+  const bool qneg = a.hadamard && a.signs && a.signs[tl] < 0;
 
   const int bK = a.bits[(a.layer * a.H + h) * 2 + 0];
   const int bV = a.bits[(a.layer * a.H + h) * 2 + 1];
   const bool valid = bK >= 1 && bK <= 8 && bV >= 1 && bV <= 8;
-  if (!valid && threadIdx.x == 0) set_status(a.status, RQ_STATUS_BAD_BITS);
+  if (!valid && tl == 0) set_status(a.status, RQ_STATUS_BAD_BITS);
   const uint64_t* offp =
       a.offsets + ((static_cast<long long>(a.layer) * a.B + batch) * a.H + h) * 2;
   const uint8_t* kbase = a.packed + (valid ? offp[0] : 0);
@@ -808,7 +855,7 @@ __global__ void __launch_bounds__(kThreads, RQ_DECODE_MIN_BLOCKS) decode_split_k
   dr.kg = a.kg;
   dr.vg = a.vg;
   const bool lmk = valid && a.kq == RQ_LLOYDMAX, lmv = valid && a.vq == RQ_LLOYDMAX;
-  for (int i = threadIdx.x; i < 256; i += kThreads) {
+  for (int i = tl; i < 256; i += kThreads) {
     if (lmk && i < (1 << bK)) lmtab[0][i] = a.lm.lv[lm_offset(bK) + i];
     if (lmv && i < (1 << bV)) lmtab[1][i] = a.lm.lv[lm_offset(bV) + i];
   }
@@ -851,9 +898,9 @@ __global__ void __launch_bounds__(kThreads, RQ_DECODE_MIN_BLOCKS) decode_split_k
   // q into shared memory, rotated into the cache's domain when the cache is
   // Hadamard-rotated (rows >= g stay zero)
 #pragma unroll
-  for (int n = 0; n < kMaxHeads; ++n) qs[n * kD + threadIdx.x] = qneg ? -qreg[n] : qreg[n];
-  __syncthreads();
-  if (a.hadamard) fwht_smem(qs, a.g);
+  for (int n = 0; n < kMaxHeads; ++n) qs[n * kD + tl] = qneg ? -qreg[n] : qreg[n];
+  group_sync(grp);
+  if (a.hadamard) fwht_smem_group(qs, a.g, tl, grp);
   // q enters the MMAs scaled by a power of two only (no rounding beyond its
   // fp16 conversion); the rest of the softmax scale 1/sqrt(128) * log2(e) is
   // applied to the fp32 scores (log2 units).
@@ -887,7 +934,7 @@ __global__ void __launch_bounds__(kThreads, RQ_DECODE_MIN_BLOCKS) decode_split_k
     const float* qr = qs + (lane & 7) * kD + 32 * (lane >> 3);
     for (int c = 0; c < 32; ++c) qgsum += __half2float(__float2half_rn(qr[c] * qpow));
   }
-  __syncthreads();                  // qs is read; its space becomes the q operand table
+  group_sync(grp);                  // qs is read; its space becomes the q operand table
   uint8_t* qtab = smem_raw;
   if (warp == 0) {
 #pragma unroll
@@ -899,7 +946,7 @@ __global__ void __launch_bounds__(kThreads, RQ_DECODE_MIN_BLOCKS) decode_split_k
     }
     if (a.kg == RQ_PER_TOKEN) reinterpret_cast<float*>(qtab + 2048)[lane] = qgsum;   // [G][n]
   }
-  __syncthreads();
+  group_sync(grp);
 
   SoftmaxAcc acc;
 #pragma unroll
@@ -957,7 +1004,7 @@ __global__ void __launch_bounds__(kThreads, RQ_DECODE_MIN_BLOCKS) decode_split_k
   }
   // merge the four warps (log-sum-exp), one partial record per query head;
   // the merge buffer reuses the rings
-  __syncthreads();
+  group_sync(grp);
   float* red_o = reinterpret_cast<float*>(rings);   // [warp][head][channel]
 #pragma unroll
   for (int mt = 0; mt < 8; ++mt) {
@@ -976,8 +1023,8 @@ __global__ void __launch_bounds__(kThreads, RQ_DECODE_MIN_BLOCKS) decode_split_k
     red_l[warp][2 * tig] = l0;
     red_l[warp][2 * tig + 1] = l1;
   }
-  __syncthreads();
-  const int d = threadIdx.x;
+  group_sync(grp);
+  const int d = tl;
   for (int n = 0; n < a.g; ++n) {
     float M = -INFINITY;
 #pragma unroll
@@ -1285,13 +1332,17 @@ inline rq_status launch_decode_t(const DecodeArgs& a, float* out, const void* re
                                  cudaStream_t s) {
   // a token count per batch row: every row may hold residual tokens
   auto kern = decode_split_kernel<T>;
-  if (cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, kSmemBytes) != cudaSuccess ||
+  if (cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, kSplitSmem) != cudaSuccess ||
       cudaFuncSetAttribute(kern, cudaFuncAttributePreferredSharedMemoryCarveout,
                            cudaSharedmemCarveoutMaxShared) != cudaSuccess)
     return RQ_ERR_CUDA;
   const long long nlo = static_cast<long long>(a.u_lo) * a.s_lo;
-  const long long ncta = nlo + (static_cast<long long>(a.B) * a.H - a.u_lo) * a.splits;
-  kern<<<static_cast<unsigned>(ncta), kThreads, kSmemBytes, s>>>(a);
+  const long long nsplit = nlo + (static_cast<long long>(a.B) * a.H - a.u_lo) * a.splits;
+  // four groups per CTA when the query group takes the merged hi/lo MMA
+  // (g <= 4: measured 2-3 % faster on those layers), one otherwise (g = 8:
+  // 2-3 % slower as four groups)
+  const int G = a.g <= kMaxHeads / 2 ? kGroups : 1;
+  kern<<<static_cast<unsigned>((nsplit + G - 1) / G), kThreads * G, G * kGroupBytes, s>>>(a);
   if (cudaGetLastError() != cudaSuccess) return RQ_ERR_CUDA;
   // a whole row per CTA for a rotated cache (the rotation mixes channels),
   // a quarter of the channels otherwise (four times the CTAs), an eighth when
@@ -1318,17 +1369,21 @@ inline rq_status launch_decode_t(const DecodeArgs& a, float* out, const void* re
   return launch_status();
 }
 
-// Resident split-kernel CTAs per SM on the current device (occupancy query).
+// Resident splits per SM on the current device: the smaller of the resident
+// one-group CTAs and kGroups x the resident four-group CTAs (occupancy
+// queries; both are 4 on GB300).
 template <typename T>
 inline rq_status split_ctas_per_sm_t(int* per_sm) {
   auto kern = decode_split_kernel<T>;
-  if (cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, kSmemBytes) != cudaSuccess ||
+  if (cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, kSplitSmem) != cudaSuccess ||
       cudaFuncSetAttribute(kern, cudaFuncAttributePreferredSharedMemoryCarveout,
                            cudaSharedmemCarveoutMaxShared) != cudaSuccess)
     return RQ_ERR_CUDA;
-  int v = 0;
-  if (cudaOccupancyMaxActiveBlocksPerMultiprocessor(&v, kern, kThreads, kSmemBytes) != cudaSuccess)
+  int v1 = 0, v4 = 0;
+  if (cudaOccupancyMaxActiveBlocksPerMultiprocessor(&v1, kern, kThreads, kGroupBytes) != cudaSuccess ||
+      cudaOccupancyMaxActiveBlocksPerMultiprocessor(&v4, kern, kThreads * kGroups, kSplitSmem) != cudaSuccess)
     return RQ_ERR_CUDA;
+  const int v = std::min(v1, v4 * kGroups);
   *per_sm = v > 0 ? v : 1;
   return RQ_OK;
 }
