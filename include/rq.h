@@ -255,10 +255,9 @@ rq_status rq_decode_attention(const rq_cache_desc* desc, int32_t layer, const vo
  *    RQ_STATIC_SCRATCH_BYTES; larger shapes return RQ_ERR_WORKSPACE before
  *    anything is launched.
  *  - The first call on a device looks up the array's device address
- *    (cudaGetSymbolAddress) with that device current; make that first call
- *    before any stream capture. The address is cached for the life of the
- *    process: a device reset (cudaDeviceReset) invalidates it and is not
- *    supported.
+ *    (cudaGetSymbolAddress, a host-side runtime call) with that device
+ *    current. The address is cached for the life of the process: a device
+ *    reset (cudaDeviceReset) invalidates it and is not supported.
  *  - Every call on a device shares the one array, which keeps the previous
  *    call's contents (each call overwrites every record it reads, so nothing
  *    needs clearing). Calls that can overlap on the GPU (different streams
@@ -332,8 +331,8 @@ rq_status rq_append_rows(const rq_cache_desc* desc, int32_t layer, const int32_t
  * first n_dev[b] tokens (device int32 [B], 4-byte aligned; 1 <= n <= desc->S):
  * the packed blocks below 32 * (n / 32) and the last n % 32 from its residual
  * windows, as rq_decode_attention_len does for one n. residual is required.
- * The split plan is that of the capacity desc->S; each row's split CTAs stop
- * at its own packed length. A count outside 1..desc->S sets
+ * The split plan is that of the capacity desc->S; each row's splits stop at
+ * its own packed length. A count outside 1..desc->S sets
  * RQ_STATUS_BAD_POSITION and that row's output is 0. Workspace and other
  * arguments as rq_decode_attention_len. */
 rq_status rq_decode_attention_rows(const rq_cache_desc* desc, int32_t layer, const int32_t* n_dev,
