@@ -1025,6 +1025,11 @@ __global__ void __launch_bounds__(kThreads * kGroups, 1) decode_split_kernel(Dec
   }
   group_sync(grp);
   const int d = tl;
+  // The split grid may start while the previous decode call's merge grid
+  // still reads the workspace (that merge lets its dependents launch at its
+  // start); the records are written only once it has finished. Everything
+  // read above is an input no decode kernel writes.
+  asm volatile("griddepcontrol.wait;\n" ::: "memory");
   for (int n = 0; n < a.g; ++n) {
     float M = -INFINITY;
 #pragma unroll
@@ -1134,6 +1139,9 @@ __global__ void __launch_bounds__(kThreads) decode_merge_kernel(const float* par
                                                                 const T* q, const T* residual,
                                                                 int R, const int32_t* n_rows,
                                                                 int cap) {
+  // the next decode call's split grid may launch now (it waits for this grid
+  // before writing the workspace)
+  asm volatile("griddepcontrol.launch_dependents;\n" ::: "memory");
   // everything up to the wait reads only this call's inputs, so it overlaps
   // the split grid's tail
   bool row_ok = true;
@@ -1342,8 +1350,20 @@ inline rq_status launch_decode_t(const DecodeArgs& a, float* out, const void* re
   // (g <= 4: measured 2-3 % faster on those layers), one otherwise (g = 8:
   // 2-3 % slower as four groups)
   const int G = a.g <= kMaxHeads / 2 ? kGroups : 1;
-  kern<<<static_cast<unsigned>((nsplit + G - 1) / G), kThreads * G, G * kGroupBytes, s>>>(a);
-  if (cudaGetLastError() != cudaSuccess) return RQ_ERR_CUDA;
+  // a programmatic dependent of whatever precedes it in the stream: it
+  // launches early only after a grid that allows it (a decode merge), and
+  // waits for that grid before writing
+  cudaLaunchConfig_t scfg = {};
+  scfg.gridDim = dim3(static_cast<unsigned>((nsplit + G - 1) / G));
+  scfg.blockDim = dim3(kThreads * G);
+  scfg.dynamicSmemBytes = G * kGroupBytes;
+  scfg.stream = s;
+  cudaLaunchAttribute sattr[1];
+  sattr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+  sattr[0].val.programmaticStreamSerializationAllowed = 1;
+  scfg.attrs = sattr;
+  scfg.numAttrs = 1;
+  if (cudaLaunchKernelEx(&scfg, kern, a) != cudaSuccess) return RQ_ERR_CUDA;
   // a whole row per CTA for a rotated cache (the rotation mixes channels),
   // a quarter of the channels otherwise (four times the CTAs), an eighth when
   // there are few (batch, kv head) units (the records of a unit are then
