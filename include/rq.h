@@ -210,8 +210,12 @@ rq_status rq_calibrate_distortion(const void* x, int32_t dtype, int32_t n, int32
  * for min-max scale = fp16(fp32(max - min) / (2^b - 1)), zero = fp16(min),
  * codes c = clamp(rint((x - zero) * (1/scale)), 0, 2^b - 1) in fp32, written
  * to packed + offsets[layer][batch][head][kind] in the block format of
- * rq_packed_layout. k, v: device [B][H_kv][S][128] of desc->dtype (16-byte
- * aligned). bits_dev: device [L][H_kv][2]; offsets_dev: device copy of the
+ * rq_packed_layout. k, v: [B][H_kv][S][128] of desc->dtype (16-byte
+ * aligned) in device memory, or in page-locked host memory the device can
+ * address (cudaHostAlloc / cudaHostRegister under unified addressing): the
+ * kernel then reads the cache over the host link itself, with no staging
+ * copy (on GB300's NVLink-C2C about twice the rate of copy-engine transfers
+ * of the same buffers). bits_dev: device [L][H_kv][2]; offsets_dev: device copy of the
  * rq_packed_layout offsets; packed: device buffer of total_bytes (16-byte
  * aligned). signs_dev as in rq_calibrate_distortion.
  * Errors: RQ_ERR_INVALID_ARG, RQ_ERR_SHAPE, RQ_ERR_ALIGNMENT, RQ_ERR_CUDA. */

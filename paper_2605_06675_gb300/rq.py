@@ -119,6 +119,19 @@ def _dp(t):
     return ctypes.c_void_p(t.data_ptr())
 
 
+def _dp_readable(t):
+    """Pointer the device can read: a CUDA tensor, or a pinned (page-locked)
+    host tensor, whose address the device uses directly under unified
+    addressing (the kernel then reads it over the host link)."""
+    if t is not None and not t.is_cuda:
+        if not t.is_pinned():
+            raise ValueError("expected a CUDA tensor or a pinned host tensor")
+        if not t.is_contiguous():
+            raise ValueError("expected a contiguous tensor")
+        return ctypes.c_void_p(t.data_ptr())
+    return _dp(t)
+
+
 def _stream(stream):
     if stream is None:
         import torch
@@ -226,9 +239,10 @@ def rq_calibrate_distortion(x, k_grouping, v_grouping, hadamard, signs, mse, ws,
 
 def rq_quantize_pack(desc, layer, k, v, signs, bits_dev, offsets_dev, packed, status=None,
                      stream=None):
+    """k, v: CUDA tensors, or pinned host tensors read by the kernel in place."""
     _check("rq_quantize_pack", lib().rq_quantize_pack(
-        ctypes.byref(desc), layer, _dp(k), _dp(v), _dp(signs), _dp(bits_dev), _dp(offsets_dev),
-        _dp(packed), _dp(status), _stream(stream)))
+        ctypes.byref(desc), layer, _dp_readable(k), _dp_readable(v), _dp(signs), _dp(bits_dev),
+        _dp(offsets_dev), _dp(packed), _dp(status), _stream(stream)))
 
 
 def rq_decode_workspace_bytes(desc) -> int:
