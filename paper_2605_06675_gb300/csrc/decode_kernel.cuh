@@ -759,9 +759,10 @@ __device__ __forceinline__ void blocks_dyn(const WarpStream& ws, const DynRing& 
 }
 
 // Key of the compile-time path, or -1: keys 0..15 for the KIVI layout
-// (per-channel K, per-token V) at widths {2, 3, 4, 8}; keys 16..24 for
-// per-token K and V (the rotated caches) at widths {3, 4, 5}, the widths an
-// allocation at about 4 bits per code mostly gives.
+// (per-channel K, per-token V) at widths {2, 3, 4, 8}; keys 16..31 for
+// per-token K and V (the rotated caches) at key widths 3..6 and value widths
+// 2..5, the widths an allocation at about 4 bits per code gives (keys take
+// the wider ones).
 __device__ __forceinline__ int fast_key(int bK, int bV, int kg, int vg) {
   if (kg == RQ_PER_CHANNEL && vg == RQ_PER_TOKEN) {
     auto idx = [](int b) { return b == 2 ? 0 : b == 3 ? 1 : b == 4 ? 2 : b == 8 ? 3 : -1; };
@@ -769,9 +770,8 @@ __device__ __forceinline__ int fast_key(int bK, int bV, int kg, int vg) {
     return (ik < 0 || iv < 0) ? -1 : 4 * ik + iv;
   }
   if (kg == RQ_PER_TOKEN && vg == RQ_PER_TOKEN) {
-    auto idx = [](int b) { return b >= 3 && b <= 5 ? b - 3 : -1; };
-    const int ik = idx(bK), iv = idx(bV);
-    return (ik < 0 || iv < 0) ? -1 : 16 + 3 * ik + iv;
+    const int ik = bK >= 3 && bK <= 6 ? bK - 3 : -1, iv = bV >= 2 && bV <= 5 ? bV - 2 : -1;
+    return (ik < 0 || iv < 0) ? -1 : 16 + 4 * ik + iv;
   }
   return -1;
 }
@@ -780,8 +780,8 @@ __device__ __forceinline__ int fast_key(int bK, int bV, int kg, int vg) {
   X(0, 2, 2) X(1, 2, 3) X(2, 2, 4) X(3, 2, 8) X(4, 3, 2) X(5, 3, 3) X(6, 3, 4) X(7, 3, 8) \
   X(8, 4, 2) X(9, 4, 3) X(10, 4, 4) X(11, 4, 8) X(12, 8, 2) X(13, 8, 3) X(14, 8, 4) X(15, 8, 8)
 #define RQ_TOKEN_CASES(X) \
-  X(16, 3, 3) X(17, 3, 4) X(18, 3, 5) X(19, 4, 3) X(20, 4, 4) X(21, 4, 5) X(22, 5, 3) X(23, 5, 4) \
-  X(24, 5, 5)
+  X(16, 3, 2) X(17, 3, 3) X(18, 3, 4) X(19, 3, 5) X(20, 4, 2) X(21, 4, 3) X(22, 4, 4) X(23, 4, 5) \
+  X(24, 5, 2) X(25, 5, 3) X(26, 5, 4) X(27, 5, 5) X(28, 6, 2) X(29, 6, 3) X(30, 6, 4) X(31, 6, 5)
 
 template <typename T>
 __global__ void __launch_bounds__(kThreads * kGroups, 1) decode_split_kernel(DecodeArgs a) {
