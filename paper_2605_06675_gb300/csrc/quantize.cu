@@ -219,6 +219,24 @@ size_t calib_smem_bytes(bool hadamard, int kg, int vg) {
 }  // namespace
 }  // namespace rq
 
+namespace rq {
+namespace {
+// K/V may be device memory or page-locked host memory (which the kernel then
+// reads over the host link); plain pageable host memory is refused before any
+// launch. cudaPointerGetAttributes reports memory it does not know as
+// unregistered.
+bool device_readable(const void* p) {
+  cudaPointerAttributes at{};
+  if (cudaPointerGetAttributes(&at, p) != cudaSuccess) {
+    cudaGetLastError();          // reset the error state the failed query left
+    return false;
+  }
+  return at.type == cudaMemoryTypeDevice || at.type == cudaMemoryTypeManaged ||
+         at.type == cudaMemoryTypeHost;
+}
+}  // namespace
+}  // namespace rq
+
 extern "C" rq_status rq_quantize_pack(const rq_cache_desc* desc, int32_t layer, const void* k,
                                       const void* v, const int8_t* signs_dev,
                                       const uint8_t* bits_dev, const uint64_t* offsets_dev,
@@ -234,6 +252,7 @@ extern "C" rq_status rq_quantize_pack(const rq_cache_desc* desc, int32_t layer, 
     return RQ_ERR_INVALID_ARG;
   if (desc->d != kD || desc->group != kG || desc->S % kTile != 0) return RQ_ERR_SHAPE;
   if (!aligned16(k) || !aligned16(v) || !aligned16(packed)) return RQ_ERR_ALIGNMENT;
+  if (!device_readable(k) || !device_readable(v)) return RQ_ERR_INVALID_ARG;
   QuantArgs a;
   a.k = k;
   a.v = v;

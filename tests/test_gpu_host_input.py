@@ -5,6 +5,8 @@ page-locked host tensors it reads them over the host link with no staging
 copy. The packed cache must equal, byte for byte, the one packed from the same
 values in device memory, and the decode over it must match the oracle. A host
 tensor that is not pinned is refused by the binding."""
+import ctypes
+
 import numpy as np
 import pytest
 import torch
@@ -54,12 +56,22 @@ def test_pinned_host_kv_packs_identically(kg, hadamard, dtype):
 
 
 def test_unpinned_host_kv_is_refused():
-    ensure_built()
+    rq = ensure_built()
     wl = Workload("hostkv2", L=1, B=1, H_kv=2, H_q=8, S=64, dtype="bfloat16",
                   k_grouping=PER_CHANNEL, v_grouping=PER_TOKEN, hadamard=False,
                   allowed=(2, 3, 4), avg_bits=3.0, sigma_lnw=0.5, value_dist="gaussian", seed=84)
     path = PackedKVPath(wl, DEV)
     path.set_bits(np.full((1, 2, 2), 3, dtype=np.uint8))
     k, v = synth.kv_layer(wl.B, wl.H_kv, wl.S, wl.dtype, wl.seed, 0)
-    with pytest.raises(ValueError):
+    with pytest.raises(ValueError):          # the binding
         path.quantize(0, k, v)
+    # the C ABI itself: pageable host memory is refused before any launch
+    st = rq.lib().rq_quantize_pack(ctypes.byref(path.desc), 0, ctypes.c_void_p(k.data_ptr()),
+                                   ctypes.c_void_p(v.data_ptr()), None,
+                                   ctypes.c_void_p(path.bits.data_ptr()),
+                                   ctypes.c_void_p(path.offsets.data_ptr()),
+                                   ctypes.c_void_p(path.packed.data_ptr()),
+                                   ctypes.c_void_p(path.status.data_ptr()), None)
+    assert rq.STATUS_NAMES[st] == "RQ_ERR_INVALID_ARG"
+    torch.cuda.synchronize()
+    assert int(path.status.item()) == 0
