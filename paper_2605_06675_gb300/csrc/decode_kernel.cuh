@@ -60,10 +60,10 @@ struct DecodeArgs {
   float* partial;            // [B][H_q][splits][132]
   const int32_t* n_rows;     // tokens attended per batch row (rq_decode_attention_rows) or null
   uint32_t* status;
-  // split plan: (batch, kv head) units [0, u_lo) take s_lo CTAs of bps_lo
-  // blocks, the others `splits` CTAs of bps blocks (splits = s_lo or s_lo + 1;
-  // it is also the record stride per query row); the grid is 1-D, the
-  // s_lo-split units' (larger) CTAs first
+  // split plan: (batch, kv head) units [0, u_lo) take s_lo splits of bps_lo
+  // blocks, the others `splits` splits of bps blocks (splits = s_lo or
+  // s_lo + 1; it is also the record stride per query row); splits are
+  // numbered unit by unit, the s_lo-split units' (larger) ones first
   int layer, B, H, Hq, g, nblk, splits, bps, s_lo, bps_lo, u_lo, kg, vg, hadamard;
   int kq, vq;                // rq_quantizer of keys / values
   LMBook lm;                 // RQ_LLOYDMAX codebooks
