@@ -25,8 +25,9 @@ NVCC_FLAGS = ["-O3", "-lineinfo", "-std=c++17", "-Xcompiler", "-fPIC", "-Xcompil
               "-Xcompiler", "-ffp-contract=off",
               "-prec-div=true", "-prec-sqrt=true", f"-I{INCLUDE}", f"-I{CSRC}"]
 SOURCES = ["host.cpp", "quantize.cu", "quantize_k_f16.cu", "quantize_k_f16_rot.cu",
-           "quantize_k_bf16.cu", "quantize_k_bf16_rot.cu", "decode.cu", "decode_f16.cu",
-           "decode_bf16.cu"]
+           "quantize_k_bf16.cu", "quantize_k_bf16_rot.cu", "quantize_lm_f16.cu",
+           "quantize_lm_f16_rot.cu", "quantize_lm_bf16.cu", "quantize_lm_bf16_rot.cu",
+           "decode.cu", "decode_f16.cu", "decode_bf16.cu"]
 
 
 def nvcc() -> str:

@@ -237,6 +237,22 @@ bool device_readable(const void* p) {
 }  // namespace
 }  // namespace rq
 
+namespace rq {
+namespace {
+// the quantize instance for the dtype and rotation; the Lloyd-Max kernel when
+// both kinds are Lloyd-Max
+rq_status launch_quantize(const QuantArgs& a, int32_t dtype, cudaStream_t st) {
+  const bool lm = a.kq == RQ_LLOYDMAX && a.vq == RQ_LLOYDMAX;
+  if (dtype == RQ_F16) {
+    if (lm) return a.hadamard ? launch_quantize_lm_f16_rot(a, st) : launch_quantize_lm_f16(a, st);
+    return a.hadamard ? launch_quantize_f16_rot(a, st) : launch_quantize_f16(a, st);
+  }
+  if (lm) return a.hadamard ? launch_quantize_lm_bf16_rot(a, st) : launch_quantize_lm_bf16(a, st);
+  return a.hadamard ? launch_quantize_bf16_rot(a, st) : launch_quantize_bf16(a, st);
+}
+}  // namespace
+}  // namespace rq
+
 extern "C" rq_status rq_quantize_pack(const rq_cache_desc* desc, int32_t layer, const void* k,
                                       const void* v, const int8_t* signs_dev,
                                       const uint8_t* bits_dev, const uint64_t* offsets_dev,
@@ -280,9 +296,7 @@ extern "C" rq_status rq_quantize_pack(const rq_cache_desc* desc, int32_t layer, 
   a.ntiles = static_cast<long long>(desc->B) * desc->H_kv * 2 * a.nblk;
   if (a.ntiles == 0) return RQ_OK;
   cudaStream_t st = static_cast<cudaStream_t>(stream);
-  if (desc->dtype == RQ_F16)
-    return a.hadamard ? launch_quantize_f16_rot(a, st) : launch_quantize_f16(a, st);
-  return a.hadamard ? launch_quantize_bf16_rot(a, st) : launch_quantize_bf16(a, st);
+  return launch_quantize(a, desc->dtype, st);
 }
 
 extern "C" size_t rq_calibrate_workspace_bytes(int32_t n, int32_t T) {
@@ -436,9 +450,7 @@ extern "C" rq_status rq_append(const rq_cache_desc* desc, int32_t layer, int32_t
   a.row_pos = nullptr;
   a.cap = desc->S;
   a.ntiles = static_cast<long long>(desc->B) * desc->H_kv * 2;
-  if (desc->dtype == RQ_F16)
-    return a.hadamard ? launch_quantize_f16_rot(a, st) : launch_quantize_f16(a, st);
-  return a.hadamard ? launch_quantize_bf16_rot(a, st) : launch_quantize_bf16(a, st);
+  return launch_quantize(a, desc->dtype, st);
 }
 
 // ---- decode-time append with a position per batch row ----------------------
@@ -496,7 +508,5 @@ extern "C" rq_status rq_append_rows(const rq_cache_desc* desc, int32_t layer,
   a.row_pos = pos_dev;
   a.cap = desc->S;
   a.ntiles = static_cast<long long>(desc->B) * desc->H_kv * 2;
-  if (desc->dtype == RQ_F16)
-    return a.hadamard ? launch_quantize_f16_rot(a, st) : launch_quantize_f16(a, st);
-  return a.hadamard ? launch_quantize_bf16_rot(a, st) : launch_quantize_bf16(a, st);
+  return launch_quantize(a, desc->dtype, st);
 }

@@ -76,6 +76,11 @@ rq_status launch_quantize_f16(const QuantArgs& a, cudaStream_t s);
 rq_status launch_quantize_f16_rot(const QuantArgs& a, cudaStream_t s);
 rq_status launch_quantize_bf16(const QuantArgs& a, cudaStream_t s);
 rq_status launch_quantize_bf16_rot(const QuantArgs& a, cudaStream_t s);
+// the same, when both kinds of the layer are Lloyd-Max
+rq_status launch_quantize_lm_f16(const QuantArgs& a, cudaStream_t s);
+rq_status launch_quantize_lm_f16_rot(const QuantArgs& a, cudaStream_t s);
+rq_status launch_quantize_lm_bf16(const QuantArgs& a, cudaStream_t s);
+rq_status launch_quantize_lm_bf16_rot(const QuantArgs& a, cudaStream_t s);
 
 namespace {
 
@@ -106,9 +111,12 @@ struct alignas(16) QSmem {
   uint8_t tile[2][kTileBytes];
   float nz[kD];                 // -zero of every group (channel c, or 32 G + t)
   float inv[kD];                // 1 / scale (0 for a group without codes)
-  uint2 xchg[kThreads];         // per-channel min/max of half the tokens (rotated tiles)
+  union {
+    uint2 xchg[kThreads];       // per-channel min/max of half the tokens (rotated tiles)
+    uint8_t lm_lut[1024];       // Lloyd-Max kernel (per-token groups only): code bucket of x / scale
+  };
   float top;                    // magic + the largest code of the tile's quantizer
-  float lm_mid[256];            // Lloyd-Max: midpoints of the tile width's levels
+  float lm_mid[257];            // Lloyd-Max: midpoints of the width's levels (+inf after, Lloyd-Max kernel)
   alignas(16) uint32_t negw[4][16];   // rotation signs (read as uint4): word k of row G flips the sign bits (15, 31)
                                 //   of the raw pair of channels 32 G + 2k, 32 G + 2k + 1
 };
@@ -793,10 +801,60 @@ __device__ __forceinline__ void emit_lm(uint32_t (&uw)[B], int x, int y, float2 
   fmt::place<B>(uw, x, y, lm_code<B>(v.x, sf.x, mid) | (lm_code<B>(v.y, sf.y, mid) << 16));
 }
 
+// The same code in the Lloyd-Max kernel (every stream of the layer Lloyd-Max),
+// found in two steps: the bucket of u = v / sf among 1024 equal bins over
+// [-5, 5) (lm_lut: c0 = the number of midpoints below the bin's lower edge by
+// more than 1e-5), then one exact comparison with threshold c0. Exact because
+// no window [edge_k - 1e-5, edge_k+1 + 1e-5) holds more than one of the
+// codebooks' fp32 midpoints (the narrowest gap, at 8 bits, is 0.0169 against
+// bins of 0.0098; none lies beyond +-4.4), while u and the thresholds are
+// within 2e-6 of their exact values; a host test checks the property on the
+// library's codebooks. (In the general kernel this code's extra registers
+// raised the spills of the min-max loops, so it has a kernel of its own.)
+constexpr int kLmBins = 1024;
+constexpr float kLmBinScale = 102.4f;          // bins per unit of u
+constexpr float kLmBinStep = 0.009765625f;     // 1 / 102.4, exact
+constexpr float kLmDelta = 1e-5f;
+
+template <int B>
+__device__ __forceinline__ uint32_t lm_code_lut(float v, float sf, float inv, const float* mid,
+                                                const uint8_t* lut) {
+  const float t = __fmaf_rn(__fmul_rn(v, inv), kLmBinScale, 0.5f * kLmBins);
+  const int k = min(max(__float2int_rd(t), 0), kLmBins - 1);
+  const int c0 = lut[k];
+  const int c = c0 + (v >= __fmul_rn(mid[c0], sf) ? 1 : 0);
+  return sf != 0.0f ? static_cast<uint32_t>(c) : 0u;
+}
+
+template <int B, bool LUT>
+__device__ __forceinline__ void emit_lm2(uint32_t (&uw)[B], int x, int y, float2 v, float2 sf,
+                                         float2 inv, const QSmem& sm) {
+  if constexpr (LUT)
+    fmt::place<B>(uw, x, y, lm_code_lut<B>(v.x, sf.x, inv.x, sm.lm_mid, sm.lm_lut) |
+                                (lm_code_lut<B>(v.y, sf.y, inv.y, sm.lm_mid, sm.lm_lut) << 16));
+  else
+    emit_lm<B>(uw, x, y, v, sf, sm.lm_mid);
+}
+
+// lm_lut from the segment's midpoints (sm.lm_mid, nmid of them): bin kb gets
+// the number of midpoints below its lower edge by more than kLmDelta.
+__device__ __forceinline__ void lm_lut_build(QSmem& sm, int nmid) {
+  for (int kb = threadIdx.x; kb < kLmBins; kb += kThreads) {
+    const float e = __fsub_rn(static_cast<float>(kb - kLmBins / 2) * kLmBinStep, kLmDelta);
+    int lo = 0, hi = nmid;
+    while (lo < hi) {
+      const int md = (lo + hi) >> 1;
+      if (sm.lm_mid[md] < e) lo = md + 1;
+      else hi = md;
+    }
+    sm.lm_lut[kb] = static_cast<uint8_t>(lo);
+  }
+}
+
 // Thread -> (lane gid/tig of the packed format, unit u). K: warp = unit,
 // lane = format lane. V: a half warp is (gid 0..7) x (two units), so the
 // 8-byte reads of one token row hit 16 distinct bank pairs.
-template <int MODE, typename T, int B, bool CLAMP, bool F32>
+template <int MODE, typename T, int B, bool CLAMP, bool F32, bool LUT = false>
 __device__ __forceinline__ void phase2(const uint8_t* tile, const float* x32, const QSmem& sm,
                                        uint32_t* blk) {
   const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
@@ -838,11 +896,12 @@ __device__ __forceinline__ void phase2(const uint8_t* tile, const float* x32, co
 #pragma unroll
     for (int x = 0; x < 4; ++x) {
       const int t = 8 * x + gid;
-      const float sf = sm.nz[32 * u + t];
+      const float sf = sm.nz[32 * u + t], inv = LUT ? __frcp_rn(sf) : 0.0f;
       float2 v[4];
       load_pairs<T, F32>(tile, x32, t, c, v);
 #pragma unroll
-      for (int y = 0; y < 4; ++y) emit_lm<B>(uw, x, y, v[y], make_float2(sf, sf), sm.lm_mid);
+      for (int y = 0; y < 4; ++y)
+        emit_lm2<B, LUT>(uw, x, y, v[y], make_float2(sf, sf), make_float2(inv, inv), sm);
     }
   } else if constexpr (MODE == kModeKT) {
     // token 8x + gid, channels 32u + 8tig + 2y + h; group = (token, G = u)
@@ -872,8 +931,9 @@ __device__ __forceinline__ void phase2(const uint8_t* tile, const float* x32, co
       load_quad<T, F32>(tile, x32, t + 1, c, b);
       if constexpr (MODE == kModeVTL) {
         const float2 sf = *reinterpret_cast<const float2*>(sm.nz + 32 * u + t);
+        const float2 inv = LUT ? make_float2(__frcp_rn(sf.x), __frcp_rn(sf.y)) : make_float2(0.0f, 0.0f);
 #pragma unroll
-        for (int x = 0; x < 4; ++x) emit_lm<B>(uw, x, y, make_float2(a[x], b[x]), sf, sm.lm_mid);
+        for (int x = 0; x < 4; ++x) emit_lm2<B, LUT>(uw, x, y, make_float2(a[x], b[x]), sf, inv, sm);
       } else if constexpr (MODE == kModeVT) {
         const float2 nz = *reinterpret_cast<const float2*>(sm.nz + 32 * u + t);
         const float2 iv = *reinterpret_cast<const float2*>(sm.inv + 32 * u + t);
@@ -969,7 +1029,7 @@ __host__ __device__ constexpr int mode_of(int kind, int grouping, bool lloydmax)
 // time: per tile, wait for it, prefetch the next, phase 1 (group
 // parameters, meta words), phase 2 (codes) in the clamping variant only when
 // phase 1 flagged the tile. Returns the ring position after the segment.
-template <typename T, bool HAD, int MODE, int B>
+template <typename T, bool HAD, int MODE, int B, bool LUT = false>
 __device__ __forceinline__ int run_segment(const QuantArgs& a, QSmem& sm, float* x32,
                                            const Segment& seg, int it) {
   constexpr int kTileSrcBytes = kTile * kD * static_cast<int>(sizeof(T));
@@ -990,11 +1050,26 @@ __device__ __forceinline__ int run_segment(const QuantArgs& a, QSmem& sm, float*
     uint8_t* meta = blk + 512 * B;
     if (threadIdx.x == 0)        // read by phase 2, after the barrier below
       sm.top = kRoundMagic + static_cast<float>(sym ? (1 << B) - 2 : (1 << B) - 1);
-    if constexpr (LM) {          // the thresholds' midpoints, exact in fp32
+    if constexpr (LM && !LUT) {  // the thresholds' midpoints, exact in fp32
       for (int i = threadIdx.x; i < (1 << B) - 1; i += kThreads) {
         const float l0 = __half2float(__ushort_as_half(a.lm.lv[lm_offset(B) + i]));
         const float l1 = __half2float(__ushort_as_half(a.lm.lv[lm_offset(B) + i + 1]));
         sm.lm_mid[i] = __fmul_rn(__fadd_rn(l0, l1), 0.5f);
+      }
+    }
+    if constexpr (LM && LUT) {
+      if (k == 0) {              // once per segment (one width): midpoints, then buckets
+        for (int i = threadIdx.x; i < (1 << B); i += kThreads) {
+          float m = INFINITY;    // exact in fp32; +inf after the last
+          if (i < (1 << B) - 1) {
+            const float l0 = __half2float(__ushort_as_half(a.lm.lv[lm_offset(B) + i]));
+            const float l1 = __half2float(__ushort_as_half(a.lm.lv[lm_offset(B) + i + 1]));
+            m = __fmul_rn(__fadd_rn(l0, l1), 0.5f);
+          }
+          sm.lm_mid[i] = m;
+        }
+        __syncthreads();
+        lm_lut_build(sm, (1 << B) - 1);
       }
     }
     GroupOut g;
@@ -1005,7 +1080,7 @@ __device__ __forceinline__ int run_segment(const QuantArgs& a, QSmem& sm, float*
     const bool slow = __syncthreads_or(g.slow) != 0;
     uint32_t* blk32 = reinterpret_cast<uint32_t*>(blk);
     if (slow) phase2_clamp_call<MODE, T, B, HAD>(it & 1, blk32);
-    else phase2<MODE, T, B, false, HAD>(buf, x32, sm, blk32);
+    else phase2<MODE, T, B, false, HAD, LUT>(buf, x32, sm, blk32);
   }
   return it;
 }
@@ -1025,25 +1100,27 @@ __device__ __forceinline__ int skip_segment(const QuantArgs& a, QSmem& sm, const
   return it;
 }
 
-template <typename T, bool HAD, int MODE>
+template <typename T, bool HAD, int MODE, bool LUT = false>
 __device__ __forceinline__ int run_segment_b(const QuantArgs& a, QSmem& sm, float* x32,
                                              const Segment& seg, int it, int b) {
   switch (b) {
-    case 1: return run_segment<T, HAD, MODE, 1>(a, sm, x32, seg, it);
-    case 2: return run_segment<T, HAD, MODE, 2>(a, sm, x32, seg, it);
-    case 3: return run_segment<T, HAD, MODE, 3>(a, sm, x32, seg, it);
-    case 4: return run_segment<T, HAD, MODE, 4>(a, sm, x32, seg, it);
-    case 5: return run_segment<T, HAD, MODE, 5>(a, sm, x32, seg, it);
-    case 6: return run_segment<T, HAD, MODE, 6>(a, sm, x32, seg, it);
-    case 7: return run_segment<T, HAD, MODE, 7>(a, sm, x32, seg, it);
-    default: return run_segment<T, HAD, MODE, 8>(a, sm, x32, seg, it);
+    case 1: return run_segment<T, HAD, MODE, 1, LUT>(a, sm, x32, seg, it);
+    case 2: return run_segment<T, HAD, MODE, 2, LUT>(a, sm, x32, seg, it);
+    case 3: return run_segment<T, HAD, MODE, 3, LUT>(a, sm, x32, seg, it);
+    case 4: return run_segment<T, HAD, MODE, 4, LUT>(a, sm, x32, seg, it);
+    case 5: return run_segment<T, HAD, MODE, 5, LUT>(a, sm, x32, seg, it);
+    case 6: return run_segment<T, HAD, MODE, 6, LUT>(a, sm, x32, seg, it);
+    case 7: return run_segment<T, HAD, MODE, 7, LUT>(a, sm, x32, seg, it);
+    default: return run_segment<T, HAD, MODE, 8, LUT>(a, sm, x32, seg, it);
   }
 }
 
 // A CTA owns a contiguous range of tiles (block j of stream sk = (batch * H
 // + h) * 2 + kind, tile index sk * nblk + j); the range is walked one stream
 // segment at a time, each with its own compile-time loop.
-template <typename T, bool HAD>
+// LMK: the Lloyd-Max kernel, launched when both kinds of the layer are
+// Lloyd-Max (every segment then is); it holds the Lloyd-Max loops only.
+template <typename T, bool HAD, bool LMK = false>
 __global__ void __launch_bounds__(kThreads, RQ_QUANT_MIN_BLOCKS) quantize_pack_kernel(QuantArgs a) {
   extern __shared__ __align__(16) unsigned char smem_raw[];
   QSmem& sm = *reinterpret_cast<QSmem*>(smem_raw);
@@ -1080,13 +1157,18 @@ __global__ void __launch_bounds__(kThreads, RQ_QUANT_MIN_BLOCKS) quantize_pack_k
       it = skip_segment(a, sm, seg, it, kTileSrcBytes, !cur.skip);
     } else {
       const bool lm = (cur.kind ? a.vq : a.kq) == RQ_LLOYDMAX;
-      switch (mode_of(cur.kind, cur.grouping, lm)) {
-        case kModeKC: it = run_segment_b<T, HAD, kModeKC>(a, sm, x32, seg, it, b); break;
-        case kModeKT: it = run_segment_b<T, HAD, kModeKT>(a, sm, x32, seg, it, b); break;
-        case kModeVT: it = run_segment_b<T, HAD, kModeVT>(a, sm, x32, seg, it, b); break;
-        case kModeKTL: it = run_segment_b<T, HAD, kModeKTL>(a, sm, x32, seg, it, b); break;
-        case kModeVTL: it = run_segment_b<T, HAD, kModeVTL>(a, sm, x32, seg, it, b); break;
-        default: it = run_segment_b<T, HAD, kModeVC>(a, sm, x32, seg, it, b); break;
+      if constexpr (LMK) {
+        if (cur.kind == 0) it = run_segment_b<T, HAD, kModeKTL, true>(a, sm, x32, seg, it, b);
+        else it = run_segment_b<T, HAD, kModeVTL, true>(a, sm, x32, seg, it, b);
+      } else {
+        switch (mode_of(cur.kind, cur.grouping, lm)) {
+          case kModeKC: it = run_segment_b<T, HAD, kModeKC>(a, sm, x32, seg, it, b); break;
+          case kModeKT: it = run_segment_b<T, HAD, kModeKT>(a, sm, x32, seg, it, b); break;
+          case kModeVT: it = run_segment_b<T, HAD, kModeVT>(a, sm, x32, seg, it, b); break;
+          case kModeKTL: it = run_segment_b<T, HAD, kModeKTL>(a, sm, x32, seg, it, b); break;
+          case kModeVTL: it = run_segment_b<T, HAD, kModeVTL>(a, sm, x32, seg, it, b); break;
+          default: it = run_segment_b<T, HAD, kModeVC>(a, sm, x32, seg, it, b); break;
+        }
       }
     }
     t = end;

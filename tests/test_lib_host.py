@@ -188,3 +188,21 @@ def test_lloydmax_codebook_matches_the_oracle(rq):
         assert np.array_equal(got.view(np.uint16), want.view(np.uint16)), b
     with pytest.raises(rq.RQError):
         rq.rq_lloydmax_levels(9)
+
+
+def test_lloydmax_midpoints_fit_the_quantizer_buckets(rq):
+    """The quantize kernel finds a Lloyd-Max code from a bucket of u = v / scale
+    (1024 equal bins over [-5, 5)) and one exact threshold comparison; that is
+    exact only if no bin widened by 1e-5 on each side holds more than one of the
+    codebook's fp32 midpoints and none lies in the end bins. Checked here on
+    the library's own codebooks, every width."""
+    bins, r, delta = 1024, 5.0, 1e-5
+    w = 2 * r / bins
+    assert w == 0.009765625                        # the kernel's exact bin step
+    for b in range(1, 9):
+        lv = rq.rq_lloydmax_levels(b).view(np.float16).astype(np.float32)
+        mid = ((lv[:-1] + lv[1:]) * np.float32(0.5)).astype(np.float64)
+        assert np.all(np.abs(mid) < r - w), b
+        for k in range(bins):
+            lo, hi = -r + k * w - delta, -r + (k + 1) * w + delta
+            assert int(((mid >= lo) & (mid < hi)).sum()) <= 1, (b, k)
