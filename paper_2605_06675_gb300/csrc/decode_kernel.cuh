@@ -44,9 +44,9 @@ constexpr int kRingBytes = 11264;    // per-warp ring of shared-memory slots
 constexpr int kMaxSlots = 8;
 constexpr int kQBytes = kMaxHeads * kD * 4;
 constexpr int kSmemBytes = kQBytes + kWarps * kRingBytes;   // 49152: q table and rings of a split group
-// a split group's shared memory: q table, rings, the warps' (m, l) and two
-// Lloyd-Max codebooks (50432 bytes, a multiple of 128)
-constexpr int kGroupBytes = kSmemBytes + 2 * kWarps * kMaxHeads * 4 + 2 * 256 * 2;
+// a split group's shared memory: q table, rings, the warps' (m, l), two
+// Lloyd-Max codebooks and two code-pair tables (52480 bytes, a multiple of 128)
+constexpr int kGroupBytes = kSmemBytes + 2 * kWarps * kMaxHeads * 4 + 2 * 256 * 2 + 2 * 256 * 4;
 constexpr int kSplitSmem = kGroups * kGroupBytes;            // per four-group CTA
 static_assert(kGroupBytes % 128 == 0, "group areas start on 128-byte boundaries");
 static_assert(kWarps * kMaxHeads * kD * 4 <= kWarps * kRingBytes, "merge buffer aliases rings");
@@ -172,10 +172,14 @@ __device__ __forceinline__ uint32_t dequant(uint32_t sub, uint32_t m, uint32_t z
 // Lloyd-Max pair: the two codes of an extracted register (at bit E of each
 // half) looked up in the width's fp16 codebook (shared memory), scaled by m
 // and shifted by z2 (one fp16x2 FMA)
+// Widths up to 4 read both levels of a register at once from a table of
+// code pairs (entry c0 + 2^BW c1 = the fp16x2 pair (L_c0, L_c1)): one
+// shared-memory read per register instead of two; `tab` then points to it.
 template <int BW>
 __device__ __forceinline__ uint32_t lm_pair(uint32_t sub, int E, const uint16_t* tab) {
   const uint32_t c0 = (sub >> E) & ((1u << BW) - 1u), c1 = (sub >> (16 + E)) & ((1u << BW) - 1u);
-  return static_cast<uint32_t>(tab[c0]) | (static_cast<uint32_t>(tab[c1]) << 16);
+  if constexpr (BW <= 4) return reinterpret_cast<const uint32_t*>(tab)[c0 | (c1 << BW)];
+  else return static_cast<uint32_t>(tab[c0]) | (static_cast<uint32_t>(tab[c1]) << 16);
 }
 
 // ------------------------------------------------------------ block math ----
@@ -855,12 +859,26 @@ __global__ void __launch_bounds__(kThreads * kGroups, 1) decode_split_kernel(Dec
   dr.kg = a.kg;
   dr.vg = a.vg;
   const bool lmk = valid && a.kq == RQ_LLOYDMAX, lmv = valid && a.vq == RQ_LLOYDMAX;
-  for (int i = tl; i < 256; i += kThreads) {
-    if (lmk && i < (1 << bK)) lmtab[0][i] = a.lm.lv[lm_offset(bK) + i];
-    if (lmv && i < (1 << bV)) lmtab[1][i] = a.lm.lv[lm_offset(bV) + i];
+  // code-pair tables (widths <= 4) after the codebooks
+  uint32_t (*lmpair)[256] = reinterpret_cast<uint32_t (*)[256]>(lmtab + 2);
+  if (lmk || lmv) {
+    for (int i = tl; i < 256; i += kThreads) {
+      if (lmk && i < (1 << bK)) lmtab[0][i] = a.lm.lv[lm_offset(bK) + i];
+      if (lmv && i < (1 << bV)) lmtab[1][i] = a.lm.lv[lm_offset(bV) + i];
+#pragma unroll
+      for (int kind = 0; kind < 2; ++kind) {
+        const int bw = kind ? bV : bK;
+        if ((kind ? lmv : lmk) && bw <= 4 && i < (1 << (2 * bw))) {
+          const uint16_t* lv = a.lm.lv + lm_offset(bw);
+          lmpair[kind][i] = static_cast<uint32_t>(lv[i & ((1 << bw) - 1)]) |
+                            static_cast<uint32_t>(lv[i >> bw]) << 16;
+        }
+      }
+    }
   }
-  dr.lmK = lmk ? lmtab[0] : nullptr;               // read after the barriers of the q prologue
-  dr.lmV = lmv ? lmtab[1] : nullptr;
+  // read after the barriers of the q prologue; the pair table for widths <= 4
+  dr.lmK = lmk ? (bK <= 4 ? reinterpret_cast<const uint16_t*>(lmpair[0]) : lmtab[0]) : nullptr;
+  dr.lmV = lmv ? (bV <= 4 ? reinterpret_cast<const uint16_t*>(lmpair[1]) : lmtab[1]) : nullptr;
   dr.sK = 512 * (bK + 1);
   dr.sV = 512 * (bV + 1);
   dr.slot = max(dr.sK, dr.sV);
