@@ -66,6 +66,7 @@ struct DecodeArgs {
   // numbered unit by unit, the s_lo-split units' (larger) ones first
   int layer, B, H, Hq, g, nblk, splits, bps, s_lo, bps_lo, u_lo, kg, vg, hadamard;
   int kq, vq;                // rq_quantizer of keys / values
+  int early;                 // let the merge grid launch before the blocks (else after)
   LMBook lm;                 // RQ_LLOYDMAX codebooks
 };
 
@@ -787,298 +788,21 @@ __device__ __forceinline__ int fast_key(int bK, int bV, int kg, int vg) {
   X(16, 3, 2) X(17, 3, 3) X(18, 3, 4) X(19, 3, 5) X(20, 4, 2) X(21, 4, 3) X(22, 4, 4) X(23, 4, 5) \
   X(24, 5, 2) X(25, 5, 3) X(26, 5, 4) X(27, 5, 5) X(28, 6, 2) X(29, 6, 3) X(30, 6, 4) X(31, 6, 5)
 
+// Two register budgets for the same code (the body below is included in
+// both). At 128 registers a thread the split CTAs of an SM take all 65,536
+// of its registers, so a merge CTA starts on an SM only where a split CTA has
+// left. At 120 (28 bytes of spill stores), 4,096 stay free on every SM: one
+// merge CTA of 128 threads at <= 32 registers fits beside the split CTAs
+// when its shared memory does too, and waits there for the split grid to
+// end. (A launch bound of 512 threads on the 120-register kernel, or the body
+// as an inlined function, made the compiler spill several times more.)
 template <typename T>
 __global__ void __launch_bounds__(kThreads * kGroups, 1) decode_split_kernel(DecodeArgs a) {
-  // A CTA is G = blockDim.x / kThreads (1 or kGroups) independent groups of
-  // kWarps warps, one split each (split c = group * CTAs + CTA index, so that
-  // with four groups every CTA takes splits from each quarter of the plan: as
-  // many of the larger ones as the others); a group synchronises on its own
-  // named barrier. The warp schedulers serve the warps of one CTA evenly but
-  // favour the CTAs that reached an SM first: four one-group CTAs per SM
-  // finish far apart (the last ones alone on their SMs), one four-group CTA
-  // per SM finishes together but streams a little slower per SM. The launch
-  // picks the layout per query-group size.
-  // No static shared memory: every group's area starts on a 128-byte
-  // boundary, so its cp.async rings take whole 128-byte lines per 8 lanes (a
-  // ring off that boundary doubles the L2 sectors every copy moves).
-  extern __shared__ __align__(128) unsigned char smem_dyn[];
-  const int grp = threadIdx.x / kThreads, tl = threadIdx.x % kThreads;   // G = blockDim.x / kThreads
-  const long long c = static_cast<long long>(grp) * gridDim.x + blockIdx.x;
-  {
-    const long long units = static_cast<long long>(a.B) * a.H;
-    if (c >= units * a.s_lo + (units - a.u_lo) * (a.splits - a.s_lo)) return;   // no split
-  }
-  unsigned char* smem_raw = smem_dyn + grp * kGroupBytes;
-  float* qs = reinterpret_cast<float*>(smem_raw);                  // [8][128]
-  uint8_t* rings = smem_raw + kQBytes;
-  float (*red_m)[kMaxHeads] = reinterpret_cast<float (*)[kMaxHeads]>(smem_raw + kSmemBytes);
-  float (*red_l)[kMaxHeads] = red_m + kWarps;
-  // Lloyd-Max codebooks of the group's widths
-  uint16_t (*lmtab)[256] = reinterpret_cast<uint16_t (*)[256]>(red_l + kWarps);
-  int unit, split, bps;
-  {
-    const int nlo = a.u_lo * a.s_lo;
-    if (c < nlo) {
-      unit = c / a.s_lo;
-      split = c - unit * a.s_lo;
-      bps = a.bps_lo;
-    } else {
-      const int c2 = c - nlo, u2 = c2 / a.splits;
-      unit = a.u_lo + u2;
-      split = c2 - u2 * a.splits;
-      bps = a.bps;
-    }
-  }
-  const int batch = unit / a.H, h = unit - batch * a.H;
-  const int lane = tl & 31, warp = tl >> 5;
-  const int gid = lane >> 2, tig = lane & 3;
-
-  // q of the g query heads of this kv head (rows >= g are zero), sign-flipped
-  // for a Hadamard-rotated cache. Its loads go out first: issued after the
-  // ring's first copies (every CTA's at once) they would queue behind them,
-  // and the q prologue, which the block loop waits for, with them.
-  static_assert(kD == kThreads, "thread d loads channel d of every row");
-  const T* qp = static_cast<const T*>(a.q) + (static_cast<long long>(batch) * a.Hq +
-                                              static_cast<long long>(h) * a.g) * kD;
-  float qreg[kMaxHeads];
-#pragma unroll
-  for (int n = 0; n < kMaxHeads; ++n) qreg[n] = n < a.g ? to_f32<T>(qp[n * kD + tl]) : 0.0f;
-  const bool qneg = a.hadamard && a.signs && a.signs[tl] < 0;
-
-  const int bK = a.bits[(a.layer * a.H + h) * 2 + 0];
-  const int bV = a.bits[(a.layer * a.H + h) * 2 + 1];
-  const bool valid = bK >= 1 && bK <= 8 && bV >= 1 && bV <= 8;
-  if (!valid && tl == 0) set_status(a.status, RQ_STATUS_BAD_BITS);
-  const uint64_t* offp =
-      a.offsets + ((static_cast<long long>(a.layer) * a.B + batch) * a.H + h) * 2;
-  const uint8_t* kbase = a.packed + (valid ? offp[0] : 0);
-  const uint8_t* vbase = a.packed + (valid ? offp[1] : 0);
-  DynRing dr;
-  dr.bK = bK;
-  dr.bV = bV;
-  dr.kg = a.kg;
-  dr.vg = a.vg;
-  const bool lmk = valid && a.kq == RQ_LLOYDMAX, lmv = valid && a.vq == RQ_LLOYDMAX;
-  // code-pair tables (widths <= 4) after the codebooks
-  uint32_t (*lmpair)[256] = reinterpret_cast<uint32_t (*)[256]>(lmtab + 2);
-  if (lmk || lmv) {
-    for (int i = tl; i < 256; i += kThreads) {
-      if (lmk && i < (1 << bK)) lmtab[0][i] = a.lm.lv[lm_offset(bK) + i];
-      if (lmv && i < (1 << bV)) lmtab[1][i] = a.lm.lv[lm_offset(bV) + i];
-#pragma unroll
-      for (int kind = 0; kind < 2; ++kind) {
-        const int bw = kind ? bV : bK;
-        if ((kind ? lmv : lmk) && bw <= 4 && i < (1 << (2 * bw))) {
-          const uint16_t* lv = a.lm.lv + lm_offset(bw);
-          lmpair[kind][i] = static_cast<uint32_t>(lv[i & ((1 << bw) - 1)]) |
-                            static_cast<uint32_t>(lv[i >> bw]) << 16;
-        }
-      }
-    }
-  }
-  // read after the barriers of the q prologue; the pair table for widths <= 4
-  dr.lmK = lmk ? (bK <= 4 ? reinterpret_cast<const uint16_t*>(lmpair[0]) : lmtab[0]) : nullptr;
-  dr.lmV = lmv ? (bV <= 4 ? reinterpret_cast<const uint16_t*>(lmpair[1]) : lmtab[1]) : nullptr;
-  dr.sK = 512 * (bK + 1);
-  dr.sV = 512 * (bV + 1);
-  dr.slot = max(dr.sK, dr.sV);
-  dr.ns = valid ? min(kMaxSlots, kRingBytes / dr.slot) : 2;
-  // the packed blocks of this batch row: all nblk, or those below 32 * floor(n / 32)
-  // of its own token count n (1 <= n <= 32 * nblk; another n attends nothing)
-  int nblk_row = a.nblk;
-  if (a.n_rows) {
-    const int n = a.n_rows[batch];
-    nblk_row = (n >= 1 && n <= a.nblk * kTile) ? n / kTile : 0;
-  }
-  const int blk0 = split * bps;
-  const int blk1 = min(nblk_row, blk0 + bps);
-  const int blk_first = blk0 + warp;
-  WarpStream ws;
-  ws.lane = lane;
-  ws.nb = valid && blk_first < blk1 ? (blk1 - blk_first + kWarps - 1) / kWarps : 0;
-  ws.ring_ptr = rings + warp * kRingBytes;
-  ws.ring = smem_u32(ws.ring_ptr);
-  ws.kwarp = kbase + static_cast<size_t>(blk_first) * dr.sK;
-  ws.vwarp = vbase + static_cast<size_t>(blk_first) * dr.sV;
-  const int key = valid && a.kq != RQ_LLOYDMAX && a.vq != RQ_LLOYDMAX ? fast_key(bK, bV, a.kg, a.vg) : -1;
-  ws.merged = a.g <= kMaxHeads / 2 && key >= 0 && key < 16;   // the compile-time KIVI paths only
-  ws.mneg = ws.merged && gid >= kMaxHeads / 2 ? 0xBC00BC00u : 0x80008000u;
-
-  // start streaming the first entries before the q prologue
-  switch (key) {
-#define RQ_PRO(k, BK, BV) case k: prologue_static<BK, BV>(ws); break;
-    RQ_FAST_CASES(RQ_PRO)
-    RQ_TOKEN_CASES(RQ_PRO)
-#undef RQ_PRO
-    default: prologue_dyn(ws, dr); break;
-  }
-
-  // q into shared memory, rotated into the cache's domain when the cache is
-  // Hadamard-rotated (rows >= g stay zero)
-#pragma unroll
-  for (int n = 0; n < kMaxHeads; ++n) qs[n * kD + tl] = qneg ? -qreg[n] : qreg[n];
-  group_sync(grp);
-  if (a.hadamard) fwht_smem_group(qs, a.g, tl, grp);
-  // q enters the MMAs scaled by a power of two only (no rounding beyond its
-  // fp16 conversion); the rest of the softmax scale 1/sqrt(128) * log2(e) is
-  // applied to the fp32 scores (log2 units).
-  // K unit u, pair x of lane (gid, tig) is channels 32u + 8tig + 2x (+1);
-  // qf carries the per-channel-key codes' 2^-E(x) as well.
-  // q is scaled by a power of two only (exact: headroom for q . scale in
-  // fp16), the rest of the softmax scale is applied in fp32
-  const float qpow = a.hadamard ? 0.015625f : 0.125f;
-  const float qscale = kLog2e * kInvSqrt128 * (a.hadamard ? kInvSqrt128 : 1.0f) / qpow;
-  uint32_t qb[4][4], qf[4][4];
-  uint32_t ef[4];
-#pragma unroll
-  for (int x = 0; x < 4; ++x) ef[x] = pow2_neg_h2(a.kg == RQ_PER_CHANNEL && valid ? fmt::exponent(bK, x) : 0);
-  if (warp == 0) {
-    // merged (g <= 4): columns 4..7 repeat heads 0..3 (they carry lo in the
-    // scores MMA; elsewhere they give duplicate results that are not stored)
-    const int qrow = ws.merged ? (gid & 3) : gid;
-#pragma unroll
-    for (int u = 0; u < 4; ++u)
-#pragma unroll
-      for (int x = 0; x < 4; ++x) {
-        const float* qr = qs + qrow * kD + 32 * u + 8 * tig + 2 * x;
-        qb[u][x] = pack_f16x2(qr[0] * qpow, qr[1] * qpow);
-        qf[u][x] = hmul2u(qb[u][x], ef[x]);
-      }
-  }
-  // per-token keys: sum over each 32-channel group of the q operand the MMA
-  // sees (fp16 q scaled by qpow), [group G = lane / 8][head n = lane % 8]
-  float qgsum = 0.0f;
-  if (warp == 0 && a.kg == RQ_PER_TOKEN) {
-    const float* qr = qs + (lane & 7) * kD + 32 * (lane >> 3);
-    for (int c = 0; c < 32; ++c) qgsum += __half2float(__float2half_rn(qr[c] * qpow));
-  }
-  group_sync(grp);                  // qs is read; its space becomes the q operand table
-  uint8_t* qtab = smem_raw;
-  if (warp == 0) {
-#pragma unroll
-    for (int u = 0; u < 4; ++u) {
-      *reinterpret_cast<uint4*>(qtab + 16 * (32 * u + lane)) = make_uint4(qb[u][0], qb[u][1], qb[u][2], qb[u][3]);
-      if (a.kg == RQ_PER_CHANNEL)
-        *reinterpret_cast<uint4*>(qtab + 2048 + 16 * (32 * u + lane)) =
-            make_uint4(qf[u][0], qf[u][1], qf[u][2], qf[u][3]);
-    }
-    if (a.kg == RQ_PER_TOKEN) reinterpret_cast<float*>(qtab + 2048)[lane] = qgsum;   // [G][n]
-  }
-  group_sync(grp);
-  // The merge grid launches once every split CTA has passed its trigger (or
-  // exited) and waits for this grid to finish before it reads a record; a
-  // merge CTA takes SM room only where a split CTA has left. One-group CTAs
-  // (a quarter of an SM each) trigger here, before the blocks: the merge's
-  // CTAs then fill the slots of the first splits to finish, and the 70B
-  // shape (B 1, 8 kv heads, g 8: 608 splits) decodes 11-14 % faster than with
-  // the trigger after the blocks. A four-group CTA holds a whole SM, so a
-  // merge CTA parked on it keeps the next call's splits off that SM until the
-  // merge ends; those trigger after their blocks (early, they were 0-1 %
-  // slower).
-  if (blockDim.x == kThreads) asm volatile("griddepcontrol.launch_dependents;\n" ::: "memory");
-
-  SoftmaxAcc acc;
-#pragma unroll
-  for (int mt = 0; mt < 8; ++mt)
-#pragma unroll
-    for (int r = 0; r < 4; ++r) acc.o[mt][r] = 0.0f;
-#pragma unroll
-  for (int gp = 0; gp < 2; ++gp)
-#pragma unroll
-    for (int r = 0; r < 4; ++r) acc.bz[gp][r] = 0.0f;
-  acc.m0 = acc.m1 = -INFINITY;
-  acc.l0 = acc.l1 = 0.0f;
-
-  switch (key) {
-#define RQ_BLK(k, BK, BV)                                                                        \
-  case k:                                                                                        \
-    if (ws.merged) blocks_static<BK, RQ_PER_CHANNEL, BV, RQ_PER_TOKEN, true>(ws, qtab, qscale, acc); \
-    else blocks_static<BK, RQ_PER_CHANNEL, BV, RQ_PER_TOKEN, false>(ws, qtab, qscale, acc);        \
-    break;
-    RQ_FAST_CASES(RQ_BLK)
-#undef RQ_BLK
-#define RQ_TBLK(k, BK, BV)                                                                  \
-  case k: blocks_static<BK, RQ_PER_TOKEN, BV, RQ_PER_TOKEN, false>(ws, qtab, qscale, acc); break;
-    RQ_TOKEN_CASES(RQ_TBLK)
-#undef RQ_TBLK
-    default: blocks_dyn(ws, dr, qtab, qscale, acc); break;
-  }
-  // four-group CTAs let the merge grid launch only now (one-group CTAs did
-  // before the blocks)
-  if (blockDim.x != kThreads) asm volatile("griddepcontrol.launch_dependents;\n" ::: "memory");
-  if (a.vg == RQ_PER_TOKEN && valid) {
-    // rows of m-tile mt are classes x = 2 (mt & 1) + r of unit mt / 2: undo
-    // their codes' 2^(E(x) - 24), then add group G's zero-point sum (rows gid
-    // of bz[G / 2] for even G, rows gid + 8 for odd G)
-    float rf[4];
-#pragma unroll
-    for (int x = 0; x < 4; ++x)       // 2^(24 - E); 1 for codebook levels
-      rf[x] = lmv ? 1.0f : __int_as_float((127 + 24 - fmt::exponent(bV, x)) << 23);
-#pragma unroll
-    for (int mt = 0; mt < 8; ++mt) {
-      const int G = mt >> 1;
-      const float z0 = (G & 1) ? acc.bz[G >> 1][2] : acc.bz[G >> 1][0];
-      const float z1 = (G & 1) ? acc.bz[G >> 1][3] : acc.bz[G >> 1][1];
-      const float f0 = rf[2 * (mt & 1)], f1 = rf[2 * (mt & 1) + 1];
-      acc.o[mt][0] = __fmaf_rn(acc.o[mt][0], f0, z0);
-      acc.o[mt][1] = __fmaf_rn(acc.o[mt][1], f0, z1);
-      acc.o[mt][2] = __fmaf_rn(acc.o[mt][2], f1, z0);
-      acc.o[mt][3] = __fmaf_rn(acc.o[mt][3], f1, z1);
-    }
-  }
-  float m0 = acc.m0, m1 = acc.m1, l0 = acc.l0, l1 = acc.l1;
-#pragma unroll
-  for (int off = 4; off <= 16; off <<= 1) {
-    l0 += __shfl_xor_sync(0xffffffffu, l0, off);
-    l1 += __shfl_xor_sync(0xffffffffu, l1, off);
-  }
-  // merge the four warps (log-sum-exp), one partial record per query head;
-  // the merge buffer reuses the rings
-  group_sync(grp);
-  float* red_o = reinterpret_cast<float*>(rings);   // [warp][head][channel]
-#pragma unroll
-  for (int mt = 0; mt < 8; ++mt) {
-    // row r of m-tile mt is channel 32 (mt / 2) + 4 gid + 2 (mt & 1) + r
-    float* r0 = red_o + (warp * kMaxHeads + 2 * tig) * kD;
-    float* r1 = r0 + kD;
-    const int ch = 32 * (mt >> 1) + 4 * gid + 2 * (mt & 1);
-    r0[ch] = acc.o[mt][0];
-    r1[ch] = acc.o[mt][1];
-    r0[ch + 1] = acc.o[mt][2];
-    r1[ch + 1] = acc.o[mt][3];
-  }
-  if (gid == 0) {
-    red_m[warp][2 * tig] = m0;
-    red_m[warp][2 * tig + 1] = m1;
-    red_l[warp][2 * tig] = l0;
-    red_l[warp][2 * tig + 1] = l1;
-  }
-  group_sync(grp);
-  const int d = tl;
-  // The split grid may start while the previous decode call's merge grid
-  // still reads the workspace (that merge lets its dependents launch at its
-  // start); the records are written only once it has finished. Everything
-  // read above is an input no decode kernel writes.
-  asm volatile("griddepcontrol.wait;\n" ::: "memory");
-  for (int n = 0; n < a.g; ++n) {
-    float M = -INFINITY;
-#pragma unroll
-    for (int w = 0; w < kWarps; ++w) M = fmaxf(M, red_m[w][n]);
-    float osum = 0.0f, lsum = 0.0f;
-#pragma unroll
-    for (int w = 0; w < kWarps; ++w) {
-      const float mw = red_m[w][n];
-      const float sc = (mw == -INFINITY) ? 0.0f : exp2f(mw - M);
-      osum += sc * red_o[(w * kMaxHeads + n) * kD + d];
-      lsum += sc * red_l[w][n];
-    }
-    float* dst = a.partial + ((static_cast<long long>(batch) * a.Hq + h * a.g + n) * a.splits + split) * kPart;
-    dst[d] = osum;
-    if (d == 0) {
-      dst[kD] = M;
-      dst[kD + 1] = lsum;
-    }
-  }
+#include "decode_split_body.inc"
+}
+template <typename T>
+__global__ void __maxnreg__(120) decode_split_kernel_co(DecodeArgs a) {
+#include "decode_split_body.inc"
 }
 
 // ------------------------------------------------------------ split merge ----
@@ -1161,14 +885,14 @@ __device__ __forceinline__ void residual_record(const T* q, const T* res, int R,
 }
 
 template <int CQ, typename T>
-__global__ void __launch_bounds__(kThreads) decode_merge_kernel(const float* partial, float* out,
+__global__ void __launch_bounds__(kThreads, 16) decode_merge_kernel(const float* partial, float* out,
                                                                 const int8_t* signs,
                                                                 uint32_t* status, int Hq, int H,
                                                                 int g, int splits, int s_lo,
                                                                 int u_lo, int hadamard,
                                                                 const T* q, const T* residual,
                                                                 int R, const int32_t* n_rows,
-                                                                int cap) {
+                                                                int cap, int msm_bytes) {
   // the next decode call's split grid may launch now (it waits for this grid
   // before writing the workspace)
   asm volatile("griddepcontrol.launch_dependents;\n" ::: "memory");
@@ -1205,7 +929,7 @@ __global__ void __launch_bounds__(kThreads) decode_merge_kernel(const float* par
       if (signs[(tid + kThreads * k) % CW] < 0) negmask |= 1u << k;
   }
   // splits per chunk: shared budget, and at most kMergeChunk (four weights per lane)
-  const int cs_max = min(kMergeChunk, kMergeSmem / (g * SLOT * 16));
+  const int cs_max = min(kMergeChunk, msm_bytes / (g * SLOT * 16));
   if (tid < kMaxHeads) {
     run_m[tid] = -INFINITY;
     run_l[tid] = 0.0f;
@@ -1362,24 +1086,70 @@ __global__ void __launch_bounds__(kThreads) decode_merge_kernel(const float* par
   }
 }
 
+// The merge's shared-memory records area for channel parts of 128 / cq: one
+// round trip for every split of a unit when it fits (at most kMergeSmem), the
+// residual record's 38 KB when rows may hold residual tokens.
+inline int merge_smem_bytes(const DecodeArgs& a, int cq, bool residual) {
+  const long long need = static_cast<long long>(a.g) * a.splits * (kD / cq / 4 + 1) * 16;
+  const long long res = residual ? (kMaxHeads * kD + kTile * (kD + 1) + kTile * kD + kMaxHeads * kTile) * 4 : 0;
+  return static_cast<int>(std::min<long long>(kMergeSmem, std::max(need, res)));
+}
+
 // split kernel, then the merge kernel as its programmatic dependent (it
 // overlaps the split grid's tail and waits for it before reading); res_layer:
 // this layer's residual windows (R > 0 tokens) or null
 template <typename T>
-inline rq_status launch_decode_t(const DecodeArgs& a, float* out, const void* res_layer, int R,
+inline rq_status launch_decode_t(DecodeArgs a, float* out, const void* res_layer, int R,
                                  cudaStream_t s) {
-  // a token count per batch row: every row may hold residual tokens
-  auto kern = decode_split_kernel<T>;
-  if (cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, kSplitSmem) != cudaSuccess ||
-      cudaFuncSetAttribute(kern, cudaFuncAttributePreferredSharedMemoryCarveout,
-                           cudaSharedmemCarveoutMaxShared) != cudaSuccess)
+  int dev = 0, sms = 0, smem_sm = 0, reserved = 0;
+  if (cudaGetDevice(&dev) != cudaSuccess ||
+      cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess ||
+      cudaDeviceGetAttribute(&smem_sm, cudaDevAttrMaxSharedMemoryPerMultiprocessor, dev) != cudaSuccess ||
+      cudaDeviceGetAttribute(&reserved, cudaDevAttrReservedSharedMemoryPerBlock, dev) != cudaSuccess)
     return RQ_ERR_CUDA;
+  const long long units = static_cast<long long>(a.B) * a.H;
   const long long nlo = static_cast<long long>(a.u_lo) * a.s_lo;
-  const long long nsplit = nlo + (static_cast<long long>(a.B) * a.H - a.u_lo) * a.splits;
+  const long long nsplit = nlo + (units - a.u_lo) * a.splits;
   // four groups per CTA when the query group takes the merged hi/lo MMA
   // (g <= 4: measured 2-3 % faster on those layers), one otherwise (g = 8:
   // 2-3 % slower as four groups)
   const int G = a.g <= kMaxHeads / 2 ? kGroups : 1;
+  const bool residual = R > 0 || a.n_rows != nullptr;
+  auto merge_kernel = [](int cq) {
+    return cq == 1 ? decode_merge_kernel<1, T> : cq == 2 ? decode_merge_kernel<2, T>
+                   : cq == 4 ? decode_merge_kernel<4, T> : decode_merge_kernel<8, T>;
+  };
+  // Merge CTAs beside the split CTAs: one fits on an SM (its <= 32
+  // registers a thread take the 4,096 the 120-register split kernel leaves),
+  // so the merge grid may have at most one CTA per SM. A whole row per CTA
+  // for a rotated cache (the rotation mixes channels), else the most channel
+  // parts (8, 4, 2) that keep units x parts within the SMs; and its shared
+  // memory must fit in what the split CTAs of an SM leave.
+  int cq = a.hadamard ? 1 : 8;
+  while (cq > 1 && units * cq > sms) cq >>= 1;
+  int msm = merge_smem_bytes(a, cq, residual);
+  bool co = units <= sms;
+  if (co) {
+    cudaFuncAttributes fa;
+    if (cudaFuncGetAttributes(&fa, merge_kernel(cq)) != cudaSuccess) return RQ_ERR_CUDA;
+    const int split_ctas = kGroups / G;                 // resident per SM
+    const int left = smem_sm - split_ctas * (G * kGroupBytes + reserved);
+    co = static_cast<int>(fa.sharedSizeBytes) + msm + reserved <= left;
+  }
+  if (!co) {
+    // a whole row per CTA for a rotated cache, a quarter of the channels
+    // otherwise (four times the CTAs), an eighth when there are few (batch,
+    // kv head) units (the records of a unit are then many, and more CTAs
+    // pull them in parallel)
+    cq = a.hadamard ? 1 : (units <= 32 ? 8 : 4);
+    msm = kMergeSmem;
+  }
+  a.early = (co || G == 1) ? 1 : 0;
+  auto kern = co ? decode_split_kernel_co<T> : decode_split_kernel<T>;
+  if (cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, kSplitSmem) != cudaSuccess ||
+      cudaFuncSetAttribute(kern, cudaFuncAttributePreferredSharedMemoryCarveout,
+                           cudaSharedmemCarveoutMaxShared) != cudaSuccess)
+    return RQ_ERR_CUDA;
   // a programmatic dependent of whatever precedes it in the stream: it
   // launches early only after a grid that allows it (a decode merge), and
   // waits for that grid before writing
@@ -1394,27 +1164,24 @@ inline rq_status launch_decode_t(const DecodeArgs& a, float* out, const void* re
   scfg.attrs = sattr;
   scfg.numAttrs = 1;
   if (cudaLaunchKernelEx(&scfg, kern, a) != cudaSuccess) return RQ_ERR_CUDA;
-  // a whole row per CTA for a rotated cache (the rotation mixes channels),
-  // a quarter of the channels otherwise (four times the CTAs), an eighth when
-  // there are few (batch, kv head) units (the records of a unit are then
-  // many, and more CTAs pull them in parallel)
-  const int cq = a.hadamard ? 1 : (static_cast<long long>(a.B) * a.H <= 32 ? 8 : 4);
   cudaLaunchConfig_t cfg = {};
-  cfg.gridDim = dim3(static_cast<unsigned>(a.B * a.H), static_cast<unsigned>(cq));
+  cfg.gridDim = dim3(static_cast<unsigned>(units), static_cast<unsigned>(cq));
   cfg.blockDim = dim3(kThreads);
-  cfg.dynamicSmemBytes = kMergeSmem;
+  cfg.dynamicSmemBytes = msm;
   cfg.stream = s;
   cudaLaunchAttribute attr[1];
   attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
   attr[0].val.programmaticStreamSerializationAllowed = 1;
   cfg.attrs = attr;
   cfg.numAttrs = 1;
-  auto mk = cq == 1 ? decode_merge_kernel<1, T> : cq == 8 ? decode_merge_kernel<8, T> : decode_merge_kernel<4, T>;
-  if (cudaFuncSetAttribute(mk, cudaFuncAttributeMaxDynamicSharedMemorySize, kMergeSmem) != cudaSuccess)
+  auto mk = merge_kernel(cq);
+  if (cudaFuncSetAttribute(mk, cudaFuncAttributeMaxDynamicSharedMemorySize, kMergeSmem) != cudaSuccess ||
+      cudaFuncSetAttribute(mk, cudaFuncAttributePreferredSharedMemoryCarveout,
+                           cudaSharedmemCarveoutMaxShared) != cudaSuccess)
     return RQ_ERR_CUDA;
   if (cudaLaunchKernelEx(&cfg, mk, static_cast<const float*>(a.partial), out, a.signs, a.status,
                          a.Hq, a.H, a.g, a.splits, a.s_lo, a.u_lo, a.hadamard, static_cast<const T*>(a.q),
-                         static_cast<const T*>(res_layer), R, a.n_rows, a.nblk * kTile) != cudaSuccess)
+                         static_cast<const T*>(res_layer), R, a.n_rows, a.nblk * kTile, msm) != cudaSuccess)
     return RQ_ERR_CUDA;
   return launch_status();
 }
