@@ -67,8 +67,8 @@ struct SplitPlan {
 // rest s_lo + 1, so that every SM holds the same number of splits (units x
 // s_lo splits would leave some SMs one split short and the others, with
 // their full complement, setting the time). The s_lo-split units' splits
-// (the larger ones) come first in the plan; the kernel deals the plan's
-// quarters to the four groups of its CTAs, so every SM gets a like mix.
+// (the larger ones) come first in the plan; the kernel gives consecutive
+// splits to the groups of a CTA, so a CTA holds splits of one size.
 // nblk: the packed blocks attended (<= the capacity's); splits <= the
 // capacity's split bound (max_splits), which sizes the workspace.
 int max_splits(const rq_cache_desc* desc, int slots) {
