@@ -236,7 +236,8 @@ rq_status rq_decode_workspace_bytes(const rq_cache_desc* desc, size_t* bytes);
  * desc->hadamard the rotated cache is used as Q(XR)R^T (App. W "QuaRot kernel").
  * Split-K over the sequence, then a log-sum-exp merge kernel launched as a
  * programmatic dependent of the split kernel (it overlaps the split grid's
- * tail and waits for it before reading).
+ * tail and waits for it before reading; where its shared memory fits, its
+ * CTAs start beside the split CTAs and wait there).
  * q: device [B][H_q][128] of desc->dtype; out: device fp32 [B][H_q][128];
  * ws: device workspace of at least rq_decode_workspace_bytes, 16-byte
  * aligned, contents arbitrary on entry; one call at a time per workspace.
