@@ -134,6 +134,9 @@ size_t workspace_bytes(const rq_cache_desc* desc, int splits) {
   return static_cast<size_t>(desc->B) * desc->H_q * splits * kPart * sizeof(float);
 }
 
+// rq_decode_set_pattern's setting
+std::atomic<int> g_decode_pattern{RQ_DECODE_BACK_TO_BACK};
+
 void fill_args(DecodeArgs& a, const rq_cache_desc* desc, int32_t layer, const void* q,
                const void* packed, const uint8_t* bits_dev, const uint64_t* offsets_dev,
                const int8_t* signs_dev, void* ws, uint32_t* status_dev, const SplitPlan& plan) {
@@ -159,6 +162,7 @@ void fill_args(DecodeArgs& a, const rq_cache_desc* desc, int32_t layer, const vo
   a.kg = stored_grouping(desc->k_grouping);   // wide per-token groups are stored as groups of 32
   a.vg = stored_grouping(desc->v_grouping);
   a.hadamard = desc->hadamard ? 1 : 0;
+  a.mix = g_decode_pattern.load(std::memory_order_relaxed) == RQ_DECODE_INTERLEAVED ? 1 : 0;
   a.kq = desc->k_quantizer;
   a.vq = desc->v_quantizer;
   if (a.kq == RQ_LLOYDMAX || a.vq == RQ_LLOYDMAX) fill_lm_book(a.lm);
@@ -173,6 +177,12 @@ rq_status launch_decode(const DecodeArgs& a, const rq_cache_desc* desc, float* o
 
 }  // namespace
 }  // namespace rq
+
+extern "C" rq_status rq_decode_set_pattern(int32_t pattern) {
+  if (pattern != RQ_DECODE_BACK_TO_BACK && pattern != RQ_DECODE_INTERLEAVED) return RQ_ERR_INVALID_ARG;
+  rq::g_decode_pattern.store(pattern, std::memory_order_relaxed);
+  return RQ_OK;
+}
 
 extern "C" rq_status rq_decode_workspace_bytes(const rq_cache_desc* desc, size_t* bytes) {
   using namespace rq;

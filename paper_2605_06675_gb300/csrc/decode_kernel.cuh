@@ -67,6 +67,7 @@ struct DecodeArgs {
   int layer, B, H, Hq, g, nblk, splits, bps, s_lo, bps_lo, u_lo, kg, vg, hadamard;
   int kq, vq;                // rq_quantizer of keys / values
   int early;                 // let the merge grid launch before the blocks (else after)
+  int mix;                   // deal each CTA one split per quarter of the plan (else consecutive)
   LMBook lm;                 // RQ_LLOYDMAX codebooks
 };
 

@@ -23,6 +23,8 @@ RQ_CAP_5X = 1
 RQ_STATUS_NUMERIC = 1
 RQ_STATUS_BAD_BITS = 2
 RQ_STATUS_BAD_POSITION = 4
+RQ_DECODE_BACK_TO_BACK = 0      # rq_decode_pattern
+RQ_DECODE_INTERLEAVED = 1
 RQ_STATIC_SCRATCH_BYTES = 8 << 20
 HEAD_DIM = 128
 GROUP = 32
@@ -35,7 +37,8 @@ EXPORTS = ["rq_status_string", "rq_abi_version", "rq_lloydmax_levels", "rq_fit_d
            "rq_alloc_continuous", "rq_packed_layout", "rq_calibrate_workspace_bytes",
            "rq_calibrate_distortion", "rq_quantize_pack", "rq_decode_workspace_bytes",
            "rq_decode_attention", "rq_decode_attention_static", "rq_residual_bytes",
-           "rq_append", "rq_decode_attention_len", "rq_append_rows", "rq_decode_attention_rows"]
+           "rq_append", "rq_decode_attention_len", "rq_append_rows", "rq_decode_attention_rows",
+           "rq_decode_set_pattern"]
 
 
 class RQError(RuntimeError):
@@ -86,6 +89,7 @@ def lib() -> ctypes.CDLL:
             "rq_append_rows": ([_P, _I, _P, _P, _P, _P, _P, _P, _P, _P, _P, _P], _I),
             "rq_decode_attention_rows": ([_P, _I, _P, _P, _P, _P, _P, _P, _P, _P, _P, _SZ, _P, _P],
                                          _I),
+            "rq_decode_set_pattern": ([_I], _I),
         }
         for name, (args, res) in sig.items():
             f = getattr(L, name)
@@ -258,6 +262,14 @@ def rq_decode_attention(desc, layer, q, packed, bits_dev, offsets_dev, signs, ou
         ctypes.byref(desc), layer, _dp(q), _dp(packed), _dp(bits_dev), _dp(offsets_dev),
         _dp(signs), _dp(out), _dp(ws), ws.numel() * ws.element_size(), _dp(status),
         _stream(stream)))
+
+
+def rq_decode_set_pattern(pattern: int) -> None:
+    """How this process issues decode calls: RQ_DECODE_BACK_TO_BACK (the
+    default; calls follow one another on the stream) or RQ_DECODE_INTERLEAVED
+    (other kernels run between them). Sets how the split kernel deals splits
+    to its CTAs; results are bit-identical either way."""
+    _check("rq_decode_set_pattern", lib().rq_decode_set_pattern(pattern))
 
 
 def rq_decode_attention_static(desc, layer, q, packed, bits_dev, offsets_dev, signs, out,

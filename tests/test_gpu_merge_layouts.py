@@ -142,6 +142,34 @@ def test_both_layouts_back_to_back(name, B, H, g, S, kg, hadamard, co):
     assert int(path.status.item()) == 0
 
 
+@pytest.mark.parametrize("name,B,H,g,S", [
+    ("pat_g4", 16, 4, 4, 32 * 38),     # 64 units: splits of two sizes, four-group CTAs
+    ("pat_g8", 4, 8, 8, 32 * 40),      # one-group CTAs
+    ("pat_late", 1, 4, 4, 32 * 200),   # the late merge layout
+])
+def test_call_patterns_are_bit_identical(name, B, H, g, S):
+    """RQ_DECODE_INTERLEAVED deals every CTA one split from each quarter of
+    the plan, RQ_DECODE_BACK_TO_BACK consecutive splits: the same splits
+    either way, so the same records and the same output, bit for bit."""
+    rq = ensure_built()
+    wl = _wl(name, B, H, g, S, seed=13)
+    path, signs, k, v, q = _setup(wl)
+    outs = []
+    try:
+        for pattern in (rq.RQ_DECODE_BACK_TO_BACK, rq.RQ_DECODE_INTERLEAVED):
+            rq.rq_decode_set_pattern(pattern)
+            out = torch.full((wl.B, wl.H_q, 128), float("nan"), dtype=torch.float32, device=DEV)
+            path.decode(0, q, out)
+            torch.cuda.synchronize()
+            outs.append(out)
+    finally:
+        rq.rq_decode_set_pattern(rq.RQ_DECODE_BACK_TO_BACK)
+    assert int(path.status.item()) == 0
+    assert torch.isfinite(outs[0]).all()
+    assert torch.equal(outs[0], outs[1])
+    check_layer(path, wl, 0, k, v, q, outs[1], signs, streams=_sampled_streams(wl))
+
+
 @pytest.mark.parametrize("late", [False, True])
 def test_residual_tokens_both_layouts(late):
     """decode_len over a packed prefix plus raw tokens in the residual

@@ -38,6 +38,15 @@ def test_exports_every_header_symbol(rq):
     assert rq.rq_status_string(3) == "unsupported shape"
 
 
+def test_decode_pattern_setting(rq):
+    # host-only: the two documented values are accepted, any other refused
+    lib = rq.lib()
+    assert lib.rq_decode_set_pattern(rq.RQ_DECODE_INTERLEAVED) == rq.RQ_OK
+    assert lib.rq_decode_set_pattern(rq.RQ_DECODE_BACK_TO_BACK) == rq.RQ_OK
+    for bad in (-1, 2, 7):
+        assert rq.STATUS_NAMES[lib.rq_decode_set_pattern(bad)] == "RQ_ERR_INVALID_ARG"
+
+
 def _mse_rows(rng, n):
     a = rng.uniform(0.5, 20, n)
     beta = rng.uniform(3.5, 6.0, n)
