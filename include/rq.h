@@ -226,8 +226,8 @@ rq_status rq_quantize_pack(const rq_cache_desc* desc, int32_t layer, const void*
 
 /* How this process issues its decode calls (a library setting; the paper
  * has no counterpart). It sets how the split kernel deals the splits of a
- * call to the four split groups of its CTAs; results are bit-identical
- * either way. Process-wide, read by every later decode call on any device;
+ * call to the four split groups of its CTAs, and where the merge kernel's
+ * CTAs start; results are bit-identical either way. Process-wide, read by every later decode call on any device;
  * the default is RQ_DECODE_BACK_TO_BACK.
  *  - RQ_DECODE_BACK_TO_BACK: decode calls follow one another on the stream
  *    (a loop over layers): a CTA takes consecutive splits of the plan, all of
@@ -235,7 +235,9 @@ rq_status rq_quantize_pack(const rq_cache_desc* desc, int32_t layer, const void*
  *    the next call's splits.
  *  - RQ_DECODE_INTERLEAVED: other kernels run between the calls (a model's
  *    layers): every CTA takes one split from each quarter of the plan, the
- *    same work per SM, so a call on its own ends sooner.
+ *    same work per SM, and the merge CTAs start where split CTAs have left
+ *    (the split kernel keeps all 128 registers a thread), so a call on its
+ *    own ends sooner.
  * Errors: RQ_ERR_INVALID_ARG (another value). */
 typedef enum { RQ_DECODE_BACK_TO_BACK = 0, RQ_DECODE_INTERLEAVED = 1 } rq_decode_pattern;
 rq_status rq_decode_set_pattern(int32_t pattern);

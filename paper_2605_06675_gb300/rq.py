@@ -268,7 +268,8 @@ def rq_decode_set_pattern(pattern: int) -> None:
     """How this process issues decode calls: RQ_DECODE_BACK_TO_BACK (the
     default; calls follow one another on the stream) or RQ_DECODE_INTERLEAVED
     (other kernels run between them). Sets how the split kernel deals splits
-    to its CTAs; results are bit-identical either way."""
+    to its CTAs and where the merge CTAs start; results are bit-identical
+    either way."""
     _check("rq_decode_set_pattern", lib().rq_decode_set_pattern(pattern))
 
 

@@ -149,8 +149,10 @@ def test_both_layouts_back_to_back(name, B, H, g, S, kg, hadamard, co):
 ])
 def test_call_patterns_are_bit_identical(name, B, H, g, S):
     """RQ_DECODE_INTERLEAVED deals every CTA one split from each quarter of
-    the plan, RQ_DECODE_BACK_TO_BACK consecutive splits: the same splits
-    either way, so the same records and the same output, bit for bit."""
+    the plan and starts the merge CTAs where split CTAs have left (128
+    registers), RQ_DECODE_BACK_TO_BACK deals consecutive splits and, where it
+    fits, starts them beside the split CTAs: the same splits and the same
+    arithmetic either way, so the same output, bit for bit."""
     rq = ensure_built()
     wl = _wl(name, B, H, g, S, seed=13)
     path, signs, k, v, q = _setup(wl)
