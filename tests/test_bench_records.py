@@ -67,3 +67,18 @@ def test_only_included_headers_enter_the_hash(tmp_path, monkeypatch):
     assert bench.kernel_source_hash("k.cu") == h0
     (tmp_path / "include" / "rq.h").write_text("int rq_x(void); int rq_y(void);\n")  # included via a.cuh
     assert bench.kernel_source_hash("k.cu") != h0
+
+
+def test_a_body_included_inside_a_function_enters_the_hash(tmp_path, monkeypatch):
+    # the decode split kernel's body is a file included inside two kernels
+    csrc = tmp_path / "paper_2605_06675_gb300" / "csrc"
+    csrc.mkdir(parents=True)
+    (tmp_path / "include").mkdir()
+    (tmp_path / "include" / "rq.h").write_text("int rq_x(void);\n")
+    (csrc / "body.inc").write_text("  *p += 1;\n")
+    (csrc / "k.cu").write_text('__global__ void k(int* p) {\n#include "body.inc"\n}\n'
+                               '__global__ void k2(int* p) {\n  #include "body.inc"\n}\n')
+    monkeypatch.setattr(bench, "ROOT", str(tmp_path))
+    h0 = bench.kernel_source_hash("k.cu")
+    (csrc / "body.inc").write_text("  *p += 2;\n")
+    assert bench.kernel_source_hash("k.cu") != h0
